@@ -1,0 +1,170 @@
+"""CPU oracle of the integer-only relative-positional MHSA (I-Parakeet, Sec. 3.1).
+
+TEST INFRASTRUCTURE ONLY.  Only ``tests/``, ``__graft_entry__.smoke()`` and
+the CPU-baseline leg of ``bench.py`` may import this package.  It shares no
+code with the GPU library: the arithmetic lives in ``ipo_mhsa.c`` (plain
+int64 C, built here with gcc) and the offline integer constants in
+``consts.py`` (float64, as the paper precomputes them offline, Eq. 7 and
+Eq. 11).  Every function cites the passage it follows.
+
+Pins: ``tests/test_oracle_*.py`` check this oracle against what the paper
+and the mathematics fix (the literal Transformer-XL relative-shift route,
+a float64 relative-position attention, closed forms of the integer softmax
+and brute force on tiny inputs).
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+from .consts import (IBERT_A, IBERT_B, IBERT_C, LayerConstants, dyadic,
+                     dyadic_pair, isoftmax_params, layer_constants)
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "ipo_mhsa.c")
+_LIB = os.path.join(_HERE, "libipo_mhsa.so")
+_lock = threading.Lock()
+_lib = None
+
+
+def build(force: bool = False) -> str:
+    """Compile the C oracle into ``oracle/libipo_mhsa.so`` (gcc, OpenMP)."""
+    if not force and os.path.exists(_LIB) and os.path.getmtime(_LIB) >= max(
+            os.path.getmtime(_SRC), os.path.getmtime(os.path.join(_HERE, "ipo_mhsa.h"))):
+        return _LIB
+    tmp = _LIB + f".tmp{os.getpid()}"
+    cmd = ["gcc", "-O2", "-std=c11", "-fPIC", "-shared", "-fopenmp", "-Wall",
+           "-Wextra", "-o", tmp, _SRC]
+    subprocess.run(cmd, check=True, cwd=_HERE)
+    os.replace(tmp, _LIB)
+    return _LIB
+
+
+class _Params(ctypes.Structure):
+    _fields_ = [("q_ln2", ctypes.c_int32), ("q_b", ctypes.c_int32),
+                ("q_c", ctypes.c_int32)]
+
+
+def _load():
+    global _lib
+    with _lock:
+        if _lib is None:
+            lib = ctypes.CDLL(build())
+            P = ctypes.c_void_p
+            i32 = ctypes.c_int32
+            lib.ipo_relpos_mhsa_i8.argtypes = [P] * 10 + [ctypes.c_int] * 4 + [P]
+            lib.ipo_content_scores_i32.argtypes = [P, P, P] + [ctypes.c_int] * 4 + [P]
+            lib.ipo_position_scores_i32.argtypes = [P, P, P] + [ctypes.c_int] * 4 + [P]
+            lib.ipo_fused_scores_i8.argtypes = [P] * 5 + [i32, i32, i32] + [ctypes.c_int] * 4 + [P]
+            lib.ipo_iexp.argtypes = [i32, P]
+            lib.ipo_iexp.restype = ctypes.c_int64
+            lib.ipo_isoftmax_u8.argtypes = [P, P, ctypes.c_int, ctypes.c_int, P, P]
+            lib.ipo_set_threads.argtypes = [ctypes.c_int]
+            for f in (lib.ipo_relpos_mhsa_i8, lib.ipo_content_scores_i32,
+                      lib.ipo_position_scores_i32, lib.ipo_fused_scores_i8,
+                      lib.ipo_isoftmax_u8, lib.ipo_set_threads):
+                f.restype = ctypes.c_int
+            _lib = lib
+    return _lib
+
+
+def _ptr(a: np.ndarray | None):
+    if a is None:
+        return None
+    assert a.flags["C_CONTIGUOUS"]
+    return a.ctypes.data
+
+
+def _params(c: LayerConstants) -> _Params:
+    return _Params(*c.softmax)
+
+
+class OracleError(RuntimeError):
+    pass
+
+
+def _check(rc: int, what: str):
+    if rc != 0:
+        raise OracleError(f"{what} returned {rc}")
+
+
+def set_threads(n: int) -> int:
+    """OpenMP threads for :func:`relpos_mhsa` (<= 0: all available)."""
+    return _load().ipo_set_threads(n)
+
+
+def relpos_mhsa(q, k, v, p, u, vb, c: LayerConstants, lengths=None) -> np.ndarray:
+    """Whole integer rel-pos MHSA layer (Eqs. 8-11, I-BERT softmax, Eq. 9 and
+    Eq. 7), int8 [B, H, T, dh]."""
+    lib = _load()
+    B, H, T, dh = q.shape
+    out = np.empty_like(q)
+    mult = np.array(c.multipliers, dtype=np.int32)
+    sh = np.array(c.shifts, dtype=np.int32)
+    sm = _params(c)
+    lens = None if lengths is None else np.ascontiguousarray(lengths, dtype=np.int32)
+    rc = lib.ipo_relpos_mhsa_i8(_ptr(q), _ptr(k), _ptr(v), _ptr(p), _ptr(u), _ptr(vb),
+                                _ptr(mult), _ptr(sh), ctypes.addressof(sm), _ptr(lens),
+                                B, H, T, dh, _ptr(out))
+    _check(rc, "ipo_relpos_mhsa_i8")
+    return out
+
+
+def content_scores(q, k, u) -> np.ndarray:
+    """A^c = (Q + 1u^T) K^T of Eq. 8, int32 [B, H, T, T]."""
+    B, H, T, dh = q.shape
+    out = np.empty((B, H, T, T), dtype=np.int32)
+    _check(_load().ipo_content_scores_i32(_ptr(q), _ptr(k), _ptr(u), B, H, T, dh, _ptr(out)),
+           "ipo_content_scores_i32")
+    return out
+
+
+def position_scores(q, p, vb) -> np.ndarray:
+    """Phi((Q + 1v^T) P^T) of Eq. 8 through the static index map, int32 [B, H, T, T]."""
+    B, H, T, dh = q.shape
+    out = np.empty((B, H, T, T), dtype=np.int32)
+    _check(_load().ipo_position_scores_i32(_ptr(q), _ptr(p), _ptr(vb), B, H, T, dh, _ptr(out)),
+           "ipo_position_scores_i32")
+    return out
+
+
+def fused_scores(q, k, p, u, vb, m_c: int, m_p: int, s_s: int) -> np.ndarray:
+    """Eq. 11 fused integer scores on the int8 grid, [B, H, T, T] (no mask)."""
+    B, H, T, dh = q.shape
+    out = np.empty((B, H, T, T), dtype=np.int8)
+    _check(_load().ipo_fused_scores_i8(_ptr(q), _ptr(k), _ptr(p), _ptr(u), _ptr(vb),
+                                       m_c, m_p, s_s, B, H, T, dh, _ptr(out)),
+           "ipo_fused_scores_i8")
+    return out
+
+
+def iexp(d: int, softmax: tuple[int, int, int]) -> int:
+    """I-BERT integer exponential of one integer d <= 0."""
+    sm = _Params(*softmax)
+    return int(_load().ipo_iexp(int(d), ctypes.addressof(sm)))
+
+
+def isoftmax(scores: np.ndarray, softmax: tuple[int, int, int], valid=None) -> np.ndarray:
+    """I-BERT integer softmax along the last axis of int8 scores; ``valid``
+    gives per-row valid-key counts (default: all).  u8 on the grid 2^-8."""
+    s = np.ascontiguousarray(scores, dtype=np.int8)
+    n = s.shape[-1]
+    rows = s.size // n
+    if valid is None:
+        valid = np.full(rows, n, dtype=np.int32)
+    valid = np.ascontiguousarray(np.broadcast_to(valid, s.shape[:-1]).reshape(rows), dtype=np.int32)
+    out = np.empty(s.shape, dtype=np.uint8)
+    sm = _Params(*softmax)
+    _check(_load().ipo_isoftmax_u8(_ptr(s), _ptr(valid), rows, n, ctypes.addressof(sm), _ptr(out)),
+           "ipo_isoftmax_u8")
+    return out
+
+
+__all__ = ["build", "relpos_mhsa", "content_scores", "position_scores",
+           "fused_scores", "iexp", "isoftmax", "set_threads", "dyadic",
+           "dyadic_pair", "isoftmax_params", "layer_constants", "LayerConstants",
+           "IBERT_A", "IBERT_B", "IBERT_C", "OracleError"]

@@ -1,0 +1,88 @@
+"""Offline integer constants of the oracle (float64 on the host, as the paper
+precomputes its multipliers offline, Sec. 2.2 under Eq. 7).
+
+TEST INFRASTRUCTURE ONLY (see the package docstring).
+
+* Dyadic multipliers (Eq. 7, Eq. 11).  The paper writes a real ratio r as
+  m 2^-n with n = 16.  Here the same dyadic form carries more bits: m is a
+  31-bit integer, normalised into [2^30, 2^31) when possible, and the total
+  right shift is n = 31 + s with 0 <= s <= 31 (so r = m 2^-(31+s)).
+* Fused-branch pair (Eq. 11): m_c and m_p share one shift, taken from the
+  larger ratio; the smaller multiplier is rounded on the same shift.
+* I-BERT softmax constants (Kim et al., ICML 2021, integer-only exponential):
+  exp(p) on [-ln2, 0] ~ a (p + b)^2 + c with a = 0.3585, b = 1.353,
+  c = 0.344, and on the grid S: q_ln2 = floor(ln2/S), q_b = floor(b/S),
+  q_c = floor(c / (a S^2)).
+"""
+from __future__ import annotations
+
+import math
+from dataclasses import dataclass
+
+IBERT_A = 0.3585
+IBERT_B = 1.353
+IBERT_C = 0.344
+LN2 = math.log(2.0)
+SOFTMAX_BITS = 8          # attention probabilities on the grid 2^-8
+
+
+def dyadic(ratio: float) -> tuple[int, int]:
+    """(m, s) with m 2^-(31+s) the nearest such value to ``ratio`` and
+    m in [2^30, 2^31) unless s had to be clipped to 31."""
+    if not (ratio > 0.0) or not math.isfinite(ratio):
+        raise ValueError(f"ratio must be positive and finite, got {ratio!r}")
+    frac, exp = math.frexp(ratio)          # ratio = frac 2^exp, frac in [0.5, 1)
+    s = -exp
+    if s > 31:
+        s = 31
+        m = math.floor(ratio * 2.0 ** 62 + 0.5)
+        return int(m), s
+    if s < 0:
+        raise ValueError(f"ratio {ratio!r} >= 1/2^0 cannot be encoded with s >= 0")
+    m = math.floor(frac * 2.0 ** 31 + 0.5)
+    if m == 2 ** 31:
+        m, s = 2 ** 30, s - 1
+        if s < 0:
+            raise ValueError(f"ratio {ratio!r} rounds to 1")
+    return int(m), int(s)
+
+
+def dyadic_pair(r_c: float, r_p: float) -> tuple[int, int, int]:
+    """(m_c, m_p, s) for the two branch ratios of Eq. 11 on one shared shift."""
+    m_big, s = dyadic(max(r_c, r_p))
+    scale = 2.0 ** (31 + s)
+    m_c = int(math.floor(r_c * scale + 0.5))
+    m_p = int(math.floor(r_p * scale + 0.5))
+    if max(m_c, m_p) >= 2 ** 31:
+        raise ValueError("multiplier overflow")
+    return m_c, m_p, s
+
+
+def isoftmax_params(S: float) -> tuple[int, int, int]:
+    """(q_ln2, q_b, q_c) of I-BERT's integer exponential on the grid S."""
+    q_ln2 = math.floor(LN2 / S)
+    q_b = math.floor(IBERT_B / S)
+    q_c = math.floor(IBERT_C / (IBERT_A * (S * S)))
+    return int(q_ln2), int(q_b), int(q_c)
+
+
+@dataclass(frozen=True)
+class LayerConstants:
+    multipliers: tuple[int, int, int]     # m_c, m_p, m_o
+    shifts: tuple[int, int]               # s_s, s_o  (total shift 31 + s)
+    softmax: tuple[int, int, int]         # q_ln2, q_b, q_c
+
+
+def layer_constants(scales: dict, dh: int) -> LayerConstants:
+    """Integer constants of one layer from its declared real scales.
+
+    Eq. 11: r_c = S_Q S_K / (S_s sqrt(dh)), r_p = S_Q S_P / (S_s sqrt(dh)).
+    Eq. 7 for A.V: r_o = 2^-8 S_V / S_O (probabilities on the grid 2^-8).
+    """
+    root = math.sqrt(dh)
+    r_c = scales["S_Q"] * scales["S_K"] / (scales["S_s"] * root)
+    r_p = scales["S_Q"] * scales["S_P"] / (scales["S_s"] * root)
+    r_o = scales["S_V"] / (scales["S_O"] * 2.0 ** SOFTMAX_BITS)
+    m_c, m_p, s_s = dyadic_pair(r_c, r_p)
+    m_o, s_o = dyadic(r_o)
+    return LayerConstants((m_c, m_p, m_o), (s_s, s_o), isoftmax_params(scales["S_s"]))

@@ -1,0 +1,182 @@
+"""Seeded synthetic workloads for the integer relative-positional MHSA.
+
+This module draws inputs only.  It holds none of the attention arithmetic:
+it produces int8 tensors shaped like the Conformer encoder of a
+Parakeet-CTC-0.6B model (d_model = 1024, 8 heads of 128, Sec. 2.1) together
+with the real-valued quantisation scales that an offline calibration would
+declare for them (Eq. 6, min-max ranges).  Both the CPU oracle and the CUDA
+path consume exactly what this module returns; each turns the declared
+scales into its own integer constants.
+
+Recipe (numpy PCG64, seed = 1000 * config + layer unless given):
+
+* Q, K, V, u, v : round(N(0, 30^2)) clipped to [-127, 127]
+  (long-form workload: Q, K, V = round(t_3 * 25) clipped to [-127, 127]).
+* P : the tiny workload draws it like Q.  The others build it the way the
+  model does (Sec. 3.1): the 2T-1 sinusoidal relative-position embeddings
+  (row r <-> relative distance T-1-r, d = 1024), quantised to int8 with
+  S = 1/127, projected through a seeded int8 W_pos [1024, 1024] ~
+  round(N(0, 20^2)), requantised to int8 by its min-max range and split into
+  8 heads of 128.
+* lengths (masked workload): uniform integers in [T/2, T].
+* declared scales: alpha_X ~ U[2, 6] for X in {Q, K, V, P}, S_X = alpha_X/127
+  (u and v live on Q's grid).  S_s, the fused-score grid, is the min-max
+  range estimated from second moments (kappa_s * sigma, kappa_s ~ U[3.5, 5]),
+  so that a few scores saturate at +-127.  S_O = kappa_O * S_V with
+  kappa_O ~ U[1.0625, 1.9375] keeps the output requantisation shift at 8.
+"""
+from __future__ import annotations
+
+import math
+from dataclasses import dataclass, field
+
+import numpy as np
+
+D_MODEL = 1024
+N_HEADS = 8
+D_HEAD = 128
+
+
+@dataclass(frozen=True)
+class Workload:
+    """One named workload: shape and input distribution."""
+    key: int
+    name: str
+    B: int
+    T: int
+    layers: int = 1
+    H: int = N_HEADS
+    dh: int = D_HEAD
+    p_mode: str = "sinusoid"      # "random" | "sinusoid"
+    dist: str = "normal"          # "normal" | "t3"
+    masked: bool = False
+
+    @property
+    def R(self) -> int:
+        return 2 * self.T - 1
+
+    def useful_ops(self) -> int:
+        """Useful integer ops of the whole workload: 6 * dh * T^2 per (b, h)
+        per layer (content, position and attn.V products, one MAC = 2 ops)."""
+        return 6 * self.dh * self.T * self.T * self.B * self.H * self.layers
+
+    def describe(self) -> str:
+        return (f"{self.name}: B={self.B} H={self.H} dh={self.dh} T={self.T} "
+                f"layers={self.layers} P={self.p_mode} dist={self.dist} "
+                f"masked={self.masked}")
+
+
+WORKLOADS = {
+    0: Workload(0, "tiny-T64", B=1, T=64, p_mode="random"),
+    1: Workload(1, "utt10s-T125", B=1, T=125),
+    2: Workload(2, "batch20s-masked-T250", B=16, T=250, masked=True),
+    3: Workload(3, "encoder24-B32-T375", B=32, T=375, layers=24),
+    4: Workload(4, "longform-T1500-t3", B=4, T=1500, dist="t3"),
+}
+
+
+@dataclass
+class Layer:
+    """Inputs of one attention layer.  Arrays are C-contiguous numpy."""
+    q: np.ndarray            # int8 [B, H, T, dh]
+    k: np.ndarray            # int8 [B, H, T, dh]
+    v: np.ndarray            # int8 [B, H, T, dh]
+    p: np.ndarray            # int8 [H, 2T-1, dh]
+    u: np.ndarray            # int8 [H, dh]
+    vb: np.ndarray           # int8 [H, dh]
+    lengths: np.ndarray | None   # int32 [B] or None (all T)
+    scales: dict = field(default_factory=dict)   # declared real scales
+
+    @property
+    def shape(self):
+        B, H, T, dh = self.q.shape
+        return B, H, T, dh
+
+
+def _int8_normal(rng, shape, sigma):
+    x = rng.standard_normal(size=shape, dtype=np.float32)
+    x *= np.float32(sigma)
+    np.rint(x, out=x)
+    np.clip(x, -127, 127, out=x)
+    return x.astype(np.int8)
+
+
+def _int8_t3(rng, shape, scale):
+    x = rng.standard_t(3, size=shape) * scale
+    return np.clip(np.rint(x), -127, 127).astype(np.int8)
+
+
+def sinusoid_relpos(T: int, d: int = D_MODEL) -> np.ndarray:
+    """Sinusoidal embeddings of the 2T-1 relative distances, row r <->
+    distance T-1-r, interleaved sin/cos with frequencies 10000^(-2k/d)."""
+    pos = (T - 1 - np.arange(2 * T - 1, dtype=np.float64))[:, None]
+    freq = np.power(10000.0, -np.arange(0, d, 2, dtype=np.float64) / d)[None, :]
+    pe = np.empty((2 * T - 1, d), dtype=np.float64)
+    pe[:, 0::2] = np.sin(pos * freq)
+    pe[:, 1::2] = np.cos(pos * freq)
+    return pe
+
+
+def _projected_p(rng, T: int, H: int, dh: int) -> np.ndarray:
+    d = H * dh
+    e = np.rint(sinusoid_relpos(T, d) * 127.0)                 # int8 grid, S = 1/127
+    w = np.clip(np.rint(rng.standard_normal((d, d)) * 20.0), -127, 127)
+    acc = e @ w.T                                              # exact: |acc| < 2^53
+    amax = float(np.max(np.abs(acc)))
+    p = np.clip(np.rint(acc * (127.0 / amax)), -127, 127).astype(np.int8)
+    return np.ascontiguousarray(p.reshape(2 * T - 1, H, dh).transpose(1, 0, 2))
+
+
+def _rms(x: np.ndarray) -> float:
+    xf = x.astype(np.float64)
+    return float(np.sqrt(np.mean(xf * xf)))
+
+
+def draw(B: int, H: int, T: int, dh: int, seed: int, *, p_mode: str = "random",
+         dist: str = "normal", masked: bool = False,
+         lengths: np.ndarray | None = None) -> Layer:
+    """Draw one layer of inputs of an arbitrary shape."""
+    rng = np.random.Generator(np.random.PCG64(seed))
+    shape = (B, H, T, dh)
+    if dist == "t3":
+        q, k, v = (_int8_t3(rng, shape, 25.0) for _ in range(3))
+    elif dist == "normal":
+        q, k, v = (_int8_normal(rng, shape, 30.0) for _ in range(3))
+    else:
+        raise ValueError(f"unknown distribution {dist!r}")
+    u = _int8_normal(rng, (H, dh), 30.0)
+    vb = _int8_normal(rng, (H, dh), 30.0)
+    if p_mode == "random":
+        p = _int8_normal(rng, (H, 2 * T - 1, dh), 30.0)
+    elif p_mode == "sinusoid":
+        p = _projected_p(rng, T, H, dh)
+    else:
+        raise ValueError(f"unknown P mode {p_mode!r}")
+    if lengths is None and masked:
+        lengths = rng.integers(T // 2, T, size=B, endpoint=True).astype(np.int32)
+    elif lengths is not None:
+        lengths = np.ascontiguousarray(lengths, dtype=np.int32)
+
+    a_q, a_k, a_v, a_p = rng.uniform(2.0, 6.0, size=4)
+    s_q, s_k, s_v, s_p = a_q / 127, a_k / 127, a_v / 127, a_p / 127
+    # Second-moment estimate of the real fused score (Q+u)K^T + (Q+v)P^T,
+    # divided by sqrt(dh); its min-max range is taken as kappa_s sigma.
+    rq = _rms(q)
+    sig_c = math.sqrt(dh) * math.hypot(rq, _rms(u)) * _rms(k) * s_q * s_k
+    sig_p = math.sqrt(dh) * math.hypot(rq, _rms(vb)) * _rms(p) * s_q * s_p
+    sigma = math.hypot(sig_c, sig_p) / math.sqrt(dh)
+    kappa_s = rng.uniform(3.5, 5.0)
+    s_s = kappa_s * sigma / 127
+    s_o = rng.uniform(1.0625, 1.9375) * s_v
+    scales = dict(S_Q=s_q, S_K=s_k, S_V=s_v, S_P=s_p, S_s=s_s, S_O=s_o)
+    return Layer(q=q, k=k, v=v, p=p, u=u, vb=vb, lengths=lengths, scales=scales)
+
+
+def layer(workload: int | Workload, index: int = 0, seed: int | None = None) -> Layer:
+    """Inputs of layer `index` of a named workload."""
+    w = WORKLOADS[workload] if isinstance(workload, int) else workload
+    if seed is None:
+        seed = 1000 * w.key + index
+    return draw(w.B, w.H, w.T, w.dh, seed, p_mode=w.p_mode, dist=w.dist,
+                masked=w.masked)
+

@@ -1,0 +1,79 @@
+"""The pins must catch plausible mistakes in the oracle.
+
+Each case plants one mistake in a copy of the oracle's C source (on the
+CPU, in a temporary directory), rebuilds it there and runs the fast pins
+against the copy in a subprocess: every mutant must make at least one pin
+fail.
+"""
+import os
+import shutil
+import subprocess
+import sys
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+MUTANTS = {
+    # mirrored relative shift (i - j instead of j - i)
+    "phi_direction": ("int r = j - i + T - 1;", "int r = i - j + T - 1;"),
+    # content branch without the u bias
+    "drop_u": ("((int64_t)qi[d] + (int64_t)u[d]) * (int64_t)kj[d]",
+               "((int64_t)qi[d]) * (int64_t)kj[d]"),
+    # position branch without the v bias
+    "drop_v": ("((int64_t)qi[d] + (int64_t)vb[d]) * (int64_t)pr[d]",
+               "((int64_t)qi[d]) * (int64_t)pr[d]"),
+    # truncation instead of rounding in Eq. 11 / Eq. 7
+    "floor_not_round": ("return floor_div_pow2(x + ((int64_t)1 << (n - 1)), n);",
+                        "return floor_div_pow2(x, n);"),
+    # shift of 2^-n off by one
+    "shift_off_by_one": ("return clamp_i8(round_shift(x, 31 + s_s));",
+                         "return clamp_i8(round_shift(x, 30 + s_s));"),
+    # exponential without the 2^-z factor
+    "iexp_no_shift": ("return L >> z; /* L >= 0 */", "return L; /* L >= 0 */"),
+    # exponential with the sign of q_b flipped
+    "iexp_sign": ("int64_t t = p + sm->q_b;", "int64_t t = p - sm->q_b;"),
+    # normaliser with the wrong output grid
+    "softmax_grid": ("int64_t y = (e[j] * f) >> 24;", "int64_t y = (e[j] * f) >> 25;"),
+    # masked keys still counted in the softmax
+    "mask_keys": ("isoftmax_row(srow, len, len, sm, e, a);",
+                  "for (int j = len; j < T; ++j) srow[j] = srow[0];\n        isoftmax_row(srow, T, T, sm, e, a);"),
+    # transposed operand in A.V
+    "av_transpose": ("acc += (int64_t)a[j] * (int64_t)vh[(size_t)j * dh + d];",
+                     "acc += (int64_t)a[j] * (int64_t)vh[(size_t)d * dh + j % dh];"),
+}
+
+PINS = [
+    "tests/test_oracle_relshift.py",
+    "tests/test_oracle_scores.py",
+    "tests/test_oracle_softmax.py::test_iexp_polynomial_accuracy",
+    "tests/test_oracle_softmax.py::test_iexp_halving_identity",
+    "tests/test_oracle_softmax.py::test_softmax_uniform_closed_form",
+    "tests/test_oracle_softmax.py::test_softmax_single_key_is_255",
+    "tests/test_oracle_layer.py::test_layer_vs_float64_attention",
+    "tests/test_oracle_layer.py::test_masked_layer_equals_truncated_problem",
+    "tests/test_oracle_layer.py::test_single_frame_closed_form",
+]
+
+
+def _copy_tree(dst):
+    for name in ("oracle", "synth", "tests"):
+        shutil.copytree(os.path.join(ROOT, name), os.path.join(dst, name),
+                        ignore=shutil.ignore_patterns("*.so", "__pycache__", "*.tmp*"))
+
+
+@pytest.mark.slow
+@pytest.mark.parametrize("name", sorted(MUTANTS))
+def test_mutant_is_caught(tmp_path, name):
+    old, new = MUTANTS[name]
+    _copy_tree(tmp_path)
+    src = tmp_path / "oracle" / "ipo_mhsa.c"
+    text = src.read_text()
+    assert text.count(old) == 1, f"mutation site for {name} not found"
+    src.write_text(text.replace(old, new))
+    env = dict(os.environ, PYTHONPATH=str(tmp_path))
+    res = subprocess.run([sys.executable, "-m", "pytest", "-x", "-q", "-p", "no:cacheprovider",
+                          "-m", "not gpu and not slow"] + PINS,
+                         cwd=tmp_path, env=env, capture_output=True, text=True, timeout=600)
+    assert res.returncode != 0, f"mutant {name} survived the pins:\n{res.stdout[-2000:]}"
+    assert "failed" in res.stdout or "error" in res.stdout.lower()
