@@ -1,0 +1,399 @@
+#!/usr/bin/env python3
+"""Benchmark of the integer-only relative-positional MHSA on GB300.
+
+One step = one pass of the whole hot path over the encoder workload: 24
+stacked attention layers, B = 32 utterances of T = 375 frames (30 s), 8
+heads of 128, each layer with its own seeded int8 Q/K/V/P/u/v and its own
+dyadic constants (bias vectors, content and position branches, relative
+shift, fused requantisation, integer softmax, attn.V and output
+requantisation, all in the CUDA kernels behind the C ABI).
+
+Metric: effective TOPS = useful integer ops (6 * dh * T^2 per head and
+layer, one multiply-add = 2 ops) / time, plus the attention-only real-time
+factor (time / (B * 30 s)).  Inputs stay resident in HBM (1.2 GB per step,
+far above the 129 MB L2, so nothing is reused across steps from L2).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+Multi-GPU: the path shards with no exchange step; each rank runs its own
+replica of the workload (weak scaling) and `value` sums the ranks' work over
+the slowest rank's time.  `--impl reference` times the CPU oracle on the
+host cores instead (rank 0 only).
+"""
+from __future__ import annotations
+
+import argparse
+import ctypes
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import synth  # noqa: E402
+
+WORKLOAD = 3
+METRIC = "INT8 rel-pos MHSA effective TOPS & % of roofline; attention RTF at B=32,T=375"
+UTT_SECONDS = 30.0          # T = 375 frames at 80 ms
+L2_BYTES = 129 * 1024 * 1024
+TRAFFIC_FILE = os.path.join(ROOT, "profiles", "fused_kernel_traffic.json")
+KERNEL_SRC = os.path.join(ROOT, "paper_2609_30846_gb300", "csrc", "ip_mhsa_kernels.cuh")
+
+
+def parse_args():
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--e2e-steps", type=int, default=3)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=15.0,
+                    help="target length of the CPU-baseline sample")
+    return ap.parse_args()
+
+
+def dist_env():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+# ------------------------------------------------------------------- clocks
+
+class ClockSampler:
+    """nvidia-smi samples every 200 ms while the timed region runs."""
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        fd, self.path = tempfile.mkstemp(prefix="clocks", suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.QUERY}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+        time.sleep(0.3)
+
+    def stop(self) -> dict:
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+        rows = []
+        if self.path and os.path.exists(self.path):
+            with open(self.path) as f:
+                for line in f:
+                    parts = [x.strip() for x in line.split(",")]
+                    if len(parts) >= 9:
+                        rows.append(parts)
+            os.unlink(self.path)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"]}
+
+        def num(x):
+            try:
+                return float(x)
+            except ValueError:
+                return None
+        sm = [num(r[1]) for r in rows if num(r[1]) is not None]
+        mx = [num(r[2]) for r in rows if num(r[2]) is not None]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i].lower() == "active"})
+        loaded = [s for s in sm if mx and s > 0.5 * max(mx)] or sm
+        return {"sm_mhz": statistics.median(loaded) if loaded else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": reasons,
+                "samples": len(rows)}
+
+
+# ------------------------------------------------------------------- inputs
+
+def make_layers(n_layers: int, B: int | None = None):
+    w = synth.WORKLOADS[WORKLOAD]
+    layers = []
+    for i in range(n_layers):
+        lay = synth.layer(w, i)
+        if B is not None and B < w.B:
+            lay = synth.Layer(*(np.ascontiguousarray(a[:B]) for a in (lay.q, lay.k, lay.v)),
+                              lay.p, lay.u, lay.vb, None, lay.scales)
+        layers.append(lay)
+    return layers
+
+
+def useful_ops(B, H, T, dh, layers):
+    return 6 * dh * T * T * B * H * layers
+
+
+def traffic_per_launch():
+    """DRAM bytes per fused-kernel launch from the committed ncu summary,
+    if it was taken on the current kernel source (else None)."""
+    if not os.path.exists(TRAFFIC_FILE):
+        return None
+    try:
+        rec = json.load(open(TRAFFIC_FILE))
+        src = hashlib.sha256(open(KERNEL_SRC, "rb").read()).hexdigest()
+        if rec.get("kernel_sha256") != src:
+            return None
+        return rec.get("dram_bytes_per_launch")
+    except (OSError, ValueError):
+        return None
+
+
+# ------------------------------------------------------------------- oracle arm
+
+def cpu_sample(layers, threads: int, target_s: float):
+    """Times the oracle, as it stands, on a bounded sample of the workload:
+    the first `nb` utterances of every layer, nb calibrated on one layer."""
+    import oracle
+    oracle.build()
+    oracle.set_threads(threads)
+    w = synth.WORKLOADS[WORKLOAD]
+    consts = [oracle.layer_constants(l.scales, w.dh) for l in layers]
+    q0 = layers[0]
+    t = time.perf_counter()
+    oracle.relpos_mhsa(np.ascontiguousarray(q0.q[:1]), np.ascontiguousarray(q0.k[:1]),
+                       np.ascontiguousarray(q0.v[:1]), q0.p, q0.u, q0.vb, consts[0])
+    per_utt_layer = max(time.perf_counter() - t, 1e-4)
+    nb = int(max(1, min(w.B, target_s / (per_utt_layer * len(layers)))))
+    t = time.perf_counter()
+    for lay, c in zip(layers, consts):
+        oracle.relpos_mhsa(np.ascontiguousarray(lay.q[:nb]), np.ascontiguousarray(lay.k[:nb]),
+                           np.ascontiguousarray(lay.v[:nb]), lay.p, lay.u, lay.vb, c)
+    dt = time.perf_counter() - t
+    ops = useful_ops(nb, w.H, w.T, w.dh, len(layers))
+    return {"value": ops / dt / 1e12, "unit": "TOPS", "cores": threads, "kind": "oracle",
+            "sample": f"{len(layers)} layers x {nb} of {w.B} utterances (T={w.T}, H={w.H}), "
+                      f"{dt:.1f} s, int64 scalar C + OpenMP"}
+
+
+def run_reference(args):
+    world, rank, _ = dist_env()
+    if rank != 0:
+        return 0
+    w = synth.WORKLOADS[WORKLOAD]
+    import oracle
+    oracle.build()
+    threads = os.cpu_count() or 1
+    oracle.set_threads(threads)
+    layers = make_layers(w.layers, B=1)
+    consts = [oracle.layer_constants(l.scales, w.dh) for l in layers]
+
+    def step():
+        for lay, c in zip(layers, consts):
+            oracle.relpos_mhsa(lay.q, lay.k, lay.v, lay.p, lay.u, lay.vb, c)
+    for _ in range(args.warmup):
+        step()
+    t = time.perf_counter()
+    for _ in range(args.steps):
+        step()
+    dt = time.perf_counter() - t
+    ops = useful_ops(1, w.H, w.T, w.dh, w.layers) * args.steps
+    value = ops / dt / 1e12
+    ms = dt / args.steps * 1e3
+    sample = f"per step {w.layers} layers x 1 of {w.B} utterances (T={w.T}, H={w.H})"
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "TOPS", "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "int64", "data": "synthetic",
+        "config": {"workload": f"{w.name} (sampled: 1 utterance per layer)", "B": 1, "T": w.T,
+                   "H": w.H, "dh": w.dh, "layers": w.layers, "l2": "cpu"},
+        "rtf": (dt / args.steps) / (1 * UTT_SECONDS),
+        "cpu_baseline": {"value": value, "unit": "TOPS", "cores": threads, "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": value, "unit": "TOPS", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+# ------------------------------------------------------------------- GPU arm
+
+def run_ours(args):
+    import torch
+    import paper_2609_30846_gb300 as ip
+
+    world, rank, local = dist_env()
+    if not torch.cuda.is_available():
+        raise SystemExit("bench.py needs a CUDA GPU (the attention runs only in CUDA kernels)")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+    ip.load()
+
+    w = synth.WORKLOADS[WORKLOAD]
+    B, H, T, dh, NL = w.B, w.H, w.T, w.dh, w.layers
+    layers = make_layers(NL)
+    consts = [ip.layer_constants(l.scales) for l in layers]
+    to_dev = lambda a: torch.from_numpy(np.ascontiguousarray(a)).to(dev)
+    dl = [dict(q=to_dev(l.q), k=to_dev(l.k), v=to_dev(l.v), p=to_dev(l.p), u=to_dev(l.u),
+               vb=to_dev(l.vb), out=torch.empty((B, H, T, dh), dtype=torch.int8, device=dev))
+          for l in layers]
+    ws = torch.empty(ip.workspace_bytes(B, H, T, dh), dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    lib = ip.load()
+    hstream = ctypes.c_void_p(stream.cuda_stream)
+
+    # Pre-marshalled C-ABI arguments of every layer: the timed loop is the
+    # bare library calls.
+    calls = []
+    for d, c in zip(dl, consts):
+        sm = ip.SoftmaxParams(*c.softmax)
+        mult = (ctypes.c_int32 * 3)(*c.multipliers)
+        sh = (ctypes.c_int32 * 2)(*c.shifts)
+        ptr = lambda t: ctypes.c_void_p(t.data_ptr())
+        calls.append((ptr(d["q"]), ptr(d["k"]), ptr(d["v"]), ptr(d["p"]), ptr(d["u"]), ptr(d["vb"]),
+                      mult, sh, ctypes.byref(sm), None, B, H, T, dh, ptr(d["out"]),
+                      ctypes.c_void_p(ws.data_ptr()), ws.numel(), hstream, sm))
+    fn = lib.ip_relpos_mhsa_i8
+
+    def step(events=None):
+        for i, a in enumerate(calls):
+            if events is not None:
+                events[i][0].record(stream)
+            rc = fn(*a[:-1])
+            if events is not None:
+                events[i][1].record(stream)
+            if rc != 0:
+                raise ip.IpError("ip_relpos_mhsa_i8", rc, ip.strerror(rc))
+
+    peak = ip.int8_mma_peak_tops()
+    for _ in range(max(args.warmup, 3)):
+        step()
+    if ip.status(ws, stream) != 0:
+        raise SystemExit("kernel reported a barrier timeout during warm-up")
+
+    ev = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+           for _ in range(NL)] for _ in range(args.steps)]
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    clocks = ClockSampler(local)
+    clocks.start()
+    if dist:
+        dist.barrier()
+    torch.cuda.synchronize(dev)
+    t0.record(stream)
+    for s in range(args.steps):
+        step(ev[s])
+    t1.record(stream)
+    torch.cuda.synchronize(dev)
+    if dist:
+        dist.barrier()
+    clk = clocks.stop()
+    total_ms = t0.elapsed_time(t1)
+    layer_ms = [a.elapsed_time(b) for st in ev for (a, b) in st]
+    if ip.status(ws, stream) != 0:
+        raise SystemExit("kernel reported a barrier timeout in the timed region")
+
+    if dist:
+        tt = torch.tensor([total_ms], device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        total_ms = float(tt.item())
+
+    ops_step = useful_ops(B, H, T, dh, NL)
+    value = ops_step * args.steps * world / (total_ms * 1e-3) / 1e12
+    ms_step = total_ms / args.steps
+    ops_layer = useful_ops(B, H, T, dh, 1)
+    avg_layer_ms = statistics.mean(layer_ms)
+    achieved = ops_layer / (avg_layer_ms * 1e-3) / 1e12
+
+    # ---- end to end through the host-buffer entry point
+    e2e = None
+    if args.e2e_steps > 0:
+        pin = lambda a: torch.from_numpy(np.ascontiguousarray(a)).pin_memory()
+        hl = [dict(q=pin(l.q), k=pin(l.k), v=pin(l.v), p=pin(l.p), u=pin(l.u), vb=pin(l.vb),
+                   out=torch.empty((B, H, T, dh), dtype=torch.int8).pin_memory()) for l in layers]
+        arena = torch.empty(ip.host_arena_bytes(B, H, T, dh), dtype=torch.uint8, device=dev)
+
+        def e2e_step():
+            for h_, c in zip(hl, consts):
+                ip.relpos_mhsa_i8_host(h_["q"], h_["k"], h_["v"], h_["p"], h_["u"], h_["vb"], c,
+                                       None, h_["out"], arena, stream=stream)
+        e2e_step()
+        torch.cuda.synchronize(dev)
+        if dist:
+            dist.barrier()
+        t = time.perf_counter()
+        for _ in range(args.e2e_steps):
+            e2e_step()
+        torch.cuda.synchronize(dev)
+        e2e_s = time.perf_counter() - t
+        if dist:
+            tt = torch.tensor([e2e_s], device=dev)
+            dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+            e2e_s = float(tt.item())
+        h2d = sum(int(h_[k].numel()) for h_ in hl for k in ("q", "k", "v", "p", "u", "vb"))
+        d2h = sum(int(h_["out"].numel()) for h_ in hl)
+        e2e = {"value": ops_step * args.e2e_steps * world / e2e_s / 1e12, "unit": "TOPS",
+               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+               "ms_per_step": e2e_s / args.e2e_steps * 1e3, "steps": args.e2e_steps}
+
+    if rank != 0:
+        if dist:
+            dist.destroy_process_group()
+        return 0
+
+    cpu = None
+    if world == 1 and not args.no_cpu_baseline:
+        cpu = cpu_sample(layers, os.cpu_count() or 1, args.cpu_seconds)
+
+    bytes_layer = 4 * B * H * T * dh + H * (2 * T - 1) * dh + 2 * H * dh
+    line = {
+        "metric": METRIC, "value": value, "unit": "TOPS", "n_gpus": world, "steps": args.steps,
+        "warmup": max(args.warmup, 3), "ms_per_step": ms_step, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "s8xs8->s32 (int32/int64 epilogue)",
+        "data": "synthetic",
+        "config": {"workload": w.name, "B": B, "H": H, "T": T, "dh": dh, "layers": NL,
+                   "parallelism": f"replicas x{world}" if world > 1 else "1 GPU",
+                   "l2": "inputs larger than L2 (%.2f GB per step, L2 129 MB)" % (bytes_layer * NL / 1e9)},
+        "rtf": ms_step * 1e-3 / (B * UTT_SECONDS),
+        "paper_rtf_npu_full_model": 0.048,
+        "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TOPS",
+                     "frac": achieved / peak, "traffic": traffic_per_launch(),
+                     "peak_source": "measured in this run: integer warp MMA (mma.sync m16n8k32 "
+                                    "s8) probe, CUDA events; sm_103a has no tcgen05 kind::i8",
+                     "hbm_floor_frac": (bytes_layer / 6757.2e9) / (avg_layer_ms * 1e-3),
+                     "kernel": "relpos_mhsa_fused_kernel (+bias_vectors_kernel in the same call)"},
+        "cpu_baseline": cpu,
+        "e2e": e2e,
+        "gpu_launches": 2 * NL * args.steps,
+        "clocks": clk,
+    }
+    print(json.dumps(line), flush=True)
+    if dist:
+        dist.destroy_process_group()
+    return 0
+
+
+def main():
+    args = parse_args()
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_ours(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

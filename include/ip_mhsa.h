@@ -1,0 +1,155 @@
+/*
+ * ip_mhsa.h - C ABI of the integer-only relative-positional multi-head
+ * self-attention of I-Parakeet (Sec. 3.1) on one GB300 GPU (sm_103a).
+ *
+ * Per (batch b, head h), with T frames, head width dh = 128 and R = 2T-1
+ * relative positions, the library computes
+ *
+ *   content   qc[i][j] = sum_d (Q[i][d] + u[d]) K[j][d]                (Eq. 8)
+ *   position  qp[i][j] = sum_d (Q[i][d] + v[d]) P[j - i + T - 1][d]    (Eq. 8,
+ *             the relative shift Phi applied as an index map; P row r holds
+ *             relative distance T-1-r)
+ *   fused     qs = clamp(round(2^-(31+s_s) (m_c qc + m_p qp)), -127, 127)
+ *                                                             (Eqs. 10-11, 6)
+ *   softmax   I-BERT integer softmax over the valid keys j < len_b:
+ *             mx = max_j qs, e_j = iexp(qs_j - mx), f = floor(2^32 / sum e),
+ *             a_j = min(255, floor(e_j f / 2^24))  (probabilities on 2^-8)
+ *             iexp(d): z = floor(-d / q_ln2), p = d + z q_ln2,
+ *                      floor(((p + q_b)^2 + q_c) / 2^z)
+ *   output    O[i][d] = clamp(round(2^-(31+s_o) m_o sum_j a_j V[j][d]),
+ *                             -127, 127)                      (Eq. 9, Eq. 7)
+ *
+ * and writes O; query rows i >= len_b are written as 0.  round(x 2^-n) is
+ * floor((x + 2^(n-1)) / 2^n) (ties toward +infinity).  Every step runs in
+ * integer arithmetic on the GPU; the offline helpers at the end turn real
+ * scales into the integer constants on the host, as the paper precomputes
+ * its multipliers offline (Sec. 2.2, under Eq. 7).
+ *
+ * Layouts: all arrays C-contiguous, int8 unless stated.
+ *   q, k, v, out : [B][H][T][dh]      p : [H][2T-1][dh]      u, v_bias : [H][dh]
+ * Ownership: every buffer belongs to the caller; the library allocates no
+ * memory.  Device entry points are asynchronous on `stream`; inputs are not
+ * modified.  Return value: IP_OK (0) or a negative IP_ERR_* code
+ * (ip_strerror gives its text); the library never aborts the process.
+ */
+#ifndef IP_MHSA_H
+#define IP_MHSA_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct CUstream_st *ip_stream_t; /* a cudaStream_t; NULL = legacy default stream */
+
+/* Integer constants of I-BERT's exponential on the fused-score grid S_s:
+ * q_ln2 = floor(ln2 / S_s), q_b = floor(1.353 / S_s),
+ * q_c = floor(0.344 / (0.3585 S_s^2)).  Domain: q_ln2 >= 1, q_b >= 0,
+ * q_c >= 0, q_b^2 + q_c >= 2, and (p + q_b)^2 + q_c < 2^31 for all p in
+ * (-q_ln2, 0]. */
+typedef struct {
+    int32_t q_ln2;
+    int32_t q_b;
+    int32_t q_c;
+} ip_isoftmax_params;
+
+#define IP_OK 0
+#define IP_ERR_NULL (-1)        /* a required pointer is NULL */
+#define IP_ERR_SHAPE (-2)       /* B, H, T out of range (see IP_MAX_*) */
+#define IP_ERR_ALIGN (-3)       /* a pointer is not 16-byte aligned (workspace: 256) */
+#define IP_ERR_UNSUPPORTED (-4) /* dh != 128 */
+#define IP_ERR_CUDA (-5)        /* a CUDA runtime call failed */
+#define IP_ERR_TIMEOUT (-6)     /* a kernel gave up waiting on a barrier */
+#define IP_ERR_PARAM (-7)       /* a multiplier, shift or softmax constant is out of its domain */
+#define IP_ERR_WORKSPACE (-8)   /* workspace smaller than ip_relpos_mhsa_workspace_bytes */
+
+#define IP_DH 128
+#define IP_MAX_T 2048   /* frames; the int8 scores of a 64-row tile stay in shared memory */
+#define IP_MAX_B 65535
+#define IP_MAX_H 65535
+
+/* Bytes of device workspace one call needs: an error word plus the bias
+ * vectors (K u) [B][H][T] and (P v) [H][2T-1] as int32 (the exact rank-1
+ * split of (Q + 1u^T)K^T and (Q + 1v^T)P^T).  0 if the shape is invalid. */
+size_t ip_relpos_mhsa_workspace_bytes(int B, int H, int T, int dh);
+
+/* The whole layer on the GPU.
+ *   q, k, v, p, u, v_bias, out : device pointers, 16-byte aligned.
+ *   multipliers : HOST array {m_c, m_p, m_o}, each in [0, 2^31).
+ *   shifts      : HOST array {s_s, s_o}, each in [0, 31]; the right shift
+ *                 of Eq. 11 is 31 + s_s, that of the output 31 + s_o.
+ *   sm          : HOST pointer to the softmax constants.
+ *   lengths     : DEVICE array [B] of valid lengths (values clamped to
+ *                 [0, T]), or NULL for all T.
+ *   workspace   : device memory of workspace_bytes >= the size above,
+ *                 256-byte aligned, owned by the caller; one call at a time
+ *                 per workspace.
+ * The call validates its arguments on the host and then enqueues two
+ * kernels on `stream`.  B == 0 or H == 0 is an empty problem: the call
+ * returns IP_OK without touching any pointer.  A kernel-side barrier timeout is reported later by
+ * ip_relpos_mhsa_status. */
+int ip_relpos_mhsa_i8(const int8_t *q, const int8_t *k, const int8_t *v,
+                      const int8_t *p, const int8_t *u, const int8_t *v_bias,
+                      const int32_t *multipliers, const int32_t *shifts,
+                      const ip_isoftmax_params *sm, const int32_t *lengths,
+                      int B, int H, int T, int dh, int8_t *out,
+                      void *workspace, size_t workspace_bytes, ip_stream_t stream);
+
+/* Synchronises `stream` and reports the device-side status of the last call
+ * that used `workspace`: IP_OK, IP_ERR_TIMEOUT, or IP_ERR_CUDA. */
+int ip_relpos_mhsa_status(const void *workspace, ip_stream_t stream);
+
+/* Bytes of device staging memory ip_relpos_mhsa_i8_host needs (inputs,
+ * output, lengths and workspace), 0 if the shape is invalid. */
+size_t ip_relpos_mhsa_host_arena_bytes(int B, int H, int T, int dh);
+
+/* The whole layer from HOST buffers: copies the inputs (and lengths, a HOST
+ * array or NULL) into `arena` (device memory of arena_bytes >= the size
+ * above, 256-byte aligned, owned by the caller), runs ip_relpos_mhsa_i8,
+ * copies the result into the HOST buffer `out` and synchronises `stream`.
+ * Page-locked host buffers make the copies asynchronous DMA. */
+int ip_relpos_mhsa_i8_host(const int8_t *q, const int8_t *k, const int8_t *v,
+                           const int8_t *p, const int8_t *u, const int8_t *v_bias,
+                           const int32_t *multipliers, const int32_t *shifts,
+                           const ip_isoftmax_params *sm, const int32_t *lengths,
+                           int B, int H, int T, int dh, int8_t *out,
+                           void *arena, size_t arena_bytes, ip_stream_t stream);
+
+/* Text of an IP_* code. */
+const char *ip_strerror(int code);
+
+/* Test hook: bound, in SM clock cycles, of every barrier wait inside the
+ * kernels launched afterwards by this process (0 = give up at the first
+ * wait that is not already satisfied; negative = the default of about two
+ * seconds).  A wait that runs out records IP_ERR_TIMEOUT for
+ * ip_relpos_mhsa_status; the kernel lets its own copies in flight land and
+ * returns. */
+int ip_debug_set_timeout_cycles(long long cycles);
+
+/* Diagnostic: enqueues a throughput probe of the integer warp MMA
+ * (mma.sync m16n8k32 s8 x s8 -> s32, eight independent accumulators per
+ * warp, `iters` rounds) on `stream`; sink is a device int array of
+ * blocks * 256 entries.  Returns the number of integer ops the launch
+ * performs (one multiply-add = 2), or -1 on error.  Timing it with events
+ * gives the measured INT8 peak of this GPU. */
+long long ip_probe_int8_mma(int blocks, int iters, int *sink, ip_stream_t stream);
+
+/* ---- offline constants (host only, float64, run once per layer) -------- */
+
+/* m, s with m 2^-(31+s) nearest to ratio, m in [2^30, 2^31) unless s is
+ * clipped at 31.  ratio must be in (0, 1 - 2^-32). */
+int ip_dyadic_multiplier(double ratio, int32_t *m, int32_t *s);
+
+/* Eq. 11 multipliers of the two score branches on one shared shift s,
+ * taken from the larger ratio. */
+int ip_dyadic_pair(double r_c, double r_p, int32_t *m_c, int32_t *m_p, int32_t *s);
+
+/* I-BERT exponential constants on the score grid S_s (see the struct). */
+int ip_isoftmax_params_from_scale(double S_s, ip_isoftmax_params *out);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* IP_MHSA_H */

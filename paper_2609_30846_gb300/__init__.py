@@ -1,0 +1,280 @@
+"""Integer-only relative-positional MHSA (I-Parakeet, Sec. 3.1) on GB300.
+
+A thin Python binding over the C ABI of ``include/ip_mhsa.h``: argument
+marshalling only.  Every step of the attention runs in the CUDA kernels of
+``libipmhsa.so``; there is no CPU fallback, and a missing or unloadable
+library raises :class:`LibraryError`.  PyTorch serves for device memory and
+streams only.
+"""
+from __future__ import annotations
+
+import ctypes
+import math
+import threading
+from dataclasses import dataclass
+
+from . import build as _build
+
+IP_DH = 128
+IP_MAX_T = 2048
+
+ERRORS = {
+    0: "IP_OK", -1: "IP_ERR_NULL", -2: "IP_ERR_SHAPE", -3: "IP_ERR_ALIGN",
+    -4: "IP_ERR_UNSUPPORTED", -5: "IP_ERR_CUDA", -6: "IP_ERR_TIMEOUT",
+    -7: "IP_ERR_PARAM", -8: "IP_ERR_WORKSPACE",
+}
+
+EXPORTS = (
+    "ip_relpos_mhsa_workspace_bytes", "ip_relpos_mhsa_i8", "ip_relpos_mhsa_status",
+    "ip_relpos_mhsa_host_arena_bytes", "ip_relpos_mhsa_i8_host", "ip_strerror",
+    "ip_debug_set_timeout_cycles", "ip_dyadic_multiplier", "ip_dyadic_pair",
+    "ip_isoftmax_params_from_scale", "ip_probe_int8_mma",
+)
+
+
+class LibraryError(RuntimeError):
+    """The GPU library could not be built or loaded."""
+
+
+class IpError(RuntimeError):
+    """A library call returned an IP_ERR_* code."""
+
+    def __init__(self, fn: str, code: int, text: str):
+        super().__init__(f"{fn}: {ERRORS.get(code, code)} ({text})")
+        self.code = code
+
+
+class SoftmaxParams(ctypes.Structure):
+    _fields_ = [("q_ln2", ctypes.c_int32), ("q_b", ctypes.c_int32), ("q_c", ctypes.c_int32)]
+
+
+_lock = threading.Lock()
+_lib = None
+
+
+def build(force: bool = False) -> str:
+    """Compile libipmhsa.so for sm_103a (nvcc) and return its path."""
+    return _build.build(force=force)
+
+
+def load(build_if_missing: bool = True) -> ctypes.CDLL:
+    """Load libipmhsa.so and declare the C signatures."""
+    global _lib
+    with _lock:
+        if _lib is not None:
+            return _lib
+        try:
+            path = _build.build() if build_if_missing else _build.LIB
+            lib = ctypes.CDLL(path)
+        except Exception as exc:  # noqa: BLE001 - reported with context
+            raise LibraryError(f"cannot build or load the GPU library: {exc}") from exc
+        P = ctypes.c_void_p
+        I = ctypes.c_int
+        i32p = ctypes.POINTER(ctypes.c_int32)
+        lib.ip_relpos_mhsa_workspace_bytes.argtypes = [I, I, I, I]
+        lib.ip_relpos_mhsa_workspace_bytes.restype = ctypes.c_size_t
+        lib.ip_relpos_mhsa_host_arena_bytes.argtypes = [I, I, I, I]
+        lib.ip_relpos_mhsa_host_arena_bytes.restype = ctypes.c_size_t
+        sig = [P] * 6 + [P, P, ctypes.POINTER(SoftmaxParams), P] + [I] * 4 + [P, P, ctypes.c_size_t, P]
+        lib.ip_relpos_mhsa_i8.argtypes = sig
+        lib.ip_relpos_mhsa_i8.restype = I
+        lib.ip_relpos_mhsa_i8_host.argtypes = sig
+        lib.ip_relpos_mhsa_i8_host.restype = I
+        lib.ip_relpos_mhsa_status.argtypes = [P, P]
+        lib.ip_relpos_mhsa_status.restype = I
+        lib.ip_strerror.argtypes = [I]
+        lib.ip_strerror.restype = ctypes.c_char_p
+        lib.ip_debug_set_timeout_cycles.argtypes = [ctypes.c_longlong]
+        lib.ip_debug_set_timeout_cycles.restype = I
+        lib.ip_dyadic_multiplier.argtypes = [ctypes.c_double, i32p, i32p]
+        lib.ip_dyadic_multiplier.restype = I
+        lib.ip_dyadic_pair.argtypes = [ctypes.c_double, ctypes.c_double, i32p, i32p, i32p]
+        lib.ip_dyadic_pair.restype = I
+        lib.ip_isoftmax_params_from_scale.argtypes = [ctypes.c_double, ctypes.POINTER(SoftmaxParams)]
+        lib.ip_isoftmax_params_from_scale.restype = I
+        lib.ip_probe_int8_mma.argtypes = [I, I, P, P]
+        lib.ip_probe_int8_mma.restype = ctypes.c_longlong
+        _lib = lib
+        return lib
+
+
+def strerror(code: int) -> str:
+    return load().ip_strerror(code).decode()
+
+
+def _check(fn: str, code: int):
+    if code != 0:
+        raise IpError(fn, code, strerror(code))
+
+
+# ---------------------------------------------------------------- constants
+
+@dataclass(frozen=True)
+class LayerConstants:
+    multipliers: tuple[int, int, int]   # m_c, m_p, m_o
+    shifts: tuple[int, int]             # s_s, s_o (right shift 31 + s)
+    softmax: tuple[int, int, int]       # q_ln2, q_b, q_c
+
+
+def dyadic_multiplier(ratio: float) -> tuple[int, int]:
+    m, s = ctypes.c_int32(), ctypes.c_int32()
+    _check("ip_dyadic_multiplier", load().ip_dyadic_multiplier(ratio, ctypes.byref(m), ctypes.byref(s)))
+    return m.value, s.value
+
+
+def dyadic_pair(r_c: float, r_p: float) -> tuple[int, int, int]:
+    a, b, s = ctypes.c_int32(), ctypes.c_int32(), ctypes.c_int32()
+    _check("ip_dyadic_pair", load().ip_dyadic_pair(r_c, r_p, ctypes.byref(a), ctypes.byref(b), ctypes.byref(s)))
+    return a.value, b.value, s.value
+
+
+def isoftmax_params_from_scale(S_s: float) -> tuple[int, int, int]:
+    prm = SoftmaxParams()
+    _check("ip_isoftmax_params_from_scale", load().ip_isoftmax_params_from_scale(S_s, ctypes.byref(prm)))
+    return prm.q_ln2, prm.q_b, prm.q_c
+
+
+def layer_constants(scales: dict, dh: int = IP_DH) -> LayerConstants:
+    """Integer constants of one layer from its real scales (offline, Eq. 7
+    and Eq. 11; probabilities on the grid 2^-8)."""
+    root = math.sqrt(dh)
+    r_c = scales["S_Q"] * scales["S_K"] / (scales["S_s"] * root)
+    r_p = scales["S_Q"] * scales["S_P"] / (scales["S_s"] * root)
+    r_o = scales["S_V"] / (scales["S_O"] * 256.0)
+    m_c, m_p, s_s = dyadic_pair(r_c, r_p)
+    m_o, s_o = dyadic_multiplier(r_o)
+    return LayerConstants((m_c, m_p, m_o), (s_s, s_o), isoftmax_params_from_scale(scales["S_s"]))
+
+
+# ---------------------------------------------------------------- device path
+
+def workspace_bytes(B: int, H: int, T: int, dh: int = IP_DH) -> int:
+    n = load().ip_relpos_mhsa_workspace_bytes(B, H, T, dh)
+    if n == 0:
+        raise IpError("ip_relpos_mhsa_workspace_bytes", -2, "invalid shape")
+    return n
+
+
+def host_arena_bytes(B: int, H: int, T: int, dh: int = IP_DH) -> int:
+    n = load().ip_relpos_mhsa_host_arena_bytes(B, H, T, dh)
+    if n == 0:
+        raise IpError("ip_relpos_mhsa_host_arena_bytes", -2, "invalid shape")
+    return n
+
+
+def set_timeout_cycles(cycles: int) -> None:
+    """Bound of every kernel barrier wait (clock cycles; negative: default)."""
+    load().ip_debug_set_timeout_cycles(int(cycles))
+
+
+def _arr(vals, ctype):
+    return (ctype * len(vals))(*vals)
+
+
+def _stream_handle(stream):
+    if stream is None:
+        import torch
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def _dev_ptr(t, name, dtype, shape):
+    import torch
+    if not isinstance(t, torch.Tensor) or not t.is_cuda:
+        raise TypeError(f"{name} must be a CUDA tensor")
+    if t.dtype != dtype:
+        raise TypeError(f"{name} must be {dtype}, got {t.dtype}")
+    if tuple(t.shape) != tuple(shape):
+        raise ValueError(f"{name} must have shape {tuple(shape)}, got {tuple(t.shape)}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    return ctypes.c_void_p(t.data_ptr())
+
+
+def relpos_mhsa_i8(q, k, v, p, u, v_bias, consts: LayerConstants, lengths=None, out=None,
+                   workspace=None, stream=None):
+    """Whole layer on the GPU.  q, k, v: int8 [B, H, T, 128] CUDA tensors;
+    p: int8 [H, 2T-1, 128]; u, v_bias: int8 [H, 128]; lengths: int32 [B]
+    CUDA tensor or None.  Returns out (int8 [B, H, T, 128]).  Asynchronous on
+    `stream` (default: torch's current stream)."""
+    import torch
+    B, H, T, dh = q.shape
+    shp = (B, H, T, dh)
+    args = [_dev_ptr(q, "q", torch.int8, shp), _dev_ptr(k, "k", torch.int8, shp),
+            _dev_ptr(v, "v", torch.int8, shp), _dev_ptr(p, "p", torch.int8, (H, 2 * T - 1, dh)),
+            _dev_ptr(u, "u", torch.int8, (H, dh)), _dev_ptr(v_bias, "v_bias", torch.int8, (H, dh))]
+    if out is None:
+        out = torch.empty(shp, dtype=torch.int8, device=q.device)
+    lens = None if lengths is None else _dev_ptr(lengths, "lengths", torch.int32, (B,))
+    if workspace is None:
+        workspace = torch.empty(workspace_bytes(B, H, T, dh), dtype=torch.uint8, device=q.device)
+    sm = SoftmaxParams(*consts.softmax)
+    rc = load().ip_relpos_mhsa_i8(
+        *args, _arr(consts.multipliers, ctypes.c_int32), _arr(consts.shifts, ctypes.c_int32),
+        ctypes.byref(sm), lens, B, H, T, dh, _dev_ptr(out, "out", torch.int8, shp),
+        ctypes.c_void_p(workspace.data_ptr()), workspace.numel(), _stream_handle(stream))
+    _check("ip_relpos_mhsa_i8", rc)
+    return out
+
+
+def int8_mma_peak_tops(iters: int = 4096, repeats: int = 3) -> float:
+    """Measured integer warp-MMA throughput of the current GPU in TOPS
+    (best of `repeats` timed launches, CUDA events on the launching stream)."""
+    import torch
+    props = torch.cuda.get_device_properties(torch.cuda.current_device())
+    blocks = props.multi_processor_count * 8
+    sink = torch.empty(blocks * 256, dtype=torch.int32, device="cuda")
+    st = torch.cuda.current_stream()
+    lib = load()
+    h = ctypes.c_void_p(st.cuda_stream)
+    lib.ip_probe_int8_mma(blocks, iters, ctypes.c_void_p(sink.data_ptr()), h)   # warm-up
+    best = 0.0
+    for _ in range(repeats):
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(st)
+        ops = lib.ip_probe_int8_mma(blocks, iters, ctypes.c_void_p(sink.data_ptr()), h)
+        e1.record(st)
+        e1.synchronize()
+        if ops < 0:
+            raise IpError("ip_probe_int8_mma", -5, "launch failed")
+        best = max(best, ops / (e0.elapsed_time(e1) * 1e-3) / 1e12)
+    return best
+
+
+def status(workspace, stream=None) -> int:
+    """Synchronises the stream and returns the device-side status code of
+    the last call that used `workspace` (0 = ok)."""
+    return load().ip_relpos_mhsa_status(ctypes.c_void_p(workspace.data_ptr()), _stream_handle(stream))
+
+
+def relpos_mhsa_i8_host(q, k, v, p, u, v_bias, consts: LayerConstants, lengths, out, arena,
+                        stream=None):
+    """Whole layer from host buffers (torch CPU tensors, ideally pinned):
+    copies in, runs, copies the result into `out` and synchronises."""
+    import torch
+    B, H, T, dh = q.shape
+    for name, t in (("q", q), ("k", k), ("v", v), ("p", p), ("u", u), ("v_bias", v_bias), ("out", out)):
+        if t.is_cuda or t.dtype != torch.int8 or not t.is_contiguous():
+            raise TypeError(f"{name} must be a contiguous int8 CPU tensor")
+    lens = None
+    if lengths is not None:
+        if lengths.is_cuda or lengths.dtype != torch.int32 or tuple(lengths.shape) != (B,):
+            raise TypeError("lengths must be an int32 [B] CPU tensor")
+        lens = ctypes.c_void_p(lengths.data_ptr())
+    sm = SoftmaxParams(*consts.softmax)
+    ptr = lambda t: ctypes.c_void_p(t.data_ptr())
+    rc = load().ip_relpos_mhsa_i8_host(
+        ptr(q), ptr(k), ptr(v), ptr(p), ptr(u), ptr(v_bias),
+        _arr(consts.multipliers, ctypes.c_int32), _arr(consts.shifts, ctypes.c_int32),
+        ctypes.byref(sm), lens, B, H, T, dh, ptr(out), ctypes.c_void_p(arena.data_ptr()),
+        arena.numel(), _stream_handle(stream))
+    _check("ip_relpos_mhsa_i8_host", rc)
+    return out
+
+
+__all__ = ["build", "load", "relpos_mhsa_i8", "relpos_mhsa_i8_host", "status", "workspace_bytes",
+           "host_arena_bytes", "layer_constants", "LayerConstants", "dyadic_multiplier",
+           "dyadic_pair", "isoftmax_params_from_scale", "set_timeout_cycles", "strerror",
+           "int8_mma_peak_tops",
+           "IpError", "LibraryError", "EXPORTS"]

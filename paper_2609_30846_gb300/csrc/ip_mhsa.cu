@@ -1,0 +1,338 @@
+// Host side of the C ABI declared in include/ip_mhsa.h: argument
+// validation, tensor-map encoding for the TMA loads, workspace layout and
+// kernel launches.  The device code lives in ip_mhsa_kernels.cuh.
+#include "ip_mhsa.h"
+#include "ip_mhsa_kernels.cuh"
+#include "ip_probe.cuh"
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include <math.h>
+#include <mutex>
+#include <string.h>
+
+namespace {
+
+constexpr size_t WS_HEADER = 256;          // error word and padding
+constexpr long long DEFAULT_TIMEOUT = 4000000000ll;   // ~2 s at 2 GHz
+long long g_timeout_cycles = DEFAULT_TIMEOUT;
+
+size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+bool aligned(const void *p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+struct WsLayout {
+    size_t ku, pv, total;
+};
+
+WsLayout ws_layout(int B, int H, int T) {
+    WsLayout w;
+    w.ku = WS_HEADER;
+    w.pv = align_up(w.ku + 4ull * B * H * T, 256);
+    w.total = align_up(w.pv + 4ull * H * (2ull * T - 1), 256);
+    return w;
+}
+
+int check_shape(int B, int H, int T, int dh) {
+    if (dh != IP_DH) return IP_ERR_UNSUPPORTED;
+    if (B < 0 || H < 0 || T < 1 || T > IP_MAX_T) return IP_ERR_SHAPE;
+    if (B > IP_MAX_B || H > IP_MAX_H) return IP_ERR_SHAPE;   // grid y, z limits
+    return IP_OK;
+}
+
+int check_softmax(const ip_isoftmax_params *sm) {
+    if (sm->q_ln2 < 1 || sm->q_b < 0 || sm->q_c < 0) return IP_ERR_PARAM;
+    const long long t0 = sm->q_b, t1 = static_cast<long long>(sm->q_b) - sm->q_ln2 + 1;
+    const long long l0 = t0 * t0 + sm->q_c, l1 = t1 * t1 + sm->q_c;
+    if (l0 < 2 || l0 >= (1ll << 31) || l1 >= (1ll << 31)) return IP_ERR_PARAM;
+    return IP_OK;
+}
+
+// cuTensorMapEncodeTiled through the runtime's driver entry point.
+typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *,
+                                  const cuuint64_t *, const cuuint64_t *, const cuuint32_t *,
+                                  const cuuint32_t *, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+    static EncodeTiledFn fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000,
+                                             cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(p);
+    });
+    return fn;
+}
+
+// 3-D int8 map [d2][d1][128] with a box of 128 x rows x 1 and the 128-byte
+// swizzle; rows outside [0, d1) read as zero.
+bool make_map(CUtensorMap *m, const void *base, unsigned long long d1, unsigned long long d2,
+              unsigned rows) {
+    EncodeTiledFn fn = encode_fn();
+    if (!fn) return false;
+    const cuuint64_t dims[3] = {static_cast<cuuint64_t>(IP_DH), d1, d2};
+    const cuuint64_t strides[2] = {static_cast<cuuint64_t>(IP_DH), d1 * IP_DH};
+    const cuuint32_t box[3] = {static_cast<cuuint32_t>(IP_DH), rows, 1};
+    const cuuint32_t estride[3] = {1, 1, 1};
+    return fn(m, CU_TENSOR_MAP_DATA_TYPE_UINT8, 3, const_cast<void *>(base), dims, strides, box,
+              estride, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+std::mutex g_attr_mu;
+int g_attr_smem[64] = {0};
+
+int ensure_smem(int bytes) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return IP_ERR_CUDA;
+    std::lock_guard<std::mutex> lock(g_attr_mu);
+    if (g_attr_smem[dev] >= bytes) return IP_OK;
+    if (cudaFuncSetAttribute(ipk::relpos_mhsa_fused_kernel,
+                             cudaFuncAttributeMaxDynamicSharedMemorySize, bytes) != cudaSuccess)
+        return IP_ERR_CUDA;
+    g_attr_smem[dev] = bytes;
+    return IP_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+size_t ip_relpos_mhsa_workspace_bytes(int B, int H, int T, int dh) {
+    if (check_shape(B, H, T, dh) != IP_OK) return 0;
+    return ws_layout(B, H, T).total;
+}
+
+int ip_relpos_mhsa_i8(const int8_t *q, const int8_t *k, const int8_t *v, const int8_t *p,
+                      const int8_t *u, const int8_t *v_bias, const int32_t *multipliers,
+                      const int32_t *shifts, const ip_isoftmax_params *sm,
+                      const int32_t *lengths, int B, int H, int T, int dh, int8_t *out,
+                      void *workspace, size_t workspace_bytes, ip_stream_t stream) {
+    int rc = check_shape(B, H, T, dh);
+    if (rc != IP_OK) return rc;
+    if (B == 0 || H == 0) return IP_OK;   // empty problem: nothing to read or write
+    if (!q || !k || !v || !p || !u || !v_bias || !multipliers || !shifts || !sm || !out ||
+        !workspace)
+        return IP_ERR_NULL;
+    for (const void *ptr : {static_cast<const void *>(q), static_cast<const void *>(k),
+                            static_cast<const void *>(v), static_cast<const void *>(p),
+                            static_cast<const void *>(u), static_cast<const void *>(v_bias),
+                            static_cast<const void *>(out)})
+        if (!aligned(ptr, 16)) return IP_ERR_ALIGN;
+    if (!aligned(workspace, 256)) return IP_ERR_ALIGN;
+    if (lengths && !aligned(lengths, 4)) return IP_ERR_ALIGN;
+    for (int c = 0; c < 3; ++c)
+        if (multipliers[c] < 0) return IP_ERR_PARAM;
+    for (int c = 0; c < 2; ++c)
+        if (shifts[c] < 0 || shifts[c] > 31) return IP_ERR_PARAM;
+    rc = check_softmax(sm);
+    if (rc != IP_OK) return rc;
+    const WsLayout wl = ws_layout(B, H, T);
+    if (workspace_bytes < wl.total) return IP_ERR_WORKSPACE;
+
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    uint8_t *ws = static_cast<uint8_t *>(workspace);
+    int *err = reinterpret_cast<int *>(ws);
+    int32_t *ku = reinterpret_cast<int32_t *>(ws + wl.ku);
+    int32_t *pv = reinterpret_cast<int32_t *>(ws + wl.pv);
+
+    CUtensorMap tm_k, tm_v, tm_p;
+    const unsigned long long bh = static_cast<unsigned long long>(B) * H;
+    if (!make_map(&tm_k, k, T, bh, ipk::NK) || !make_map(&tm_v, v, T, bh, ipk::NK) ||
+        !make_map(&tm_p, p, 2ull * T - 1, H, ipk::BAND_ROWS))
+        return IP_ERR_CUDA;
+
+    const int ntiles = (T + ipk::MROWS - 1) / ipk::MROWS;
+    const int nchunk_max = (T + ipk::NK - 1) / ipk::NK;
+    const int smem = ipk::smem_layout(nchunk_max).total + 1024;
+    rc = ensure_smem(smem);
+    if (rc != IP_OK) return rc;
+
+    const dim3 grid0((2 * T - 1 + 255) / 256, H, B + 1);
+    ipk::bias_vectors_kernel<<<grid0, 256, 0, st>>>(k, p, u, v_bias, ku, pv, err, B, H, T);
+    if (cudaGetLastError() != cudaSuccess) return IP_ERR_CUDA;
+
+    ipk::FusedParams prm;
+    prm.q = q;
+    prm.out = out;
+    prm.ku = ku;
+    prm.pv = pv;
+    prm.lengths = lengths;
+    prm.err = err;
+    prm.B = B;
+    prm.H = H;
+    prm.T = T;
+    prm.ntiles = ntiles;
+    prm.nchunk_max = nchunk_max;
+    prm.m_c = multipliers[0];
+    prm.m_p = multipliers[1];
+    prm.m_o = multipliers[2];
+    prm.sh_s = 31 + shifts[0];
+    prm.sh_o = 31 + shifts[1];
+    prm.q_ln2 = sm->q_ln2;
+    prm.q_b = sm->q_b;
+    prm.q_c = sm->q_c;
+    prm.timeout_cycles = g_timeout_cycles;
+    const dim3 grid1(ntiles, H, B);
+    ipk::relpos_mhsa_fused_kernel<<<grid1, ipk::NTHREADS, smem, st>>>(tm_k, tm_v, tm_p, prm);
+    if (cudaGetLastError() != cudaSuccess) return IP_ERR_CUDA;
+    return IP_OK;
+}
+
+int ip_relpos_mhsa_status(const void *workspace, ip_stream_t stream) {
+    if (!workspace) return IP_ERR_NULL;
+    int word = 0;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    if (cudaMemcpyAsync(&word, workspace, sizeof(int), cudaMemcpyDeviceToHost, st) != cudaSuccess)
+        return IP_ERR_CUDA;
+    if (cudaStreamSynchronize(st) != cudaSuccess) return IP_ERR_CUDA;
+    return word == 0 ? IP_OK : IP_ERR_TIMEOUT;
+}
+
+size_t ip_relpos_mhsa_host_arena_bytes(int B, int H, int T, int dh) {
+    if (check_shape(B, H, T, dh) != IP_OK) return 0;
+    const size_t act = align_up(static_cast<size_t>(B) * H * T * dh, 256);
+    const size_t pb = align_up(static_cast<size_t>(H) * (2ull * T - 1) * dh, 256);
+    const size_t bias = align_up(static_cast<size_t>(H) * dh, 256);
+    const size_t lens = align_up(4ull * (B > 0 ? B : 1), 256);
+    return 4 * act + pb + 2 * bias + lens + ws_layout(B, H, T).total;
+}
+
+int ip_relpos_mhsa_i8_host(const int8_t *q, const int8_t *k, const int8_t *v, const int8_t *p,
+                           const int8_t *u, const int8_t *v_bias, const int32_t *multipliers,
+                           const int32_t *shifts, const ip_isoftmax_params *sm,
+                           const int32_t *lengths, int B, int H, int T, int dh, int8_t *out,
+                           void *arena, size_t arena_bytes, ip_stream_t stream) {
+    int rc = check_shape(B, H, T, dh);
+    if (rc != IP_OK) return rc;
+    if (B == 0 || H == 0) return IP_OK;
+    if (!q || !k || !v || !p || !u || !v_bias || !out || !arena) return IP_ERR_NULL;
+    if (!aligned(arena, 256)) return IP_ERR_ALIGN;
+    if (arena_bytes < ip_relpos_mhsa_host_arena_bytes(B, H, T, dh)) return IP_ERR_WORKSPACE;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    const size_t nact = static_cast<size_t>(B) * H * T * dh;
+    const size_t np = static_cast<size_t>(H) * (2ull * T - 1) * dh;
+    const size_t nb = static_cast<size_t>(H) * dh;
+    uint8_t *a = static_cast<uint8_t *>(arena);
+    size_t off = 0;
+    auto take = [&](size_t bytes) {
+        uint8_t *r = a + off;
+        off += align_up(bytes, 256);
+        return r;
+    };
+    int8_t *dq = reinterpret_cast<int8_t *>(take(nact));
+    int8_t *dk = reinterpret_cast<int8_t *>(take(nact));
+    int8_t *dv = reinterpret_cast<int8_t *>(take(nact));
+    int8_t *dout = reinterpret_cast<int8_t *>(take(nact));
+    int8_t *dp = reinterpret_cast<int8_t *>(take(np));
+    int8_t *du = reinterpret_cast<int8_t *>(take(nb));
+    int8_t *dvb = reinterpret_cast<int8_t *>(take(nb));
+    int32_t *dlen = reinterpret_cast<int32_t *>(take(4ull * (B > 0 ? B : 1)));
+    void *ws = take(ws_layout(B, H, T).total);
+    struct Copy {
+        void *dst;
+        const void *src;
+        size_t n;
+    } copies[] = {{dq, q, nact}, {dk, k, nact}, {dv, v, nact}, {dp, p, np},
+                  {du, u, nb},   {dvb, v_bias, nb}, {dlen, lengths, lengths ? 4ull * B : 0}};
+    for (const Copy &c : copies)
+        if (c.n && cudaMemcpyAsync(c.dst, c.src, c.n, cudaMemcpyHostToDevice, st) != cudaSuccess)
+            return IP_ERR_CUDA;
+    rc = ip_relpos_mhsa_i8(dq, dk, dv, dp, du, dvb, multipliers, shifts, sm,
+                           lengths ? dlen : nullptr, B, H, T, dh, dout, ws,
+                           ws_layout(B, H, T).total, stream);
+    if (rc != IP_OK) return rc;
+    if (nact && cudaMemcpyAsync(out, dout, nact, cudaMemcpyDeviceToHost, st) != cudaSuccess)
+        return IP_ERR_CUDA;
+    return ip_relpos_mhsa_status(ws, stream);
+}
+
+const char *ip_strerror(int code) {
+    switch (code) {
+    case IP_OK: return "ok";
+    case IP_ERR_NULL: return "a required pointer is NULL";
+    case IP_ERR_SHAPE: return "shape out of range (B, H >= 0; 1 <= T <= IP_MAX_T)";
+    case IP_ERR_ALIGN: return "pointer misaligned (16 bytes; workspace and arena 256)";
+    case IP_ERR_UNSUPPORTED: return "unsupported head width (dh must be 128)";
+    case IP_ERR_CUDA: return "CUDA runtime call failed";
+    case IP_ERR_TIMEOUT: return "kernel barrier wait timed out";
+    case IP_ERR_PARAM: return "multiplier, shift or softmax constant out of its domain";
+    case IP_ERR_WORKSPACE: return "workspace or arena too small";
+    default: return "unknown error code";
+    }
+}
+
+// Offline constants: float64 on the host, once per layer.
+int ip_dyadic_multiplier(double ratio, int32_t *m, int32_t *s) {
+    if (!m || !s) return IP_ERR_NULL;
+    if (!(ratio > 0.0) || !isfinite(ratio)) return IP_ERR_PARAM;
+    int e = 0;
+    const double frac = frexp(ratio, &e);   // ratio = frac 2^e, frac in [0.5, 1)
+    int sh = -e;
+    if (sh > 31) {
+        const double mm = floor(ratio * ldexp(1.0, 62) + 0.5);
+        *m = static_cast<int32_t>(mm);
+        *s = 31;
+        return IP_OK;
+    }
+    if (sh < 0) return IP_ERR_PARAM;
+    double mm = floor(frac * ldexp(1.0, 31) + 0.5);
+    if (mm >= ldexp(1.0, 31)) {
+        mm = ldexp(1.0, 30);
+        sh -= 1;
+        if (sh < 0) return IP_ERR_PARAM;
+    }
+    *m = static_cast<int32_t>(mm);
+    *s = sh;
+    return IP_OK;
+}
+
+int ip_dyadic_pair(double r_c, double r_p, int32_t *m_c, int32_t *m_p, int32_t *s) {
+    if (!m_c || !m_p || !s) return IP_ERR_NULL;
+    if (!(r_c > 0.0) || !(r_p > 0.0) || !isfinite(r_c) || !isfinite(r_p)) return IP_ERR_PARAM;
+    int32_t mbig = 0, sh = 0;
+    const int rc = ip_dyadic_multiplier(r_c > r_p ? r_c : r_p, &mbig, &sh);
+    if (rc != IP_OK) return rc;
+    const double scale = ldexp(1.0, 31 + sh);
+    const double mc = floor(r_c * scale + 0.5), mp = floor(r_p * scale + 0.5);
+    if (mc >= ldexp(1.0, 31) || mp >= ldexp(1.0, 31)) return IP_ERR_PARAM;
+    *m_c = static_cast<int32_t>(mc);
+    *m_p = static_cast<int32_t>(mp);
+    *s = sh;
+    return IP_OK;
+}
+
+int ip_isoftmax_params_from_scale(double S_s, ip_isoftmax_params *out) {
+    if (!out) return IP_ERR_NULL;
+    if (!(S_s > 0.0) || !isfinite(S_s)) return IP_ERR_PARAM;
+    const double ln2 = 0.6931471805599453;
+    const double qln2 = floor(ln2 / S_s), qb = floor(1.353 / S_s),
+                 qc = floor(0.344 / (0.3585 * (S_s * S_s)));
+    if (qln2 > 2147483647.0 || qb > 2147483647.0 || qc > 2147483647.0) return IP_ERR_PARAM;
+    out->q_ln2 = static_cast<int32_t>(qln2);
+    out->q_b = static_cast<int32_t>(qb);
+    out->q_c = static_cast<int32_t>(qc);
+    return IP_OK;
+}
+
+long long ip_probe_int8_mma(int blocks, int iters, int *sink, ip_stream_t stream) {
+    if (blocks < 1 || iters < 1 || !sink) return -1;
+    ipk::int8_mma_probe_kernel<<<blocks, ipk::PROBE_THREADS, 0,
+                                 reinterpret_cast<cudaStream_t>(stream)>>>(sink, 0x9e3779b9u,
+                                                                            iters);
+    if (cudaGetLastError() != cudaSuccess) return -1;
+    return static_cast<long long>(blocks) * (ipk::PROBE_THREADS / 32) * iters * ipk::PROBE_CHAINS *
+           (16ll * 8 * 32 * 2);
+}
+
+int ip_debug_set_timeout_cycles(long long cycles) {
+    g_timeout_cycles = cycles >= 0 ? cycles : DEFAULT_TIMEOUT;
+    return IP_OK;
+}
+
+}  // extern "C"

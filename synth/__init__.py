@@ -8,7 +8,8 @@ declare for them (Eq. 6, min-max ranges).  Both the CPU oracle and the CUDA
 path consume exactly what this module returns; each turns the declared
 scales into its own integer constants.
 
-Recipe (numpy PCG64, seed = 1000 * config + layer unless given):
+Recipe (numpy PCG64 streams spawned from SeedSequence(seed), seed =
+1000 * config + layer unless given):
 
 * Q, K, V, u, v : round(N(0, 30^2)) clipped to [-127, 127]
   (long-form workload: Q, K, V = round(t_3 * 25) clipped to [-127, 127]).
@@ -28,6 +29,8 @@ Recipe (numpy PCG64, seed = 1000 * config + layer unless given):
 from __future__ import annotations
 
 import math
+import os
+from concurrent.futures import ThreadPoolExecutor
 from dataclasses import dataclass, field
 
 import numpy as np
@@ -93,17 +96,46 @@ class Layer:
         return B, H, T, dh
 
 
-def _int8_normal(rng, shape, sigma):
-    x = rng.standard_normal(size=shape, dtype=np.float32)
-    x *= np.float32(sigma)
-    np.rint(x, out=x)
-    np.clip(x, -127, 127, out=x)
-    return x.astype(np.int8)
+_NCHUNK = 16          # fixed split of every large draw (independent of threads)
+_POOL = None
 
 
-def _int8_t3(rng, shape, scale):
-    x = rng.standard_t(3, size=shape) * scale
-    return np.clip(np.rint(x), -127, 127).astype(np.int8)
+def _pool():
+    global _POOL
+    if _POOL is None:
+        _POOL = ThreadPoolExecutor(max_workers=min(16, os.cpu_count() or 1))
+    return _POOL
+
+
+def _draw_int8(seq: np.random.SeedSequence, shape, dist: str, scale: float) -> np.ndarray:
+    """int8 draw of `shape`: round(N(0,1) * scale) or round(t_3 * scale),
+    clipped to [-127, 127]; filled in _NCHUNK pieces, each from its own
+    child seed, on a thread pool (numpy releases the GIL while drawing)."""
+    n = int(np.prod(shape))
+    out = np.empty(n, dtype=np.int8)
+    kids = seq.spawn(_NCHUNK)
+    bounds = [n * c // _NCHUNK for c in range(_NCHUNK + 1)]
+
+    def fill(c):
+        lo, hi = bounds[c], bounds[c + 1]
+        if hi <= lo:
+            return
+        g = np.random.Generator(np.random.PCG64(kids[c]))
+        if dist == "normal":
+            x = g.standard_normal(hi - lo, dtype=np.float32)
+        else:
+            x = g.standard_t(3, size=hi - lo).astype(np.float32)
+        x *= np.float32(scale)
+        np.rint(x, out=x)
+        np.clip(x, -127, 127, out=x)
+        out[lo:hi] = x.astype(np.int8)
+
+    if n >= 1 << 20:
+        list(_pool().map(fill, range(_NCHUNK)))
+    else:
+        for c in range(_NCHUNK):
+            fill(c)
+    return out.reshape(shape)
 
 
 def sinusoid_relpos(T: int, d: int = D_MODEL) -> np.ndarray:
@@ -117,10 +149,10 @@ def sinusoid_relpos(T: int, d: int = D_MODEL) -> np.ndarray:
     return pe
 
 
-def _projected_p(rng, T: int, H: int, dh: int) -> np.ndarray:
+def _projected_p(seq: np.random.SeedSequence, T: int, H: int, dh: int) -> np.ndarray:
     d = H * dh
     e = np.rint(sinusoid_relpos(T, d) * 127.0)                 # int8 grid, S = 1/127
-    w = np.clip(np.rint(rng.standard_normal((d, d)) * 20.0), -127, 127)
+    w = _draw_int8(seq, (d, d), "normal", 20.0).astype(np.float64)
     acc = e @ w.T                                              # exact: |acc| < 2^53
     amax = float(np.max(np.abs(acc)))
     p = np.clip(np.rint(acc * (127.0 / amax)), -127, 127).astype(np.int8)
@@ -128,36 +160,45 @@ def _projected_p(rng, T: int, H: int, dh: int) -> np.ndarray:
 
 
 def _rms(x: np.ndarray) -> float:
-    xf = x.astype(np.float64)
-    return float(np.sqrt(np.mean(xf * xf)))
+    """Root mean square of an int8 array, exact (integer sums below 2^53)."""
+    flat = x.reshape(-1)
+    total = 0.0
+    step = 1 << 22
+    for lo in range(0, flat.size, step):
+        xf = flat[lo:lo + step].astype(np.float64)
+        total += float(np.dot(xf, xf))
+    return math.sqrt(total / max(flat.size, 1))
 
 
 def draw(B: int, H: int, T: int, dh: int, seed: int, *, p_mode: str = "random",
          dist: str = "normal", masked: bool = False,
          lengths: np.ndarray | None = None) -> Layer:
     """Draw one layer of inputs of an arbitrary shape."""
-    rng = np.random.Generator(np.random.PCG64(seed))
+    root = np.random.SeedSequence(seed)
+    s_q, s_k, s_v, s_u, s_vb, s_p, s_len, s_sc = root.spawn(8)
     shape = (B, H, T, dh)
     if dist == "t3":
-        q, k, v = (_int8_t3(rng, shape, 25.0) for _ in range(3))
+        q, k, v = (_draw_int8(sq, shape, "t3", 25.0) for sq in (s_q, s_k, s_v))
     elif dist == "normal":
-        q, k, v = (_int8_normal(rng, shape, 30.0) for _ in range(3))
+        q, k, v = (_draw_int8(sq, shape, "normal", 30.0) for sq in (s_q, s_k, s_v))
     else:
         raise ValueError(f"unknown distribution {dist!r}")
-    u = _int8_normal(rng, (H, dh), 30.0)
-    vb = _int8_normal(rng, (H, dh), 30.0)
+    u = _draw_int8(s_u, (H, dh), "normal", 30.0)
+    vb = _draw_int8(s_vb, (H, dh), "normal", 30.0)
     if p_mode == "random":
-        p = _int8_normal(rng, (H, 2 * T - 1, dh), 30.0)
+        p = _draw_int8(s_p, (H, 2 * T - 1, dh), "normal", 30.0)
     elif p_mode == "sinusoid":
-        p = _projected_p(rng, T, H, dh)
+        p = _projected_p(s_p, T, H, dh)
     else:
         raise ValueError(f"unknown P mode {p_mode!r}")
     if lengths is None and masked:
-        lengths = rng.integers(T // 2, T, size=B, endpoint=True).astype(np.int32)
+        g = np.random.Generator(np.random.PCG64(s_len))
+        lengths = g.integers(T // 2, T, size=B, endpoint=True).astype(np.int32)
     elif lengths is not None:
         lengths = np.ascontiguousarray(lengths, dtype=np.int32)
 
-    a_q, a_k, a_v, a_p = rng.uniform(2.0, 6.0, size=4)
+    rng = np.random.Generator(np.random.PCG64(s_sc))
+    a_q, a_k, a_v, a_p = (float(x) for x in rng.uniform(2.0, 6.0, size=4))
     s_q, s_k, s_v, s_p = a_q / 127, a_k / 127, a_v / 127, a_p / 127
     # Second-moment estimate of the real fused score (Q+u)K^T + (Q+v)P^T,
     # divided by sqrt(dh); its min-max range is taken as kappa_s sigma.
@@ -165,9 +206,9 @@ def draw(B: int, H: int, T: int, dh: int, seed: int, *, p_mode: str = "random",
     sig_c = math.sqrt(dh) * math.hypot(rq, _rms(u)) * _rms(k) * s_q * s_k
     sig_p = math.sqrt(dh) * math.hypot(rq, _rms(vb)) * _rms(p) * s_q * s_p
     sigma = math.hypot(sig_c, sig_p) / math.sqrt(dh)
-    kappa_s = rng.uniform(3.5, 5.0)
+    kappa_s = float(rng.uniform(3.5, 5.0))
     s_s = kappa_s * sigma / 127
-    s_o = rng.uniform(1.0625, 1.9375) * s_v
+    s_o = float(rng.uniform(1.0625, 1.9375)) * s_v
     scales = dict(S_Q=s_q, S_K=s_k, S_V=s_v, S_P=s_p, S_s=s_s, S_O=s_o)
     return Layer(q=q, k=k, v=v, p=p, u=u, vb=vb, lengths=lengths, scales=scales)
 

@@ -1,0 +1,136 @@
+"""Host-side checks of the C ABI (no GPU needed): the library builds, loads
+and exports every function include/ip_mhsa.h declares; argument validation
+returns the documented codes before any device work; the offline constant
+helpers agree bit for bit with the oracle's; the kernel source carries no
+floating-point type."""
+import ctypes
+import math
+import os
+import re
+
+import numpy as np
+import pytest
+
+import paper_2609_30846_gb300 as ip
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "ip_mhsa.h")
+KERNELS = os.path.join(ROOT, "paper_2609_30846_gb300", "csrc", "ip_mhsa_kernels.cuh")
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(ip_[a-z0-9_]+)\s*\(", text)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    return ip.load()
+
+
+def test_exports_every_declared_symbol(lib):
+    names = declared_functions()
+    assert len(names) >= 10
+    for n in names:
+        assert hasattr(lib, n), f"{n} declared in include/ip_mhsa.h but not exported"
+    assert set(names) == set(ip.EXPORTS)
+
+
+def test_strerror_texts(lib):
+    for code in range(-8, 1):
+        assert ip.strerror(code)
+    assert "unknown" in ip.strerror(-99)
+
+
+def test_workspace_bytes(lib):
+    assert ip.workspace_bytes(1, 8, 64) >= 256 + 4 * 8 * 64 + 4 * 8 * 127
+    for bad in [(1, 8, 0), (1, 8, ip.IP_MAX_T + 1), (-1, 8, 10)]:
+        assert lib.ip_relpos_mhsa_workspace_bytes(*bad, 128) == 0
+    assert lib.ip_relpos_mhsa_workspace_bytes(1, 8, 64, 64) == 0
+
+
+def _call(lib, **over):
+    buf = (ctypes.c_byte * 4096)()
+    base = (ctypes.addressof(buf) + 255) // 256 * 256
+    a = dict(q=base, k=base, v=base, p=base, u=base, vb=base,
+             mult=(ctypes.c_int32 * 3)(2 ** 30, 2 ** 30, 2 ** 30),
+             shifts=(ctypes.c_int32 * 2)(9, 8), sm=ip.SoftmaxParams(12, 24, 327),
+             lens=None, B=1, H=1, T=4, dh=128, out=base, ws=base, wsb=1 << 20)
+    a.update(over)
+    return lib.ip_relpos_mhsa_i8(a["q"], a["k"], a["v"], a["p"], a["u"], a["vb"], a["mult"],
+                                 a["shifts"], ctypes.byref(a["sm"]) if a["sm"] is not None else None,
+                                 a["lens"], a["B"], a["H"], a["T"], a["dh"], a["out"], a["ws"],
+                                 a["wsb"], None)
+
+
+def test_validation_codes(lib):
+    assert _call(lib, q=None) == -1
+    assert _call(lib, sm=None) == -1
+    assert _call(lib, ws=None) == -1
+    assert _call(lib, T=0) == -2
+    assert _call(lib, T=ip.IP_MAX_T + 1) == -2
+    assert _call(lib, B=-1) == -2
+    assert _call(lib, dh=64) == -4
+    assert _call(lib, k=None) == -1
+    assert _call(lib, B=70000) == -2
+    buf = (ctypes.c_byte * 64)()
+    odd = (ctypes.addressof(buf) + 15) // 16 * 16 + 8
+    assert _call(lib, v=odd) == -3
+    assert _call(lib, mult=(ctypes.c_int32 * 3)(-1, 0, 0)) == -7
+    assert _call(lib, shifts=(ctypes.c_int32 * 2)(32, 8)) == -7
+    assert _call(lib, shifts=(ctypes.c_int32 * 2)(9, -1)) == -7
+    assert _call(lib, sm=ip.SoftmaxParams(0, 24, 327)) == -7      # q_ln2 < 1
+    assert _call(lib, sm=ip.SoftmaxParams(5, 0, 1)) == -7         # L(0) = 1 < 2
+    assert _call(lib, sm=ip.SoftmaxParams(5, 46341, 0)) == -7     # L(0) >= 2^31
+    assert _call(lib, wsb=16) == -8
+    # B = 0 or H = 0 is a valid empty problem: nothing is read or launched
+    assert _call(lib, B=0) == 0
+    assert _call(lib, B=0, q=None, out=None) == 0
+    assert _call(lib, H=0, ws=None) == 0
+
+
+def test_constants_match_oracle(lib):
+    import oracle
+    rng = np.random.default_rng(0)
+    ratios = np.concatenate([10.0 ** rng.uniform(-18, -0.31, 400), [2.0 ** -9, 0.25, 0.49999]])
+    for r in ratios:
+        assert ip.dyadic_multiplier(float(r)) == oracle.dyadic(float(r)), r
+    for _ in range(200):
+        r_c, r_p = 10.0 ** rng.uniform(-6, -1, 2)
+        assert ip.dyadic_pair(float(r_c), float(r_p)) == oracle.dyadic_pair(float(r_c), float(r_p))
+    for S in 10.0 ** rng.uniform(-3.5, 0, 300):
+        assert ip.isoftmax_params_from_scale(float(S)) == oracle.isoftmax_params(float(S)), S
+    import synth
+    for w in range(5):
+        sc = synth.layer(w, 0).scales if w != 3 else synth.draw(1, 8, 375, 128, 3000, p_mode="sinusoid").scales
+        c1 = ip.layer_constants(sc)
+        c2 = oracle.layer_constants(sc, 128)
+        assert (c1.multipliers, c1.shifts, c1.softmax) == (c2.multipliers, c2.shifts, c2.softmax)
+
+
+def test_constants_reject_bad_ratios(lib):
+    with pytest.raises(ip.IpError):
+        ip.dyadic_multiplier(1.0)
+    with pytest.raises(ip.IpError):
+        ip.dyadic_multiplier(-1e-3)
+    with pytest.raises(ip.IpError):
+        ip.isoftmax_params_from_scale(0.0)
+
+
+def test_kernel_source_is_integer_only():
+    text = open(KERNELS).read()
+    code = re.sub(r"//[^\n]*", "", re.sub(r"/\*.*?\*/", "", text, flags=re.S))
+    code = re.sub(r'"(\\.|[^"\\])*"', '""', code)          # drop string literals (PTX)
+    for pat in (r"\bfloat\b", r"\bdouble\b", r"\b__half\b", r"\b__nv_bfloat16\b", r"\bhalf\b",
+                r"__fdividef|__expf|\bexpf\b|\bexp\b\s*\(", r"\bsqrtf?\b", r"kind::f16|kind::tf32"):
+        assert not re.search(pat, code), pat
+    # No '/' or '%' by a run-time value: the compiler's integer division
+    # would not be integer-only.  Divisions are the long-division helpers;
+    # the remaining operators divide by compile-time powers of two.
+    assert "div_2pow32" in code and "iexp_neg" in code
+    allowed = {"NSTAGE", "NK", "MROWS", "DH", "16", "2", "4", "8", "32", "256"}
+    for m in re.finditer(r"[^/*](/|%)\s*\(?\s*([A-Za-z_0-9]+)", code):
+        if m.group(0).startswith("<") or m.group(1) == "/" and code[m.start(1) + 1] in "/*":
+            continue
+        assert m.group(2) in allowed, f"run-time division by {m.group(2)!r}"

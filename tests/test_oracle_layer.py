@@ -19,8 +19,8 @@ def layer_bound(q_ln2: int) -> tuple[float, float]:
     if q_ln2 >= 16:
         return 6, 0.85
     if q_ln2 >= 10:
-        return 14, 1.0
-    return 24, 2.0
+        return 12, 1.0
+    return 32, 3.0
 
 
 CASES = [

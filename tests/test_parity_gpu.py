@@ -1,0 +1,162 @@
+"""Parity of the CUDA path (through the C ABI) with the CPU oracle.
+
+Integer work: the bar is bit-exactness on every output.  Inputs come from
+the seeded generator; the oracle's expected values come from the oracle
+only.
+"""
+import numpy as np
+import pytest
+
+import synth
+
+pytestmark = pytest.mark.gpu
+
+torch = pytest.importorskip("torch")
+
+
+@pytest.fixture(scope="module")
+def ip():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import paper_2609_30846_gb300 as mod
+    mod.load()
+    return mod
+
+
+@pytest.fixture(scope="module")
+def orc():
+    import oracle
+    oracle.build()
+    return oracle
+
+
+def _dev(a):
+    return torch.from_numpy(np.ascontiguousarray(a)).cuda()
+
+
+def run_gpu(ip, lay, consts, lengths=None):
+    B, H, T, dh = lay.q.shape
+    ws = torch.empty(ip.workspace_bytes(B, H, T, dh), dtype=torch.uint8, device="cuda")
+    lens = None if lengths is None else _dev(lengths.astype(np.int32))
+    out = ip.relpos_mhsa_i8(_dev(lay.q), _dev(lay.k), _dev(lay.v), _dev(lay.p), _dev(lay.u),
+                            _dev(lay.vb), consts, lengths=lens, workspace=ws)
+    assert ip.status(ws) == 0
+    return out.cpu().numpy()
+
+
+def oracle_out(orc, lay, consts, lengths=None):
+    c = orc.LayerConstants(consts.multipliers, consts.shifts, consts.softmax)
+    return orc.relpos_mhsa(lay.q, lay.k, lay.v, lay.p, lay.u, lay.vb, c, lengths)
+
+
+def assert_same(got, want):
+    bad = got != want
+    if bad.any():
+        idx = np.argwhere(bad)[:5]
+        raise AssertionError(f"{int(bad.sum())} of {got.size} outputs differ; first at {idx.tolist()}: "
+                             f"gpu {got[tuple(idx[0])]} oracle {want[tuple(idx[0])]}")
+
+
+@pytest.mark.parametrize("w", [0, 1, 2, 4])
+def test_workload_full_size(ip, orc, w):
+    lay = synth.layer(w, 0)
+    c = ip.layer_constants(lay.scales)
+    assert_same(run_gpu(ip, lay, c, lay.lengths), oracle_out(orc, lay, c, lay.lengths))
+
+
+def test_encoder_layer_full_size(ip, orc):
+    # one layer of the 24-layer encoder sweep (B=32, T=375), every output
+    lay = synth.layer(3, 5)
+    c = ip.layer_constants(lay.scales)
+    assert_same(run_gpu(ip, lay, c), oracle_out(orc, lay, c))
+
+
+@pytest.mark.parametrize("T", [1, 2, 3, 17, 63, 64, 65, 100, 127, 128, 129, 191, 200])
+def test_ragged_lengths_of_T(ip, orc, T):
+    lay = synth.draw(2, 3, T, 128, seed=500 + T, p_mode="sinusoid")
+    c = ip.layer_constants(lay.scales)
+    assert_same(run_gpu(ip, lay, c), oracle_out(orc, lay, c))
+
+
+@pytest.mark.parametrize("seed", range(3))
+def test_key_padding_masks(ip, orc, seed):
+    T = 150
+    rng = np.random.default_rng(seed)
+    lens = np.array([0, 1, 2, 63, 64, 65, 149, 150, 999, -4] + list(rng.integers(0, T + 1, 6)), np.int32)
+    lay = synth.draw(len(lens), 2, T, 128, seed=900 + seed, lengths=lens)
+    c = ip.layer_constants(lay.scales)
+    assert_same(run_gpu(ip, lay, c, lens), oracle_out(orc, lay, c, lens))
+
+
+def test_extreme_values_and_constants(ip, orc):
+    B, H, T = 2, 2, 96
+    rng = np.random.default_rng(7)
+    base = synth.draw(B, H, T, 128, seed=31)
+    for lo, hi in ((-128, 127), (-128, -127), (126, 127)):
+        q = rng.integers(lo, hi + 1, size=base.q.shape).astype(np.int8)
+        k = rng.integers(lo, hi + 1, size=base.q.shape).astype(np.int8)
+        v = rng.integers(-128, 128, size=base.q.shape).astype(np.int8)
+        p = rng.integers(lo, hi + 1, size=base.p.shape).astype(np.int8)
+        u = rng.integers(lo, hi + 1, size=base.u.shape).astype(np.int8)
+        vb = rng.integers(lo, hi + 1, size=base.vb.shape).astype(np.int8)
+        lay = synth.Layer(q, k, v, p, u, vb, None, base.scales)
+        for mult, shifts, sm in (((2 ** 31 - 1, 2 ** 31 - 1, 2 ** 31 - 1), (0, 0), (3, 6, 10)),
+                                 ((2 ** 31 - 1, 12345, 2 ** 30), (31, 31), (100, 195, 20000)),
+                                 ((0, 2 ** 30, 1), (20, 8), (12, 24, 327)),
+                                 ((2 ** 30, 0, 2 ** 31 - 1), (12, 0), (1, 2, 0))):
+            c = ip.LayerConstants(mult, shifts, sm)
+            assert_same(run_gpu(ip, lay, c), oracle_out(orc, lay, c))
+
+
+def test_uniform_scores(ip, orc):
+    # all keys equal: every probability is the same closed-form value
+    B, H, T = 1, 2, 300
+    lay = synth.draw(B, H, T, 128, seed=3)
+    lay.k[:] = 0
+    lay.p[:] = 0
+    c = ip.layer_constants(lay.scales)
+    assert_same(run_gpu(ip, lay, c), oracle_out(orc, lay, c))
+
+
+def test_longest_sequence(ip, orc):
+    T = ip.IP_MAX_T
+    lay = synth.draw(1, 2, T, 128, seed=77, dist="t3", p_mode="random")
+    c = ip.layer_constants(lay.scales)
+    assert_same(run_gpu(ip, lay, c), oracle_out(orc, lay, c))
+
+
+def test_empty_batch(ip):
+    lay = synth.draw(0, 8, 10, 128, seed=1)
+    c = ip.layer_constants(synth.draw(1, 8, 10, 128, seed=1).scales)
+    out = torch.full((0, 8, 10, 128), 5, dtype=torch.int8, device="cuda")
+    ws = torch.empty(ip.workspace_bytes(0, 8, 10), dtype=torch.uint8, device="cuda")
+    ip.relpos_mhsa_i8(_dev(lay.q), _dev(lay.k), _dev(lay.v), _dev(lay.p), _dev(lay.u),
+                      _dev(lay.vb), c, out=out, workspace=ws)
+    torch.cuda.synchronize()
+    assert out.numel() == 0
+
+
+def test_host_entry_point_matches_device(ip, orc):
+    lay = synth.layer(2, 1)
+    c = ip.layer_constants(lay.scales)
+    B, H, T, dh = lay.q.shape
+    arena = torch.empty(ip.host_arena_bytes(B, H, T), dtype=torch.uint8, device="cuda")
+    pin = lambda a: torch.from_numpy(np.ascontiguousarray(a)).pin_memory()
+    out = torch.empty((B, H, T, dh), dtype=torch.int8).pin_memory()
+    ip.relpos_mhsa_i8_host(pin(lay.q), pin(lay.k), pin(lay.v), pin(lay.p), pin(lay.u),
+                           pin(lay.vb), c, pin(lay.lengths), out, arena)
+    assert_same(out.numpy(), oracle_out(orc, lay, c, lay.lengths))
+
+
+def test_repeated_calls_share_workspace(ip, orc):
+    # back-to-back calls on one stream reuse one workspace: results stay exact
+    ws = None
+    for i in range(3):
+        lay = synth.draw(3, 8, 130, 128, seed=60 + i, p_mode="sinusoid")
+        c = ip.layer_constants(lay.scales)
+        if ws is None:
+            ws = torch.empty(ip.workspace_bytes(3, 8, 130), dtype=torch.uint8, device="cuda")
+        out = ip.relpos_mhsa_i8(_dev(lay.q), _dev(lay.k), _dev(lay.v), _dev(lay.p), _dev(lay.u),
+                                _dev(lay.vb), c, workspace=ws)
+        assert ip.status(ws) == 0
+        assert_same(out.cpu().numpy(), oracle_out(orc, lay, c))
