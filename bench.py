@@ -59,6 +59,10 @@ def parse_args():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0,
                     help="target length of the CPU-baseline sample")
+    ap.add_argument("--layers", type=int, default=None,
+                    help="profiling only: fewer layers than the workload's 24")
+    ap.add_argument("--batch", type=int, default=None,
+                    help="profiling only: fewer utterances than the workload's 32")
     return ap.parse_args()
 
 
@@ -246,7 +250,12 @@ def run_ours(args):
 
     w = synth.WORKLOADS[WORKLOAD]
     B, H, T, dh, NL = w.B, w.H, w.T, w.dh, w.layers
-    layers = make_layers(NL)
+    if args.layers:
+        NL = min(NL, args.layers)
+    if args.batch:
+        B = min(B, args.batch)
+    reduced = (NL, B) != (w.layers, w.B)
+    layers = make_layers(NL, B)
     consts = [ip.layer_constants(l.scales) for l in layers]
     to_dev = lambda a: torch.from_numpy(np.ascontiguousarray(a)).to(dev)
     dl = [dict(q=to_dev(l.q), k=to_dev(l.k), v=to_dev(l.v), p=to_dev(l.p), u=to_dev(l.u),
@@ -366,7 +375,8 @@ def run_ours(args):
         "warmup": max(args.warmup, 3), "ms_per_step": ms_step, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "s8xs8->s32 (int32/int64 epilogue)",
         "data": "synthetic",
-        "config": {"workload": w.name, "B": B, "H": H, "T": T, "dh": dh, "layers": NL,
+        "config": {"workload": w.name + (" (REDUCED, profiling only)" if reduced else ""),
+                   "B": B, "H": H, "T": T, "dh": dh, "layers": NL,
                    "parallelism": f"replicas x{world}" if world > 1 else "1 GPU",
                    "l2": "inputs larger than L2 (%.2f GB per step, L2 129 MB)" % (bytes_layer * NL / 1e9)},
         "rtf": ms_step * 1e-3 / (B * UTT_SECONDS),
