@@ -70,9 +70,10 @@ typedef struct {
 #define IP_MAX_B 65535
 #define IP_MAX_H 65535
 
-/* Bytes of device workspace one call needs: an error word plus the bias
- * vectors (K u) [B][H][T] and (P v) [H][2T-1] as int32 (the exact rank-1
- * split of (Q + 1u^T)K^T and (Q + 1v^T)P^T).  0 if the shape is invalid. */
+/* Bytes of device workspace a call needs: the device-side status word of
+ * the calls that use it.  The caller zero-fills the workspace once before
+ * its first use; ip_relpos_mhsa_status reads and clears it.  0 if the shape
+ * is invalid. */
 size_t ip_relpos_mhsa_workspace_bytes(int B, int H, int T, int dh);
 
 /* The whole layer on the GPU.
@@ -86,8 +87,8 @@ size_t ip_relpos_mhsa_workspace_bytes(int B, int H, int T, int dh);
  *   workspace   : device memory of workspace_bytes >= the size above,
  *                 256-byte aligned, owned by the caller; one call at a time
  *                 per workspace.
- * The call validates its arguments on the host and then enqueues two
- * kernels on `stream`.  B == 0 or H == 0 is an empty problem: the call
+ * The call validates its arguments on the host and then enqueues one
+ * kernel on `stream`.  B == 0 or H == 0 is an empty problem: the call
  * returns IP_OK without touching any pointer.  A kernel-side barrier timeout is reported later by
  * ip_relpos_mhsa_status. */
 int ip_relpos_mhsa_i8(const int8_t *q, const int8_t *k, const int8_t *v,
@@ -97,8 +98,9 @@ int ip_relpos_mhsa_i8(const int8_t *q, const int8_t *k, const int8_t *v,
                       int B, int H, int T, int dh, int8_t *out,
                       void *workspace, size_t workspace_bytes, ip_stream_t stream);
 
-/* Synchronises `stream` and reports the device-side status of the last call
- * that used `workspace`: IP_OK, IP_ERR_TIMEOUT, or IP_ERR_CUDA. */
+/* Synchronises `stream`, reports the device-side status of the calls that
+ * used `workspace` since the previous status call (IP_OK, IP_ERR_TIMEOUT,
+ * or IP_ERR_CUDA) and clears it. */
 int ip_relpos_mhsa_status(const void *workspace, ip_stream_t stream);
 
 /* Bytes of device staging memory ip_relpos_mhsa_i8_host needs (inputs,

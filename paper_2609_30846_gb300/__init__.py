@@ -207,7 +207,7 @@ def relpos_mhsa_i8(q, k, v, p, u, v_bias, consts: LayerConstants, lengths=None, 
         out = torch.empty(shp, dtype=torch.int8, device=q.device)
     lens = None if lengths is None else _dev_ptr(lengths, "lengths", torch.int32, (B,))
     if workspace is None:
-        workspace = torch.empty(workspace_bytes(B, H, T, dh), dtype=torch.uint8, device=q.device)
+        workspace = torch.zeros(workspace_bytes(B, H, T, dh), dtype=torch.uint8, device=q.device)
     sm = SoftmaxParams(*consts.softmax)
     rc = load().ip_relpos_mhsa_i8(
         *args, _arr(consts.multipliers, ctypes.c_int32), _arr(consts.shifts, ctypes.c_int32),

@@ -22,17 +22,8 @@ size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 bool aligned(const void *p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 
-struct WsLayout {
-    size_t ku, pv, total;
-};
-
-WsLayout ws_layout(int B, int H, int T) {
-    WsLayout w;
-    w.ku = WS_HEADER;
-    w.pv = align_up(w.ku + 4ull * B * H * T, 256);
-    w.total = align_up(w.pv + 4ull * H * (2ull * T - 1), 256);
-    return w;
-}
+// The workspace holds the device error word of the calls that use it.
+size_t ws_bytes() { return WS_HEADER; }
 
 int check_shape(int B, int H, int T, int dh) {
     if (dh != IP_DH) return IP_ERR_UNSUPPORTED;
@@ -105,7 +96,7 @@ extern "C" {
 
 size_t ip_relpos_mhsa_workspace_bytes(int B, int H, int T, int dh) {
     if (check_shape(B, H, T, dh) != IP_OK) return 0;
-    return ws_layout(B, H, T).total;
+    return ws_bytes();
 }
 
 int ip_relpos_mhsa_i8(const int8_t *q, const int8_t *k, const int8_t *v, const int8_t *p,
@@ -132,14 +123,10 @@ int ip_relpos_mhsa_i8(const int8_t *q, const int8_t *k, const int8_t *v, const i
         if (shifts[c] < 0 || shifts[c] > 31) return IP_ERR_PARAM;
     rc = check_softmax(sm);
     if (rc != IP_OK) return rc;
-    const WsLayout wl = ws_layout(B, H, T);
-    if (workspace_bytes < wl.total) return IP_ERR_WORKSPACE;
+    if (workspace_bytes < ws_bytes()) return IP_ERR_WORKSPACE;
 
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-    uint8_t *ws = static_cast<uint8_t *>(workspace);
-    int *err = reinterpret_cast<int *>(ws);
-    int32_t *ku = reinterpret_cast<int32_t *>(ws + wl.ku);
-    int32_t *pv = reinterpret_cast<int32_t *>(ws + wl.pv);
+    int *err = static_cast<int *>(workspace);
 
     CUtensorMap tm_k, tm_v, tm_p;
     const unsigned long long bh = static_cast<unsigned long long>(B) * H;
@@ -153,21 +140,16 @@ int ip_relpos_mhsa_i8(const int8_t *q, const int8_t *k, const int8_t *v, const i
     rc = ensure_smem(smem);
     if (rc != IP_OK) return rc;
 
-    const dim3 grid0((2 * T - 1 + 255) / 256, H, B + 1);
-    ipk::bias_vectors_kernel<<<grid0, 256, 0, st>>>(k, p, u, v_bias, ku, pv, err, B, H, T);
-    if (cudaGetLastError() != cudaSuccess) return IP_ERR_CUDA;
-
     ipk::FusedParams prm;
     prm.q = q;
+    prm.u = u;
+    prm.vb = v_bias;
     prm.out = out;
-    prm.ku = ku;
-    prm.pv = pv;
     prm.lengths = lengths;
     prm.err = err;
     prm.B = B;
     prm.H = H;
     prm.T = T;
-    prm.ntiles = ntiles;
     prm.nchunk_max = nchunk_max;
     prm.m_c = multipliers[0];
     prm.m_p = multipliers[1];
@@ -190,6 +172,8 @@ int ip_relpos_mhsa_status(const void *workspace, ip_stream_t stream) {
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
     if (cudaMemcpyAsync(&word, workspace, sizeof(int), cudaMemcpyDeviceToHost, st) != cudaSuccess)
         return IP_ERR_CUDA;
+    if (cudaMemsetAsync(const_cast<void *>(workspace), 0, sizeof(int), st) != cudaSuccess)
+        return IP_ERR_CUDA;
     if (cudaStreamSynchronize(st) != cudaSuccess) return IP_ERR_CUDA;
     return word == 0 ? IP_OK : IP_ERR_TIMEOUT;
 }
@@ -200,7 +184,7 @@ size_t ip_relpos_mhsa_host_arena_bytes(int B, int H, int T, int dh) {
     const size_t pb = align_up(static_cast<size_t>(H) * (2ull * T - 1) * dh, 256);
     const size_t bias = align_up(static_cast<size_t>(H) * dh, 256);
     const size_t lens = align_up(4ull * (B > 0 ? B : 1), 256);
-    return 4 * act + pb + 2 * bias + lens + ws_layout(B, H, T).total;
+    return 4 * act + pb + 2 * bias + lens + ws_bytes();
 }
 
 int ip_relpos_mhsa_i8_host(const int8_t *q, const int8_t *k, const int8_t *v, const int8_t *p,
@@ -233,7 +217,8 @@ int ip_relpos_mhsa_i8_host(const int8_t *q, const int8_t *k, const int8_t *v, co
     int8_t *du = reinterpret_cast<int8_t *>(take(nb));
     int8_t *dvb = reinterpret_cast<int8_t *>(take(nb));
     int32_t *dlen = reinterpret_cast<int32_t *>(take(4ull * (B > 0 ? B : 1)));
-    void *ws = take(ws_layout(B, H, T).total);
+    void *ws = take(ws_bytes());
+    if (cudaMemsetAsync(ws, 0, ws_bytes(), st) != cudaSuccess) return IP_ERR_CUDA;
     struct Copy {
         void *dst;
         const void *src;
@@ -244,8 +229,7 @@ int ip_relpos_mhsa_i8_host(const int8_t *q, const int8_t *k, const int8_t *v, co
         if (c.n && cudaMemcpyAsync(c.dst, c.src, c.n, cudaMemcpyHostToDevice, st) != cudaSuccess)
             return IP_ERR_CUDA;
     rc = ip_relpos_mhsa_i8(dq, dk, dv, dp, du, dvb, multipliers, shifts, sm,
-                           lengths ? dlen : nullptr, B, H, T, dh, dout, ws,
-                           ws_layout(B, H, T).total, stream);
+                           lengths ? dlen : nullptr, B, H, T, dh, dout, ws, ws_bytes(), stream);
     if (rc != IP_OK) return rc;
     if (nact && cudaMemcpyAsync(out, dout, nact, cudaMemcpyDeviceToHost, st) != cudaSuccess)
         return IP_ERR_CUDA;

@@ -1,23 +1,30 @@
 // Device code of the integer-only relative-positional MHSA (I-Parakeet,
 // Sec. 3.1) for sm_103a.  Integer arithmetic only: no floating-point type
-// appears in this file.
+// appears in this file, and no division by a run-time value (the two
+// divisions the method needs are done by binary long division).
 //
 // sm_103a has no integer tcgen05 MMA kind, so the three contractions use the
-// integer warp MMA (mma.sync m16n8k32, s8 x s8 and u8 x s8 -> s32), fed from
-// shared memory tiles that the tensor-memory accelerator (TMA) stages with
-// the 128-byte swizzle.
+// integer warp MMA (mma.sync m16n8k32, s8 x s8 and u8 x s8 -> s32, which
+// runs on the tensor pipe), fed from shared-memory tiles that the tensor
+// memory accelerator (TMA) stages with the 128-byte swizzle.
 //
 // One CTA owns 64 query rows of one (b, h): four consumer warps of 16 rows
-// and one producer warp that issues the TMA loads.  Per CTA:
-//   pass 1  for each chunk of 64 keys: the position band Q (P_band)^T and
-//           the content Q K^T (bias vectors preloaded into the accumulators),
-//           the relative shift as an index remap through shared memory, the
-//           fused requantisation of Eq. 11 and the key mask; int8 scores are
-//           kept in shared memory, row maxima in registers;
-//   pass 2  integer exponentials from a 256-entry table and row sums;
-//   pass 3  probabilities on the grid 2^-8 fed as the u8 operand of the
-//           A.V MMA against V tiles, then the output requantisation and
-//           16-byte stores.
+// and one producer warp.  The producer issues the TMA loads and prepares each
+// staged chunk for the consumers: for the score pass it computes the bias
+// vectors K u and P v of the chunk (the exact rank-1 split of (Q + 1u^T)K^T
+// and (Q + 1v^T)P^T, since Q + u does not fit an int8 operand), for the
+// attn.V pass it transposes the V tile into the operand layout of the MMA.
+// The consumers, per CTA:
+//   pass 1  for each chunk of 64 keys: the content MMAs Q K^T, the MMAs of
+//           the position band Q P_band^T for the next chunk (issued before
+//           this chunk's epilogue so that the tensor pipe stays busy), the
+//           relative shift as an index remap through shared memory, the
+//           fused requantisation of Eq. 11 and the key mask; int8 scores
+//           stay in shared memory, row maxima in registers;
+//   pass 2  integer exponentials (a 256-entry table, one copy per row
+//           group to spread the banks) and row sums;
+//   pass 3  probabilities on the grid 2^-8 as the u8 operand of the A.V
+//           MMA, then the output requantisation and 16-byte stores.
 #pragma once
 
 #include <cuda.h>
@@ -32,39 +39,45 @@ constexpr int NTHREADS = (NCWARPS + 1) * 32;
 constexpr int NK = 64;                    // keys per chunk
 constexpr int NSTAGE = 2;
 constexpr int BAND_ROWS = 128;            // P rows staged per chunk (NK + MROWS - 1, padded)
-constexpr int K_TILE_BYTES = NK * DH;     // also the V tile
-constexpr int P_TILE_BYTES = BAND_ROWS * DH;
-constexpr int STAGE_BYTES = K_TILE_BYTES + P_TILE_BYTES;
+constexpr int K_TILE_BYTES = NK * DH;     // K (pass 1) or V (pass 3) tile
+constexpr int P_TILE_BYTES = BAND_ROWS * DH;   // P band (pass 1) or transposed V (pass 3)
+constexpr int KU_OFF = K_TILE_BYTES + P_TILE_BYTES;   // int32 K u of the chunk's keys
+constexpr int PV_OFF = KU_OFF + NK * 4;                // int32 P v of the band rows
+constexpr int STAGE_BYTES = 25600;        // PV_OFF + BAND_ROWS * 4, rounded to 1024
 constexpr int BAND_TILES = 10;            // n8 tiles of one warp's band: 16 + NK - 1 -> 80
 constexpr int REMAP_STRIDE = 88;          // int32 words per band row in the remap buffer
 constexpr int REMAP_BYTES = 16 * REMAP_STRIDE * 4;
 constexpr int LUT_ENTRIES = 256;
+constexpr int LUT_COPIES = 8;             // one per MMA row group
 constexpr int CHUNK_SCORE_BYTES = 16 * NK;   // one warp's int8 scores of one chunk
+
+static_assert(PV_OFF + BAND_ROWS * 4 <= STAGE_BYTES, "stage layout");
+static_assert(STAGE_BYTES % 1024 == 0, "the 128-byte swizzle needs 1024-byte aligned tiles");
 
 struct SmemLayout {
     int stages, scores, remap, lut, bars, total;
 };
 
-// Offsets from a 1024-byte aligned base (the 128-byte swizzle needs it).
+// Offsets from a 1024-byte aligned base.
 __host__ __device__ inline SmemLayout smem_layout(int nchunk_max) {
     SmemLayout L;
     L.stages = 0;
     L.scores = NSTAGE * STAGE_BYTES;
     L.remap = L.scores + NCWARPS * nchunk_max * CHUNK_SCORE_BYTES;
     L.lut = L.remap + NCWARPS * REMAP_BYTES;
-    L.bars = L.lut + LUT_ENTRIES * 4;
+    L.bars = L.lut + LUT_ENTRIES * LUT_COPIES * 4;
     L.total = L.bars + 64;
     return L;
 }
 
 struct FusedParams {
     const int8_t *q;
+    const int8_t *u;          // [H][DH]
+    const int8_t *vb;         // [H][DH]
     int8_t *out;
-    const int32_t *ku;        // [B*H*T]   K u
-    const int32_t *pv;        // [H*(2T-1)] P v
     const int32_t *lengths;   // [B] or nullptr
     int *err;                 // device error word
-    int B, H, T, ntiles, nchunk_max;
+    int B, H, T, nchunk_max;
     int32_t m_c, m_p, m_o;
     int32_t sh_s, sh_o;       // total right shifts, 31 + s
     int32_t q_ln2, q_b, q_c;
@@ -73,6 +86,8 @@ struct FusedParams {
 
 constexpr int ERR_TIMEOUT_FULL = 1;
 constexpr int ERR_TIMEOUT_EMPTY = 2;
+constexpr int ERR_TIMEOUT_READY = 4;
+constexpr long long DRAIN_CYCLES = 2000000000ll;
 
 // ---------------------------------------------------------------- helpers --
 
@@ -139,6 +154,33 @@ __device__ __forceinline__ uint4 lds128(uint32_t addr) {
     return v;
 }
 
+__device__ __forceinline__ uint32_t lds32(uint32_t addr) {
+    uint32_t v;
+    asm volatile("ld.shared.u32 %0, [%1];" : "=r"(v) : "r"(addr));
+    return v;
+}
+
+__device__ __forceinline__ int2 lds64(uint32_t addr) {
+    int2 v;
+    asm volatile("ld.shared.v2.s32 {%0,%1}, [%2];" : "=r"(v.x), "=r"(v.y) : "r"(addr));
+    return v;
+}
+
+__device__ __forceinline__ void sts32(uint32_t addr, uint32_t v) {
+    asm volatile("st.shared.u32 [%0], %1;" ::"r"(addr), "r"(v) : "memory");
+}
+
+__device__ __forceinline__ void sts64(uint32_t addr, int x, int y) {
+    asm volatile("st.shared.v2.s32 [%0], {%1,%2};" ::"r"(addr), "r"(x), "r"(y) : "memory");
+}
+
+__device__ __forceinline__ void sts128(uint32_t addr, uint32_t x, uint32_t y, uint32_t z,
+                                       uint32_t w) {
+    asm volatile("st.shared.v4.u32 [%0], {%1,%2,%3,%4};" ::"r"(addr), "r"(x), "r"(y), "r"(z),
+                 "r"(w)
+                 : "memory");
+}
+
 // D += A B with A 16x32 s8 (row), B 32x8 s8 (col), D 16x8 s32.
 __device__ __forceinline__ void mma_s8s8(int (&d)[4], const uint32_t (&a)[4], uint32_t b0,
                                          uint32_t b1) {
@@ -171,14 +213,46 @@ __device__ __forceinline__ void transpose4(uint32_t x0, uint32_t x1, uint32_t x2
     y3 = __byte_perm(t1, t3, 0x7632);
 }
 
-// Offset of byte-chunk `chunk` (16 bytes) of row `row` in a tile written by
-// TMA with the 128-byte swizzle (rows of 128 bytes, 1024-byte aligned).
+// Sign-extended byte I of w (prmt with the sign-replicate bit set in the
+// three upper selector nibbles).
+template <int I>
+__device__ __forceinline__ int sbyte(uint32_t w) {
+    constexpr uint32_t s = 8u | I;
+    constexpr uint32_t sel = (s << 12) | (s << 8) | (s << 4) | I;
+    uint32_t r;
+    asm("prmt.b32 %0, %1, 0, %2;" : "=r"(r) : "r"(w), "n"(sel));
+    return static_cast<int>(r);
+}
+
+// Packs the low bytes of four values: [a.b0, b.b0, c.b0, d.b0].
+__device__ __forceinline__ uint32_t pack4(uint32_t a, uint32_t b, uint32_t c, uint32_t d) {
+    return __byte_perm(__byte_perm(a, b, 0x0040), __byte_perm(c, d, 0x0040), 0x5410);
+}
+
+// Address of exp table entry d (0 <= d <= 255 by construction: the row
+// maximum minus a score of the row; the mask keeps it inside the table).
+__device__ __forceinline__ uint32_t lut_addr(uint32_t lut_g, int d) {
+    return lut_g + (static_cast<uint32_t>(d) & 0xffu) * (LUT_COPIES * 4);
+}
+
+// Offset of the 16-byte chunk `chunk` of row `row` in a tile written by TMA
+// with the 128-byte swizzle (rows of 128 bytes, 1024-byte aligned).
 __device__ __forceinline__ uint32_t swz(int row, int chunk) {
     return static_cast<uint32_t>(row * 128 + (((chunk ^ row) & 7) << 4));
 }
 
-// floor(2^32 / s) for s >= 2 by restoring binary long division (integer
-// only; the quotient is below 2^31).
+// Transposed V tile of one chunk: for each 32-key k step ks, half hf (keys
+// 16 hf .. 16 hf + 15 of the step) and MMA n8 tile nt, one 8 x 16-byte
+// matrix whose row r holds d = nt + 16 r and whose byte 4t + i holds key
+// 32 ks + 16 hf + 2t + (i & 1) + 8 (i >> 1) (the k order of the A operand).
+// Rows are placed at slot r ^ 2((nt >> 2) & 3) to spread the banks.
+__device__ __forceinline__ uint32_t vt_row(int ks, int hf, int nt, int r) {
+    return static_cast<uint32_t>((((ks * 2 + hf) * 16 + nt) << 7) +
+                                 ((r ^ (((nt >> 2) & 3) << 1)) << 4));
+}
+
+// floor(2^32 / s) for s >= 2 by restoring binary long division (the
+// quotient is at most 2^31).
 __device__ __forceinline__ uint32_t div_2pow32(unsigned long long s) {
     if (s > (1ull << 32)) return 0u;
     unsigned long long rem = 1ull << 32;
@@ -217,51 +291,234 @@ __device__ __forceinline__ int clamp127(long long x) {
     return x > 127 ? 127 : (x < -127 ? -127 : static_cast<int>(x));
 }
 
-// ------------------------------------------------------------ bias vectors --
-// Grid (ceil((2T-1)/256), H, B+1).  z < B: ku[(z*H + y)*T + j] =
-// sum_d u[y][d] K[z][y][j][d] for j < T.  z == B: pv[y*(2T-1) + r] =
-// sum_d v[y][d] P[y][r][d] for r < 2T-1.
-__global__ void __launch_bounds__(256) bias_vectors_kernel(const int8_t *__restrict__ k,
-                                                           const int8_t *__restrict__ p,
-                                                           const int8_t *__restrict__ u,
-                                                           const int8_t *__restrict__ vb,
-                                                           int32_t *__restrict__ ku,
-                                                           int32_t *__restrict__ pv, int *err,
-                                                           int B, int H, int T) {
-    const int j = blockIdx.x * blockDim.x + threadIdx.x;
-    const int h = blockIdx.y;
-    const int b = blockIdx.z;
-    if (j == 0 && h == 0 && b == 0) *err = 0;
-    const int8_t *row;
-    const int8_t *bias;
-    int32_t *dst;
-    if (b < B) {
-        if (j >= T) return;
-        const size_t r = (static_cast<size_t>(b) * H + h) * T + j;
-        row = k + r * DH;
-        bias = u + static_cast<size_t>(h) * DH;
-        dst = ku + r;
-    } else {
-        const int R = 2 * T - 1;
-        if (j >= R) return;
-        const size_t r = static_cast<size_t>(h) * R + j;
-        row = p + r * DH;
-        bias = vb + static_cast<size_t>(h) * DH;
-        dst = pv + r;
-    }
-    const int4 *r4 = reinterpret_cast<const int4 *>(row);
-    const int4 *b4 = reinterpret_cast<const int4 *>(bias);
-    int acc = 0;
+// ---------------------------------------------------------- consumer parts --
+
+// Position band of one warp: acc[nt] = Pv + Q P_band^T over 80 band columns
+// (P rows rw0 .. rw0 + 79, staged at ptile rows 0 .. 79; pv = shared address
+// of their P v).  Tiles go in groups of five so that the two MMAs into one
+// accumulator are separated by four independent ones.
+__device__ __forceinline__ void band_mma(int (&acc)[BAND_TILES][4], const uint32_t (&qa)[4][4],
+                                         uint32_t ptile, uint32_t pv, int lane) {
+    const int t4 = lane & 3;
 #pragma unroll
-    for (int c = 0; c < DH / 16; ++c) {
-        const int4 x = __ldg(r4 + c);
-        const int4 y = __ldg(b4 + c);
-        acc = __dp4a(x.x, y.x, acc);
-        acc = __dp4a(x.y, y.y, acc);
-        acc = __dp4a(x.z, y.z, acc);
-        acc = __dp4a(x.w, y.w, acc);
+    for (int nt = 0; nt < BAND_TILES; ++nt) {
+        const int2 v = lds64(pv + (nt * 8 + 2 * t4) * 4);
+        acc[nt][0] = v.x;
+        acc[nt][1] = v.y;
+        acc[nt][2] = v.x;
+        acc[nt][3] = v.y;
     }
-    *dst = acc;
+    const int lm_row = lane & 7, lm_mat = lane >> 3;
+#pragma unroll
+    for (int grp = 0; grp < BAND_TILES; grp += 5) {
+#pragma unroll
+        for (int kh = 0; kh < 2; ++kh) {
+            uint32_t b[5][4];
+#pragma unroll
+            for (int i = 0; i < 5; ++i)
+                ldsm_x4(ptile + swz((grp + i) * 8 + lm_row, kh * 4 + lm_mat), b[i][0], b[i][1],
+                        b[i][2], b[i][3]);
+#pragma unroll
+            for (int i = 0; i < 5; ++i) mma_s8s8(acc[grp + i], qa[2 * kh], b[i][0], b[i][1]);
+#pragma unroll
+            for (int i = 0; i < 5; ++i) mma_s8s8(acc[grp + i], qa[2 * kh + 1], b[i][2], b[i][3]);
+        }
+    }
+}
+
+// Content scores of one warp: acc[nt] = Ku + Q K^T over the chunk's 64 keys
+// (ku = shared address of the chunk's K u).
+__device__ __forceinline__ void content_mma(int (&acc)[8][4], const uint32_t (&qa)[4][4],
+                                            uint32_t ktile, uint32_t ku, int lane) {
+    const int t4 = lane & 3;
+#pragma unroll
+    for (int nt = 0; nt < 8; ++nt) {
+        const int2 v = lds64(ku + (nt * 8 + 2 * t4) * 4);
+        acc[nt][0] = v.x;
+        acc[nt][1] = v.y;
+        acc[nt][2] = v.x;
+        acc[nt][3] = v.y;
+    }
+    const int lm_row = lane & 7, lm_mat = lane >> 3;
+#pragma unroll
+    for (int grp = 0; grp < 8; grp += 4) {
+#pragma unroll
+        for (int kh = 0; kh < 2; ++kh) {
+            uint32_t b[4][4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+                ldsm_x4(ktile + swz((grp + i) * 8 + lm_row, kh * 4 + lm_mat), b[i][0], b[i][1],
+                        b[i][2], b[i][3]);
+#pragma unroll
+            for (int i = 0; i < 4; ++i) mma_s8s8(acc[grp + i], qa[2 * kh], b[i][0], b[i][1]);
+#pragma unroll
+            for (int i = 0; i < 4; ++i) mma_s8s8(acc[grp + i], qa[2 * kh + 1], b[i][2], b[i][3]);
+        }
+    }
+}
+
+// Eq. 11 for one n8 tile of the content accumulator: the fused int8 scores
+// of rows g, g+8 and keys 8nt + 2t, 8nt + 2t + 1 (Phi as the index remap
+// jj - rho + 15 into the band), key mask, running row maxima; returns the
+// four scores packed [g:2t, g:2t+1, g+8:2t, g+8:2t+1].
+template <bool MASK>
+__device__ __forceinline__ uint32_t score_tile(const int (&c)[4], int nt, uint32_t remap, int lane,
+                                               long long m_c, long long m_p, long long half_s,
+                                               int s_s, int kvalid, int &mx0, int &mx1) {
+    const int g = lane >> 2, t4 = lane & 3;
+    uint32_t v[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+        const int rho = g + ((e >> 1) << 3);
+        const int jj = nt * 8 + 2 * t4 + (e & 1);
+        const int qp = static_cast<int>(lds32(remap + (rho * (REMAP_STRIDE - 1) + jj + 15) * 4));
+        // |x| < 2^55, so x >> 31 fits 32 bits; >> (31 + s_s) = (x >> 31) >> s_s
+        const long long x = m_c * c[e] + m_p * qp + half_s;
+        const int y = static_cast<int>(__funnelshift_r(static_cast<uint32_t>(x),
+                                                       static_cast<uint32_t>(x >> 32), 31));
+        int sc = min(max(y >> s_s, -127), 127);
+        if (MASK && jj >= kvalid) sc = -128;
+        if (e < 2) mx0 = max(mx0, sc);
+        else mx1 = max(mx1, sc);
+        v[e] = static_cast<uint32_t>(sc);
+    }
+    return pack4(v[0], v[1], v[2], v[3]);
+}
+
+// Eq. 11 for a whole chunk (8 tiles) and the store of the packed scores.
+template <bool MASK>
+__device__ __forceinline__ void score_epilogue(const int (&cacc)[8][4], uint32_t remap,
+                                               uint32_t sdst, int lane, long long m_c,
+                                               long long m_p, long long half_s, int s_s,
+                                               int kvalid, int &mx0, int &mx1) {
+    uint32_t packed[8];
+#pragma unroll
+    for (int nt = 0; nt < 8; ++nt)
+        packed[nt] = score_tile<MASK>(cacc[nt], nt, remap, lane, m_c, m_p, half_s, s_s, kvalid,
+                                      mx0, mx1);
+    sts128(sdst + lane * 16, packed[0], packed[1], packed[2], packed[3]);
+    sts128(sdst + 512 + lane * 16, packed[4], packed[5], packed[6], packed[7]);
+}
+
+// Sum of the integer exponentials of one stored half chunk (16 scores per
+// thread: rows g and g+8, 8 keys each).
+template <bool MASK>
+__device__ __forceinline__ void exp_sums(uint4 sv, uint32_t lut_g, int mx0, int mx1, int t4,
+                                         int kbase, int kvalid, unsigned long long &s0,
+                                         unsigned long long &s1) {
+    const uint32_t wv[4] = {sv.x, sv.y, sv.z, sv.w};
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        const int sc[4] = {sbyte<0>(wv[q]), sbyte<1>(wv[q]), sbyte<2>(wv[q]), sbyte<3>(wv[q])};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const int mx = e < 2 ? mx0 : mx1;
+            uint32_t ev = lds32(lut_addr(lut_g, mx - sc[e]));
+            if (MASK && kbase + q * 8 + 2 * t4 + (e & 1) >= kvalid) ev = 0u;
+            if (e < 2) s0 += ev;
+            else s1 += ev;
+        }
+    }
+}
+
+// Probabilities of one packed score word (rows g, g+8 x two keys) on the
+// grid 2^-8.  Masked keys (score -128) are zeroed by the caller.
+__device__ __forceinline__ uint32_t prob_word(uint32_t wv, uint32_t lut_g, int mx0, int mx1,
+                                              uint32_t f0, uint32_t f1) {
+    const int sc[4] = {sbyte<0>(wv), sbyte<1>(wv), sbyte<2>(wv), sbyte<3>(wv)};
+    uint32_t a[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+        const int mx = e < 2 ? mx0 : mx1;
+        const uint32_t f = e < 2 ? f0 : f1;
+        const uint32_t ev = lds32(lut_addr(lut_g, mx - sc[e]));
+        const unsigned long long y = (static_cast<unsigned long long>(ev) * f) >> 24;
+        a[e] = static_cast<uint32_t>(min(y, 255ull));
+    }
+    return pack4(a[0], a[1], a[2], a[3]);
+}
+
+// Byte mask of a probability word of tile q of a 32-key step whose first
+// key is kbase: keys kbase + 8q + 2t (bytes 0, 2) and + 1 (bytes 1, 3)
+// are kept when below kvalid.
+__device__ __forceinline__ uint32_t key_mask(int kbase, int q, int t4, int kvalid) {
+    const int k0 = kbase + 8 * q + 2 * t4;
+    return (k0 < kvalid ? 0x00ff00ffu : 0u) | (k0 + 1 < kvalid ? 0xff00ff00u : 0u);
+}
+
+// The u8 A operand of the A.V MMA from the four probability words of a
+// 32-key step (k order: keys 2t, 2t+1, 8+2t, 9+2t, then the same + 16).
+__device__ __forceinline__ void prob_operand(const uint32_t (&pw)[4], uint32_t (&af)[4]) {
+    af[0] = __byte_perm(pw[0], pw[1], 0x5410);
+    af[1] = __byte_perm(pw[0], pw[1], 0x7632);
+    af[2] = __byte_perm(pw[2], pw[3], 0x5410);
+    af[3] = __byte_perm(pw[2], pw[3], 0x7632);
+}
+
+// ---------------------------------------------------------- producer parts --
+
+// K u for the chunk's 64 keys and P v for the 128 staged band rows; lane l
+// takes keys l, l+32 and band rows l, l+32, l+64, l+96.
+__device__ __forceinline__ void prep_bias(uint32_t ktile, uint32_t ptile, uint32_t ku, uint32_t pv,
+                                          const uint32_t (&uw)[32], const uint32_t (&vw)[32],
+                                          int lane) {
+#pragma unroll
+    for (int k = 0; k < 2; ++k) {
+        const int row = lane + 32 * k;
+        int acc = 0;
+#pragma unroll
+        for (int ch = 0; ch < 8; ++ch) {
+            const uint4 x = lds128(ktile + swz(row, ch));
+            acc = __dp4a(static_cast<int>(x.x), static_cast<int>(uw[4 * ch + 0]), acc);
+            acc = __dp4a(static_cast<int>(x.y), static_cast<int>(uw[4 * ch + 1]), acc);
+            acc = __dp4a(static_cast<int>(x.z), static_cast<int>(uw[4 * ch + 2]), acc);
+            acc = __dp4a(static_cast<int>(x.w), static_cast<int>(uw[4 * ch + 3]), acc);
+        }
+        sts32(ku + row * 4, static_cast<uint32_t>(acc));
+    }
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        const int row = lane + 32 * k;
+        int acc = 0;
+#pragma unroll
+        for (int ch = 0; ch < 8; ++ch) {
+            const uint4 x = lds128(ptile + swz(row, ch));
+            acc = __dp4a(static_cast<int>(x.x), static_cast<int>(vw[4 * ch + 0]), acc);
+            acc = __dp4a(static_cast<int>(x.y), static_cast<int>(vw[4 * ch + 1]), acc);
+            acc = __dp4a(static_cast<int>(x.z), static_cast<int>(vw[4 * ch + 2]), acc);
+            acc = __dp4a(static_cast<int>(x.w), static_cast<int>(vw[4 * ch + 3]), acc);
+        }
+        sts32(pv + row * 4, static_cast<uint32_t>(acc));
+    }
+}
+
+// Transposes the staged V tile (rows = keys, 128-byte swizzle) into the
+// MMA operand layout of vt_row.  Work unit: 4 keys x 4 d; lane l, round k:
+// t = l & 3, 4-d block db = (l >> 2) + 8 (k & 3), half hf = (k >> 2) & 1,
+// k step ks = k >> 3.
+__device__ __forceinline__ void prep_vt(uint32_t vtile, uint32_t vt, int lane) {
+    const int t4 = lane & 3;
+#pragma unroll 4
+    for (int k = 0; k < 16; ++k) {
+        const int db = (lane >> 2) + 8 * (k & 3);
+        const int hf = (k >> 2) & 1;
+        const int ks = k >> 3;
+        const int d0 = 4 * db;
+        const int kb = 32 * ks + 16 * hf + 2 * t4;
+        uint32_t x[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const int key = kb + (i & 1) + 8 * (i >> 1);
+            x[i] = lds32(vtile + swz(key, d0 >> 4) + (d0 & 15));
+        }
+        uint32_t y[4];
+        transpose4(x[0], x[1], x[2], x[3], y[0], y[1], y[2], y[3]);
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+            const int d = d0 + c;
+            sts32(vt + vt_row(ks, hf, d & 15, d >> 4) + 4 * t4, y[c]);
+        }
+    }
 }
 
 // ------------------------------------------------------------ fused kernel --
@@ -298,59 +555,100 @@ __global__ void __launch_bounds__(NTHREADS, 2)
         return;
     }
     const int nchunks = (len + NK - 1) / NK;
+    const int total = 2 * nchunks;   // uses of the stage ring: pass-1 chunks, then pass-3 chunks
 
-    uint32_t *lut = reinterpret_cast<uint32_t *>(smem + L.lut);
+    const uint32_t lut = smem_u32(smem + L.lut);
     const uint32_t bar_base = smem_u32(smem + L.bars);
     auto full_bar = [&](int s) { return bar_base + 8u * s; };
-    auto empty_bar = [&](int s) { return bar_base + 8u * (NSTAGE + s); };
+    auto ready_bar = [&](int s) { return bar_base + 8u * (NSTAGE + s); };
+    auto empty_bar = [&](int s) { return bar_base + 8u * (2 * NSTAGE + s); };
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < NSTAGE; ++s) {
             mbar_init(full_bar(s), 1);
+            mbar_init(ready_bar(s), 1);
             mbar_init(empty_bar(s), NCWARPS);
         }
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
     }
-    for (int d = threadIdx.x; d < LUT_ENTRIES; d += NTHREADS)
-        lut[d] = iexp_neg(d, prm.q_ln2, prm.q_b, prm.q_c);
+    for (int d = threadIdx.x; d < LUT_ENTRIES; d += NTHREADS) {
+        const uint32_t e = iexp_neg(d, prm.q_ln2, prm.q_b, prm.q_c);
+#pragma unroll
+        for (int c = 0; c < LUT_COPIES; ++c) sts32(lut + (d * LUT_COPIES + c) * 4, e);
+    }
     __syncthreads();
 
     const uint32_t stage_base = smem_u32(smem + L.stages);
+    auto stage_addr = [&](int s) { return stage_base + s * STAGE_BYTES; };
 
     // ------------------------------------------------------------ producer
+    // Use `it` of the stage ring (stage it & 1, phase it >> 1): TMA lands
+    // (full), the producer prepares it (ready), the consumers release it
+    // (empty), and the stage is refilled with use it + 2.
     if (warp == NCWARPS) {
+        uint32_t uw[32], vw[32];
+        {
+            const uint4 *u4 = reinterpret_cast<const uint4 *>(prm.u + static_cast<size_t>(h) * DH);
+            const uint4 *v4 = reinterpret_cast<const uint4 *>(prm.vb + static_cast<size_t>(h) * DH);
+#pragma unroll
+            for (int c = 0; c < 8; ++c) {
+                const uint4 a = __ldg(u4 + c), bq = __ldg(v4 + c);
+                uw[4 * c] = a.x; uw[4 * c + 1] = a.y; uw[4 * c + 2] = a.z; uw[4 * c + 3] = a.w;
+                vw[4 * c] = bq.x; vw[4 * c + 1] = bq.y; vw[4 * c + 2] = bq.z; vw[4 * c + 3] = bq.w;
+            }
+        }
+        auto issue = [&](int it) {
+            const int s = it & 1;
+            const uint32_t dst = stage_addr(s);
+            if (it < nchunks) {
+                const int j0 = it * NK;
+                mbar_expect_tx(full_bar(s), K_TILE_BYTES + P_TILE_BYTES);
+                tma_load_3d(dst, &tm_k, 0, j0, bh, full_bar(s));
+                tma_load_3d(dst + K_TILE_BYTES, &tm_p, 0, j0 - i0 - (MROWS - 1) + T - 1, h,
+                            full_bar(s));
+            } else {
+                const int j0 = (it - nchunks) * NK;
+                mbar_expect_tx(full_bar(s), K_TILE_BYTES);
+                tma_load_3d(dst, &tm_v, 0, j0, bh, full_bar(s));
+            }
+        };
+        int issued = total > 1 ? 2 : 1, landed = 0;
+        bool ok = true;
         if (lane == 0) {
-            int uses[NSTAGE] = {0};
-            bool ok = true;
-            const int total = 2 * nchunks;
-            for (int it = 0; it < total && ok; ++it) {
-                const int s = it % NSTAGE;
-                if (uses[s] > 0 && !mbar_wait(empty_bar(s), (uses[s] - 1) & 1, prm.timeout_cycles)) {
-                    atomicOr(prm.err, ERR_TIMEOUT_EMPTY);
+            issue(0);
+            if (total > 1) issue(1);
+        }
+        for (int it = 0; it < total; ++it) {
+            const int s = it & 1;
+            if (!mbar_wait(full_bar(s), (it >> 1) & 1, prm.timeout_cycles)) {
+                if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_FULL);
+                ok = false;
+                break;
+            }
+            landed = it + 1;
+            if (it < nchunks)
+                prep_bias(stage_addr(s), stage_addr(s) + K_TILE_BYTES, stage_addr(s) + KU_OFF,
+                          stage_addr(s) + PV_OFF, uw, vw, lane);
+            else
+                prep_vt(stage_addr(s), stage_addr(s) + K_TILE_BYTES, lane);
+            __syncwarp();
+            if (lane == 0) mbar_arrive(ready_bar(s));
+            if (it + 2 < total) {
+                if (!mbar_wait(empty_bar(s), (it >> 1) & 1, prm.timeout_cycles)) {
+                    if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_EMPTY);
                     ok = false;
                     break;
                 }
-                const uint32_t dst = stage_base + s * STAGE_BYTES;
-                if (it < nchunks) {
-                    const int j0 = it * NK;
-                    mbar_expect_tx(full_bar(s), K_TILE_BYTES + P_TILE_BYTES);
-                    tma_load_3d(dst, &tm_k, 0, j0, bh, full_bar(s));
-                    tma_load_3d(dst + K_TILE_BYTES, &tm_p, 0, j0 - i0 - (MROWS - 1) + T - 1, h,
-                                full_bar(s));
-                } else {
-                    const int j0 = (it - nchunks) * NK;
-                    mbar_expect_tx(full_bar(s), K_TILE_BYTES);
-                    tma_load_3d(dst, &tm_v, 0, j0, bh, full_bar(s));
-                }
-                ++uses[s];
+                if (lane == 0) issue(it + 2);
+                issued = it + 3;
             }
-            if (!ok) {
-                // Let the copies already issued land before the CTA exits
-                // (bounded by a fixed budget independent of the caller's).
-                for (int s = 0; s < NSTAGE; ++s)
-                    if (uses[s] > 0) mbar_wait(full_bar(s), (uses[s] - 1) & 1, 2000000000ll);
-            }
+        }
+        if (!ok) {
+            // Let the copies already issued land before the CTA exits
+            // (bounded by a fixed budget independent of the caller's).
+            for (int it = landed; it < issued; ++it)
+                mbar_wait(full_bar(it & 1), (it >> 1) & 1, DRAIN_CYCLES);
         }
         return;
     }
@@ -375,113 +673,86 @@ __global__ void __launch_bounds__(NTHREADS, 2)
         }
     }
 
-    int32_t *remap = reinterpret_cast<int32_t *>(smem + L.remap) + warp * (16 * REMAP_STRIDE);
-    uint8_t *scores = smem + L.scores + warp * (prm.nchunk_max * CHUNK_SCORE_BYTES);
-    const int32_t *ku = prm.ku + static_cast<size_t>(bh) * T;
-    const int32_t *pv = prm.pv + static_cast<size_t>(h) * (2 * T - 1);
+    const uint32_t remap = smem_u32(smem + L.remap) + warp * REMAP_BYTES;
+    const uint32_t scores = smem_u32(smem + L.scores) + warp * (prm.nchunk_max * CHUNK_SCORE_BYTES);
+    const long long m_c = prm.m_c, m_p = prm.m_p;
     const long long half_s = 1ll << (prm.sh_s - 1);
-    int mx0 = -128, mx1 = -128;   // running maxima of rows g and g + 8
-    bool ok = true;
+    const int s_s = prm.sh_s - 31;
+    const int band_row0 = 48 - 16 * warp;      // this warp's first row in the staged band
+    int mx0 = -128, mx1 = -128;                // running maxima of rows g and g + 8
 
-    // lane address pattern of ldmatrix.x4: matrix lane>>3, row lane&7
-    const int lm_row = lane & 7;
-    const int lm_mat = lane >> 3;
-
+    // ---- pass 1: scores.  A warp that issues an integer MMA waits until the
+    // tensor pipe accepts it, so the band MMAs of chunk c+1 are issued in
+    // groups with the epilogue of chunk c between them: the epilogue runs
+    // while the pipe works through the band.
+    int bacc[BAND_TILES][4];
+    if (!mbar_wait(ready_bar(0), 0, prm.timeout_cycles)) {
+        if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_READY);
+        return;
+    }
+    band_mma(bacc, qa, stage_addr(0) + K_TILE_BYTES + band_row0 * 128,
+             stage_addr(0) + PV_OFF + band_row0 * 4, lane);
+    const int lm_row = lane & 7, lm_mat = lane >> 3;
     for (int c = 0; c < nchunks; ++c) {
-        const int s = c % NSTAGE;
-        if (!mbar_wait(full_bar(s), (c / NSTAGE) & 1, prm.timeout_cycles)) {
-            atomicOr(prm.err, ERR_TIMEOUT_FULL);
-            ok = false;
-            break;
+        const int s = c & 1;
+        __syncwarp();
+#pragma unroll
+        for (int nt = 0; nt < BAND_TILES; ++nt) {
+            sts64(remap + (g * REMAP_STRIDE + nt * 8 + 2 * t4) * 4, bacc[nt][0], bacc[nt][1]);
+            sts64(remap + ((g + 8) * REMAP_STRIDE + nt * 8 + 2 * t4) * 4, bacc[nt][2], bacc[nt][3]);
         }
-        const uint32_t ktile = stage_base + s * STAGE_BYTES;
-        const uint32_t ptile = ktile + K_TILE_BYTES + (48 - 16 * warp) * 128;
-        const int j0 = c * NK;
-        const int rw0 = j0 - wrow0 - 15 + T - 1;   // P row of band column 0
-
-        // ---- position band: 16 rows x 80 relative positions
-        {
-            int bacc[BAND_TILES][4];
-#pragma unroll
-            for (int nt = 0; nt < BAND_TILES; ++nt) {
-#pragma unroll
-                for (int e = 0; e < 2; ++e) {
-                    const int r = rw0 + nt * 8 + 2 * t4 + e;
-                    const int val = (r >= 0 && r <= 2 * T - 2) ? pv[r] : 0;
-                    bacc[nt][e] = val;
-                    bacc[nt][2 + e] = val;
-                }
-            }
-#pragma unroll
-            for (int nt = 0; nt < BAND_TILES; ++nt) {
-#pragma unroll
-                for (int kh = 0; kh < 2; ++kh) {
-                    uint32_t b0, b1, b2, b3;
-                    ldsm_x4(ptile + swz(nt * 8 + lm_row, kh * 4 + lm_mat), b0, b1, b2, b3);
-                    mma_s8s8(bacc[nt], qa[2 * kh], b0, b1);
-                    mma_s8s8(bacc[nt], qa[2 * kh + 1], b2, b3);
-                }
-            }
-            __syncwarp();
-#pragma unroll
-            for (int nt = 0; nt < BAND_TILES; ++nt) {
-                *reinterpret_cast<int2 *>(remap + g * REMAP_STRIDE + nt * 8 + 2 * t4) =
-                    make_int2(bacc[nt][0], bacc[nt][1]);
-                *reinterpret_cast<int2 *>(remap + (g + 8) * REMAP_STRIDE + nt * 8 + 2 * t4) =
-                    make_int2(bacc[nt][2], bacc[nt][3]);
-            }
-        }
-
-        // ---- content: 16 rows x 64 keys
         int cacc[8][4];
-#pragma unroll
-        for (int nt = 0; nt < 8; ++nt) {
-#pragma unroll
-            for (int e = 0; e < 2; ++e) {
-                const int j = j0 + nt * 8 + 2 * t4 + e;
-                const int val = j < T ? ku[j] : 0;
-                cacc[nt][e] = val;
-                cacc[nt][2 + e] = val;
-            }
-        }
-#pragma unroll
-        for (int nt = 0; nt < 8; ++nt) {
-#pragma unroll
-            for (int kh = 0; kh < 2; ++kh) {
-                uint32_t b0, b1, b2, b3;
-                ldsm_x4(ktile + swz(nt * 8 + lm_row, kh * 4 + lm_mat), b0, b1, b2, b3);
-                mma_s8s8(cacc[nt], qa[2 * kh], b0, b1);
-                mma_s8s8(cacc[nt], qa[2 * kh + 1], b2, b3);
-            }
-        }
+        content_mma(cacc, qa, stage_addr(s), stage_addr(s) + KU_OFF, lane);
         __syncwarp();
         if (lane == 0) mbar_arrive(empty_bar(s));
-
-        // ---- Eq. 11 with Phi as an index remap, key mask, row max
-        uint32_t packed[8];
-#pragma unroll
-        for (int nt = 0; nt < 8; ++nt) {
-            uint32_t w = 0;
-#pragma unroll
-            for (int e = 0; e < 4; ++e) {
-                const int rho = g + ((e >> 1) << 3);
-                const int jj = nt * 8 + 2 * t4 + (e & 1);
-                const int qp = remap[rho * REMAP_STRIDE + jj - rho + 15];
-                const long long x = static_cast<long long>(prm.m_c) * cacc[nt][e] +
-                                    static_cast<long long>(prm.m_p) * qp + half_s;
-                int sc = clamp127(x >> prm.sh_s);
-                if (j0 + jj >= len) sc = -128;
-                if (e < 2) mx0 = sc > mx0 ? sc : mx0;
-                else mx1 = sc > mx1 ? sc : mx1;
-                w |= (static_cast<uint32_t>(sc) & 0xffu) << (8 * e);
+        const uint32_t sdst = scores + c * CHUNK_SCORE_BYTES;
+        if (c + 1 < nchunks) {
+            if (!mbar_wait(ready_bar(s ^ 1), ((c + 1) >> 1) & 1, prm.timeout_cycles)) {
+                if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_READY);
+                return;
             }
-            packed[nt] = w;
+            const uint32_t ptile = stage_addr(s ^ 1) + K_TILE_BYTES + band_row0 * 128;
+            const uint32_t pvs = stage_addr(s ^ 1) + PV_OFF + band_row0 * 4;
+#pragma unroll
+            for (int nt = 0; nt < BAND_TILES; ++nt) {
+                const int2 v = lds64(pvs + (nt * 8 + 2 * t4) * 4);
+                bacc[nt][0] = v.x;
+                bacc[nt][1] = v.y;
+                bacc[nt][2] = v.x;
+                bacc[nt][3] = v.y;
+            }
+            __syncwarp();
+            uint32_t packed[8];
+#pragma unroll
+            for (int m = 0; m < 4; ++m) {
+                const int kh = m >> 1, t0 = (m & 1) * 5;
+                uint32_t b[5][4];
+#pragma unroll
+                for (int i = 0; i < 5; ++i)
+                    ldsm_x4(ptile + swz((t0 + i) * 8 + lm_row, kh * 4 + lm_mat), b[i][0], b[i][1],
+                            b[i][2], b[i][3]);
+#pragma unroll
+                for (int i = 0; i < 5; ++i) mma_s8s8(bacc[t0 + i], qa[2 * kh], b[i][0], b[i][1]);
+                packed[2 * m] = score_tile<false>(cacc[2 * m], 2 * m, remap, lane, m_c, m_p, half_s,
+                                                  s_s, NK, mx0, mx1);
+#pragma unroll
+                for (int i = 0; i < 5; ++i) mma_s8s8(bacc[t0 + i], qa[2 * kh + 1], b[i][2], b[i][3]);
+                packed[2 * m + 1] = score_tile<false>(cacc[2 * m + 1], 2 * m + 1, remap, lane, m_c,
+                                                      m_p, half_s, s_s, NK, mx0, mx1);
+            }
+            sts128(sdst + lane * 16, packed[0], packed[1], packed[2], packed[3]);
+            sts128(sdst + 512 + lane * 16, packed[4], packed[5], packed[6], packed[7]);
+        } else {
+            __syncwarp();
+            const int kvalid = len - c * NK;
+            if (kvalid < NK)
+                score_epilogue<true>(cacc, remap, sdst, lane, m_c, m_p, half_s, s_s, kvalid,
+                                     mx0, mx1);
+            else
+                score_epilogue<false>(cacc, remap, sdst, lane, m_c, m_p, half_s, s_s, kvalid,
+                                      mx0, mx1);
         }
-        uint8_t *sdst = scores + c * CHUNK_SCORE_BYTES + lane * 16;
-        *reinterpret_cast<uint4 *>(sdst) = make_uint4(packed[0], packed[1], packed[2], packed[3]);
-        *reinterpret_cast<uint4 *>(sdst + 512) = make_uint4(packed[4], packed[5], packed[6], packed[7]);
     }
-    if (!ok) return;
 
     // ---- row maxima across the quad
     mx0 = max(mx0, __shfl_xor_sync(0xffffffffu, mx0, 1));
@@ -490,23 +761,17 @@ __global__ void __launch_bounds__(NTHREADS, 2)
     mx1 = max(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
 
     // ---- pass 2: sums of the integer exponentials
+    const uint32_t lut_g = lut + 4 * g;
     unsigned long long sum0 = 0, sum1 = 0;
     for (int c = 0; c < nchunks; ++c) {
+        const int kvalid = len - c * NK;
 #pragma unroll
         for (int hf = 0; hf < 2; ++hf) {
-            const uint4 sv = *reinterpret_cast<const uint4 *>(scores + c * CHUNK_SCORE_BYTES + hf * 512 + lane * 16);
-            const uint32_t wv[4] = {sv.x, sv.y, sv.z, sv.w};
-#pragma unroll
-            for (int q = 0; q < 4; ++q) {
-#pragma unroll
-                for (int e = 0; e < 4; ++e) {
-                    const int sc = static_cast<int>(static_cast<int8_t>((wv[q] >> (8 * e)) & 0xffu));
-                    const int mx = e < 2 ? mx0 : mx1;
-                    const uint32_t ev = sc == -128 ? 0u : lut[mx - sc];
-                    if (e < 2) sum0 += ev;
-                    else sum1 += ev;
-                }
-            }
+            const uint4 sv = lds128(scores + c * CHUNK_SCORE_BYTES + hf * 512 + lane * 16);
+            if (kvalid < NK)
+                exp_sums<true>(sv, lut_g, mx0, mx1, t4, 32 * hf, kvalid, sum0, sum1);
+            else
+                exp_sums<false>(sv, lut_g, mx0, mx1, t4, 32 * hf, kvalid, sum0, sum1);
         }
     }
     sum0 += __shfl_xor_sync(0xffffffffu, sum0, 1);
@@ -516,76 +781,69 @@ __global__ void __launch_bounds__(NTHREADS, 2)
     const uint32_t f0 = div_2pow32(sum0);
     const uint32_t f1 = div_2pow32(sum1);
 
-    // ---- pass 3: probabilities x V
+    // ---- pass 3: probabilities x V.  The A operand of the next 32-key step
+    // is computed between the MMA groups of the current one.
     int oacc[16][4];
 #pragma unroll
     for (int nt = 0; nt < 16; ++nt) oacc[nt][0] = oacc[nt][1] = oacc[nt][2] = oacc[nt][3] = 0;
-
+    const int nsteps = 2 * nchunks;
+    uint32_t af[4];
+    const int kvalid_last = len - (nchunks - 1) * NK;   // valid keys of the last chunk
+    {
+        const uint4 sv = lds128(scores + lane * 16);
+        uint32_t pw[4] = {prob_word(sv.x, lut_g, mx0, mx1, f0, f1),
+                          prob_word(sv.y, lut_g, mx0, mx1, f0, f1),
+                          prob_word(sv.z, lut_g, mx0, mx1, f0, f1),
+                          prob_word(sv.w, lut_g, mx0, mx1, f0, f1)};
+        if (nchunks == 1 && kvalid_last < NK) {
+#pragma unroll
+            for (int q = 0; q < 4; ++q) pw[q] &= key_mask(0, q, t4, kvalid_last);
+        }
+        prob_operand(pw, af);
+    }
     for (int c = 0; c < nchunks; ++c) {
         const int it = nchunks + c;
-        const int s = it % NSTAGE;
-        if (!mbar_wait(full_bar(s), (it / NSTAGE) & 1, prm.timeout_cycles)) {
-            atomicOr(prm.err, ERR_TIMEOUT_FULL);
-            ok = false;
-            break;
+        const int s = it & 1;
+        if (!mbar_wait(ready_bar(s), (it >> 1) & 1, prm.timeout_cycles)) {
+            if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_READY);
+            return;
         }
-        const uint32_t vtile = stage_base + s * STAGE_BYTES;
+        const uint32_t vt = stage_addr(s) + K_TILE_BYTES;
 #pragma unroll
-        for (int hf = 0; hf < 2; ++hf) {
-            const uint4 sv = *reinterpret_cast<const uint4 *>(scores + c * CHUNK_SCORE_BYTES + hf * 512 + lane * 16);
-            const uint32_t wv[4] = {sv.x, sv.y, sv.z, sv.w};
+        for (int ks = 0; ks < 2; ++ks) {
+            const int nxt = min(2 * c + ks + 1, nsteps - 1);
+            const uint4 svn = lds128(scores + (nxt >> 1) * CHUNK_SCORE_BYTES + (nxt & 1) * 512 + lane * 16);
+            const uint32_t wn[4] = {svn.x, svn.y, svn.z, svn.w};
             uint32_t pw[4];
 #pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                uint32_t w = 0;
+            for (int grp = 0; grp < 4; ++grp) {
+                uint32_t b[2][4];
 #pragma unroll
-                for (int e = 0; e < 4; ++e) {
-                    const int sc = static_cast<int>(static_cast<int8_t>((wv[q] >> (8 * e)) & 0xffu));
-                    const int mx = e < 2 ? mx0 : mx1;
-                    const uint32_t f = e < 2 ? f0 : f1;
-                    const uint32_t ev = sc == -128 ? 0u : lut[mx - sc];
-                    unsigned long long y = (static_cast<unsigned long long>(ev) * f) >> 24;
-                    const uint32_t a = y > 255ull ? 255u : static_cast<uint32_t>(y);
-                    w |= a << (8 * e);
+                for (int i = 0; i < 2; ++i) {
+                    // matrix m = lm_mat: tile nt = 4 grp + 2 i + (m >> 1), half hf = m & 1
+                    ldsm_x4(vt + vt_row(ks, lm_mat & 1, 4 * grp + 2 * i + (lm_mat >> 1), lm_row),
+                            b[i][0], b[i][1], b[i][2], b[i][3]);
                 }
-                pw[q] = w;
-            }
-            uint32_t af[4];
-            af[0] = __byte_perm(pw[0], pw[1], 0x5410);
-            af[1] = __byte_perm(pw[0], pw[1], 0x7632);
-            af[2] = __byte_perm(pw[2], pw[3], 0x5410);
-            af[3] = __byte_perm(pw[2], pw[3], 0x7632);
-
-            // V rows of this k step in the MMA's k order:
-            // b0 <- keys {2t, 2t+1, 8+2t, 9+2t}, b1 <- the same + 16.
-            uint32_t bf0[16], bf1[16];
 #pragma unroll
-            for (int half16 = 0; half16 < 2; ++half16) {
-                uint32_t x[4][4];
-#pragma unroll
-                for (int kk = 0; kk < 4; ++kk) {
-                    const int key = hf * 32 + half16 * 16 + 2 * t4 + (kk & 1) + 8 * (kk >> 1);
-                    const uint4 v4 = lds128(vtile + swz(key, g));
-                    x[kk][0] = v4.x;
-                    x[kk][1] = v4.y;
-                    x[kk][2] = v4.z;
-                    x[kk][3] = v4.w;
+                for (int i = 0; i < 2; ++i) {
+                    mma_u8s8(oacc[4 * grp + 2 * i], af, b[i][0], b[i][1]);
+                    mma_u8s8(oacc[4 * grp + 2 * i + 1], af, b[i][2], b[i][3]);
                 }
-                uint32_t *dst = half16 ? bf1 : bf0;
-#pragma unroll
-                for (int w = 0; w < 4; ++w)
-                    transpose4(x[0][w], x[1][w], x[2][w], x[3][w], dst[4 * w + 0], dst[4 * w + 1],
-                               dst[4 * w + 2], dst[4 * w + 3]);
+                pw[grp] = prob_word(wn[grp], lut_g, mx0, mx1, f0, f1);
             }
+            if ((nxt >> 1) == nchunks - 1 && kvalid_last < NK) {
+                const int kbase = (nxt & 1) * 32;
 #pragma unroll
-            for (int nt = 0; nt < 16; ++nt) mma_u8s8(oacc[nt], af, bf0[nt], bf1[nt]);
+                for (int q = 0; q < 4; ++q) pw[q] &= key_mask(kbase, q, t4, kvalid_last);
+            }
+            prob_operand(pw, af);
         }
         __syncwarp();
         if (lane == 0) mbar_arrive(empty_bar(s));
     }
-    if (!ok) return;
 
     // ---- output requantisation (Eq. 7) and 16-byte stores
+    const long long m_o = prm.m_o;
     const long long half_o = 1ll << (prm.sh_o - 1);
 #pragma unroll
     for (int rr = 0; rr < 2; ++rr) {
@@ -600,7 +858,7 @@ __global__ void __launch_bounds__(NTHREADS, 2)
 #pragma unroll
                 for (int e = 0; e < 4; ++e) {
                     const int nt = wq * 4 + e;
-                    const long long x = static_cast<long long>(prm.m_o) * oacc[nt][2 * rr + hh] + half_o;
+                    const long long x = m_o * oacc[nt][2 * rr + hh] + half_o;
                     const int o = row < len ? clamp127(x >> prm.sh_o) : 0;
                     w |= (static_cast<uint32_t>(o) & 0xffu) << (8 * e);
                 }

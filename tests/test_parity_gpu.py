@@ -36,7 +36,7 @@ def _dev(a):
 
 def run_gpu(ip, lay, consts, lengths=None):
     B, H, T, dh = lay.q.shape
-    ws = torch.empty(ip.workspace_bytes(B, H, T, dh), dtype=torch.uint8, device="cuda")
+    ws = torch.zeros(ip.workspace_bytes(B, H, T, dh), dtype=torch.uint8, device="cuda")
     lens = None if lengths is None else _dev(lengths.astype(np.int32))
     out = ip.relpos_mhsa_i8(_dev(lay.q), _dev(lay.k), _dev(lay.v), _dev(lay.p), _dev(lay.u),
                             _dev(lay.vb), consts, lengths=lens, workspace=ws)
@@ -129,7 +129,7 @@ def test_empty_batch(ip):
     lay = synth.draw(0, 8, 10, 128, seed=1)
     c = ip.layer_constants(synth.draw(1, 8, 10, 128, seed=1).scales)
     out = torch.full((0, 8, 10, 128), 5, dtype=torch.int8, device="cuda")
-    ws = torch.empty(ip.workspace_bytes(0, 8, 10), dtype=torch.uint8, device="cuda")
+    ws = torch.zeros(ip.workspace_bytes(0, 8, 10), dtype=torch.uint8, device="cuda")
     ip.relpos_mhsa_i8(_dev(lay.q), _dev(lay.k), _dev(lay.v), _dev(lay.p), _dev(lay.u),
                       _dev(lay.vb), c, out=out, workspace=ws)
     torch.cuda.synchronize()
@@ -155,7 +155,7 @@ def test_repeated_calls_share_workspace(ip, orc):
         lay = synth.draw(3, 8, 130, 128, seed=60 + i, p_mode="sinusoid")
         c = ip.layer_constants(lay.scales)
         if ws is None:
-            ws = torch.empty(ip.workspace_bytes(3, 8, 130), dtype=torch.uint8, device="cuda")
+            ws = torch.zeros(ip.workspace_bytes(3, 8, 130), dtype=torch.uint8, device="cuda")
         out = ip.relpos_mhsa_i8(_dev(lay.q), _dev(lay.k), _dev(lay.v), _dev(lay.p), _dev(lay.u),
                                 _dev(lay.vb), c, workspace=ws)
         assert ip.status(ws) == 0
