@@ -130,6 +130,13 @@ const char *ip_strerror(int code);
  * returns. */
 int ip_debug_set_timeout_cycles(long long cycles);
 
+/* Test hook: when on, the kernels launched afterwards by this process first
+ * make every consumer warp wait on a barrier that nothing arrives on, so
+ * that the bounded wait runs out and the error path (IP_ERR_TIMEOUT, copies
+ * in flight drained, early return) is exercised without faulting or hanging
+ * the GPU.  Off by default. */
+int ip_debug_set_stall_injection(int on);
+
 /* Diagnostic: enqueues a throughput probe of the integer warp MMA
  * (mma.sync m16n8k32 s8 x s8 -> s32, eight independent accumulators per
  * warp, `iters` rounds) on `stream`; sink is a device int array of

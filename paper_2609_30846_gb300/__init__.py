@@ -27,7 +27,8 @@ ERRORS = {
 EXPORTS = (
     "ip_relpos_mhsa_workspace_bytes", "ip_relpos_mhsa_i8", "ip_relpos_mhsa_status",
     "ip_relpos_mhsa_host_arena_bytes", "ip_relpos_mhsa_i8_host", "ip_strerror",
-    "ip_debug_set_timeout_cycles", "ip_dyadic_multiplier", "ip_dyadic_pair",
+    "ip_debug_set_timeout_cycles", "ip_debug_set_stall_injection", "ip_dyadic_multiplier",
+    "ip_dyadic_pair",
     "ip_isoftmax_params_from_scale", "ip_probe_int8_mma",
 )
 
@@ -86,6 +87,8 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
         lib.ip_strerror.restype = ctypes.c_char_p
         lib.ip_debug_set_timeout_cycles.argtypes = [ctypes.c_longlong]
         lib.ip_debug_set_timeout_cycles.restype = I
+        lib.ip_debug_set_stall_injection.argtypes = [I]
+        lib.ip_debug_set_stall_injection.restype = I
         lib.ip_dyadic_multiplier.argtypes = [ctypes.c_double, i32p, i32p]
         lib.ip_dyadic_multiplier.restype = I
         lib.ip_dyadic_pair.argtypes = [ctypes.c_double, ctypes.c_double, i32p, i32p, i32p]
@@ -165,6 +168,11 @@ def host_arena_bytes(B: int, H: int, T: int, dh: int = IP_DH) -> int:
 def set_timeout_cycles(cycles: int) -> None:
     """Bound of every kernel barrier wait (clock cycles; negative: default)."""
     load().ip_debug_set_timeout_cycles(int(cycles))
+
+
+def set_stall_injection(on: bool) -> None:
+    """Test hook: make the kernels wait on a barrier nothing arrives on."""
+    load().ip_debug_set_stall_injection(1 if on else 0)
 
 
 def _arr(vals, ctype):
@@ -276,5 +284,5 @@ def relpos_mhsa_i8_host(q, k, v, p, u, v_bias, consts: LayerConstants, lengths, 
 __all__ = ["build", "load", "relpos_mhsa_i8", "relpos_mhsa_i8_host", "status", "workspace_bytes",
            "host_arena_bytes", "layer_constants", "LayerConstants", "dyadic_multiplier",
            "dyadic_pair", "isoftmax_params_from_scale", "set_timeout_cycles", "strerror",
-           "int8_mma_peak_tops",
+           "int8_mma_peak_tops", "set_stall_injection",
            "IpError", "LibraryError", "EXPORTS"]

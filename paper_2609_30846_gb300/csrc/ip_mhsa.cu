@@ -17,6 +17,7 @@ namespace {
 constexpr size_t WS_HEADER = 256;          // error word and padding
 constexpr long long DEFAULT_TIMEOUT = 4000000000ll;   // ~2 s at 2 GHz
 long long g_timeout_cycles = DEFAULT_TIMEOUT;
+int g_stall_injection = 0;
 
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
@@ -160,6 +161,7 @@ int ip_relpos_mhsa_i8(const int8_t *q, const int8_t *k, const int8_t *v, const i
     prm.q_b = sm->q_b;
     prm.q_c = sm->q_c;
     prm.timeout_cycles = g_timeout_cycles;
+    prm.stall_injection = g_stall_injection;
     const dim3 grid1(ntiles, H, B);
     ipk::relpos_mhsa_fused_kernel<<<grid1, ipk::NTHREADS, smem, st>>>(tm_k, tm_v, tm_p, prm);
     if (cudaGetLastError() != cudaSuccess) return IP_ERR_CUDA;
@@ -316,6 +318,11 @@ long long ip_probe_int8_mma(int blocks, int iters, int *sink, ip_stream_t stream
 
 int ip_debug_set_timeout_cycles(long long cycles) {
     g_timeout_cycles = cycles >= 0 ? cycles : DEFAULT_TIMEOUT;
+    return IP_OK;
+}
+
+int ip_debug_set_stall_injection(int on) {
+    g_stall_injection = on ? 1 : 0;
     return IP_OK;
 }
 

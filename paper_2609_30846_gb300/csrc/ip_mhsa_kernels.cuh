@@ -82,11 +82,13 @@ struct FusedParams {
     int32_t sh_s, sh_o;       // total right shifts, 31 + s
     int32_t q_ln2, q_b, q_c;
     long long timeout_cycles; // bound of every barrier wait
+    int stall_injection;      // test hook: consumers first wait on a barrier nobody arrives on
 };
 
 constexpr int ERR_TIMEOUT_FULL = 1;
 constexpr int ERR_TIMEOUT_EMPTY = 2;
 constexpr int ERR_TIMEOUT_READY = 4;
+constexpr int ERR_TIMEOUT_INJECTED = 8;
 constexpr long long DRAIN_CYCLES = 2000000000ll;
 
 // ---------------------------------------------------------------- helpers --
@@ -128,6 +130,13 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, long lo
         if (clock64() - t0 > limit) return false;
     }
     return true;
+}
+
+// Warp-wide wait: every lane polls, then the warp agrees on the outcome, so
+// that a timeout takes all lanes down the same path.
+__device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, long long limit) {
+    const bool ok = mbar_wait(bar, parity, limit);
+    return __all_sync(0xffffffffu, ok) != 0;
 }
 
 __device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap *map, int c0, int c1,
@@ -562,6 +571,7 @@ __global__ void __launch_bounds__(NTHREADS, 2)
     auto full_bar = [&](int s) { return bar_base + 8u * s; };
     auto ready_bar = [&](int s) { return bar_base + 8u * (NSTAGE + s); };
     auto empty_bar = [&](int s) { return bar_base + 8u * (2 * NSTAGE + s); };
+    const uint32_t never_bar = bar_base + 8u * (3 * NSTAGE);   // test hook only
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < NSTAGE; ++s) {
@@ -569,6 +579,7 @@ __global__ void __launch_bounds__(NTHREADS, 2)
             mbar_init(ready_bar(s), 1);
             mbar_init(empty_bar(s), NCWARPS);
         }
+        mbar_init(never_bar, 1);
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
     }
@@ -621,7 +632,7 @@ __global__ void __launch_bounds__(NTHREADS, 2)
         }
         for (int it = 0; it < total; ++it) {
             const int s = it & 1;
-            if (!mbar_wait(full_bar(s), (it >> 1) & 1, prm.timeout_cycles)) {
+            if (!warp_wait(full_bar(s), (it >> 1) & 1, prm.timeout_cycles)) {
                 if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_FULL);
                 ok = false;
                 break;
@@ -635,7 +646,7 @@ __global__ void __launch_bounds__(NTHREADS, 2)
             __syncwarp();
             if (lane == 0) mbar_arrive(ready_bar(s));
             if (it + 2 < total) {
-                if (!mbar_wait(empty_bar(s), (it >> 1) & 1, prm.timeout_cycles)) {
+                if (!warp_wait(empty_bar(s), (it >> 1) & 1, prm.timeout_cycles)) {
                     if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_EMPTY);
                     ok = false;
                     break;
@@ -686,7 +697,11 @@ __global__ void __launch_bounds__(NTHREADS, 2)
     // groups with the epilogue of chunk c between them: the epilogue runs
     // while the pipe works through the band.
     int bacc[BAND_TILES][4];
-    if (!mbar_wait(ready_bar(0), 0, prm.timeout_cycles)) {
+    if (prm.stall_injection && !warp_wait(never_bar, 0, prm.timeout_cycles)) {
+        if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_INJECTED);
+        return;
+    }
+    if (!warp_wait(ready_bar(0), 0, prm.timeout_cycles)) {
         if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_READY);
         return;
     }
@@ -707,7 +722,7 @@ __global__ void __launch_bounds__(NTHREADS, 2)
         if (lane == 0) mbar_arrive(empty_bar(s));
         const uint32_t sdst = scores + c * CHUNK_SCORE_BYTES;
         if (c + 1 < nchunks) {
-            if (!mbar_wait(ready_bar(s ^ 1), ((c + 1) >> 1) & 1, prm.timeout_cycles)) {
+            if (!warp_wait(ready_bar(s ^ 1), ((c + 1) >> 1) & 1, prm.timeout_cycles)) {
                 if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_READY);
                 return;
             }
@@ -804,7 +819,7 @@ __global__ void __launch_bounds__(NTHREADS, 2)
     for (int c = 0; c < nchunks; ++c) {
         const int it = nchunks + c;
         const int s = it & 1;
-        if (!mbar_wait(ready_bar(s), (it >> 1) & 1, prm.timeout_cycles)) {
+        if (!warp_wait(ready_bar(s), (it >> 1) & 1, prm.timeout_cycles)) {
             if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_READY);
             return;
         }
