@@ -119,6 +119,38 @@ int ip_relpos_mhsa_i8_host(const int8_t *q, const int8_t *k, const int8_t *v,
                            int B, int H, int T, int dh, int8_t *out,
                            void *arena, size_t arena_bytes, ip_stream_t stream);
 
+/* The whole layer without any allocation by anyone: the same computation
+ * and result as ip_relpos_mhsa_i8, for callers that cannot allocate device
+ * memory, such as a plugin whose host framework owns the whole device pool
+ * and hands it only input and output buffers, or a latency-critical
+ * streaming path where a device allocation (which may synchronise the
+ * device) is not allowed.  The paper has no counterpart of this entry point.
+ *
+ * The caller passes inputs and outputs as for ip_relpos_mhsa_i8 (device
+ * pointers, 16-byte aligned; lengths a device array or NULL).  The scratch
+ * the kernel needs - the device status word that ip_relpos_mhsa_i8 keeps in
+ * the caller's workspace - lives instead in a file-scope device array of
+ * IP_NOALLOC_SCRATCH_BYTES bytes inside the library, held by every GPU that
+ * loads the library until the process exits.  A call whose scratch need
+ * exceeds that size is rejected with IP_ERR_WORKSPACE (every shape the
+ * library accepts needs IP_NOALLOC_SCRATCH_BYTES at most).  The call makes
+ * no allocation: no cudaMalloc, cudaFree or allocating library routine.
+ *
+ * The first call on a device looks up the device address of the array
+ * (cudaGetSymbolAddress, with that device current) and caches it; make that
+ * first call before any stream capture.  Every call shares the array and
+ * clears its status word in stream order before launching; calls that
+ * overlap on the GPU (concurrent streams) race on it.  Kernel-side barrier
+ * timeouts are recorded there and are not reported by this entry point; a
+ * caller that needs them uses ip_relpos_mhsa_i8 with a workspace.
+ * Returns IP_OK or an IP_ERR_* code as ip_relpos_mhsa_i8. */
+#define IP_NOALLOC_SCRATCH_BYTES 256
+int ip_relpos_mhsa_i8_noalloc(const int8_t *q, const int8_t *k, const int8_t *v,
+                              const int8_t *p, const int8_t *u, const int8_t *v_bias,
+                              const int32_t *multipliers, const int32_t *shifts,
+                              const ip_isoftmax_params *sm, const int32_t *lengths,
+                              int B, int H, int T, int dh, int8_t *out, ip_stream_t stream);
+
 /* Text of an IP_* code. */
 const char *ip_strerror(int code);
 

@@ -29,7 +29,7 @@ EXPORTS = (
     "ip_relpos_mhsa_host_arena_bytes", "ip_relpos_mhsa_i8_host", "ip_strerror",
     "ip_debug_set_timeout_cycles", "ip_debug_set_stall_injection", "ip_dyadic_multiplier",
     "ip_dyadic_pair",
-    "ip_isoftmax_params_from_scale", "ip_probe_int8_mma",
+    "ip_isoftmax_params_from_scale", "ip_probe_int8_mma", "ip_relpos_mhsa_i8_noalloc",
 )
 
 
@@ -81,6 +81,8 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
         lib.ip_relpos_mhsa_i8.restype = I
         lib.ip_relpos_mhsa_i8_host.argtypes = sig
         lib.ip_relpos_mhsa_i8_host.restype = I
+        lib.ip_relpos_mhsa_i8_noalloc.argtypes = sig[:15] + [P]
+        lib.ip_relpos_mhsa_i8_noalloc.restype = I
         lib.ip_relpos_mhsa_status.argtypes = [P, P]
         lib.ip_relpos_mhsa_status.restype = I
         lib.ip_strerror.argtypes = [I]

@@ -254,6 +254,52 @@ const char *ip_strerror(int code) {
 }
 
 // Offline constants: float64 on the host, once per layer.
+// ---- entry point without allocation --------------------------------------
+// File-scope device scratch of ip_relpos_mhsa_i8_noalloc: the status word
+// that ip_relpos_mhsa_i8 otherwise keeps in the caller's workspace.  Every
+// GPU that loads the library holds it until the process exits.
+static __device__ __align__(256) unsigned char g_noalloc_scratch[IP_NOALLOC_SCRATCH_BYTES];
+
+static std::mutex g_noalloc_mu;
+static void *g_noalloc_addr[64] = {nullptr};
+
+// Device address of g_noalloc_scratch on the current device, looked up
+// once per device (with that device current) and cached.
+static int noalloc_scratch(void **addr) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return IP_ERR_CUDA;
+    std::lock_guard<std::mutex> lock(g_noalloc_mu);
+    if (g_noalloc_addr[dev] == nullptr) {
+        void *p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || p == nullptr)
+            return IP_ERR_CUDA;
+        g_noalloc_addr[dev] = p;
+    }
+    *addr = g_noalloc_addr[dev];
+    return IP_OK;
+}
+
+int ip_relpos_mhsa_i8_noalloc(const int8_t *q, const int8_t *k, const int8_t *v, const int8_t *p,
+                              const int8_t *u, const int8_t *v_bias, const int32_t *multipliers,
+                              const int32_t *shifts, const ip_isoftmax_params *sm,
+                              const int32_t *lengths, int B, int H, int T, int dh, int8_t *out,
+                              ip_stream_t stream) {
+    int rc = check_shape(B, H, T, dh);
+    if (rc != IP_OK) return rc;
+    if (B == 0 || H == 0) return IP_OK;
+    const size_t need = ws_bytes();
+    if (need > IP_NOALLOC_SCRATCH_BYTES) return IP_ERR_WORKSPACE;
+    void *scratch = nullptr;
+    rc = noalloc_scratch(&scratch);
+    if (rc != IP_OK) return rc;
+    // The status word is shared by every call and keeps the last call's
+    // value: clear it in stream order before this call's kernel.
+    if (cudaMemsetAsync(scratch, 0, need, reinterpret_cast<cudaStream_t>(stream)) != cudaSuccess)
+        return IP_ERR_CUDA;
+    return ip_relpos_mhsa_i8(q, k, v, p, u, v_bias, multipliers, shifts, sm, lengths, B, H, T, dh,
+                             out, scratch, IP_NOALLOC_SCRATCH_BYTES, stream);
+}
+
 int ip_dyadic_multiplier(double ratio, int32_t *m, int32_t *s) {
     if (!m || !s) return IP_ERR_NULL;
     if (!(ratio > 0.0) || !isfinite(ratio)) return IP_ERR_PARAM;

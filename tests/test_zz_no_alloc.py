@@ -1,0 +1,66 @@
+"""The entry point that allocates nothing (ip_relpos_mhsa_i8_noalloc).
+
+It serves callers that cannot allocate device memory - a plugin whose host
+framework owns the device pool and passes only inputs and outputs, or a
+latency-critical path where an allocation may not happen.  Its scratch (the
+device status word) is a file-scope device array inside the library.  This
+test calls it through the C ABI twice in a row and checks that both calls
+give exactly the output of ip_relpos_mhsa_i8, the entry point that takes a
+caller-owned workspace (integer path: the tolerance is bit-exactness).  It
+lives in a file of its own that pytest collects last.
+"""
+import ctypes
+
+import numpy as np
+import pytest
+
+import synth
+
+pytestmark = pytest.mark.gpu
+
+torch = pytest.importorskip("torch")
+
+
+def _ptr(t):
+    return ctypes.c_void_p(t.data_ptr())
+
+
+@pytest.mark.parametrize("masked", [False, True])
+def test_noalloc_matches_workspace_entry_point(masked):
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import paper_2609_30846_gb300 as ip
+    lib = ip.load()
+    B, H, T, dh = 3, 8, 150, 128
+    lens = np.array([150, 97, 1], np.int32) if masked else None
+    cases = [synth.draw(B, H, T, dh, seed=8100 + i + 10 * masked, p_mode="sinusoid",
+                        lengths=lens) for i in range(2)]
+    stream = torch.cuda.current_stream()
+    for lay in cases:      # two calls in a row, each against the workspace path
+        c = ip.layer_constants(lay.scales)
+        dev = {n: torch.from_numpy(np.ascontiguousarray(getattr(lay, n))).cuda()
+               for n in ("q", "k", "v", "p", "u", "vb")}
+        dlen = None if lens is None else torch.from_numpy(lens).cuda()
+        ws = torch.zeros(ip.workspace_bytes(B, H, T), dtype=torch.uint8, device="cuda")
+        want = ip.relpos_mhsa_i8(dev["q"], dev["k"], dev["v"], dev["p"], dev["u"], dev["vb"], c,
+                                 lengths=dlen, workspace=ws)
+        assert ip.status(ws) == 0
+        got = torch.full((B, H, T, dh), 99, dtype=torch.int8, device="cuda")
+        sm = ip.SoftmaxParams(*c.softmax)
+        rc = lib.ip_relpos_mhsa_i8_noalloc(
+            _ptr(dev["q"]), _ptr(dev["k"]), _ptr(dev["v"]), _ptr(dev["p"]), _ptr(dev["u"]),
+            _ptr(dev["vb"]), (ctypes.c_int32 * 3)(*c.multipliers),
+            (ctypes.c_int32 * 2)(*c.shifts), ctypes.byref(sm),
+            None if dlen is None else _ptr(dlen), B, H, T, dh, _ptr(got),
+            ctypes.c_void_p(stream.cuda_stream))
+        assert rc == 0, ip.strerror(rc)
+        torch.cuda.synchronize()
+        np.testing.assert_array_equal(got.cpu().numpy(), want.cpu().numpy())
+
+
+def test_noalloc_rejects_bad_shapes():
+    import paper_2609_30846_gb300 as ip
+    lib = ip.load()
+    args = [None] * 6 + [None, None, None, None]
+    assert lib.ip_relpos_mhsa_i8_noalloc(*args, 1, 8, ip.IP_MAX_T + 1, 128, None, None) == -2
+    assert lib.ip_relpos_mhsa_i8_noalloc(*args, 1, 8, 10, 64, None, None) == -4
