@@ -149,6 +149,23 @@ def useful_ops(B, H, T, dh, layers):
     return 6 * dh * T * T * B * H * layers
 
 
+def slowest(dist, x: float, device=None) -> float:
+    """Max of a per-rank time over all ranks (x itself without a process
+    group): the job ends when its slowest replica ends."""
+    if dist is None:
+        return x
+    import torch
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_tops(ops_per_rank: float, world: int, seconds: float) -> float:
+    """Whole-job throughput: every replica does the same work (weak scaling),
+    all of it counted, over the slowest rank's time."""
+    return ops_per_rank * world / seconds / 1e12
+
+
 def traffic_per_launch():
     """DRAM bytes per fused-kernel launch from the committed ncu summary,
     if it was taken on the current kernel source (else None)."""
@@ -317,13 +334,10 @@ def run_ours(args):
     if ip.status(ws, stream) != 0:
         raise SystemExit("kernel reported a barrier timeout in the timed region")
 
-    if dist:
-        tt = torch.tensor([total_ms], device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        total_ms = float(tt.item())
+    total_ms = slowest(dist, total_ms, dev)
 
     ops_step = useful_ops(B, H, T, dh, NL)
-    value = ops_step * args.steps * world / (total_ms * 1e-3) / 1e12
+    value = job_tops(ops_step * args.steps, world, total_ms * 1e-3)
     ms_step = total_ms / args.steps
     ops_layer = useful_ops(B, H, T, dh, 1)
     avg_layer_ms = statistics.mean(layer_ms)
@@ -349,14 +363,10 @@ def run_ours(args):
         for _ in range(args.e2e_steps):
             e2e_step()
         torch.cuda.synchronize(dev)
-        e2e_s = time.perf_counter() - t
-        if dist:
-            tt = torch.tensor([e2e_s], device=dev)
-            dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-            e2e_s = float(tt.item())
+        e2e_s = slowest(dist, time.perf_counter() - t, dev)
         h2d = sum(int(h_[k].numel()) for h_ in hl for k in ("q", "k", "v", "p", "u", "vb"))
         d2h = sum(int(h_["out"].numel()) for h_ in hl)
-        e2e = {"value": ops_step * args.e2e_steps * world / e2e_s / 1e12, "unit": "TOPS",
+        e2e = {"value": job_tops(ops_step * args.e2e_steps, world, e2e_s), "unit": "TOPS",
                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                "ms_per_step": e2e_s / args.e2e_steps * 1e3, "steps": args.e2e_steps}
 
