@@ -169,6 +169,15 @@ int ip_debug_set_timeout_cycles(long long cycles);
  * the GPU.  Off by default. */
 int ip_debug_set_stall_injection(int on);
 
+/* Test hook: how the kernels launched afterwards by this process do the
+ * tiles of 64 query rows.  Negative (the default): as planned, i.e. when the
+ * last wave of CTAs on the GPU would be at most half full, its tiles are
+ * done as two halves of 32 rows whose warps split the keys of every chunk
+ * and combine their row maxima, exponential sums and attn.V partial sums.
+ * 0: no tile is split.  Positive: every tile is split (when the grid allows
+ * it).  The outputs are the same bit for bit in every mode. */
+int ip_debug_set_split_mode(int mode);
+
 /* Diagnostic: enqueues a throughput probe of the integer warp MMA
  * (mma.sync m16n8k32 s8 x s8 -> s32, eight independent accumulators per
  * warp, `iters` rounds) on `stream`; sink is a device int array of

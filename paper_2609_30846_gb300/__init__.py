@@ -30,6 +30,7 @@ EXPORTS = (
     "ip_debug_set_timeout_cycles", "ip_debug_set_stall_injection", "ip_dyadic_multiplier",
     "ip_dyadic_pair",
     "ip_isoftmax_params_from_scale", "ip_probe_int8_mma", "ip_relpos_mhsa_i8_noalloc",
+    "ip_debug_set_split_mode",
 )
 
 
@@ -91,6 +92,8 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
         lib.ip_debug_set_timeout_cycles.restype = I
         lib.ip_debug_set_stall_injection.argtypes = [I]
         lib.ip_debug_set_stall_injection.restype = I
+        lib.ip_debug_set_split_mode.argtypes = [I]
+        lib.ip_debug_set_split_mode.restype = I
         lib.ip_dyadic_multiplier.argtypes = [ctypes.c_double, i32p, i32p]
         lib.ip_dyadic_multiplier.restype = I
         lib.ip_dyadic_pair.argtypes = [ctypes.c_double, ctypes.c_double, i32p, i32p, i32p]
@@ -175,6 +178,12 @@ def set_timeout_cycles(cycles: int) -> None:
 def set_stall_injection(on: bool) -> None:
     """Test hook: make the kernels wait on a barrier nothing arrives on."""
     load().ip_debug_set_stall_injection(1 if on else 0)
+
+
+def set_split_mode(mode: int) -> None:
+    """Test hook: -1 planned tail split (default), 0 never split, 1 split
+    every 64-row tile into two key-split halves."""
+    load().ip_debug_set_split_mode(int(mode))
 
 
 def _arr(vals, ctype):

@@ -18,6 +18,7 @@ constexpr size_t WS_HEADER = 256;          // error word and padding
 constexpr long long DEFAULT_TIMEOUT = 4000000000ll;   // ~2 s at 2 GHz
 long long g_timeout_cycles = DEFAULT_TIMEOUT;
 int g_stall_injection = 0;
+int g_split_mode = -1;   // -1 planned, 0 never, 1 every tile (test hook)
 
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
@@ -91,6 +92,61 @@ int ensure_smem(int bytes) {
     return IP_OK;
 }
 
+// CTAs of the fused kernel resident on the whole GPU at once (its SMs x the
+// CTAs an SM holds at this shared-memory size), cached for the last query.
+std::mutex g_occ_mu;
+int g_occ_dev = -1, g_occ_smem = -1, g_occ_slots = 0;
+
+int resident_ctas(int smem) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+    std::lock_guard<std::mutex> lock(g_occ_mu);
+    if (dev == g_occ_dev && smem == g_occ_smem) return g_occ_slots;
+    int nsm = 0, per_sm = 0;
+    if (cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
+        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, ipk::relpos_mhsa_fused_kernel,
+                                                      ipk::NTHREADS, smem) != cudaSuccess)
+        return 0;
+    g_occ_dev = dev;
+    g_occ_smem = smem;
+    g_occ_slots = nsm * per_sm;
+    return g_occ_slots;
+}
+
+// Tail split.  The N tiles run in waves of `slots` CTAs; when the last wave
+// is at most half full (r = N mod slots tiles, 2 r <= slots), its r tiles
+// are done as 2 r halves of 32 rows whose warps split the keys of every
+// chunk, so the last wave takes about half as long.  The halves live in
+// grid slices after the B batch slices, which the block scheduler
+// dispatches last.
+struct SplitPlan {
+    int nsplit = 0, extra = 0, b0 = 0, h0 = 0, tile0 = 0;
+    long long first = 0;
+};
+
+SplitPlan plan_split(int B, int H, int ntiles, int slots) {
+    SplitPlan sp;
+    const long long N = static_cast<long long>(B) * H * ntiles;
+    long long ns = 0;
+    if (g_split_mode == 1) {
+        ns = N;
+    } else if (g_split_mode < 0 && slots > 0) {
+        const long long r = N % slots;
+        if (r > 0 && 2 * r <= slots) ns = r;
+    }
+    const long long per_slice = static_cast<long long>(ntiles) * H;
+    const long long extra = (2 * ns + per_slice - 1) / per_slice;
+    if (ns == 0 || B + extra > IP_MAX_B) return sp;
+    sp.nsplit = static_cast<int>(ns);
+    sp.extra = static_cast<int>(extra);
+    sp.first = N - ns;
+    sp.tile0 = static_cast<int>(sp.first % ntiles);
+    const long long bh = sp.first / ntiles;
+    sp.h0 = static_cast<int>(bh % H);
+    sp.b0 = static_cast<int>(bh / H);
+    return sp;
+}
+
 }  // namespace
 
 extern "C" {
@@ -162,7 +218,13 @@ int ip_relpos_mhsa_i8(const int8_t *q, const int8_t *k, const int8_t *v, const i
     prm.q_c = sm->q_c;
     prm.timeout_cycles = g_timeout_cycles;
     prm.stall_injection = g_stall_injection;
-    const dim3 grid1(ntiles, H, B);
+    const SplitPlan sp = plan_split(B, H, ntiles, resident_ctas(smem));
+    prm.nsplit = sp.nsplit;
+    prm.split_b0 = sp.b0;
+    prm.split_h0 = sp.h0;
+    prm.split_tile0 = sp.tile0;
+    prm.first_split = sp.first;
+    const dim3 grid1(ntiles, H, B + sp.extra);
     ipk::relpos_mhsa_fused_kernel<<<grid1, ipk::NTHREADS, smem, st>>>(tm_k, tm_v, tm_p, prm);
     if (cudaGetLastError() != cudaSuccess) return IP_ERR_CUDA;
     return IP_OK;
@@ -364,6 +426,11 @@ long long ip_probe_int8_mma(int blocks, int iters, int *sink, ip_stream_t stream
 
 int ip_debug_set_timeout_cycles(long long cycles) {
     g_timeout_cycles = cycles >= 0 ? cycles : DEFAULT_TIMEOUT;
+    return IP_OK;
+}
+
+int ip_debug_set_split_mode(int mode) {
+    g_split_mode = mode < 0 ? -1 : (mode > 0 ? 1 : 0);
     return IP_OK;
 }
 

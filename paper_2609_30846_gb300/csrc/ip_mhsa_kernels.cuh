@@ -66,7 +66,7 @@ __host__ __device__ inline SmemLayout smem_layout(int nchunk_max) {
     L.remap = L.scores + NCWARPS * nchunk_max * CHUNK_SCORE_BYTES;
     L.lut = L.remap + NCWARPS * REMAP_BYTES;
     L.bars = L.lut + LUT_ENTRIES * LUT_COPIES * 4;
-    L.total = L.bars + 64;
+    L.total = L.bars + 128;
     return L;
 }
 
@@ -83,6 +83,11 @@ struct FusedParams {
     int32_t q_ln2, q_b, q_c;
     long long timeout_cycles; // bound of every barrier wait
     int stall_injection;      // test hook: consumers first wait on a barrier nobody arrives on
+    // Tail split: the last nsplit tiles of the (b, h, tile) order, from
+    // tile split_tile0 of (split_b0, split_h0) on, are done as two halves of
+    // 32 rows each by the CTAs of the grid slices z >= B (dispatched last).
+    int nsplit, split_b0, split_h0, split_tile0;
+    long long first_split;    // linear index of the first split tile
 };
 
 constexpr int ERR_TIMEOUT_FULL = 1;
@@ -464,6 +469,111 @@ __device__ __forceinline__ void prob_operand(const uint32_t (&pw)[4], uint32_t (
     af[3] = __byte_perm(pw[2], pw[3], 0x7632);
 }
 
+// ------------------------------------------------------- split-tile parts --
+// In a split tile the two warps of a row strip take the key halves
+// [32 hk, 32 hk + 32) of every chunk.  Exchange area in each warp's remap
+// buffer (after its score pass): row maxima, exponential sums, and the
+// attn.V partial sums that the partner warp finishes.
+constexpr int XMAX_OFF = 0;      // 32 lanes x 2 int32
+constexpr int XSUM_OFF = 256;    // 32 lanes x 2 uint64
+constexpr int XO_OFF = 768;      // 32 words x 32 lanes
+static_assert(XO_OFF + 32 * 32 * 4 <= REMAP_BYTES, "exchange area");
+
+// Band n-tiles nt0 .. nt0 + 5 and content n-tiles nt0 .. nt0 + 3 of one
+// key half (nt0 = 4 hk): the band columns of keys 32 hk .. 32 hk + 31 of 16
+// rows are 32 hk .. 32 hk + 46.
+__device__ __forceinline__ void half_chunk_mma(int (&bacc)[6][4], int (&cacc)[4][4],
+                                               const uint32_t (&qa)[4][4], uint32_t ptile,
+                                               uint32_t pv, uint32_t ktile, uint32_t ku, int nt0,
+                                               int lane) {
+    const int t4 = lane & 3;
+#pragma unroll
+    for (int i = 0; i < 6; ++i) {
+        const int2 v = lds64(pv + ((nt0 + i) * 8 + 2 * t4) * 4);
+        bacc[i][0] = v.x;
+        bacc[i][1] = v.y;
+        bacc[i][2] = v.x;
+        bacc[i][3] = v.y;
+    }
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const int2 v = lds64(ku + ((nt0 + i) * 8 + 2 * t4) * 4);
+        cacc[i][0] = v.x;
+        cacc[i][1] = v.y;
+        cacc[i][2] = v.x;
+        cacc[i][3] = v.y;
+    }
+    const int lm_row = lane & 7, lm_mat = lane >> 3;
+#pragma unroll
+    for (int kh = 0; kh < 2; ++kh) {
+        uint32_t b[6][4], kb[4][4];
+#pragma unroll
+        for (int i = 0; i < 6; ++i)
+            ldsm_x4(ptile + swz((nt0 + i) * 8 + lm_row, kh * 4 + lm_mat), b[i][0], b[i][1],
+                    b[i][2], b[i][3]);
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+            ldsm_x4(ktile + swz((nt0 + i) * 8 + lm_row, kh * 4 + lm_mat), kb[i][0], kb[i][1],
+                    kb[i][2], kb[i][3]);
+#pragma unroll
+        for (int i = 0; i < 6; ++i) mma_s8s8(bacc[i], qa[2 * kh], b[i][0], b[i][1]);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) mma_s8s8(cacc[i], qa[2 * kh], kb[i][0], kb[i][1]);
+#pragma unroll
+        for (int i = 0; i < 6; ++i) mma_s8s8(bacc[i], qa[2 * kh + 1], b[i][2], b[i][3]);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) mma_s8s8(cacc[i], qa[2 * kh + 1], kb[i][2], kb[i][3]);
+    }
+}
+
+// Sends the partial sums of the partner's output n-tiles (8 (1 - HK) ..
+// + 7) to this warp's exchange area.
+template <int HK>
+__device__ __forceinline__ void send_partial(const int (&oacc)[16][4], uint32_t xo, int lane) {
+#pragma unroll
+    for (int i = 0; i < 8; ++i)
+#pragma unroll
+        for (int e = 0; e < 4; ++e)
+            sts32(xo + ((i * 4 + e) * 32 + lane) * 4, static_cast<uint32_t>(oacc[8 * (1 - HK) + i][e]));
+}
+
+// Adds the partner's partial sums of this warp's n-tiles 8 HK .. 8 HK + 7,
+// requantises them (Eq. 7) and stores two 8-byte runs per row: d =
+// nt + 32 t + 16 hh for nt in 8 HK .. 8 HK + 7.
+template <int HK>
+__device__ __forceinline__ void finish_half(int (&oacc)[16][4], uint32_t pxo, int lane, int wrow0,
+                                            int T, int len, size_t bh, long long m_o,
+                                            long long half_o, int sh_o, int8_t *out) {
+    const int g = lane >> 2, t4 = lane & 3;
+#pragma unroll
+    for (int i = 0; i < 8; ++i)
+#pragma unroll
+        for (int e = 0; e < 4; ++e)
+            oacc[8 * HK + i][e] += static_cast<int>(lds32(pxo + ((i * 4 + e) * 32 + lane) * 4));
+#pragma unroll
+    for (int rr = 0; rr < 2; ++rr) {
+        const int row = wrow0 + g + 8 * rr;
+        if (row >= T) continue;
+        int8_t *dst = out + (bh * T + row) * DH + 32 * t4 + 8 * HK;
+#pragma unroll
+        for (int hh = 0; hh < 2; ++hh) {
+            uint32_t wv[2];
+#pragma unroll
+            for (int wq = 0; wq < 2; ++wq) {
+                uint32_t w = 0;
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const long long x = m_o * oacc[8 * HK + 4 * wq + e][2 * rr + hh] + half_o;
+                    const int o = row < len ? clamp127(x >> sh_o) : 0;
+                    w |= (static_cast<uint32_t>(o) & 0xffu) << (8 * e);
+                }
+                wv[wq] = w;
+            }
+            *reinterpret_cast<uint2 *>(dst + 16 * hh) = make_uint2(wv[0], wv[1]);
+        }
+    }
+}
+
 // ---------------------------------------------------------- producer parts --
 
 // K u for the chunk's 64 keys and P v for the 128 staged band rows; lane l
@@ -541,11 +651,36 @@ __global__ void __launch_bounds__(NTHREADS, 2)
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
     const SmemLayout L = smem_layout(prm.nchunk_max);
 
-    // Grid (ntiles, H, B): no run-time division anywhere in the kernel.
+    // Grid (ntiles, H, B + extra): slices z < B hold one CTA per tile, the
+    // slices after them the halves of the split tiles.  No run-time
+    // division anywhere in the kernel.
     const int T = prm.T;
-    const int tile = blockIdx.x;
-    const int h = blockIdx.y;
-    const int b = blockIdx.z;
+    const int ntiles = static_cast<int>(gridDim.x);
+    int tile = blockIdx.x;
+    int h = blockIdx.y;
+    int b = blockIdx.z;
+    int part = -1;                 // -1: whole tile; 0, 1: half of a split tile
+    if (b >= prm.B) {
+        const long long t = blockIdx.x + static_cast<long long>(ntiles) *
+                                             (blockIdx.y + static_cast<long long>(prm.H) * (b - prm.B));
+        if (t >= 2ll * prm.nsplit) return;
+        part = static_cast<int>(t & 1);
+        tile = prm.split_tile0 + static_cast<int>(t >> 1);
+        h = prm.split_h0;
+        b = prm.split_b0;
+        while (tile >= ntiles) {   // at most nsplit / ntiles + 1 steps
+            tile -= ntiles;
+            ++h;
+        }
+        while (h >= prm.H) {
+            h -= prm.H;
+            ++b;
+        }
+    } else if (prm.nsplit > 0) {
+        const long long lin = blockIdx.x + static_cast<long long>(ntiles) *
+                                               (blockIdx.y + static_cast<long long>(prm.H) * b);
+        if (lin >= prm.first_split) return;   // done by the two halves
+    }
     const int bh = b * prm.H + h;
     const int i0 = tile * MROWS;
     int len = T;
@@ -556,12 +691,17 @@ __global__ void __launch_bounds__(NTHREADS, 2)
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
 
-    if (i0 >= len) {
-        // Every row of this tile is padding: write zeros.
-        const int rows = (T - i0) < MROWS ? (T - i0) : MROWS;
-        int4 *dst = reinterpret_cast<int4 *>(prm.out + (static_cast<size_t>(bh) * T + i0) * DH);
-        for (int c = threadIdx.x; c < rows * (DH / 16); c += NTHREADS) dst[c] = make_int4(0, 0, 0, 0);
-        return;
+    {
+        const int r0 = part < 0 ? i0 : i0 + 32 * part;
+        const int nrows = part < 0 ? MROWS : 32;
+        if (r0 >= len) {
+            // Every row of this tile (half) is padding: write zeros.
+            const int rows = (T - r0) < nrows ? (T - r0) : nrows;
+            int4 *dst = reinterpret_cast<int4 *>(prm.out + (static_cast<size_t>(bh) * T + r0) * DH);
+            for (int c = threadIdx.x; c < rows * (DH / 16); c += NTHREADS)
+                dst[c] = make_int4(0, 0, 0, 0);
+            return;
+        }
     }
     const int nchunks = (len + NK - 1) / NK;
     const int total = 2 * nchunks;   // uses of the stage ring: pass-1 chunks, then pass-3 chunks
@@ -572,6 +712,7 @@ __global__ void __launch_bounds__(NTHREADS, 2)
     auto ready_bar = [&](int s) { return bar_base + 8u * (NSTAGE + s); };
     auto empty_bar = [&](int s) { return bar_base + 8u * (2 * NSTAGE + s); };
     const uint32_t never_bar = bar_base + 8u * (3 * NSTAGE);   // test hook only
+    auto pair_bar = [&](int strip2) { return bar_base + 8u * (3 * NSTAGE + 1 + strip2); };
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < NSTAGE; ++s) {
@@ -580,6 +721,8 @@ __global__ void __launch_bounds__(NTHREADS, 2)
             mbar_init(empty_bar(s), NCWARPS);
         }
         mbar_init(never_bar, 1);
+        mbar_init(pair_bar(0), 2);
+        mbar_init(pair_bar(1), 2);
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
     }
@@ -667,7 +810,10 @@ __global__ void __launch_bounds__(NTHREADS, 2)
     // ------------------------------------------------------------ consumers
     const int g = lane >> 2;       // row group of the MMA fragments
     const int t4 = lane & 3;       // thread in group
-    const int wrow0 = i0 + warp * 16;
+    // Row strip of 16 rows: one per warp in a whole tile; in a split tile
+    // strips 2 part, 2 part + 1, each shared by warps 2s', 2s' + 1.
+    const int strip = part < 0 ? warp : 2 * part + (warp >> 1);
+    const int wrow0 = i0 + strip * 16;
     const int8_t *qbase = prm.q + static_cast<size_t>(bh) * T * DH;
 
     // Q fragments (A operand) for the four 32-wide k steps, rows >= T zero.
@@ -689,18 +835,176 @@ __global__ void __launch_bounds__(NTHREADS, 2)
     const long long m_c = prm.m_c, m_p = prm.m_p;
     const long long half_s = 1ll << (prm.sh_s - 1);
     const int s_s = prm.sh_s - 31;
-    const int band_row0 = 48 - 16 * warp;      // this warp's first row in the staged band
+    const int band_row0 = 48 - 16 * strip;     // this warp's first row in the staged band
     int mx0 = -128, mx1 = -128;                // running maxima of rows g and g + 8
+    if (prm.stall_injection && !warp_wait(never_bar, 0, prm.timeout_cycles)) {
+        if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_INJECTED);
+        return;
+    }
+
+    if (part >= 0) {
+        // ---------------------------------------------- split tile (tail)
+        const int hk = warp & 1;                   // key half of every chunk
+        const int nt0 = 4 * hk;
+        const uint32_t pair = pair_bar(warp >> 1);
+        const uint32_t xown = remap;
+        const uint32_t xpart = smem_u32(smem + L.remap) + (warp ^ 1) * REMAP_BYTES;
+        const uint32_t lut_g = lut + 4 * g;
+
+        // pass 1: scores of this warp's key half of every chunk
+        for (int c = 0; c < nchunks; ++c) {
+            const int s = c & 1;
+            if (!warp_wait(ready_bar(s), (c >> 1) & 1, prm.timeout_cycles)) {
+                if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_READY);
+                return;
+            }
+            int hb[6][4], hc[4][4];
+            half_chunk_mma(hb, hc, qa, stage_addr(s) + K_TILE_BYTES + band_row0 * 128,
+                           stage_addr(s) + PV_OFF + band_row0 * 4, stage_addr(s),
+                           stage_addr(s) + KU_OFF, nt0, lane);
+            __syncwarp();
+            if (lane == 0) mbar_arrive(empty_bar(s));
+#pragma unroll
+            for (int i = 0; i < 6; ++i) {
+                sts64(remap + (g * REMAP_STRIDE + (nt0 + i) * 8 + 2 * t4) * 4, hb[i][0], hb[i][1]);
+                sts64(remap + ((g + 8) * REMAP_STRIDE + (nt0 + i) * 8 + 2 * t4) * 4, hb[i][2],
+                      hb[i][3]);
+            }
+            __syncwarp();
+            const int kvalid = len - c * NK;
+            uint32_t pk[4];
+            if (kvalid < NK) {
+#pragma unroll
+                for (int i = 0; i < 4; ++i)
+                    pk[i] = score_tile<true>(hc[i], nt0 + i, remap, lane, m_c, m_p, half_s, s_s,
+                                             kvalid, mx0, mx1);
+            } else {
+#pragma unroll
+                for (int i = 0; i < 4; ++i)
+                    pk[i] = score_tile<false>(hc[i], nt0 + i, remap, lane, m_c, m_p, half_s, s_s,
+                                              kvalid, mx0, mx1);
+            }
+            sts128(scores + c * CHUNK_SCORE_BYTES + hk * 512 + lane * 16, pk[0], pk[1], pk[2],
+                   pk[3]);
+        }
+        mx0 = max(mx0, __shfl_xor_sync(0xffffffffu, mx0, 1));
+        mx0 = max(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
+        mx1 = max(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
+        mx1 = max(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
+        __syncwarp();   // the remap reads of the last chunk are done
+        sts64(xown + XMAX_OFF + lane * 8, mx0, mx1);
+        __syncwarp();
+        if (lane == 0) mbar_arrive(pair);
+        if (!warp_wait(pair, 0, prm.timeout_cycles)) {
+            if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_READY);
+            return;
+        }
+        {
+            const int2 pm = lds64(xpart + XMAX_OFF + lane * 8);
+            mx0 = max(mx0, pm.x);
+            mx1 = max(mx1, pm.y);
+        }
+
+        // pass 2: exponential sums of the key half, then of the whole row
+        unsigned long long sum0 = 0, sum1 = 0;
+        for (int c = 0; c < nchunks; ++c) {
+            const int kvalid = len - c * NK;
+            const uint4 sv = lds128(scores + c * CHUNK_SCORE_BYTES + hk * 512 + lane * 16);
+            if (kvalid < NK)
+                exp_sums<true>(sv, lut_g, mx0, mx1, t4, 32 * hk, kvalid, sum0, sum1);
+            else
+                exp_sums<false>(sv, lut_g, mx0, mx1, t4, 32 * hk, kvalid, sum0, sum1);
+        }
+        sum0 += __shfl_xor_sync(0xffffffffu, sum0, 1);
+        sum0 += __shfl_xor_sync(0xffffffffu, sum0, 2);
+        sum1 += __shfl_xor_sync(0xffffffffu, sum1, 1);
+        sum1 += __shfl_xor_sync(0xffffffffu, sum1, 2);
+        sts64(xown + XSUM_OFF + lane * 16, static_cast<int>(sum0), static_cast<int>(sum0 >> 32));
+        sts64(xown + XSUM_OFF + lane * 16 + 8, static_cast<int>(sum1), static_cast<int>(sum1 >> 32));
+        __syncwarp();
+        if (lane == 0) mbar_arrive(pair);
+        if (!warp_wait(pair, 1, prm.timeout_cycles)) {
+            if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_READY);
+            return;
+        }
+        {
+            const int2 a = lds64(xpart + XSUM_OFF + lane * 16);
+            const int2 bq = lds64(xpart + XSUM_OFF + lane * 16 + 8);
+            sum0 += (static_cast<unsigned long long>(static_cast<uint32_t>(a.y)) << 32) |
+                    static_cast<uint32_t>(a.x);
+            sum1 += (static_cast<unsigned long long>(static_cast<uint32_t>(bq.y)) << 32) |
+                    static_cast<uint32_t>(bq.x);
+        }
+        const uint32_t f0 = div_2pow32(sum0);
+        const uint32_t f1 = div_2pow32(sum1);
+
+        // pass 3: probabilities of the key half x V (k step hk of every chunk)
+        int oacc[16][4];
+#pragma unroll
+        for (int nt = 0; nt < 16; ++nt) oacc[nt][0] = oacc[nt][1] = oacc[nt][2] = oacc[nt][3] = 0;
+        const int kvalid_last = len - (nchunks - 1) * NK;
+        const int lm_row = lane & 7, lm_mat = lane >> 3;
+        for (int c = 0; c < nchunks; ++c) {
+            const uint4 sv = lds128(scores + c * CHUNK_SCORE_BYTES + hk * 512 + lane * 16);
+            uint32_t pw[4] = {prob_word(sv.x, lut_g, mx0, mx1, f0, f1),
+                              prob_word(sv.y, lut_g, mx0, mx1, f0, f1),
+                              prob_word(sv.z, lut_g, mx0, mx1, f0, f1),
+                              prob_word(sv.w, lut_g, mx0, mx1, f0, f1)};
+            if (c == nchunks - 1 && kvalid_last < NK) {
+#pragma unroll
+                for (int q = 0; q < 4; ++q) pw[q] &= key_mask(32 * hk, q, t4, kvalid_last);
+            }
+            uint32_t af[4];
+            prob_operand(pw, af);
+            const int it = nchunks + c;
+            const int s = it & 1;
+            if (!warp_wait(ready_bar(s), (it >> 1) & 1, prm.timeout_cycles)) {
+                if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_READY);
+                return;
+            }
+            const uint32_t vt = stage_addr(s) + K_TILE_BYTES;
+#pragma unroll
+            for (int grp = 0; grp < 4; ++grp) {
+                uint32_t bv[2][4];
+#pragma unroll
+                for (int i = 0; i < 2; ++i)
+                    ldsm_x4(vt + vt_row(hk, lm_mat & 1, 4 * grp + 2 * i + (lm_mat >> 1), lm_row),
+                            bv[i][0], bv[i][1], bv[i][2], bv[i][3]);
+#pragma unroll
+                for (int i = 0; i < 2; ++i) {
+                    mma_u8s8(oacc[4 * grp + 2 * i], af, bv[i][0], bv[i][1]);
+                    mma_u8s8(oacc[4 * grp + 2 * i + 1], af, bv[i][2], bv[i][3]);
+                }
+            }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(empty_bar(s));
+        }
+
+        // the partner finishes the other half of the output columns
+        if (hk == 0) send_partial<0>(oacc, xown + XO_OFF, lane);
+        else send_partial<1>(oacc, xown + XO_OFF, lane);
+        __syncwarp();
+        if (lane == 0) mbar_arrive(pair);
+        if (!warp_wait(pair, 0, prm.timeout_cycles)) {
+            if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_READY);
+            return;
+        }
+        const long long m_o = prm.m_o;
+        const long long half_o = 1ll << (prm.sh_o - 1);
+        if (hk == 0)
+            finish_half<0>(oacc, xpart + XO_OFF, lane, wrow0, T, len, bh, m_o, half_o, prm.sh_o,
+                           prm.out);
+        else
+            finish_half<1>(oacc, xpart + XO_OFF, lane, wrow0, T, len, bh, m_o, half_o, prm.sh_o,
+                           prm.out);
+        return;
+    }
 
     // ---- pass 1: scores.  A warp that issues an integer MMA waits until the
     // tensor pipe accepts it, so the band MMAs of chunk c+1 are issued in
     // groups with the epilogue of chunk c between them: the epilogue runs
     // while the pipe works through the band.
     int bacc[BAND_TILES][4];
-    if (prm.stall_injection && !warp_wait(never_bar, 0, prm.timeout_cycles)) {
-        if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_INJECTED);
-        return;
-    }
     if (!warp_wait(ready_bar(0), 0, prm.timeout_cycles)) {
         if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_READY);
         return;

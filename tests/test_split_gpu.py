@@ -1,0 +1,83 @@
+"""Parity of the tail split with the oracle.
+
+The kernel may do a 64-row tile as two halves of 32 rows whose warp pairs
+split the keys of every chunk and combine their row maxima, exponential
+sums and attn.V partial sums.  Integer arithmetic makes the combination
+exact, so every mode must match the oracle bit for bit: here each case runs
+with no tile split and with every tile split (the planned mode, which
+splits only the last wave, runs in the other parity tests).
+"""
+import numpy as np
+import pytest
+
+import synth
+from test_parity_gpu import assert_same, oracle_out, run_gpu
+
+pytestmark = pytest.mark.gpu
+
+torch = pytest.importorskip("torch")
+
+
+@pytest.fixture(scope="module")
+def ip():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import paper_2609_30846_gb300 as mod
+    mod.load()
+    yield mod
+    mod.set_split_mode(-1)
+
+
+@pytest.fixture(scope="module")
+def orc():
+    import oracle
+    oracle.build()
+    return oracle
+
+
+@pytest.fixture(params=[0, 1], ids=["whole", "split"])
+def mode(request, ip):
+    ip.set_split_mode(request.param)
+    yield request.param
+    ip.set_split_mode(-1)
+
+
+@pytest.mark.parametrize("T", [1, 2, 31, 32, 33, 63, 64, 65, 96, 97, 129, 200])
+def test_ragged_T(ip, orc, mode, T):
+    lay = synth.draw(2, 3, T, 128, seed=900 + T, p_mode="sinusoid")
+    c = ip.layer_constants(lay.scales)
+    assert_same(run_gpu(ip, lay, c), oracle_out(orc, lay, c))
+
+
+@pytest.mark.parametrize("seed", range(3))
+def test_masks_with_short_rows(ip, orc, mode, seed):
+    # lengths that end inside the first and the second key half of a chunk,
+    # on a half boundary, and rows that are all padding in one half
+    rng = np.random.default_rng(seed)
+    T = 150
+    lengths = np.array([1, 20, 32, 33, 64, 95, 96, 97, 150, int(rng.integers(1, T + 1))],
+                       np.int32)
+    lay = synth.draw(len(lengths), 2, T, 128, seed=930 + seed, p_mode="sinusoid",
+                     masked=True, lengths=lengths)
+    c = ip.layer_constants(lay.scales)
+    assert_same(run_gpu(ip, lay, c, lay.lengths), oracle_out(orc, lay, c, lay.lengths))
+
+
+@pytest.mark.parametrize("w", [0, 1])
+def test_workloads(ip, orc, mode, w):
+    lay = synth.layer(w, 1)
+    c = ip.layer_constants(lay.scales)
+    assert_same(run_gpu(ip, lay, c, lay.lengths), oracle_out(orc, lay, c, lay.lengths))
+
+
+def test_modes_agree_on_the_encoder_layer(ip):
+    # one full encoder layer (B=32, T=375) in all three modes
+    lay = synth.layer(3, 7)
+    c = ip.layer_constants(lay.scales)
+    outs = []
+    for m in (-1, 0, 1):
+        ip.set_split_mode(m)
+        outs.append(run_gpu(ip, lay, c))
+    ip.set_split_mode(-1)
+    assert_same(outs[1], outs[0])
+    assert_same(outs[2], outs[0])
