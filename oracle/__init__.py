@@ -22,10 +22,11 @@ import threading
 import numpy as np
 
 from .consts import (IBERT_A, IBERT_B, IBERT_C, LayerConstants, dyadic,
-                     dyadic_pair, isoftmax_params, layer_constants)
+                     dyadic_pair, isoftmax_params, layer_constants, linear_constants)
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
-_SRC = os.path.join(_HERE, "ipo_mhsa.c")
+_SRCS = [os.path.join(_HERE, f) for f in ("ipo_mhsa.c", "ipo_linear.c")]
+_HDRS = [os.path.join(_HERE, f) for f in ("ipo_mhsa.h", "ipo_linear.h")]
 _LIB = os.path.join(_HERE, "libipo_mhsa.so")
 _lock = threading.Lock()
 _lib = None
@@ -34,11 +35,11 @@ _lib = None
 def build(force: bool = False) -> str:
     """Compile the C oracle into ``oracle/libipo_mhsa.so`` (gcc, OpenMP)."""
     if not force and os.path.exists(_LIB) and os.path.getmtime(_LIB) >= max(
-            os.path.getmtime(_SRC), os.path.getmtime(os.path.join(_HERE, "ipo_mhsa.h"))):
+            os.path.getmtime(f) for f in _SRCS + _HDRS):
         return _LIB
     tmp = _LIB + f".tmp{os.getpid()}"
     cmd = ["gcc", "-O2", "-std=c11", "-fPIC", "-shared", "-fopenmp", "-Wall",
-           "-Wextra", "-o", tmp, _SRC]
+           "-Wextra", "-o", tmp] + _SRCS
     subprocess.run(cmd, check=True, cwd=_HERE)
     os.replace(tmp, _LIB)
     return _LIB
@@ -64,6 +65,9 @@ def _load():
             lib.ipo_iexp.restype = ctypes.c_int64
             lib.ipo_isoftmax_u8.argtypes = [P, P, ctypes.c_int, ctypes.c_int, P, P]
             lib.ipo_set_threads.argtypes = [ctypes.c_int]
+            lib.ipo_linear_i8.argtypes = [P, ctypes.c_int, P, P, P, P] + [ctypes.c_int] * 5 + [
+                P, ctypes.c_int]
+            lib.ipo_linear_i8.restype = ctypes.c_int
             for f in (lib.ipo_relpos_mhsa_i8, lib.ipo_content_scores_i32,
                       lib.ipo_position_scores_i32, lib.ipo_fused_scores_i8,
                       lib.ipo_isoftmax_u8, lib.ipo_set_threads):
@@ -164,7 +168,36 @@ def isoftmax(scores: np.ndarray, softmax: tuple[int, int, int], valid=None) -> n
     return out
 
 
-__all__ = ["build", "relpos_mhsa", "content_scores", "position_scores",
+ROWS = 0
+HEADS = 1
+
+
+def linear(x, w, bias, m, s, *, x_layout: int = ROWS, y_layout: int = ROWS, groups: int = 1,
+           B: int | None = None, T: int | None = None) -> np.ndarray:
+    """Integer linear layer of Eqs. 6-7 (per-channel m, s; optional int32
+    bias on the accumulator grid), int8.  ``x``: [B, T, K] (ROWS) or
+    [B, K/128, T, 128] (HEADS); ``w``: [N, K].  Output [B, T, N] (ROWS) or
+    [G, B, N/G/128, T, 128] (HEADS)."""
+    x = np.ascontiguousarray(x, dtype=np.int8)
+    w = np.ascontiguousarray(w, dtype=np.int8)
+    N, K = w.shape
+    if x_layout == ROWS:
+        B, T, _ = x.shape
+    else:
+        B, _, T, _ = x.shape
+    m = np.ascontiguousarray(m, dtype=np.int32)
+    s = np.ascontiguousarray(s, dtype=np.int32)
+    b = None if bias is None else np.ascontiguousarray(bias, dtype=np.int32)
+    if y_layout == ROWS:
+        y = np.empty((B, T, N), dtype=np.int8)
+    else:
+        y = np.empty((groups, B, N // groups // 128, T, 128), dtype=np.int8)
+    _check(_load().ipo_linear_i8(_ptr(x), x_layout, _ptr(w), _ptr(b), _ptr(m), _ptr(s),
+                                 B, T, K, N, groups, _ptr(y), y_layout), "ipo_linear_i8")
+    return y
+
+
+__all__ = ["build", "linear", "linear_constants", "ROWS", "HEADS", "relpos_mhsa", "content_scores", "position_scores",
            "fused_scores", "iexp", "isoftmax", "set_threads", "dyadic",
            "dyadic_pair", "isoftmax_params", "layer_constants", "LayerConstants",
            "IBERT_A", "IBERT_B", "IBERT_C", "OracleError"]

@@ -19,6 +19,8 @@ from __future__ import annotations
 import math
 from dataclasses import dataclass
 
+import numpy as np
+
 IBERT_A = 0.3585
 IBERT_B = 1.353
 IBERT_C = 0.344
@@ -86,3 +88,16 @@ def layer_constants(scales: dict, dh: int) -> LayerConstants:
     m_c, m_p, s_s = dyadic_pair(r_c, r_p)
     m_o, s_o = dyadic(r_o)
     return LayerConstants((m_c, m_p, m_o), (s_s, s_o), isoftmax_params(scales["S_s"]))
+
+
+def linear_constants(s_x: float, s_w, s_y) -> tuple[np.ndarray, np.ndarray]:
+    """Per-output-channel constants of Eq. 7: m[n], s[n] with
+    m 2^-(31+s) the dyadic nearest to S_x S_w[n] / S_y[n] (weights carry one
+    scale per channel, Sec. 2.2).  Returns int32 arrays (m, s)."""
+    s_w = np.asarray(s_w, dtype=np.float64)
+    s_y = np.broadcast_to(np.asarray(s_y, dtype=np.float64), s_w.shape)
+    m = np.empty(s_w.shape, dtype=np.int32)
+    s = np.empty(s_w.shape, dtype=np.int32)
+    for n in range(s_w.size):
+        m[n], s[n] = dyadic(float(s_x) * float(s_w[n]) / float(s_y[n]))
+    return m, s

@@ -221,3 +221,63 @@ def layer(workload: int | Workload, index: int = 0, seed: int | None = None) -> 
     return draw(w.B, w.H, w.T, w.dh, seed, p_mode=w.p_mode, dist=w.dist,
                 masked=w.masked)
 
+
+
+# ------------------------------------------------------------ linear layers
+
+@dataclass
+class LinearCase:
+    """Inputs of one integer linear layer (Eqs. 6-7): int8 activations x
+    [B, T, K], int8 weights w [N, K] (one row per output channel), an int32
+    bias on the accumulator grid S_x S_w[n] (or None), and the declared
+    scales: S_x, per-channel S_w [N], and S_y per output group (the G
+    stacked projections of a head-split output each have their own grid)."""
+    x: np.ndarray
+    w: np.ndarray
+    bias: np.ndarray | None
+    s_x: float
+    s_w: np.ndarray
+    s_y: np.ndarray          # [G]
+    groups: int = 1
+
+    def s_y_per_channel(self) -> np.ndarray:
+        N = self.w.shape[0]
+        return np.repeat(self.s_y, N // self.groups)
+
+
+def linear(B: int, T: int, K: int, N: int, seed: int, *, groups: int = 1,
+           bias: bool = True, dist: str = "normal", calib_frames: int = 256) -> LinearCase:
+    """Seeded linear-layer case shaped like the encoder's projections
+    (d = 1024 in and out; Q, K, V stacked as three groups).
+
+    x: round(N(0, 30^2)) (or t_3 * 25) clipped to [-127, 127]; w row n:
+    round(N(0, sigma_n^2)), sigma_n ~ U[15, 45], clipped; S_x = alpha_x/127
+    with alpha_x ~ U[2, 6]; S_w[n] = alpha_n/127 with alpha_n ~ U[0.05,
+    0.3]; real bias ~ N(0, 0.5^2) put on the accumulator grid; S_y of each
+    group = the min-max of the real output over the first `calib_frames`
+    frames / 127 (the offline calibration of Eq. 6)."""
+    seq = np.random.SeedSequence(seed)
+    kx, kw, kb, ks = seq.spawn(4)
+    x = _draw_int8(kx, (B, T, K), dist, 30.0 if dist == "normal" else 25.0)
+    g = np.random.Generator(np.random.PCG64(ks))
+    sig = g.uniform(15.0, 45.0, size=N)
+    gw = np.random.Generator(np.random.PCG64(kw))
+    wf = gw.standard_normal((N, K), dtype=np.float32) * sig[:, None].astype(np.float32)
+    w = np.clip(np.rint(wf), -127, 127).astype(np.int8)
+    s_x = g.uniform(2.0, 6.0) / 127.0
+    s_w = g.uniform(0.05, 0.3, size=N) / 127.0
+    bq = None
+    if bias:
+        gb = np.random.Generator(np.random.PCG64(kb))
+        real = gb.normal(0.0, 0.5, size=N)
+        bq = np.clip(np.rint(real / (s_x * s_w)), -(2**30 - 1), 2**30 - 1).astype(np.int32)
+    # calibration: real output of the first frames, float64
+    frames = x.reshape(-1, K)[:max(1, min(calib_frames, B * T))].astype(np.float64)
+    acc = frames @ w.astype(np.float64).T
+    if bq is not None:
+        acc += bq.astype(np.float64)
+    yr = acc * (s_x * s_w)[None, :]
+    per = N // groups
+    s_y = np.array([max(np.abs(yr[:, gi * per:(gi + 1) * per]).max(), 1e-30) / 127.0
+                    for gi in range(groups)])
+    return LinearCase(x, w, bq, float(s_x), s_w, s_y, groups)

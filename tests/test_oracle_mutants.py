@@ -43,6 +43,27 @@ MUTANTS = {
                      "acc += (int64_t)a[j] * (int64_t)vh[(size_t)d * dh + j % dh];"),
 }
 
+# mistakes planted in the linear-layer oracle (Eqs. 6-7)
+LINEAR_MUTANTS = {
+    # bias dropped
+    "lin_drop_bias": ("int64_t acc = bias ? (int64_t)bias[n] : 0;", "int64_t acc = 0;"),
+    # weights read transposed
+    "lin_w_transposed": ("acc += xr[k] * (int64_t)wn[k];",
+                         "acc += xr[k] * (int64_t)w[(size_t)k * N + n];"),
+    # truncation instead of rounding
+    "lin_floor": ("lin_floor_pow2((int64_t)m[n] * acc + ((int64_t)1 << (e - 1)), e)",
+                  "lin_floor_pow2((int64_t)m[n] * acc, e)"),
+    # shift one short
+    "lin_shift": ("int e = 31 + s[n];", "int e = 30 + s[n];"),
+    # asymmetric clamp (the int8 grid is symmetric, Eq. 6)
+    "lin_clamp": ("if (v < -127) v = -127;", "if (v < -128) v = -128;"),
+    # head index of the head-split layout swapped with the frame
+    "lin_heads": ("* heads + (size_t)(cc / 128)) * T + t) * 128",
+                  "* T + t) * heads + (size_t)(cc / 128)) * 128"),
+}
+
+LINEAR_PINS = ["tests/test_oracle_linear.py"]
+
 PINS = [
     "tests/test_oracle_relshift.py",
     "tests/test_oracle_scores.py",
@@ -63,17 +84,19 @@ def _copy_tree(dst):
 
 
 @pytest.mark.slow
-@pytest.mark.parametrize("name", sorted(MUTANTS))
+@pytest.mark.parametrize("name", sorted(MUTANTS) + sorted(LINEAR_MUTANTS))
 def test_mutant_is_caught(tmp_path, name):
-    old, new = MUTANTS[name]
+    linear = name in LINEAR_MUTANTS
+    old, new = (LINEAR_MUTANTS if linear else MUTANTS)[name]
+    pins = LINEAR_PINS if linear else PINS
     _copy_tree(tmp_path)
-    src = tmp_path / "oracle" / "ipo_mhsa.c"
+    src = tmp_path / "oracle" / ("ipo_linear.c" if linear else "ipo_mhsa.c")
     text = src.read_text()
     assert text.count(old) == 1, f"mutation site for {name} not found"
     src.write_text(text.replace(old, new))
     env = dict(os.environ, PYTHONPATH=str(tmp_path))
     res = subprocess.run([sys.executable, "-m", "pytest", "-x", "-q", "-p", "no:cacheprovider",
-                          "-m", "not gpu and not slow"] + PINS,
+                          "-m", "not gpu and not slow"] + pins,
                          cwd=tmp_path, env=env, capture_output=True, text=True, timeout=600)
     assert res.returncode != 0, f"mutant {name} survived the pins:\n{res.stdout[-2000:]}"
     assert "failed" in res.stdout or "error" in res.stdout.lower()
