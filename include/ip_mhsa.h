@@ -151,6 +151,48 @@ int ip_relpos_mhsa_i8_noalloc(const int8_t *q, const int8_t *k, const int8_t *v,
                               const ip_isoftmax_params *sm, const int32_t *lengths,
                               int B, int H, int T, int dh, int8_t *out, ip_stream_t stream);
 
+/* ---- integer linear layer (Sec. 2.2, Eqs. 6-7) ------------------------
+ *
+ * The projections around the attention: Q, K, V (and P) from the
+ * normalised frames, and the output projection of the heads.  Weights carry
+ * one scale per output channel, so Eq. 7's multiplier is per channel.
+ *
+ * Activation layouts (int8, C channels per frame, d = 128 per head):
+ *   IP_LAYOUT_ROWS   [B][T][C] row-major
+ *   IP_LAYOUT_HEADS  [G][B][C/G/128][T][128]: channel c of group g = c / (C/G)
+ *                    sits in head (c mod C/G) / 128 at d = c mod 128.  G = 1 is
+ *                    the attention's [B][H][T][128]; G = 3 writes Q, K and V
+ *                    of one stacked projection as three such tensors. */
+#define IP_LAYOUT_ROWS 0
+#define IP_LAYOUT_HEADS 1
+#define IP_LINEAR_MAX_K 32768          /* keeps the int32 accumulator exact */
+#define IP_LINEAR_MAX_N 65536
+#define IP_LINEAR_MAX_FRAMES 134217728  /* B T, 2^27 */
+
+/* For every frame (b, t) and output channel n (Eq. 7):
+ *   acc       = sum_k x[b,t,k] w[n,k] + bias[n]                   (int32)
+ *   y[b,t,n]  = clamp(round(2^-(31 + s[n]) m[n] acc), -127, 127)
+ * round(v 2^-e) = floor((v + 2^(e-1)) / 2^e).
+ * x: device int8, x_layout with C = K (IP_LAYOUT_HEADS reads K/128 heads).
+ * w: device int8 [N][K] row-major (one row per output channel).
+ * bias: device int32 [N] with |bias| < 2^30, or NULL; m: device int32 [N]
+ *   in [0, 2^31); s: device int32 [N] in [0, 31] (a value outside is
+ *   clamped into its domain and reported as IP_ERR_PARAM by
+ *   ip_relpos_mhsa_status).
+ * y: device int8, y_layout with C = N and G groups (G = 1 for ROWS).
+ * Shapes: B in [0, IP_MAX_B], T >= 1, B T <= IP_LINEAR_MAX_FRAMES, K a
+ *   multiple of 128 in [128, IP_LINEAR_MAX_K], N a multiple of 128 (of 128 G
+ *   for a HEADS output) up to IP_LINEAR_MAX_N.
+ * x, w, y 16-byte aligned; bias, m, s 4-byte aligned; workspace as for
+ *   ip_relpos_mhsa_i8 (>= 256 bytes, 256-aligned, zero-filled once; its
+ *   status word is read and cleared by ip_relpos_mhsa_status).
+ * Inputs are not modified; launch is asynchronous on `stream`; B == 0
+ * returns IP_OK without touching any pointer.  Returns IP_OK or IP_ERR_*. */
+int ip_linear_i8(const int8_t *x, int x_layout, const int8_t *w, const int32_t *bias,
+                 const int32_t *m, const int32_t *s, int B, int T, int K, int N, int G,
+                 int8_t *y, int y_layout, void *workspace, size_t workspace_bytes,
+                 ip_stream_t stream);
+
 /* Text of an IP_* code. */
 const char *ip_strerror(int code);
 

@@ -30,8 +30,11 @@ EXPORTS = (
     "ip_debug_set_timeout_cycles", "ip_debug_set_stall_injection", "ip_dyadic_multiplier",
     "ip_dyadic_pair",
     "ip_isoftmax_params_from_scale", "ip_probe_int8_mma", "ip_relpos_mhsa_i8_noalloc",
-    "ip_debug_set_split_mode",
+    "ip_debug_set_split_mode", "ip_linear_i8",
 )
+
+ROWS = 0    # IP_LAYOUT_ROWS:  [B][T][C]
+HEADS = 1   # IP_LAYOUT_HEADS: [G][B][C/G/128][T][128]
 
 
 class LibraryError(RuntimeError):
@@ -100,6 +103,8 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
         lib.ip_dyadic_pair.restype = I
         lib.ip_isoftmax_params_from_scale.argtypes = [ctypes.c_double, ctypes.POINTER(SoftmaxParams)]
         lib.ip_isoftmax_params_from_scale.restype = I
+        lib.ip_linear_i8.argtypes = [P, I, P, P, P, P, I, I, I, I, I, P, I, P, ctypes.c_size_t, P]
+        lib.ip_linear_i8.restype = I
         lib.ip_probe_int8_mma.argtypes = [I, I, P, P]
         lib.ip_probe_int8_mma.restype = ctypes.c_longlong
         _lib = lib
@@ -267,6 +272,49 @@ def status(workspace, stream=None) -> int:
     return load().ip_relpos_mhsa_status(ctypes.c_void_p(workspace.data_ptr()), _stream_handle(stream))
 
 
+def linear_constants(s_x: float, s_w, s_y):
+    """Per-output-channel constants of Eq. 7 (offline): int32 arrays m, s
+    with m[n] 2^-(31+s[n]) the dyadic nearest to S_x S_w[n] / S_y[n]."""
+    import numpy as np
+    s_w = np.asarray(s_w, dtype=np.float64)
+    s_y = np.broadcast_to(np.asarray(s_y, dtype=np.float64), s_w.shape)
+    m = np.empty(s_w.shape, dtype=np.int32)
+    s = np.empty(s_w.shape, dtype=np.int32)
+    for n in range(s_w.size):
+        m[n], s[n] = dyadic_multiplier(float(s_x) * float(s_w[n]) / float(s_y[n]))
+    return m, s
+
+
+def linear_i8(x, w, bias, m, s, *, x_layout: int = ROWS, y_layout: int = ROWS, groups: int = 1,
+              out=None, workspace=None, stream=None):
+    """Integer linear layer (Eqs. 6-7) on the GPU.  x: int8 [B, T, K] (ROWS)
+    or [B, K/128, T, 128] (HEADS); w: int8 [N, K]; bias: int32 [N] or None;
+    m, s: int32 [N] (per output channel); all CUDA tensors.  Returns out:
+    int8 [B, T, N] (ROWS) or [G, B, N/G/128, T, 128] (HEADS).  Asynchronous
+    on `stream` (default: torch's current stream)."""
+    import torch
+    N, K = w.shape
+    if x_layout == ROWS:
+        B, T, _ = x.shape
+        xs = (B, T, K)
+    else:
+        B, _, T, _ = x.shape
+        xs = (B, K // 128, T, 128)
+    ys = (B, T, N) if y_layout == ROWS else (groups, B, N // max(groups, 1) // 128, T, 128)
+    if out is None:
+        out = torch.empty(ys, dtype=torch.int8, device=w.device)
+    if workspace is None:
+        workspace = torch.zeros(256, dtype=torch.uint8, device=w.device)
+    bp = None if bias is None else _dev_ptr(bias, "bias", torch.int32, (N,))
+    rc = load().ip_linear_i8(
+        _dev_ptr(x, "x", torch.int8, xs), x_layout, _dev_ptr(w, "w", torch.int8, (N, K)), bp,
+        _dev_ptr(m, "m", torch.int32, (N,)), _dev_ptr(s, "s", torch.int32, (N,)), B, T, K, N,
+        groups, _dev_ptr(out, "out", torch.int8, ys), y_layout,
+        ctypes.c_void_p(workspace.data_ptr()), workspace.numel(), _stream_handle(stream))
+    _check("ip_linear_i8", rc)
+    return out
+
+
 def relpos_mhsa_i8_host(q, k, v, p, u, v_bias, consts: LayerConstants, lengths, out, arena,
                         stream=None):
     """Whole layer from host buffers (torch CPU tensors, ideally pinned):
@@ -295,5 +343,6 @@ def relpos_mhsa_i8_host(q, k, v, p, u, v_bias, consts: LayerConstants, lengths, 
 __all__ = ["build", "load", "relpos_mhsa_i8", "relpos_mhsa_i8_host", "status", "workspace_bytes",
            "host_arena_bytes", "layer_constants", "LayerConstants", "dyadic_multiplier",
            "dyadic_pair", "isoftmax_params_from_scale", "set_timeout_cycles", "strerror",
-           "int8_mma_peak_tops", "set_stall_injection",
+           "int8_mma_peak_tops", "set_stall_injection", "set_split_mode", "linear_i8",
+           "linear_constants", "ROWS", "HEADS",
            "IpError", "LibraryError", "EXPORTS"]

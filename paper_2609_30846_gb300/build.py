@@ -14,8 +14,10 @@ ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 LIB = os.path.join(PKG, "libipmhsa.so")
-SOURCES = [os.path.join(CSRC, "ip_mhsa.cu")]
-DEPS = SOURCES + [os.path.join(CSRC, "ip_mhsa_kernels.cuh"), os.path.join(INCLUDE, "ip_mhsa.h")]
+SOURCES = [os.path.join(CSRC, f) for f in ("ip_mhsa.cu", "ip_linear.cu")]
+DEPS = SOURCES + [os.path.join(CSRC, f) for f in ("ip_mhsa_kernels.cuh", "ip_linear_kernels.cuh",
+                                                  "ip_ptx.cuh", "ip_probe.cuh")] + [
+    os.path.join(INCLUDE, "ip_mhsa.h")]
 ARCH = "-gencode=arch=compute_103a,code=sm_103a"
 
 
@@ -26,9 +28,15 @@ def nvcc() -> str:
     raise RuntimeError("nvcc not found: the GPU library cannot be built")
 
 
-def command(out: str) -> list[str]:
-    return [nvcc(), ARCH, "-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-shared",
-            "-I" + INCLUDE, "-o", out] + SOURCES
+FLAGS = [ARCH, "-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC"]
+
+
+def compile_command(src: str, obj: str) -> list[str]:
+    return [nvcc()] + FLAGS + ["-I" + INCLUDE, "-c", "-o", obj, src]
+
+
+def link_command(objs: list[str], out: str) -> list[str]:
+    return [nvcc(), ARCH, "-shared", "-o", out] + objs
 
 
 def up_to_date() -> bool:
@@ -42,12 +50,26 @@ def build(force: bool = False, verbose: bool = False) -> str:
     """Compile (if stale) and return the path of libipmhsa.so."""
     if not force and up_to_date():
         return LIB
-    tmp = LIB + f".tmp{os.getpid()}"
-    cmd = command(tmp)
-    if verbose:
-        print(" ".join(cmd), flush=True)
-    subprocess.run(cmd, check=True, cwd=CSRC)
-    os.replace(tmp, LIB)
+    tag = f".tmp{os.getpid()}"
+    objs = [os.path.join(CSRC, os.path.basename(s) + tag + ".o") for s in SOURCES]
+    try:
+        # the translation units compile in parallel, then one link
+        procs = []
+        for src, obj in zip(SOURCES, objs):
+            cmd = compile_command(src, obj)
+            if verbose:
+                print(" ".join(cmd), flush=True)
+            procs.append((cmd, subprocess.Popen(cmd, cwd=CSRC)))
+        for cmd, p in procs:
+            if p.wait() != 0:
+                raise subprocess.CalledProcessError(p.returncode, cmd)
+        tmp = LIB + tag
+        subprocess.run(link_command(objs, tmp), check=True, cwd=CSRC)
+        os.replace(tmp, LIB)
+    finally:
+        for obj in objs:
+            if os.path.exists(obj):
+                os.unlink(obj)
     return LIB
 
 

@@ -1,0 +1,161 @@
+// Host side of the integer linear layer of the C ABI (include/ip_mhsa.h):
+// argument validation, TMA tensor maps and the launch.  Device code:
+// ip_linear_kernels.cuh.
+#include "ip_mhsa.h"
+#include "ip_linear_kernels.cuh"
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include <mutex>
+
+namespace {
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *,
+                                  const cuuint64_t *, const cuuint64_t *, const cuuint32_t *,
+                                  const cuuint32_t *, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+    static EncodeTiledFn fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000,
+                                             cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(p);
+    });
+    return fn;
+}
+
+// int8 tensor map of `rank` dimensions (innermost first; byte strides of
+// dimensions 1..rank-1) with a box of 128 x 128 (x 1 ...), 128-byte swizzle;
+// elements outside the tensor read as zero.
+bool make_map(CUtensorMap *m, const void *base, int rank, const cuuint64_t *dims,
+              const cuuint64_t *strides) {
+    EncodeTiledFn fn = encode_fn();
+    if (!fn) return false;
+    const cuuint32_t box[4] = {128, 128, 1, 1};
+    const cuuint32_t estride[4] = {1, 1, 1, 1};
+    return fn(m, CU_TENSOR_MAP_DATA_TYPE_UINT8, rank, const_cast<void *>(base), dims, strides,
+              box, estride, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) ==
+           CUDA_SUCCESS;
+}
+
+bool aligned(const void *p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+std::mutex g_mu;
+int g_smem_set[64] = {0};
+int g_sms[64] = {0};
+
+int sm_count() {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
+    std::lock_guard<std::mutex> lock(g_mu);
+    if (g_sms[dev] == 0) {
+        int n = 0;
+        if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
+        g_sms[dev] = n;
+    }
+    return g_sms[dev];
+}
+
+// Constant of udiv_magic: floor(2^64 / d) + 1, or 0 for d = 1.
+unsigned long long div_magic(unsigned long long d) {
+    if (d <= 1) return 0;
+    const unsigned __int128 one = static_cast<unsigned __int128>(1) << 64;
+    return static_cast<unsigned long long>(one / d) + 1;
+}
+
+int ensure_smem() {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return IP_ERR_CUDA;
+    std::lock_guard<std::mutex> lock(g_mu);
+    if (g_smem_set[dev]) return IP_OK;
+    if (cudaFuncSetAttribute(ipl::linear_i8_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             ipl::SMEM_LAUNCH) != cudaSuccess)
+        return IP_ERR_CUDA;
+    g_smem_set[dev] = 1;
+    return IP_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int ip_linear_i8(const int8_t *x, int x_layout, const int8_t *w, const int32_t *bias,
+                 const int32_t *m, const int32_t *s, int B, int T, int K, int N, int G,
+                 int8_t *y, int y_layout, void *workspace, size_t workspace_bytes,
+                 ip_stream_t stream) {
+    if ((x_layout != IP_LAYOUT_ROWS && x_layout != IP_LAYOUT_HEADS) ||
+        (y_layout != IP_LAYOUT_ROWS && y_layout != IP_LAYOUT_HEADS))
+        return IP_ERR_PARAM;
+    if (B < 0 || B > IP_MAX_B || T < 1 || G < 1) return IP_ERR_SHAPE;
+    if (static_cast<long long>(B) * T > IP_LINEAR_MAX_FRAMES) return IP_ERR_SHAPE;
+    if (K < 128 || K > IP_LINEAR_MAX_K || K % 128 != 0) return IP_ERR_SHAPE;
+    if (N < 128 || N > IP_LINEAR_MAX_N || N % 128 != 0) return IP_ERR_SHAPE;
+    if (y_layout == IP_LAYOUT_HEADS && N % (128 * G) != 0) return IP_ERR_SHAPE;
+    if (y_layout == IP_LAYOUT_ROWS && G != 1) return IP_ERR_SHAPE;
+    if (B == 0) return IP_OK;
+    if (!x || !w || !m || !s || !y || !workspace) return IP_ERR_NULL;
+    if (!aligned(x, 16) || !aligned(w, 16) || !aligned(y, 16) || !aligned(m, 4) ||
+        !aligned(s, 4) || (bias && !aligned(bias, 4)) || !aligned(workspace, 256))
+        return IP_ERR_ALIGN;
+    if (workspace_bytes < 256) return IP_ERR_WORKSPACE;
+
+    CUtensorMap tm_x, tm_w;
+    const cuuint64_t kk = static_cast<cuuint64_t>(K), tt = static_cast<cuuint64_t>(T);
+    bool okm;
+    if (x_layout == IP_LAYOUT_ROWS) {
+        // all frames of all utterances as one axis of B T rows
+        const cuuint64_t dims[2] = {kk, tt * static_cast<cuuint64_t>(B)};
+        const cuuint64_t strides[1] = {kk};
+        okm = make_map(&tm_x, x, 2, dims, strides);
+    } else {
+        const cuuint64_t dims[4] = {128, tt, kk / 128, static_cast<cuuint64_t>(B)};
+        const cuuint64_t strides[3] = {128, tt * 128, tt * kk};
+        okm = make_map(&tm_x, x, 4, dims, strides);
+    }
+    const cuuint64_t wdims[2] = {kk, static_cast<cuuint64_t>(N)};
+    const cuuint64_t wstrides[1] = {kk};
+    if (!okm || !make_map(&tm_w, w, 2, wdims, wstrides)) return IP_ERR_CUDA;
+    int rc = ensure_smem();
+    if (rc != IP_OK) return rc;
+
+    ipl::LinearParams prm;
+    prm.bias = bias;
+    prm.m = m;
+    prm.s = s;
+    prm.y = y;
+    prm.B = B;
+    prm.T = T;
+    prm.K = K;
+    prm.N = N;
+    prm.heads_per_group = N / G / 128;
+    prm.y_layout = y_layout;
+    prm.x_layout = x_layout;
+    prm.err = static_cast<int *>(workspace);
+    prm.timeout_cycles = 4000000000ll;
+    prm.ntn = N / ipl::BN;
+    prm.tpu = (T + ipl::BM - 1) / ipl::BM;
+    const long long frame_tiles = x_layout == IP_LAYOUT_ROWS
+                                      ? (static_cast<long long>(B) * T + ipl::BM - 1) / ipl::BM
+                                      : static_cast<long long>(B) * prm.tpu;
+    prm.ntiles = static_cast<unsigned>(frame_tiles * prm.ntn);
+    prm.magic_ntn = div_magic(prm.ntn);
+    prm.magic_T = div_magic(T);
+    prm.magic_tpu = div_magic(prm.tpu);
+    const int nsm = sm_count();
+    if (nsm <= 0) return IP_ERR_CUDA;
+    const unsigned grid = prm.ntiles < static_cast<unsigned>(nsm) ? prm.ntiles
+                                                                  : static_cast<unsigned>(nsm);
+    ipl::linear_i8_kernel<<<grid, ipl::THREADS, ipl::SMEM_LAUNCH,
+                            reinterpret_cast<cudaStream_t>(stream)>>>(tm_x, tm_w, prm);
+    if (cudaGetLastError() != cudaSuccess) return IP_ERR_CUDA;
+    return IP_OK;
+}
+
+}  // extern "C"

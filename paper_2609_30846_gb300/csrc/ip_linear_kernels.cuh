@@ -1,0 +1,286 @@
+// Device code of the integer linear layer (I-Parakeet, Sec. 2.2, Eqs. 6-7)
+// for sm_103a: Y = requant(X W^T + bias) with one dyadic multiplier per
+// output channel.  Integer arithmetic only: no floating-point type and no
+// division by a run-time value.
+//
+// Persistent kernel: one CTA per SM takes the 128 x 128 tiles of Y (128
+// frames x 128 output channels) round-robin.  With a row-major X the frames
+// of all utterances form one axis of B T rows; with a head-split X a tile
+// stays inside one utterance.  A producer warp streams K in stages of 128
+// bytes: the 128 x 128 int8 tiles of X and W land through TMA with the
+// 128-byte swizzle in a ring of four stages that runs on across tiles, so
+// the next tile's first stages load during the current tile's epilogue.  Eight consumer warps (2 along the frames x 4
+// along the channels, 64 x 32 each) feed the integer warp MMA (mma.sync
+// m16n8k32 s8 x s8 -> s32) from ldmatrix; sm_103a has no integer tcgen05
+// kind.  The epilogue adds the int32 bias, multiplies by m[n] in int64,
+// shifts right by 31 + s[n] with rounding, clamps to [-127, 127] and writes
+// each warp's 64 x 32 bytes through shared memory as 16-byte row segments,
+// either row-major [B][T][N] or head-split [G][B][N/G/128][T][128].
+#pragma once
+
+#include <cuda.h>
+#include <stdint.h>
+
+#include "ip_ptx.cuh"
+
+namespace ipl {
+
+using namespace ipk;
+
+constexpr int BM = 128;                 // frames per CTA
+constexpr int BN = 128;                 // output channels per CTA
+constexpr int BK = 128;                 // K bytes per stage
+constexpr int NCW = 8;                  // consumer warps: 2 (frames) x 4 (channels)
+constexpr int THREADS = (NCW + 1) * 32;
+constexpr int STAGES = 4;
+constexpr int A_BYTES = BM * BK;
+constexpr int B_BYTES = BN * BK;
+constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+constexpr int OUT_ROW = 48;             // staged output row of one warp: 32 bytes + pad
+constexpr int OUT_WARP_BYTES = 64 * OUT_ROW;
+constexpr int SMEM_OUT = STAGES * STAGE_BYTES;
+constexpr int SMEM_BARS = SMEM_OUT + NCW * OUT_WARP_BYTES;
+constexpr int SMEM_BYTES = SMEM_BARS + 8 * (2 * STAGES);
+constexpr int SMEM_LAUNCH = SMEM_BYTES + 1024;   // + alignment of the dynamic base
+
+constexpr int LAYOUT_ROWS = 0;
+constexpr int LAYOUT_HEADS = 1;
+constexpr int ERR_PARAM = 16;           // a multiplier, shift or bias out of its domain
+
+static_assert(STAGE_BYTES % 1024 == 0, "128-byte swizzle needs 1024-byte aligned tiles");
+static_assert((STAGES & (STAGES - 1)) == 0, "stage index by mask");
+
+struct LinearParams {
+    const int32_t *bias;      // [N] or nullptr
+    const int32_t *m;         // [N]
+    const int32_t *s;         // [N]
+    int8_t *y;
+    int B, T, K, N;
+    int ntn;                  // N / 128 channel tiles
+    int tpu;                  // frame tiles per utterance (head-split X)
+    unsigned ntiles;          // all tiles
+    unsigned long long magic_ntn, magic_T, magic_tpu;   // exact division constants
+    int heads_per_group;      // N / G / 128 (head-split output)
+    int y_layout;
+    int x_layout;
+    int *err;
+    long long timeout_cycles;
+};
+
+struct Tile {
+    int nt;        // channel tile
+    int b, t0;     // utterance and frame of the first row
+    int m0;        // flat row of the first row (b T + t0)
+};
+
+__device__ __forceinline__ Tile tile_of(unsigned idx, const LinearParams &p) {
+    Tile L;
+    const unsigned mt = udiv_magic(idx, p.magic_ntn);
+    L.nt = static_cast<int>(idx - mt * static_cast<unsigned>(p.ntn));
+    if (p.x_layout == LAYOUT_ROWS) {
+        L.m0 = static_cast<int>(mt) * BM;
+        L.b = static_cast<int>(udiv_magic(static_cast<unsigned>(L.m0), p.magic_T));
+        L.t0 = L.m0 - L.b * p.T;
+    } else {
+        L.b = static_cast<int>(udiv_magic(mt, p.magic_tpu));
+        L.t0 = (static_cast<int>(mt) - L.b * p.tpu) * BM;
+        L.m0 = L.b * p.T + L.t0;
+    }
+    return L;
+}
+
+__global__ void __launch_bounds__(THREADS, 1)
+    linear_i8_kernel(const __grid_constant__ CUtensorMap tm_x,
+                     const __grid_constant__ CUtensorMap tm_w, const LinearParams prm) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+    const int kt = prm.K / BK;     // BK is a power of two: a shift
+
+    const uint32_t base = smem_u32(smem);
+    const uint32_t bars = base + SMEM_BARS;
+    auto full_bar = [&](int s) { return bars + 8u * s; };
+    auto empty_bar = [&](int s) { return bars + 8u * (STAGES + s); };
+    auto stage = [&](int s) { return base + s * STAGE_BYTES; };
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < STAGES; ++s) {
+            mbar_init(full_bar(s), 1);
+            mbar_init(empty_bar(s), NCW);
+        }
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    }
+    __syncthreads();
+
+    // ---------------------------------------------------------- producer
+    // Use u of the ring: stage u & 3, phase (u / 4) & 1.
+    if (warp == NCW) {
+        unsigned u = 0, landed_from = 0;
+        bool ok = true;
+        for (unsigned idx = blockIdx.x; idx < prm.ntiles && ok; idx += gridDim.x) {
+            const Tile L = tile_of(idx, prm);
+            for (int it = 0; it < kt; ++it, ++u) {
+                const int s = static_cast<int>(u & (STAGES - 1));
+                if (u >= STAGES &&
+                    !warp_wait(empty_bar(s), ((u / STAGES) - 1) & 1, prm.timeout_cycles)) {
+                    if (lane == 0) atomicOr(prm.err, 2);
+                    ok = false;
+                    break;
+                }
+                if (lane == 0) {
+                    mbar_expect_tx(full_bar(s), STAGE_BYTES);
+                    if (prm.x_layout == LAYOUT_ROWS)
+                        tma_load_2d(stage(s), &tm_x, it * BK, L.m0, full_bar(s));
+                    else
+                        tma_load_4d(stage(s), &tm_x, 0, L.t0, it, L.b, full_bar(s));
+                    tma_load_2d(stage(s) + A_BYTES, &tm_w, it * BK, L.nt * BN, full_bar(s));
+                }
+            }
+        }
+        if (!ok) {
+            // let the copies in flight land before the CTA exits
+            landed_from = u > STAGES ? u - STAGES : 0;
+            for (unsigned v = landed_from; v < u; ++v)
+                mbar_wait(full_bar(static_cast<int>(v & (STAGES - 1))), (v / STAGES) & 1,
+                          2000000000ll);
+        }
+        return;
+    }
+
+    // ---------------------------------------------------------- consumers
+    const int wm = warp & 1;        // rows 64 wm .. 64 wm + 63 of the tile
+    const int wn = warp >> 1;       // channels 32 wn .. 32 wn + 31
+    const int g = lane >> 2, t4 = lane & 3;
+    const int lm_row = lane & 7, lm_mat = lane >> 3;
+    const uint32_t ob = base + SMEM_OUT + warp * OUT_WARP_BYTES;
+    const int frames = prm.B * prm.T;
+
+    unsigned u = 0;
+    for (unsigned idx = blockIdx.x; idx < prm.ntiles; idx += gridDim.x) {
+        const Tile L = tile_of(idx, prm);
+        const int n0 = L.nt * BN;
+
+        // per-channel constants of this thread's eight channels (Eq. 7)
+        int cb[8], cm[8], ce[8];
+        bool bad = false;
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+#pragma unroll
+            for (int q = 0; q < 2; ++q) {
+                const int n = n0 + 32 * wn + 8 * j + 2 * t4 + q;
+                int bi = prm.bias != nullptr ? __ldg(prm.bias + n) : 0;
+                int mi = __ldg(prm.m + n);
+                int si = __ldg(prm.s + n);
+                if (mi < 0 || si < 0 || si > 31 || bi >= (1 << 30) || bi <= -(1 << 30)) {
+                    bad = true;
+                    mi = mi < 0 ? 0 : mi;
+                    si = si < 0 ? 0 : (si > 31 ? 31 : si);
+                    bi = 0;
+                }
+                cb[2 * j + q] = bi;
+                cm[2 * j + q] = mi;
+                ce[2 * j + q] = 31 + si;
+            }
+        if (bad) atomicOr(prm.err, ERR_PARAM);
+
+        int acc[4][4][4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+#pragma unroll
+            for (int j = 0; j < 4; ++j)
+                acc[i][j][0] = acc[i][j][1] = acc[i][j][2] = acc[i][j][3] = 0;
+
+        for (int it = 0; it < kt; ++it, ++u) {
+            const int s = static_cast<int>(u & (STAGES - 1));
+            if (!warp_wait(full_bar(s), (u / STAGES) & 1, prm.timeout_cycles)) {
+                if (lane == 0) atomicOr(prm.err, 1);
+                return;
+            }
+            const uint32_t at = stage(s) + (64 * wm) * 128;
+            const uint32_t bt = stage(s) + A_BYTES + (32 * wn) * 128;
+#pragma unroll
+            for (int ks = 0; ks < 4; ++ks) {
+                uint32_t af[4][4], bf[4][2];
+#pragma unroll
+                for (int i = 0; i < 4; ++i)
+                    ldsm_x4(at + swz(16 * i + (lm_mat & 1) * 8 + lm_row, 2 * ks + (lm_mat >> 1)),
+                            af[i][0], af[i][1], af[i][2], af[i][3]);
+#pragma unroll
+                for (int jj = 0; jj < 2; ++jj)
+                    ldsm_x4(bt + swz(16 * jj + (lm_mat >> 1) * 8 + lm_row, 2 * ks + (lm_mat & 1)),
+                            bf[2 * jj][0], bf[2 * jj][1], bf[2 * jj + 1][0], bf[2 * jj + 1][1]);
+#pragma unroll
+                for (int i = 0; i < 4; ++i)
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) mma_s8s8(acc[i][j], af[i], bf[j][0], bf[j][1]);
+            }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(empty_bar(s));
+        }
+
+        // ------------------------------------------------------ epilogue
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+#pragma unroll
+            for (int j = 0; j < 4; ++j)
+#pragma unroll
+                for (int rr = 0; rr < 2; ++rr) {
+                    uint32_t two = 0;
+#pragma unroll
+                    for (int q = 0; q < 2; ++q) {
+                        const int c = 2 * j + q;
+                        const long long v = static_cast<long long>(cm[c]) *
+                                                (acc[i][j][2 * rr + q] + cb[c]) +
+                                            (1ll << (ce[c] - 1));
+                        two |= (static_cast<uint32_t>(clamp127(v >> ce[c])) & 0xffu) << (8 * q);
+                    }
+                    const int r = 16 * i + g + 8 * rr;
+                    asm volatile("st.shared.u16 [%0], %1;" ::"r"(ob + r * OUT_ROW + 8 * j + 2 * t4),
+                                 "h"(static_cast<unsigned short>(two))
+                                 : "memory");
+                }
+        __syncwarp();
+
+        int hh = L.nt, grp = 0;
+        if (prm.y_layout == LAYOUT_HEADS) {
+            while (hh >= prm.heads_per_group) {   // at most G - 1 steps
+                hh -= prm.heads_per_group;
+                ++grp;
+            }
+        }
+        // 64 rows x 32 bytes: lane -> (row 16 it + lane / 2, segment lane & 1)
+#pragma unroll
+        for (int it = 0; it < 4; ++it) {
+            const int r = 64 * wm + 16 * it + (lane >> 1);
+            const int seg = lane & 1;
+            const uint4 v = lds128(ob + (r - 64 * wm) * OUT_ROW + 16 * seg);
+            int b = L.b, t = L.t0 + r;
+            bool valid;
+            if (prm.x_layout == LAYOUT_ROWS) {
+                valid = L.m0 + r < frames;
+                if (valid && prm.y_layout == LAYOUT_HEADS)
+                    while (t >= prm.T) {   // rows of a flat tile may run into later utterances
+                        t -= prm.T;
+                        ++b;
+                    }
+            } else {
+                valid = t < prm.T;
+            }
+            if (valid) {
+                size_t off;
+                if (prm.y_layout == LAYOUT_ROWS)
+                    off = (static_cast<size_t>(b) * prm.T + t) * prm.N + n0 + 32 * wn + 16 * seg;
+                else
+                    off = (((static_cast<size_t>(grp) * prm.B + b) * prm.heads_per_group + hh) *
+                               prm.T + t) * 128 + 32 * wn + 16 * seg;
+                *reinterpret_cast<uint4 *>(prm.y + off) = v;
+            }
+        }
+        __syncwarp();
+    }
+}
+
+}  // namespace ipl

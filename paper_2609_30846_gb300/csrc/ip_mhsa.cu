@@ -239,7 +239,8 @@ int ip_relpos_mhsa_status(const void *workspace, ip_stream_t stream) {
     if (cudaMemsetAsync(const_cast<void *>(workspace), 0, sizeof(int), st) != cudaSuccess)
         return IP_ERR_CUDA;
     if (cudaStreamSynchronize(st) != cudaSuccess) return IP_ERR_CUDA;
-    return word == 0 ? IP_OK : IP_ERR_TIMEOUT;
+    if (word & 15) return IP_ERR_TIMEOUT;   // a bounded barrier wait ran out
+    return word == 0 ? IP_OK : IP_ERR_PARAM;   // a device-side constant out of its domain
 }
 
 size_t ip_relpos_mhsa_host_arena_bytes(int B, int H, int T, int dh) {

@@ -15,7 +15,10 @@ import paper_2609_30846_gb300 as ip
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 HEADER = os.path.join(ROOT, "include", "ip_mhsa.h")
-KERNELS = os.path.join(ROOT, "paper_2609_30846_gb300", "csrc", "ip_mhsa_kernels.cuh")
+CSRC = os.path.join(ROOT, "paper_2609_30846_gb300", "csrc")
+KERNELS = os.path.join(CSRC, "ip_mhsa_kernels.cuh")
+DEVICE_SOURCES = [os.path.join(CSRC, f) for f in
+                  ("ip_mhsa_kernels.cuh", "ip_linear_kernels.cuh", "ip_ptx.cuh")]
 
 
 def declared_functions():
@@ -118,8 +121,9 @@ def test_constants_reject_bad_ratios(lib):
         ip.isoftmax_params_from_scale(0.0)
 
 
-def test_kernel_source_is_integer_only():
-    text = open(KERNELS).read()
+@pytest.mark.parametrize("path", DEVICE_SOURCES, ids=os.path.basename)
+def test_kernel_source_is_integer_only(path):
+    text = open(path).read()
     code = re.sub(r"//[^\n]*", "", re.sub(r"/\*.*?\*/", "", text, flags=re.S))
     code = re.sub(r'"(\\.|[^"\\])*"', '""', code)          # drop string literals (PTX)
     for pat in (r"\bfloat\b", r"\bdouble\b", r"\b__half\b", r"\b__nv_bfloat16\b", r"\bhalf\b",
@@ -128,8 +132,10 @@ def test_kernel_source_is_integer_only():
     # No '/' or '%' by a run-time value: the compiler's integer division
     # would not be integer-only.  Divisions are the long-division helpers;
     # the remaining operators divide by compile-time powers of two.
-    assert "div_2pow32" in code and "iexp_neg" in code
-    allowed = {"NSTAGE", "NK", "MROWS", "DH", "16", "2", "4", "8", "32", "256"}
+    if path == KERNELS:
+        assert "div_2pow32" in code and "iexp_neg" in code
+    allowed = {"NSTAGE", "NK", "MROWS", "DH", "BK", "BM", "BN", "STAGES",
+               "16", "2", "4", "8", "32", "256"}
     for m in re.finditer(r"[^/*](/|%)\s*\(?\s*([A-Za-z_0-9]+)", code):
         if m.group(0).startswith("<") or m.group(1) == "/" and code[m.start(1) + 1] in "/*":
             continue
@@ -137,3 +143,44 @@ def test_kernel_source_is_integer_only():
         if tok.isdigit() and int(tok) & (int(tok) - 1) == 0:
             continue   # a literal power of two
         assert tok in allowed, f"run-time division by {tok!r}"
+
+
+def test_linear_validation_codes(lib):
+    P = ctypes.c_void_p
+    fake = P(1 << 20)           # never dereferenced: every case fails validation first
+    ws = P(1 << 21)
+
+    def call(x_layout=0, y_layout=0, B=1, T=4, K=256, N=256, G=1, x=fake, w=fake, y=fake,
+             m=fake, s=fake, bias=None, wsb=256, wsp=ws):
+        return lib.ip_linear_i8(x, x_layout, w, bias, m, s, B, T, K, N, G, y, y_layout, wsp,
+                                wsb, None)
+
+    assert call(x_layout=2) == -7
+    assert call(y_layout=-1) == -7
+    assert call(K=200) == -2                     # not a multiple of 128
+    assert call(K=65536) == -2                   # above IP_LINEAR_MAX_K
+    assert call(N=64) == -2
+    assert call(T=0) == -2
+    assert call(y_layout=1, N=256, G=3) == -2    # N not a multiple of 128 G
+    assert call(y_layout=0, G=2) == -2
+    assert call(B=0, x=None, w=None, y=None) == 0   # empty batch: nothing touched
+    assert call(w=None) == -1
+    assert call(x=P((1 << 20) + 8)) == -3        # 16-byte alignment
+    assert call(wsp=P((1 << 21) + 64)) == -3     # workspace 256-byte alignment
+    assert call(wsb=128) == -8
+
+
+def test_exact_division_constant():
+    # udiv_magic: floor(n * (floor(2^64 / d) + 1) / 2^64) == floor(n / d) for
+    # 0 <= n < 2^32, 2 <= d < 2^32 (d = 1 uses the constant 0 and returns n)
+    rng = np.random.default_rng(0)
+    ds = [2, 3, 5, 7, 24, 96, 375, 1500, 2 ** 16 + 1, 2 ** 31 - 1, 2 ** 32 - 1]
+    ds += [int(v) for v in rng.integers(2, 2 ** 32, size=40)]
+    for d in ds:
+        M = (1 << 64) // d + 1
+        ns = [0, 1, d - 1, d, d + 1, 2 * d - 1, 2 ** 32 - 1, (2 ** 32 - 1) // d * d,
+              (2 ** 32 - 1) // d * d - 1]
+        ns += [int(v) for v in rng.integers(0, 2 ** 32, size=200)]
+        for n in ns:
+            if 0 <= n < 2 ** 32:
+                assert (n * M) >> 64 == n // d, (n, d)
