@@ -22,7 +22,8 @@ import threading
 import numpy as np
 
 from .consts import (IBERT_A, IBERT_B, IBERT_C, LayerConstants, dyadic,
-                     dyadic_pair, isoftmax_params, layer_constants, linear_constants)
+                     dyadic_pair, isoftmax_params, layer_constants, linear_constants,
+                     SWISH_A, SWISH_C, SwishParams, swish_params)
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 _SRCS = [os.path.join(_HERE, f) for f in ("ipo_mhsa.c", "ipo_linear.c")]
@@ -68,6 +69,8 @@ def _load():
             lib.ipo_linear_i8.argtypes = [P, ctypes.c_int, P, P, P, P] + [ctypes.c_int] * 5 + [
                 P, ctypes.c_int]
             lib.ipo_linear_i8.restype = ctypes.c_int
+            lib.ipo_swish_i8.argtypes = [P, ctypes.c_longlong, P, P]
+            lib.ipo_swish_i8.restype = ctypes.c_int
             for f in (lib.ipo_relpos_mhsa_i8, lib.ipo_content_scores_i32,
                       lib.ipo_position_scores_i32, lib.ipo_fused_scores_i8,
                       lib.ipo_isoftmax_u8, lib.ipo_set_threads):
@@ -197,7 +200,22 @@ def linear(x, w, bias, m, s, *, x_layout: int = ROWS, y_layout: int = ROWS, grou
     return y
 
 
-__all__ = ["build", "linear", "linear_constants", "ROWS", "HEADS", "relpos_mhsa", "content_scores", "position_scores",
+class _Swish(ctypes.Structure):
+    _fields_ = [("q_c", ctypes.c_int32), ("q_one", ctypes.c_int32), ("m", ctypes.c_int32),
+                ("s", ctypes.c_int32)]
+
+
+def swish(z, p: SwishParams) -> np.ndarray:
+    """Integer minimax Swish (Eqs. 12-13) of int8 values on grid S_z, int8
+    on grid S_y (constants from :func:`swish_params`)."""
+    z = np.ascontiguousarray(z, dtype=np.int8)
+    y = np.empty_like(z)
+    prm = _Swish(p.q_c, p.q_one, p.m, p.s)
+    _check(_load().ipo_swish_i8(_ptr(z), z.size, ctypes.addressof(prm), _ptr(y)), "ipo_swish_i8")
+    return y
+
+
+__all__ = ["build", "linear", "swish", "swish_params", "SwishParams", "SWISH_A", "SWISH_C", "linear_constants", "ROWS", "HEADS", "relpos_mhsa", "content_scores", "position_scores",
            "fused_scores", "iexp", "isoftmax", "set_threads", "dyadic",
            "dyadic_pair", "isoftmax_params", "layer_constants", "LayerConstants",
            "IBERT_A", "IBERT_B", "IBERT_C", "OracleError"]

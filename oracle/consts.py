@@ -101,3 +101,31 @@ def linear_constants(s_x: float, s_w, s_y) -> tuple[np.ndarray, np.ndarray]:
     for n in range(s_w.size):
         m[n], s[n] = dyadic(float(s_x) * float(s_w[n]) / float(s_y[n]))
     return m, s
+
+
+# Minimax fit of Eq. 13 (Sec. 3.2): tanh(u) ~ sgn(u) [a (min(|u|, c) - c)^2 + 1]
+SWISH_A = -0.1240
+SWISH_C = 2.4632
+
+
+@dataclass(frozen=True)
+class SwishParams:
+    q_c: int
+    q_one: int
+    m: int
+    s: int
+
+
+def swish_params(s_z: float, s_y: float, a: float = SWISH_A, c: float = SWISH_C) -> SwishParams:
+    """Integer constants of the Swish of Eqs. 12-13 for an int8 input on
+    grid S_z and an int8 output on grid S_y (offline, float64): the clip
+    point q_c = round(2c / S_z) of |z|, the 1 of the polynomial on its grid
+    S_t = |a| (S_z/2)^2, q_one = round(1 / S_t), and the dyadic m 2^-(31+s)
+    of S_z S_t / (2 S_y)."""
+    if not (a < 0 and c > 0 and s_z > 0 and s_y > 0):
+        raise ValueError("need a < 0, c > 0 and positive grids")
+    s_t = abs(a) * (s_z / 2.0) ** 2
+    q_c = int(math.floor(2.0 * c / s_z + 0.5))
+    q_one = int(math.floor(1.0 / s_t + 0.5))
+    m, s = dyadic(s_z * s_t / (2.0 * s_y))
+    return SwishParams(q_c, q_one, m, s)

@@ -10,6 +10,10 @@
  *          by m and one rounding right shift by n = 31 + s onto the int8
  *          grid of y.  A bias, where the layer has one, is an integer on
  *          the accumulator's grid S_W S_x and is added before the shift.
+ *   Eqs. 12-13  Swish sw(x) = x sigma(x) = x (1 + tanh(x / 2)) / 2 with
+ *          tanh(u) ~ sgn(u) [a (min(|u|, c) - c)^2 + 1], (a, c) the minimax
+ *          fit (a* = -0.1240, c* = 2.4632), evaluated on integers of the
+ *          input grid; the constants come from consts.swish_params.
  */
 #include "ipo_linear.h"
 
@@ -86,4 +90,27 @@ int ipo_linear_i8(const int8_t *x, int x_layout, const int8_t *w, const int32_t 
         free(xr);
     }
     return err;
+}
+
+int ipo_swish_i8(const int8_t *z, long long n, const ipo_swish_params *p, int8_t *y) {
+    if (n < 0) return IPO_ERR_SHAPE;
+    if (n == 0) return IPO_OK;
+    if (!z || !p || !y) return IPO_ERR_NULL;
+    if (p->q_c < 1 || p->q_c >= (1 << 15) || p->q_one < 1 || p->q_one >= (1 << 23) ||
+        (int64_t)p->q_one < (int64_t)p->q_c * p->q_c || p->m < 0 || p->s < 0 || p->s > 31)
+        return IPO_ERR_PARAM;
+    int e = 31 + p->s;
+    for (long long i = 0; i < n; ++i) {
+        int64_t q = z[i];
+        int64_t a = q < 0 ? -q : q;                    /* |u| on the grid S_z / 2 */
+        int64_t dclip = (a < p->q_c ? a : p->q_c) - p->q_c;
+        int64_t L = (int64_t)p->q_one - dclip * dclip; /* |tanh|, grid S_t */
+        int64_t sg = q > 0 ? 1 : (q < 0 ? -1 : 0);
+        int64_t t = (int64_t)p->q_one + sg * L;        /* 1 + tanh */
+        int64_t v = lin_floor_pow2((int64_t)p->m * (q * t) + ((int64_t)1 << (e - 1)), e);
+        if (v > 127) v = 127;
+        if (v < -127) v = -127;
+        y[i] = (int8_t)v;
+    }
+    return IPO_OK;
 }

@@ -36,6 +36,24 @@ int ipo_linear_i8(const int8_t *x, int x_layout, const int8_t *w, const int32_t 
                   const int32_t *m, const int32_t *s, int B, int T, int K, int N, int G,
                   int8_t *y, int y_layout);
 
+/* Integer constants of the minimax Swish (Sec. 3.2, Eqs. 12-13) for an
+ * int8 input on grid S_z and an int8 output on grid S_y:
+ *   q_c   = round(2 c* / S_z)                 clip point of |z| (|u| >= c*)
+ *   q_one = round(1 / (|a*| (S_z / 2)^2))     the constant 1 on the grid
+ *                                             S_t = |a*| (S_z / 2)^2
+ *   m, s  : m 2^-(31+s) = S_z S_t / (2 S_y)   output requantisation */
+typedef struct {
+    int32_t q_c, q_one, m, s;
+} ipo_swish_params;
+
+/* Integer Swish of n int8 values (Eqs. 12-13, a* < 0):
+ *   D = min(|z|, q_c) - q_c;  L = q_one - D^2      (|tanh| on the grid S_t)
+ *   t = q_one + sgn(z) L                           (1 + tanh(z S_z / 2))
+ *   y = clamp(round(2^-(31+s) m z t), -127, 127)   (z (1 + tanh) / 2)
+ * Needs 1 <= q_c < 2^15, 1 <= q_one < 2^23, q_one >= q_c^2, m in [0, 2^31),
+ * s in [0, 31]. */
+int ipo_swish_i8(const int8_t *z, long long n, const ipo_swish_params *p, int8_t *y);
+
 #ifdef __cplusplus
 }
 #endif

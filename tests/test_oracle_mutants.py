@@ -56,13 +56,27 @@ LINEAR_MUTANTS = {
     # shift one short
     "lin_shift": ("int e = 31 + s[n];", "int e = 30 + s[n];"),
     # asymmetric clamp (the int8 grid is symmetric, Eq. 6)
-    "lin_clamp": ("if (v < -127) v = -127;", "if (v < -128) v = -128;"),
+    "lin_clamp": ("if (v < -127) v = -127;\n            y[act_index",
+                  "if (v < -128) v = -128;\n            y[act_index"),
     # head index of the head-split layout swapped with the frame
     "lin_heads": ("* heads + (size_t)(cc / 128)) * T + t) * 128",
                   "* T + t) * heads + (size_t)(cc / 128)) * 128"),
 }
 
-LINEAR_PINS = ["tests/test_oracle_linear.py"]
+LINEAR_MUTANTS.update({
+    # Swish with the sign of tanh dropped (sigma(x) = (1 + |tanh|) / 2)
+    "swish_sign": ("int64_t t = (int64_t)p->q_one + sg * L;", "int64_t t = (int64_t)p->q_one + L;"),
+    # Swish without the clip at c (the parabola turns back up)
+    "swish_clip": ("int64_t dclip = (a < p->q_c ? a : p->q_c) - p->q_c;",
+                   "int64_t dclip = a - p->q_c;"),
+    # tanh = q_one + D^2 (sign of a lost)
+    "swish_a_sign": ("int64_t L = (int64_t)p->q_one - dclip * dclip;",
+                     "int64_t L = (int64_t)p->q_one + dclip * dclip;"),
+    # x (1 + tanh) without the halving: output shift one short
+    "swish_half": ("int e = 31 + p->s;\n    for", "int e = 30 + p->s;\n    for"),
+})
+
+LINEAR_PINS = ["tests/test_oracle_linear.py", "tests/test_oracle_swish.py"]
 
 PINS = [
     "tests/test_oracle_relshift.py",
