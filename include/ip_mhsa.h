@@ -193,6 +193,35 @@ int ip_linear_i8(const int8_t *x, int x_layout, const int8_t *w, const int32_t *
                  int8_t *y, int y_layout, void *workspace, size_t workspace_bytes,
                  ip_stream_t stream);
 
+/* ---- minimax integer Swish (Sec. 3.2, Eqs. 12-13) ----------------------
+ *
+ * Swish sw(x) = x (1 + tanh(x/2)) / 2 with tanh(u) ~ sgn(u) [a (min(|u|, c)
+ * - c)^2 + 1] and the paper's minimax fit (a, c) below, on int8 inputs z of
+ * grid S_z and int8 outputs of grid S_y:
+ *   D = min(|z|, q_c) - q_c;  L = q_one - D^2;  t = q_one + sgn(z) L
+ *   y = clamp(round(2^-(31+s) m z t), -127, 127)
+ * q_c = round(2c / S_z) is the clip point of |z|, q_one = round(1 / S_t)
+ * the 1 of the polynomial on its grid S_t = |a| (S_z/2)^2, and m 2^-(31+s)
+ * is S_z S_t / (2 S_y).  Domain: 1 <= q_c < 2^15, 1 <= q_one < 2^23,
+ * q_one >= q_c^2, m in [0, 2^31), s in [0, 31]. */
+#define IP_SWISH_A (-0.1240)
+#define IP_SWISH_C 2.4632
+
+typedef struct {
+    int32_t q_c, q_one, m, s;
+} ip_swish_params;
+
+/* The feed-forward layer's first projection with the Swish fused into its
+ * epilogue: z = ip_linear_i8's output (row-major, G = 1; m, s put z on the
+ * grid S_z), then y = Swish(z) on S_y.  Arguments as ip_linear_i8 (x and y
+ * IP_LAYOUT_ROWS); sw: host, validated (IP_ERR_PARAM outside its domain). */
+int ip_linear_swish_i8(const int8_t *x, const int8_t *w, const int32_t *bias, const int32_t *m,
+                       const int32_t *s, const ip_swish_params *sw, int B, int T, int K, int N,
+                       int8_t *y, void *workspace, size_t workspace_bytes, ip_stream_t stream);
+
+/* Swish constants for the grids S_z (input) and S_y (output), host only. */
+int ip_swish_params_from_scales(double S_z, double S_y, ip_swish_params *out);
+
 /* Text of an IP_* code. */
 const char *ip_strerror(int code);
 

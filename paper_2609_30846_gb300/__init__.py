@@ -30,7 +30,7 @@ EXPORTS = (
     "ip_debug_set_timeout_cycles", "ip_debug_set_stall_injection", "ip_dyadic_multiplier",
     "ip_dyadic_pair",
     "ip_isoftmax_params_from_scale", "ip_probe_int8_mma", "ip_relpos_mhsa_i8_noalloc",
-    "ip_debug_set_split_mode", "ip_linear_i8",
+    "ip_debug_set_split_mode", "ip_linear_i8", "ip_linear_swish_i8", "ip_swish_params_from_scales",
 )
 
 ROWS = 0    # IP_LAYOUT_ROWS:  [B][T][C]
@@ -47,6 +47,11 @@ class IpError(RuntimeError):
     def __init__(self, fn: str, code: int, text: str):
         super().__init__(f"{fn}: {ERRORS.get(code, code)} ({text})")
         self.code = code
+
+
+class SwishParams(ctypes.Structure):
+    _fields_ = [("q_c", ctypes.c_int32), ("q_one", ctypes.c_int32), ("m", ctypes.c_int32),
+                ("s", ctypes.c_int32)]
 
 
 class SoftmaxParams(ctypes.Structure):
@@ -105,6 +110,12 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
         lib.ip_isoftmax_params_from_scale.restype = I
         lib.ip_linear_i8.argtypes = [P, I, P, P, P, P, I, I, I, I, I, P, I, P, ctypes.c_size_t, P]
         lib.ip_linear_i8.restype = I
+        lib.ip_linear_swish_i8.argtypes = [P, P, P, P, P, ctypes.POINTER(SwishParams), I, I, I, I,
+                                           P, P, ctypes.c_size_t, P]
+        lib.ip_linear_swish_i8.restype = I
+        lib.ip_swish_params_from_scales.argtypes = [ctypes.c_double, ctypes.c_double,
+                                                    ctypes.POINTER(SwishParams)]
+        lib.ip_swish_params_from_scales.restype = I
         lib.ip_probe_int8_mma.argtypes = [I, I, P, P]
         lib.ip_probe_int8_mma.restype = ctypes.c_longlong
         _lib = lib
@@ -315,6 +326,38 @@ def linear_i8(x, w, bias, m, s, *, x_layout: int = ROWS, y_layout: int = ROWS, g
     return out
 
 
+def swish_params_from_scales(S_z: float, S_y: float) -> tuple[int, int, int, int]:
+    """Integer constants (q_c, q_one, m, s) of the minimax Swish for an int8
+    input on grid S_z and an int8 output on grid S_y (Eqs. 12-13)."""
+    prm = SwishParams()
+    _check("ip_swish_params_from_scales",
+           load().ip_swish_params_from_scales(S_z, S_y, ctypes.byref(prm)))
+    return prm.q_c, prm.q_one, prm.m, prm.s
+
+
+def linear_swish_i8(x, w, bias, m, s, swish: tuple[int, int, int, int], *, out=None,
+                    workspace=None, stream=None):
+    """Feed-forward projection with the fused minimax Swish: x int8 [B, T, K],
+    w int8 [N, K], bias int32 [N] or None, m, s int32 [N] (onto the Swish
+    input grid), swish = (q_c, q_one, m, s).  Returns int8 [B, T, N]."""
+    import torch
+    N, K = w.shape
+    B, T, _ = x.shape
+    if out is None:
+        out = torch.empty((B, T, N), dtype=torch.int8, device=w.device)
+    if workspace is None:
+        workspace = torch.zeros(256, dtype=torch.uint8, device=w.device)
+    bp = None if bias is None else _dev_ptr(bias, "bias", torch.int32, (N,))
+    sw = SwishParams(*swish)
+    rc = load().ip_linear_swish_i8(
+        _dev_ptr(x, "x", torch.int8, (B, T, K)), _dev_ptr(w, "w", torch.int8, (N, K)), bp,
+        _dev_ptr(m, "m", torch.int32, (N,)), _dev_ptr(s, "s", torch.int32, (N,)), ctypes.byref(sw),
+        B, T, K, N, _dev_ptr(out, "out", torch.int8, (B, T, N)),
+        ctypes.c_void_p(workspace.data_ptr()), workspace.numel(), _stream_handle(stream))
+    _check("ip_linear_swish_i8", rc)
+    return out
+
+
 def relpos_mhsa_i8_host(q, k, v, p, u, v_bias, consts: LayerConstants, lengths, out, arena,
                         stream=None):
     """Whole layer from host buffers (torch CPU tensors, ideally pinned):
@@ -344,5 +387,5 @@ __all__ = ["build", "load", "relpos_mhsa_i8", "relpos_mhsa_i8_host", "status", "
            "host_arena_bytes", "layer_constants", "LayerConstants", "dyadic_multiplier",
            "dyadic_pair", "isoftmax_params_from_scale", "set_timeout_cycles", "strerror",
            "int8_mma_peak_tops", "set_stall_injection", "set_split_mode", "linear_i8",
-           "linear_constants", "ROWS", "HEADS",
+           "linear_constants", "ROWS", "HEADS", "linear_swish_i8", "swish_params_from_scales",
            "IpError", "LibraryError", "EXPORTS"]

@@ -7,6 +7,7 @@
 #include <cuda.h>
 #include <cuda_runtime.h>
 
+#include <cmath>
 #include <mutex>
 
 namespace {
@@ -75,21 +76,29 @@ int ensure_smem() {
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return IP_ERR_CUDA;
     std::lock_guard<std::mutex> lock(g_mu);
     if (g_smem_set[dev]) return IP_OK;
-    if (cudaFuncSetAttribute(ipl::linear_i8_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    if (cudaFuncSetAttribute(ipl::linear_i8_kernel<false>,
+                             cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             ipl::SMEM_LAUNCH) != cudaSuccess ||
+        cudaFuncSetAttribute(ipl::linear_i8_kernel<true>,
+                             cudaFuncAttributeMaxDynamicSharedMemorySize,
                              ipl::SMEM_LAUNCH) != cudaSuccess)
         return IP_ERR_CUDA;
     g_smem_set[dev] = 1;
     return IP_OK;
 }
 
-}  // namespace
+int check_swish(const ip_swish_params *p) {
+    if (p->q_c < 1 || p->q_c >= (1 << 15) || p->q_one < 1 || p->q_one >= (1 << 23) ||
+        static_cast<long long>(p->q_one) < static_cast<long long>(p->q_c) * p->q_c ||
+        p->m < 0 || p->s < 0 || p->s > 31)
+        return IP_ERR_PARAM;
+    return IP_OK;
+}
 
-extern "C" {
-
-int ip_linear_i8(const int8_t *x, int x_layout, const int8_t *w, const int32_t *bias,
-                 const int32_t *m, const int32_t *s, int B, int T, int K, int N, int G,
-                 int8_t *y, int y_layout, void *workspace, size_t workspace_bytes,
-                 ip_stream_t stream) {
+int linear_launch(const int8_t *x, int x_layout, const int8_t *w, const int32_t *bias,
+                  const int32_t *m, const int32_t *s, const ip_swish_params *sw, int B, int T,
+                  int K, int N, int G, int8_t *y, int y_layout, void *workspace,
+                  size_t workspace_bytes, ip_stream_t stream) {
     if ((x_layout != IP_LAYOUT_ROWS && x_layout != IP_LAYOUT_HEADS) ||
         (y_layout != IP_LAYOUT_ROWS && y_layout != IP_LAYOUT_HEADS))
         return IP_ERR_PARAM;
@@ -148,13 +157,61 @@ int ip_linear_i8(const int8_t *x, int x_layout, const int8_t *w, const int32_t *
     prm.magic_ntn = div_magic(prm.ntn);
     prm.magic_T = div_magic(T);
     prm.magic_tpu = div_magic(prm.tpu);
+    prm.sw_qc = sw ? sw->q_c : 0;
+    prm.sw_qone = sw ? sw->q_one : 0;
+    prm.sw_m = sw ? sw->m : 0;
+    prm.sw_e = sw ? 31 + sw->s : 0;
     const int nsm = sm_count();
     if (nsm <= 0) return IP_ERR_CUDA;
     const unsigned grid = prm.ntiles < static_cast<unsigned>(nsm) ? prm.ntiles
                                                                   : static_cast<unsigned>(nsm);
-    ipl::linear_i8_kernel<<<grid, ipl::THREADS, ipl::SMEM_LAUNCH,
-                            reinterpret_cast<cudaStream_t>(stream)>>>(tm_x, tm_w, prm);
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    if (sw)
+        ipl::linear_i8_kernel<true><<<grid, ipl::THREADS, ipl::SMEM_LAUNCH, st>>>(tm_x, tm_w, prm);
+    else
+        ipl::linear_i8_kernel<false><<<grid, ipl::THREADS, ipl::SMEM_LAUNCH, st>>>(tm_x, tm_w, prm);
     if (cudaGetLastError() != cudaSuccess) return IP_ERR_CUDA;
+    return IP_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int ip_linear_i8(const int8_t *x, int x_layout, const int8_t *w, const int32_t *bias,
+                 const int32_t *m, const int32_t *s, int B, int T, int K, int N, int G,
+                 int8_t *y, int y_layout, void *workspace, size_t workspace_bytes,
+                 ip_stream_t stream) {
+    return linear_launch(x, x_layout, w, bias, m, s, nullptr, B, T, K, N, G, y, y_layout,
+                         workspace, workspace_bytes, stream);
+}
+
+int ip_linear_swish_i8(const int8_t *x, const int8_t *w, const int32_t *bias, const int32_t *m,
+                       const int32_t *s, const ip_swish_params *sw, int B, int T, int K, int N,
+                       int8_t *y, void *workspace, size_t workspace_bytes, ip_stream_t stream) {
+    if (!sw) return IP_ERR_NULL;
+    const int rc = check_swish(sw);
+    if (rc != IP_OK) return rc;
+    return linear_launch(x, IP_LAYOUT_ROWS, w, bias, m, s, sw, B, T, K, N, 1, y, IP_LAYOUT_ROWS,
+                         workspace, workspace_bytes, stream);
+}
+
+int ip_swish_params_from_scales(double S_z, double S_y, ip_swish_params *out) {
+    if (!out) return IP_ERR_NULL;
+    if (!(S_z > 0.0) || !(S_y > 0.0) || !std::isfinite(S_z) || !std::isfinite(S_y))
+        return IP_ERR_PARAM;
+    const double a = IP_SWISH_A, c = IP_SWISH_C;
+    const double s_t = -a * (S_z / 2.0) * (S_z / 2.0);
+    const double qc = std::floor(2.0 * c / S_z + 0.5);
+    const double qone = std::floor(1.0 / s_t + 0.5);
+    if (qc < 1.0 || qc >= 32768.0 || qone < 1.0 || qone >= 8388608.0) return IP_ERR_PARAM;
+    ip_swish_params p;
+    p.q_c = static_cast<int32_t>(qc);
+    p.q_one = static_cast<int32_t>(qone);
+    const int rc = ip_dyadic_multiplier(S_z * s_t / (2.0 * S_y), &p.m, &p.s);
+    if (rc != IP_OK) return rc;
+    if (check_swish(&p) != IP_OK) return IP_ERR_PARAM;
+    *out = p;
     return IP_OK;
 }
 

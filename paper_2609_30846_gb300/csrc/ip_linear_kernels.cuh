@@ -13,7 +13,8 @@
 // along the channels, 64 x 32 each) feed the integer warp MMA (mma.sync
 // m16n8k32 s8 x s8 -> s32) from ldmatrix; sm_103a has no integer tcgen05
 // kind.  The epilogue adds the int32 bias, multiplies by m[n] in int64,
-// shifts right by 31 + s[n] with rounding, clamps to [-127, 127] and writes
+// shifts right by 31 + s[n] with rounding, clamps to [-127, 127] (and, in
+// the feed-forward variant, applies the minimax integer Swish) and writes
 // each warp's 64 x 32 bytes through shared memory as 16-byte row segments,
 // either row-major [B][T][N] or head-split [G][B][N/G/128][T][128].
 #pragma once
@@ -40,7 +41,8 @@ constexpr int OUT_ROW = 48;             // staged output row of one warp: 32 byt
 constexpr int OUT_WARP_BYTES = 64 * OUT_ROW;
 constexpr int SMEM_OUT = STAGES * STAGE_BYTES;
 constexpr int SMEM_BARS = SMEM_OUT + NCW * OUT_WARP_BYTES;
-constexpr int SMEM_BYTES = SMEM_BARS + 8 * (2 * STAGES);
+constexpr int SMEM_LUT = SMEM_BARS + 8 * (2 * STAGES);     // Swish of every int8 z
+constexpr int SMEM_BYTES = SMEM_LUT + 256;
 constexpr int SMEM_LAUNCH = SMEM_BYTES + 1024;   // + alignment of the dynamic base
 
 constexpr int LAYOUT_ROWS = 0;
@@ -65,6 +67,8 @@ struct LinearParams {
     int x_layout;
     int *err;
     long long timeout_cycles;
+    // minimax Swish of the requantised output (Eqs. 12-13), SWISH kernels only
+    int sw_qc, sw_qone, sw_m, sw_e;
 };
 
 struct Tile {
@@ -89,6 +93,20 @@ __device__ __forceinline__ Tile tile_of(unsigned idx, const LinearParams &p) {
     return L;
 }
 
+// Integer Swish of one int8 value z on the grid S_z (Eqs. 12-13): the
+// clipped parabola L = q_one - (min(|z|, q_c) - q_c)^2 is |tanh(z S_z / 2)|
+// on the grid S_t, t = q_one + sgn(z) L is 1 + tanh, and z t is requantised
+// onto the output grid.  |z t| < 2^31 since t <= 2 q_one < 2^24.
+__device__ __forceinline__ int swish_i8(int z, const LinearParams &p) {
+    const int a = z < 0 ? -z : z;
+    const int dc = (a < p.sw_qc ? a : p.sw_qc) - p.sw_qc;
+    const int L = p.sw_qone - dc * dc;
+    const int t = z > 0 ? p.sw_qone + L : (z < 0 ? p.sw_qone - L : p.sw_qone);
+    const long long v = static_cast<long long>(p.sw_m) * (z * t) + (1ll << (p.sw_e - 1));
+    return clamp127(v >> p.sw_e);
+}
+
+template <bool SWISH>
 __global__ void __launch_bounds__(THREADS, 1)
     linear_i8_kernel(const __grid_constant__ CUtensorMap tm_x,
                      const __grid_constant__ CUtensorMap tm_w, const LinearParams prm) {
@@ -105,6 +123,8 @@ __global__ void __launch_bounds__(THREADS, 1)
     auto empty_bar = [&](int s) { return bars + 8u * (STAGES + s); };
     auto stage = [&](int s) { return base + s * STAGE_BYTES; };
 
+    const uint32_t lut = base + SMEM_LUT;
+    const uint8_t *swish_lut = smem + SMEM_LUT;
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
             mbar_init(full_bar(s), 1);
@@ -112,6 +132,12 @@ __global__ void __launch_bounds__(THREADS, 1)
         }
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    }
+    if (SWISH && threadIdx.x < 256) {
+        // the Swish of every int8 input, entry at the byte value of z
+        const int z = static_cast<int>(static_cast<int8_t>(static_cast<uint8_t>(threadIdx.x)));
+        const uint32_t y = static_cast<uint32_t>(swish_i8(z, prm)) & 0xffu;
+        asm volatile("st.shared.u8 [%0], %1;" ::"r"(lut + threadIdx.x), "r"(y) : "memory");
     }
     __syncthreads();
 
@@ -163,29 +189,6 @@ __global__ void __launch_bounds__(THREADS, 1)
         const Tile L = tile_of(idx, prm);
         const int n0 = L.nt * BN;
 
-        // per-channel constants of this thread's eight channels (Eq. 7)
-        int cb[8], cm[8], ce[8];
-        bool bad = false;
-#pragma unroll
-        for (int j = 0; j < 4; ++j)
-#pragma unroll
-            for (int q = 0; q < 2; ++q) {
-                const int n = n0 + 32 * wn + 8 * j + 2 * t4 + q;
-                int bi = prm.bias != nullptr ? __ldg(prm.bias + n) : 0;
-                int mi = __ldg(prm.m + n);
-                int si = __ldg(prm.s + n);
-                if (mi < 0 || si < 0 || si > 31 || bi >= (1 << 30) || bi <= -(1 << 30)) {
-                    bad = true;
-                    mi = mi < 0 ? 0 : mi;
-                    si = si < 0 ? 0 : (si > 31 ? 31 : si);
-                    bi = 0;
-                }
-                cb[2 * j + q] = bi;
-                cm[2 * j + q] = mi;
-                ce[2 * j + q] = 31 + si;
-            }
-        if (bad) atomicOr(prm.err, ERR_PARAM);
-
         int acc[4][4][4];
 #pragma unroll
         for (int i = 0; i < 4; ++i)
@@ -222,6 +225,30 @@ __global__ void __launch_bounds__(THREADS, 1)
         }
 
         // ------------------------------------------------------ epilogue
+        // per-channel constants of this thread's eight channels (Eq. 7), loaded after
+        // the main loop so that they hold no registers during it
+        int cb[8], cm[8], ce[8];
+        bool bad = false;
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+#pragma unroll
+            for (int q = 0; q < 2; ++q) {
+                const int n = n0 + 32 * wn + 8 * j + 2 * t4 + q;
+                int bi = prm.bias != nullptr ? __ldg(prm.bias + n) : 0;
+                int mi = __ldg(prm.m + n);
+                int si = __ldg(prm.s + n);
+                if (mi < 0 || si < 0 || si > 31 || bi >= (1 << 30) || bi <= -(1 << 30)) {
+                    bad = true;
+                    mi = mi < 0 ? 0 : mi;
+                    si = si < 0 ? 0 : (si > 31 ? 31 : si);
+                    bi = 0;
+                }
+                cb[2 * j + q] = bi;
+                cm[2 * j + q] = mi;
+                ce[2 * j + q] = 31 + si;
+            }
+        if (bad) atomicOr(prm.err, ERR_PARAM);
+
 #pragma unroll
         for (int i = 0; i < 4; ++i)
 #pragma unroll
@@ -235,7 +262,9 @@ __global__ void __launch_bounds__(THREADS, 1)
                         const long long v = static_cast<long long>(cm[c]) *
                                                 (acc[i][j][2 * rr + q] + cb[c]) +
                                             (1ll << (ce[c] - 1));
-                        two |= (static_cast<uint32_t>(clamp127(v >> ce[c])) & 0xffu) << (8 * q);
+                        uint32_t o = static_cast<uint32_t>(clamp127(v >> ce[c])) & 0xffu;
+                        if (SWISH) o = swish_lut[o];
+                        two |= o << (8 * q);
                     }
                     const int r = 16 * i + g + 8 * rr;
                     asm volatile("st.shared.u16 [%0], %1;" ::"r"(ob + r * OUT_ROW + 8 * j + 2 * t4),

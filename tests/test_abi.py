@@ -184,3 +184,25 @@ def test_exact_division_constant():
         for n in ns:
             if 0 <= n < 2 ** 32:
                 assert (n * M) >> 64 == n // d, (n, d)
+
+
+@pytest.mark.parametrize("s_z,s_y", [(8 / 127, 8 / 127), (6 / 127, 7 / 127), (0.2, 0.05),
+                                     (3e-3, 2e-3)])
+def test_swish_constants_match_oracle(lib, s_z, s_y):
+    import oracle
+    want = oracle.swish_params(s_z, s_y)
+    assert ip.swish_params_from_scales(s_z, s_y) == (want.q_c, want.q_one, want.m, want.s)
+
+
+def test_swish_validation(lib):
+    with pytest.raises(ip.IpError):
+        ip.swish_params_from_scales(0.0, 0.1)
+    with pytest.raises(ip.IpError):
+        ip.swish_params_from_scales(1e-6, 0.1)      # q_one beyond 2^23
+    P = ctypes.c_void_p
+    fake = P(1 << 20)
+    bad = ip.SwishParams(20, 100, 2 ** 30, 0)          # q_one < q_c^2
+    assert lib.ip_linear_swish_i8(fake, fake, None, fake, fake, ctypes.byref(bad), 1, 4, 128, 128,
+                                  fake, P(1 << 21), 256, None) == -7
+    assert lib.ip_linear_swish_i8(fake, fake, None, fake, fake, None, 1, 4, 128, 128,
+                                  fake, P(1 << 21), 256, None) == -1

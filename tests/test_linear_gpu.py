@@ -149,3 +149,38 @@ def test_encoder_output_projection_full_size(ip, orc):
     got, want, st = run_both(ip, orc, xh, c.w, c.bias, m, s, x_layout=1)
     assert st == 0
     assert_same(got, want)
+
+
+def swish_case(orc, B, T, K, N, seed):
+    """FFN first projection: z on an int8 grid S_z (the linear layer's output
+    grid), then the Swish onto S_y."""
+    c = synth.linear(B, T, K, N, seed=seed)
+    m, s = orc.linear_constants(c.s_x, c.s_w, c.s_y_per_channel())
+    s_z = float(c.s_y[0])
+    sw = orc.swish_params(s_z, 0.9 * s_z)
+    return c, m, s, sw
+
+
+def run_swish(ip, orc, c, m, s, sw):
+    ws = torch.zeros(256, dtype=torch.uint8, device="cuda")
+    got = ip.linear_swish_i8(_d(c.x), _d(c.w), None if c.bias is None else _d(c.bias), _d(m),
+                             _d(s), (sw.q_c, sw.q_one, sw.m, sw.s), workspace=ws)
+    st = ip.status(ws)
+    z = orc.linear(c.x, c.w, c.bias, m, s)
+    return got.cpu().numpy(), orc.swish(z, sw), st
+
+
+@pytest.mark.parametrize("B,T,K,N", [(1, 1, 128, 128), (2, 77, 256, 384), (3, 200, 1024, 512)])
+def test_linear_swish(ip, orc, B, T, K, N):
+    c, m, s, sw = swish_case(orc, B, T, K, N, seed=900 + T)
+    got, want, st = run_swish(ip, orc, c, m, s, sw)
+    assert st == 0
+    assert_same(got, want)
+
+
+def test_ffn_first_projection_full_size(ip, orc):
+    # FFN of one encoder block: B=32, T=375, 1024 -> 4096 with the Swish
+    c, m, s, sw = swish_case(orc, 32, 375, 1024, 4096, seed=3003)
+    got, want, st = run_swish(ip, orc, c, m, s, sw)
+    assert st == 0
+    assert_same(got, want)
