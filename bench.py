@@ -63,6 +63,10 @@ def parse_args():
                     help="profiling only: fewer layers than the workload's 24")
     ap.add_argument("--batch", type=int, default=None,
                     help="profiling only: fewer utterances than the workload's 32")
+    ap.add_argument("--no-next-rows", action="store_true",
+                    help="skip the projection and feed-forward measurements")
+    ap.add_argument("--rows-only", action="store_true",
+                    help="profiling: only the projection and feed-forward measurements")
     return ap.parse_args()
 
 
@@ -248,6 +252,97 @@ def run_reference(args):
     return 0
 
 
+# ------------------------------------------------------------------- next rows
+
+# The projections around the attention of one encoder block (B=32, T=375,
+# d=1024): Q/K/V stacked and written head-split, the output projection from
+# the heads, and the feed-forward pair with the fused minimax Swish.
+NEXT_ROWS = [
+    # name, K, N, groups, x_layout, y_layout, swish
+    ("linear_qkv_1024x3072_heads", 1024, 3072, 3, 0, 1, False),
+    ("linear_out_heads_1024x1024", 1024, 1024, 1, 1, 0, False),
+    ("ffn1_swish_1024x4096", 1024, 4096, 1, 0, 0, True),
+    ("ffn2_4096x1024", 4096, 1024, 1, 0, 0, False),
+]
+
+
+def measure_next_rows(dev, peak, steps: int, cpu: bool):
+    """Each projection timed alone (CUDA events per launch, L2 flushed before
+    every timed launch), useful ops 2 B T K N, against the measured INT8
+    MMA peak; with `cpu`, the oracle on a bounded sample of frames."""
+    import torch
+    import paper_2609_30846_gb300 as ip
+    w0 = synth.WORKLOADS[WORKLOAD]
+    B, T = w0.B, w0.T
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    rows = {}
+    for name, K, N, G, xl, yl, sw in NEXT_ROWS:
+        case = synth.linear(B, T, K, N, seed=7000 + K + N + G, groups=G)
+        m, s = ip.linear_constants(case.s_x, case.s_w, case.s_y_per_channel())
+        x = torch.from_numpy(case.x).to(dev)
+        if xl == 1:
+            x = x.reshape(B, T, K // 128, 128).permute(0, 2, 1, 3).contiguous()
+        w = torch.from_numpy(case.w).to(dev)
+        b = torch.from_numpy(case.bias).to(dev)
+        md, sd = torch.from_numpy(m).to(dev), torch.from_numpy(s).to(dev)
+        ws = torch.zeros(256, dtype=torch.uint8, device=dev)
+        swp = ip.swish_params_from_scales(float(case.s_y[0]), 0.9 * float(case.s_y[0])) if sw else None
+        if sw:
+            out = torch.empty((B, T, N), dtype=torch.int8, device=dev)
+            call = lambda: ip.linear_swish_i8(x, w, b, md, sd, swp, out=out, workspace=ws,
+                                              stream=stream)
+        else:
+            ys = (B, T, N) if yl == 0 else (G, B, N // G // 128, T, 128)
+            out = torch.empty(ys, dtype=torch.int8, device=dev)
+            call = lambda: ip.linear_i8(x, w, b, md, sd, x_layout=xl, y_layout=yl, groups=G,
+                                        out=out, workspace=ws, stream=stream)
+        for _ in range(3):
+            call()
+        times = []
+        for _ in range(steps):
+            flush.zero_()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            call()
+            e1.record(stream)
+            e1.synchronize()
+            times.append(e0.elapsed_time(e1) * 1e-3)
+        if ip.status(ws, stream) != 0:
+            raise SystemExit(f"{name}: kernel reported an error")
+        t = statistics.median(times)
+        ops = 2.0 * B * T * K * N
+        row = {"value": ops / t / 1e12, "unit": "TOPS", "us_per_launch": t * 1e6,
+               "shape": {"B": B, "T": T, "K": K, "N": N, "groups": G,
+                         "x": "heads" if xl else "rows", "y": "heads" if yl else "rows",
+                         "swish": sw},
+               "roofline": {"bound": "tensor", "achieved": ops / t / 1e12, "peak": peak,
+                            "unit": "TOPS", "frac": ops / t / 1e12 / peak, "traffic": None},
+               "kernel": "linear_i8_kernel" + ("<swish>" if sw else ""), "gpu_launches": 1}
+        if cpu:
+            import oracle
+            oracle.build()
+            def run(frames):
+                xs = case.x.reshape(-1, K)[:frames].reshape(1, frames, K)
+                t0 = time.perf_counter()
+                z = oracle.linear(xs, case.w, case.bias, m, s)
+                if sw:
+                    oracle.swish(z, oracle.SwishParams(*swp))
+                return time.perf_counter() - t0
+            # a sample of about one second of oracle work
+            frames = 32
+            dt = run(frames)
+            frames = int(min(B * T, max(32, frames * 1.0 / max(dt, 1e-4))))
+            dt = run(frames)
+            row["cpu_baseline"] = {"value": 2.0 * frames * K * N / dt / 1e12, "unit": "TOPS",
+                                   "cores": os.cpu_count() or 1, "kind": "oracle",
+                                   "sample": f"{frames} frames of {B * T}, {dt:.2f} s"}
+        rows[name] = row
+        del x, w, b, out
+    del flush
+    return rows
+
+
 # ------------------------------------------------------------------- GPU arm
 
 def run_ours(args):
@@ -264,6 +359,13 @@ def run_ours(args):
         import torch.distributed as dist
         dist.init_process_group("nccl", device_id=dev)
     ip.load()
+    if args.rows_only:
+        if rank == 0:
+            rows = measure_next_rows(dev, ip.int8_mma_peak_tops(), max(args.steps, 1), cpu=False)
+            print(json.dumps({"next_rows": rows}), flush=True)
+        if dist:
+            dist.destroy_process_group()
+        return 0
 
     w = synth.WORKLOADS[WORKLOAD]
     B, H, T, dh, NL = w.B, w.H, w.T, w.dh, w.layers
@@ -378,6 +480,10 @@ def run_ours(args):
     cpu = None
     if world == 1 and not args.no_cpu_baseline:
         cpu = cpu_sample(layers, os.cpu_count() or 1, args.cpu_seconds)
+    next_rows = None
+    if not args.no_next_rows and not reduced:
+        next_rows = measure_next_rows(dev, peak, max(args.steps, 5),
+                                      cpu=world == 1 and not args.no_cpu_baseline)
 
     bytes_layer = 4 * B * H * T * dh + H * (2 * T - 1) * dh + 2 * H * dh
     line = {
@@ -401,6 +507,7 @@ def run_ours(args):
         "e2e": e2e,
         "gpu_launches": NL * args.steps,
         "clocks": clk,
+        "next_rows": next_rows,
     }
     print(json.dumps(line), flush=True)
     if dist:
