@@ -23,11 +23,12 @@ import numpy as np
 
 from .consts import (IBERT_A, IBERT_B, IBERT_C, LayerConstants, dyadic,
                      dyadic_pair, isoftmax_params, layer_constants, linear_constants,
-                     SWISH_A, SWISH_C, SwishParams, swish_params)
+                     SWISH_A, SWISH_C, SwishParams, swish_params, NormConstants,
+                     layernorm_constants)
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
-_SRCS = [os.path.join(_HERE, f) for f in ("ipo_mhsa.c", "ipo_linear.c")]
-_HDRS = [os.path.join(_HERE, f) for f in ("ipo_mhsa.h", "ipo_linear.h")]
+_SRCS = [os.path.join(_HERE, f) for f in ("ipo_mhsa.c", "ipo_linear.c", "ipo_norm.c")]
+_HDRS = [os.path.join(_HERE, f) for f in ("ipo_mhsa.h", "ipo_linear.h", "ipo_norm.h")]
 _LIB = os.path.join(_HERE, "libipo_mhsa.so")
 _lock = threading.Lock()
 _lib = None
@@ -71,6 +72,11 @@ def _load():
             lib.ipo_linear_i8.restype = ctypes.c_int
             lib.ipo_swish_i8.argtypes = [P, ctypes.c_longlong, P, P]
             lib.ipo_swish_i8.restype = ctypes.c_int
+            lib.ipo_isqrt.argtypes = [ctypes.c_int64]
+            lib.ipo_isqrt.restype = ctypes.c_int64
+            lib.ipo_layernorm_i8.argtypes = [P, ctypes.c_longlong, ctypes.c_int, ctypes.c_int64,
+                                             P, P, P, P]
+            lib.ipo_layernorm_i8.restype = ctypes.c_int
             for f in (lib.ipo_relpos_mhsa_i8, lib.ipo_content_scores_i32,
                       lib.ipo_position_scores_i32, lib.ipo_fused_scores_i8,
                       lib.ipo_isoftmax_u8, lib.ipo_set_threads):
@@ -215,7 +221,28 @@ def swish(z, p: SwishParams) -> np.ndarray:
     return y
 
 
-__all__ = ["build", "linear", "swish", "swish_params", "SwishParams", "SWISH_A", "SWISH_C", "linear_constants", "ROWS", "HEADS", "relpos_mhsa", "content_scores", "position_scores",
+def isqrt(n: int) -> int:
+    """floor(sqrt(n)) of the oracle's integer Newton iteration, 0 <= n < 2^62."""
+    return int(_load().ipo_isqrt(int(n)))
+
+
+def layernorm(x, c: "NormConstants") -> np.ndarray:
+    """Integer LayerNorm over the last axis (d channels) of int8 x; constants
+    from :func:`layernorm_constants`."""
+    x = np.ascontiguousarray(x, dtype=np.int8)
+    d = x.shape[-1]
+    rows = x.size // d
+    y = np.empty_like(x)
+    M = np.ascontiguousarray(c.M, dtype=np.int32)
+    B = np.ascontiguousarray(c.B, dtype=np.int64)
+    E = np.ascontiguousarray(c.E, dtype=np.int32)
+    _check(_load().ipo_layernorm_i8(_ptr(x), rows, d, int(c.eps_c), _ptr(M), _ptr(B), _ptr(E),
+                                    _ptr(y)), "ipo_layernorm_i8")
+    return y
+
+
+__all__ = ["build", "linear", "swish", "isqrt", "layernorm", "layernorm_constants",
+           "NormConstants", "swish_params", "SwishParams", "SWISH_A", "SWISH_C", "linear_constants", "ROWS", "HEADS", "relpos_mhsa", "content_scores", "position_scores",
            "fused_scores", "iexp", "isoftmax", "set_threads", "dyadic",
            "dyadic_pair", "isoftmax_params", "layer_constants", "LayerConstants",
            "IBERT_A", "IBERT_B", "IBERT_C", "OracleError"]

@@ -129,3 +129,40 @@ def swish_params(s_z: float, s_y: float, a: float = SWISH_A, c: float = SWISH_C)
     q_one = int(math.floor(1.0 / s_t + 0.5))
     m, s = dyadic(s_z * s_t / (2.0 * s_y))
     return SwishParams(q_c, q_one, m, s)
+
+
+@dataclass(frozen=True)
+class NormConstants:
+    eps_c: int            # epsilon on the grid of c^2, c = d (q - mean)
+    M: np.ndarray         # int32 [d]
+    B: np.ndarray         # int64 [d]
+    E: np.ndarray         # int32 [d], total right shift
+
+
+def layernorm_constants(s_x: float, gamma, beta, s_y: float, eps: float = 1e-5) -> NormConstants:
+    """Integer constants of the LayerNorm for an int8 input on grid S_x and
+    an int8 output on S_y (offline, float64).  The normalised value reaches
+    the affine step as n = (x - mean) / sqrt(var + eps) on the grid 2^-15;
+    per channel y = (gamma_i 2^-15 n + beta_i) / S_y = (M_i n + B_i) 2^-E_i,
+    with (|M_i|, E_i - 31) the dyadic of |gamma_i| 2^-15 / S_y (sign of
+    gamma_i on M_i; gamma_i = 0 gives M_i = 0, E_i = 31) and B_i =
+    round(beta_i / S_y 2^E_i).  eps_c = round(eps d^2 / S_x^2): var in units
+    of c^2 / d where c = d (q - mean)."""
+    gamma = np.asarray(gamma, dtype=np.float64)
+    beta = np.asarray(beta, dtype=np.float64)
+    d = gamma.size
+    M = np.zeros(d, dtype=np.int32)
+    E = np.full(d, 31, dtype=np.int32)
+    B = np.zeros(d, dtype=np.int64)
+    for i in range(d):
+        g = float(gamma[i])
+        if g != 0.0:
+            m, s = dyadic(abs(g) * 2.0 ** -15 / s_y)
+            M[i] = m if g > 0 else -m
+            E[i] = 31 + s
+        b = math.floor(float(beta[i]) / s_y * 2.0 ** int(E[i]) + 0.5)
+        if abs(b) >= 2 ** 61:
+            raise ValueError(f"beta/gamma ratio of channel {i} out of range")
+        B[i] = b
+    eps_c = int(math.floor(eps * d * d / (s_x * s_x) + 0.5))
+    return NormConstants(eps_c, M, B, E)

@@ -78,6 +78,26 @@ LINEAR_MUTANTS.update({
 
 LINEAR_PINS = ["tests/test_oracle_linear.py", "tests/test_oracle_swish.py"]
 
+# mistakes planted in the LayerNorm oracle
+NORM_MUTANTS = {
+    # variance around 0 instead of the mean
+    "ln_no_mean": ("int64_t c = (int64_t)d * q[i] - sum;\n            v += c * c;",
+                   "int64_t c = (int64_t)d * q[i];\n            v += c * c;"),
+    # output without subtracting the mean
+    "ln_no_centre": ("int64_t c = (int64_t)d * q[i] - sum;\n            int64_t n",
+                     "int64_t c = (int64_t)d * q[i];\n            int64_t n"),
+    # mean square not divided by d
+    "ln_var_div": ("ipo_isqrt(v / d + eps_c)", "ipo_isqrt(v / (d / 2) + eps_c)"),
+    # epsilon dropped
+    "ln_eps": ("ipo_isqrt(v / d + eps_c)", "ipo_isqrt(v / d)"),
+    # square root one too large
+    "ln_isqrt": ("if (next >= r) return r;", "if (next >= r) return r + 1;"),
+    # reciprocal on the wrong grid
+    "ln_recip": ("int64_t f = ((int64_t)1 << 31) / sigma;", "int64_t f = ((int64_t)1 << 30) / sigma;"),
+}
+
+NORM_PINS = ["tests/test_oracle_norm.py"]
+
 PINS = [
     "tests/test_oracle_relshift.py",
     "tests/test_oracle_scores.py",
@@ -97,14 +117,17 @@ def _copy_tree(dst):
                         ignore=shutil.ignore_patterns("*.so", "__pycache__", "*.tmp*"))
 
 
+GROUPS = [(MUTANTS, PINS, "ipo_mhsa.c"), (LINEAR_MUTANTS, LINEAR_PINS, "ipo_linear.c"),
+          (NORM_MUTANTS, NORM_PINS, "ipo_norm.c")]
+
+
 @pytest.mark.slow
-@pytest.mark.parametrize("name", sorted(MUTANTS) + sorted(LINEAR_MUTANTS))
+@pytest.mark.parametrize("name", [n for g in GROUPS for n in sorted(g[0])])
 def test_mutant_is_caught(tmp_path, name):
-    linear = name in LINEAR_MUTANTS
-    old, new = (LINEAR_MUTANTS if linear else MUTANTS)[name]
-    pins = LINEAR_PINS if linear else PINS
+    table, pins, fname = next(g for g in GROUPS if name in g[0])
+    old, new = table[name]
     _copy_tree(tmp_path)
-    src = tmp_path / "oracle" / ("ipo_linear.c" if linear else "ipo_mhsa.c")
+    src = tmp_path / "oracle" / fname
     text = src.read_text()
     assert text.count(old) == 1, f"mutation site for {name} not found"
     src.write_text(text.replace(old, new))
