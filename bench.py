@@ -268,14 +268,24 @@ NEXT_ROWS = [
 
 def measure_next_rows(dev, peak, steps: int, cpu: bool):
     """Each projection timed alone (CUDA events per launch, L2 flushed before
-    every timed launch), useful ops 2 B T K N, against the measured INT8
-    MMA peak; with `cpu`, the oracle on a bounded sample of frames."""
+    every timed launch: a 256 MB write, then a 256 MB read so that no dirty
+    line is written back inside the timed launch), useful ops 2 B T K N,
+    against the measured INT8 MMA peak; with `cpu`, the oracle on a bounded
+    sample of frames."""
     import torch
     import paper_2609_30846_gb300 as ip
     w0 = synth.WORKLOADS[WORKLOAD]
     B, T = w0.B, w0.T
-    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    flush_w = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    flush_r = torch.ones(256 << 18, dtype=torch.int32, device=dev)
     stream = torch.cuda.current_stream(dev)
+
+    def flush():
+        # write a buffer larger than L2, then read another one, so that the
+        # timed launch finds L2 full of clean lines (no write-back inside it)
+        flush_w.zero_()
+        flush_r.sum()
+
     rows = {}
     for name, K, N, G, xl, yl, sw in NEXT_ROWS:
         case = synth.linear(B, T, K, N, seed=7000 + K + N + G, groups=G)
@@ -301,7 +311,7 @@ def measure_next_rows(dev, peak, steps: int, cpu: bool):
             call()
         times = []
         for _ in range(steps):
-            flush.zero_()
+            flush()
             e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             e0.record(stream)
             call()
@@ -339,8 +349,87 @@ def measure_next_rows(dev, peak, steps: int, cpu: bool):
                                    "sample": f"{frames} frames of {B * T}, {dt:.2f} s"}
         rows[name] = row
         del x, w, b, out
-    del flush
+
+    # integer LayerNorm of the frames before the attention (d = 1024)
+    d = 1024
+    nc = synth.norm(B * T, d, seed=7100)
+    k = ip.layernorm_constants(nc.s_x, nc.gamma, nc.beta, nc.s_y, nc.eps)
+    x = torch.from_numpy(nc.x).to(dev)
+    Md, Bd, Ed = (torch.from_numpy(a).to(dev) for a in (k.M, k.B, k.E))
+    out = torch.empty_like(x)
+    ws = torch.zeros(256, dtype=torch.uint8, device=dev)
+    call = lambda: ip.layernorm_i8(x, Md, Bd, Ed, k.eps_c, out=out, workspace=ws, stream=stream)
+    for _ in range(3):
+        call()
+    times = []
+    for _ in range(steps):
+        flush()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        call()
+        e1.record(stream)
+        e1.synchronize()
+        times.append(e0.elapsed_time(e1) * 1e-3)
+    if ip.status(ws, stream) != 0:
+        raise SystemExit("layernorm: kernel reported an error")
+    t = statistics.median(times)
+    elems = B * T * d
+    ops = NORM_OPS_PER_ELEMENT * elems
+    alu_peak = alu_peak_tops(dev)
+    row = {"value": elems * 2 / t / 1e9, "unit": "GB/s", "us_per_launch": t * 1e6,
+           "shape": {"rows": B * T, "d": d},
+           "roofline": {"bound": "alu", "achieved": ops / t / 1e12, "peak": alu_peak,
+                        "unit": "Tops/s (int32 lane ops)", "frac": ops / t / 1e12 / alu_peak,
+                        "traffic": None, "hbm_frac": elems * 2 / t / 1e9 / HBM_GBS},
+           "kernel": "layernorm_i8_kernel<2>", "gpu_launches": 1}
+    if cpu:
+        import oracle
+        oracle.build()
+        oc = oracle.layernorm_constants(nc.s_x, nc.gamma, nc.beta, nc.s_y, nc.eps)
+        n = 512
+        t0 = time.perf_counter()
+        oracle.layernorm(nc.x[:n], oc)
+        dt = time.perf_counter() - t0
+        n = int(min(B * T, max(512, n / max(dt, 1e-4))))
+        t0 = time.perf_counter()
+        oracle.layernorm(nc.x[:n], oc)
+        dt = time.perf_counter() - t0
+        row["cpu_baseline"] = {"value": n * d * 2 / dt / 1e9, "unit": "GB/s",
+                               "cores": os.cpu_count() or 1, "kind": "oracle",
+                               "sample": f"{n} frames of {B * T}, {dt:.2f} s"}
+    rows["layernorm_1024"] = row
+    del x, out, flush_w, flush_r
     return rows
+
+
+# Integer operations of the LayerNorm per element as the method states them:
+# sum and sum of squares (2), centring d q - sum (2), c f with rounding and
+# shift (3), M n + B with rounding and shift (3), clamp (2).
+NORM_OPS_PER_ELEMENT = 12
+def _hbm_gbs() -> float:
+    """Measured copy bandwidth of this GPU type (MEASURED_PEAKS.json, written
+    by the pool's driver), else the 6.8 TB/s fallback."""
+    try:
+        return float(json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))["hbm_gbs"])
+    except (OSError, ValueError, KeyError):
+        return 6800.0
+
+
+HBM_GBS = _hbm_gbs()
+
+
+def alu_peak_tops(dev) -> float:
+    """One 32-bit integer operation per lane per cycle: SMs x 128 lanes x
+    the maximum SM clock."""
+    import torch
+    props = torch.cuda.get_device_properties(dev)
+    try:
+        import subprocess as sp
+        mhz = float(sp.run(["nvidia-smi", "--query-gpu=clocks.max.sm", "--format=csv,noheader,nounits",
+                            f"--id={dev.index or 0}"], capture_output=True, text=True).stdout.split()[0])
+    except Exception:
+        mhz = 2070.0
+    return props.multi_processor_count * 128 * mhz * 1e6 / 1e12
 
 
 # ------------------------------------------------------------------- GPU arm
@@ -501,7 +590,7 @@ def run_ours(args):
                      "frac": achieved / peak, "traffic": traffic_per_launch(),
                      "peak_source": "measured in this run: integer warp MMA (mma.sync m16n8k32 "
                                     "s8) probe, CUDA events; sm_103a has no tcgen05 kind::i8",
-                     "hbm_floor_frac": (bytes_layer / 6757.2e9) / (avg_layer_ms * 1e-3),
+                     "hbm_floor_frac": (bytes_layer / (HBM_GBS * 1e9)) / (avg_layer_ms * 1e-3),
                      "kernel": "relpos_mhsa_fused_kernel (one launch per layer)"},
         "cpu_baseline": cpu,
         "e2e": e2e,

@@ -222,6 +222,39 @@ int ip_linear_swish_i8(const int8_t *x, const int8_t *w, const int32_t *bias, co
 /* Swish constants for the grids S_z (input) and S_y (output), host only. */
 int ip_swish_params_from_scales(double S_z, double S_y, ip_swish_params *out);
 
+/* ---- integer LayerNorm (Sec. 2.1, Eqs. 1-4; integer kernel of Sec. 2.2) --
+ *
+ * For each row of d int8 values q (grid S_x), all in integers:
+ *   c_i   = d q_i - sum_j q_j                          d (q_i - mean)
+ *   sigma = max(1, isqrt(floor(sum_i c_i^2 / d) + eps_c))
+ *   f     = floor(2^31 / sigma)
+ *   n_i   = round(c_i f / 2^16)                        (q_i - mean) / std on 2^-15
+ *   y_i   = clamp(round((M_i n_i + B_i) / 2^E_i), -127, 127)
+ * round(v / 2^e) = floor((v + 2^(e-1)) / 2^e).  M, B, E per channel carry
+ * gamma, beta and the output grid S_y (ip_layernorm_constants); eps_c is the
+ * epsilon of the variance on the grid of c^2 / d. */
+#define IP_NORM_MAX_ROWS (1ll << 40)
+
+/* x, y: device int8 [rows][d] row-major (16-byte aligned); d in {512, 1024,
+ * 1536, 2048} (others: IP_ERR_UNSUPPORTED); M: device int32 [d]; B: device
+ * int64 [d] with |B| < 2^60; E: device int32 [d] in [31, 62] (a value out of
+ * its domain is clamped and reported as IP_ERR_PARAM by
+ * ip_relpos_mhsa_status); eps_c in [0, 2^40]; workspace as for
+ * ip_relpos_mhsa_i8.  rows == 0 returns IP_OK without touching any pointer.
+ * Launch asynchronous on `stream`.  Returns IP_OK or IP_ERR_*. */
+int ip_layernorm_i8(const int8_t *x, long long rows, int d, long long eps_c, const int32_t *M,
+                    const long long *B, const int32_t *E, int8_t *y, void *workspace,
+                    size_t workspace_bytes, ip_stream_t stream);
+
+/* Offline constants of the LayerNorm (host, float64): gamma, beta [d] real,
+ * input grid S_x, output grid S_y, epsilon eps.  Per channel, (|M_i|, E_i -
+ * 31) is the dyadic of |gamma_i| 2^-15 / S_y with the sign of gamma_i on M_i
+ * (gamma_i = 0: M_i = 0, E_i = 31), B_i = round(beta_i / S_y 2^E_i), and
+ * eps_c = round(eps d^2 / S_x^2).  Outputs: eps_c, M, B, E [d]. */
+int ip_layernorm_constants(double S_x, const double *gamma, const double *beta, int d,
+                           double S_y, double eps, long long *eps_c, int32_t *M, long long *B,
+                           int32_t *E);
+
 /* Text of an IP_* code. */
 const char *ip_strerror(int code);
 

@@ -161,7 +161,7 @@ def layernorm_constants(s_x: float, gamma, beta, s_y: float, eps: float = 1e-5) 
             M[i] = m if g > 0 else -m
             E[i] = 31 + s
         b = math.floor(float(beta[i]) / s_y * 2.0 ** int(E[i]) + 0.5)
-        if abs(b) >= 2 ** 61:
+        if abs(b) >= 2 ** 60:
             raise ValueError(f"beta/gamma ratio of channel {i} out of range")
         B[i] = b
     eps_c = int(math.floor(eps * d * d / (s_x * s_x) + 0.5))

@@ -51,7 +51,7 @@ int ipo_layernorm_i8(const int8_t *x, long long rows, int d, int64_t eps_c, cons
     if (!x || !M || !B || !E || !y) return IPO_ERR_NULL;
     if (eps_c < 0 || eps_c > ((int64_t)1 << 40)) return IPO_ERR_PARAM;
     for (int i = 0; i < d; ++i)
-        if (E[i] < 16 || E[i] > 62 || B[i] >= ((int64_t)1 << 61) || B[i] <= -((int64_t)1 << 61))
+        if (E[i] < 31 || E[i] > 62 || B[i] >= ((int64_t)1 << 60) || B[i] <= -((int64_t)1 << 60))
             return IPO_ERR_PARAM;
 #pragma omp parallel for schedule(static)
     for (long long r = 0; r < rows; ++r) {

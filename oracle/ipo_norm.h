@@ -26,9 +26,9 @@ int64_t ipo_isqrt(int64_t n);
  *   n_i   = round(c_i f / 2^16)                   (q_i - mean) / std on 2^-15
  *   y_i   = clamp(round((M_i n_i + B_i) / 2^E_i), -127, 127)
  * round(v / 2^e) = floor((v + 2^(e-1)) / 2^e).  M (int32), B (int64), E
- * (int32 in [16, 62]) carry gamma, beta and the output grid per channel
+ * (int32 in [31, 62]) carry gamma, beta and the output grid per channel
  * (consts.layernorm_constants); eps_c >= 0 is epsilon on the grid of c^2.
- * d in [2, 4096] (|c| < 2^20, sum c^2 < 2^52); |B_i| < 2^61.  Returns 0 or a negative error. */
+ * d in [2, 4096] (|c| < 2^20, sum c^2 < 2^52); |B_i| < 2^60.  Returns 0 or a negative error. */
 int ipo_layernorm_i8(const int8_t *x, long long rows, int d, int64_t eps_c, const int32_t *M,
                      const int64_t *B, const int32_t *E, int8_t *y);
 

@@ -31,6 +31,7 @@ EXPORTS = (
     "ip_dyadic_pair",
     "ip_isoftmax_params_from_scale", "ip_probe_int8_mma", "ip_relpos_mhsa_i8_noalloc",
     "ip_debug_set_split_mode", "ip_linear_i8", "ip_linear_swish_i8", "ip_swish_params_from_scales",
+    "ip_layernorm_i8", "ip_layernorm_constants",
 )
 
 ROWS = 0    # IP_LAYOUT_ROWS:  [B][T][C]
@@ -116,6 +117,12 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
         lib.ip_swish_params_from_scales.argtypes = [ctypes.c_double, ctypes.c_double,
                                                     ctypes.POINTER(SwishParams)]
         lib.ip_swish_params_from_scales.restype = I
+        LL = ctypes.c_longlong
+        lib.ip_layernorm_i8.argtypes = [P, LL, I, LL, P, P, P, P, P, ctypes.c_size_t, P]
+        lib.ip_layernorm_i8.restype = I
+        D = ctypes.c_double
+        lib.ip_layernorm_constants.argtypes = [D, P, P, I, D, D, ctypes.POINTER(LL), P, P, P]
+        lib.ip_layernorm_constants.restype = I
         lib.ip_probe_int8_mma.argtypes = [I, I, P, P]
         lib.ip_probe_int8_mma.restype = ctypes.c_longlong
         _lib = lib
@@ -358,6 +365,50 @@ def linear_swish_i8(x, w, bias, m, s, swish: tuple[int, int, int, int], *, out=N
     return out
 
 
+@dataclass(frozen=True)
+class NormConstants:
+    eps_c: int
+    M: "np.ndarray"     # int32 [d]
+    B: "np.ndarray"     # int64 [d]
+    E: "np.ndarray"     # int32 [d]
+
+
+def layernorm_constants(s_x: float, gamma, beta, s_y: float, eps: float = 1e-5) -> NormConstants:
+    """Offline constants of the integer LayerNorm (host, float64)."""
+    import numpy as np
+    g = np.ascontiguousarray(gamma, dtype=np.float64)
+    b = np.ascontiguousarray(beta, dtype=np.float64)
+    d = g.size
+    M = np.empty(d, np.int32)
+    B = np.empty(d, np.int64)
+    E = np.empty(d, np.int32)
+    ec = ctypes.c_longlong()
+    _check("ip_layernorm_constants", load().ip_layernorm_constants(
+        s_x, g.ctypes.data, b.ctypes.data, d, s_y, eps, ctypes.byref(ec), M.ctypes.data,
+        B.ctypes.data, E.ctypes.data))
+    return NormConstants(ec.value, M, B, E)
+
+
+def layernorm_i8(x, M, B, E, eps_c: int, *, out=None, workspace=None, stream=None):
+    """Integer LayerNorm over the last axis of int8 x (CUDA, d in {512, 1024,
+    1536, 2048}); M int32, B int64, E int32 [d] CUDA tensors.  Returns int8
+    like x.  Asynchronous on `stream`."""
+    import torch
+    d = x.shape[-1]
+    rows = x.numel() // d if d else 0
+    if out is None:
+        out = torch.empty_like(x)
+    if workspace is None:
+        workspace = torch.zeros(256, dtype=torch.uint8, device=x.device)
+    rc = load().ip_layernorm_i8(
+        _dev_ptr(x, "x", torch.int8, tuple(x.shape)), rows, d, int(eps_c),
+        _dev_ptr(M, "M", torch.int32, (d,)), _dev_ptr(B, "B", torch.int64, (d,)),
+        _dev_ptr(E, "E", torch.int32, (d,)), _dev_ptr(out, "out", torch.int8, tuple(x.shape)),
+        ctypes.c_void_p(workspace.data_ptr()), workspace.numel(), _stream_handle(stream))
+    _check("ip_layernorm_i8", rc)
+    return out
+
+
 def relpos_mhsa_i8_host(q, k, v, p, u, v_bias, consts: LayerConstants, lengths, out, arena,
                         stream=None):
     """Whole layer from host buffers (torch CPU tensors, ideally pinned):
@@ -388,4 +439,5 @@ __all__ = ["build", "load", "relpos_mhsa_i8", "relpos_mhsa_i8_host", "status", "
            "dyadic_pair", "isoftmax_params_from_scale", "set_timeout_cycles", "strerror",
            "int8_mma_peak_tops", "set_stall_injection", "set_split_mode", "linear_i8",
            "linear_constants", "ROWS", "HEADS", "linear_swish_i8", "swish_params_from_scales",
+           "layernorm_i8", "layernorm_constants", "NormConstants",
            "IpError", "LibraryError", "EXPORTS"]

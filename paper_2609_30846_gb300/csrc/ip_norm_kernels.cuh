@@ -1,0 +1,201 @@
+// Device code of the integer LayerNorm (I-Parakeet, Sec. 2.1, Eqs. 1-4, with
+// the integer kernel of Sec. 2.2) for sm_103a.  Integer arithmetic only: no
+// floating-point type, no division by a run-time value (d is a compile-time
+// multiple of 512; the square root and the reciprocal are digit-by-digit).
+//
+// One warp per batch of four rows of d channels, batches dealt round-robin
+// over the warps of the grid.  Per row: the sum and the sum of squares of the
+// int8 values (dp4a, warp reduction), floor(sum c^2 / d) = d sum q^2 -
+// (sum q)^2 exactly for the centred values c_i = d q_i - sum, sigma =
+// isqrt(that + eps_c) (at least 1), f = floor(2^31 / sigma), and per element
+// n = round(c f / 2^16), y = clamp(round((M_i n + B_i) / 2^E_i), -127, 127).
+// Lane l takes the 16-byte segments l, l + 32, ... of the row (coalesced);
+// the per-channel constants (B, M, E) of its channels sit in shared memory
+// in lane-major order, one 16-byte record per channel.
+#pragma once
+
+#include <stdint.h>
+
+#include "ip_ptx.cuh"
+
+namespace ipn {
+
+using namespace ipk;
+
+constexpr int THREADS = 256;              // 8 warps, one batch of rows each
+constexpr int NB = 4;                     // rows per warp batch
+constexpr int ERR_PARAM = 16;             // a per-channel constant out of its domain
+
+struct NormParams {
+    const int8_t *x;
+    int8_t *y;
+    long long rows;
+    long long eps_c;
+    const int32_t *M;
+    const long long *B;
+    const int32_t *E;
+    int *err;
+};
+
+// floor(sqrt(n)) for 0 <= n < 2^42, digit by digit (no division).
+__device__ __forceinline__ unsigned long long isqrt_u42(unsigned long long n) {
+    unsigned long long r = 0;
+    // the root has at most (bit length of n + 1) / 2 bits: start there
+    const int k0 = n == 0 ? -1 : (63 - __clzll(static_cast<long long>(n))) >> 1;
+#pragma unroll 1
+    for (int k = k0; k >= 0; --k) {
+        const unsigned long long bit = 1ull << (2 * k);
+        const bool take = n >= r + bit;
+        n -= take ? r + bit : 0ull;
+        r = (r >> 1) + (take ? bit : 0ull);
+    }
+    return r;
+}
+
+// floor(2^31 / s) for 1 <= s < 2^32 by restoring binary long division.
+__device__ __forceinline__ uint32_t recip_2pow31(unsigned long long s) {
+    unsigned long long rem = 1ull << 31;
+    uint32_t quo = 0;
+    // s >= 2^(L-1) for bit length L, so the quotient is below 2^(32 - L)
+    const int top = __clzll(static_cast<long long>(s)) - 32;   // 32 - L
+#pragma unroll 1
+    for (int bit = top < 31 ? top : 31; bit >= 0; --bit) {
+        const unsigned long long t = s << bit;          // s < 2^32: no overflow
+        const bool take = t <= rem;
+        rem -= take ? t : 0ull;
+        quo |= take ? (1u << bit) : 0u;
+    }
+    return quo;
+}
+
+// Sign-extended byte e of w.
+__device__ __forceinline__ int sbyte_at(uint32_t w, int e) {
+    return static_cast<int>(static_cast<int8_t>((w >> (8 * e)) & 0xffu));
+}
+
+// C = d / 512 segments of 16 channels per lane.  A warp takes NB rows at a
+// time: it reduces them, lane r computes the square root and the reciprocal
+// of row r (one chain of those scalar steps serves NB rows), then it
+// normalises the rows one after the other, reading each again (from L2, it
+// was just read).  Loops over rows stay rolled so that the code fits the
+// instruction cache.
+template <int C>
+__global__ void __launch_bounds__(THREADS)
+    layernorm_i8_kernel(const NormParams prm) {
+    constexpr int D = 512 * C;
+    extern __shared__ uint8_t smem_raw[];
+    uint4 *cst = reinterpret_cast<uint4 *>(smem_raw);   // [C * 16][32] records
+    const int lane = threadIdx.x & 31;
+
+    // per-channel records {B' lo, B' hi, M, E - 31} with B' = B + 2^(E-1)
+    // (the rounding term folded in): channel j 512 + l 16 + e of lane l goes
+    // to record (j 16 + e) 32 + l
+    bool bad = false;
+    for (int k = threadIdx.x; k < D; k += THREADS) {
+        const int j = k >> 9, l = (k >> 4) & 31, e = k & 15;
+        long long b = prm.B[k];
+        int m = prm.M[k], ex = prm.E[k];
+        if (ex < 31 || ex > 62 || b >= (1ll << 60) || b <= -(1ll << 60)) {
+            bad = true;
+            ex = ex < 31 ? 31 : (ex > 62 ? 62 : ex);
+            b = 0;
+        }
+        b += 1ll << (ex - 1);
+        cst[(j * 16 + e) * 32 + l] =
+            make_uint4(static_cast<uint32_t>(b), static_cast<uint32_t>(static_cast<unsigned long long>(b) >> 32),
+                       static_cast<uint32_t>(m), static_cast<uint32_t>(ex - 31));
+    }
+    if (bad) atomicOr(prm.err, ERR_PARAM);
+    __syncthreads();
+
+    const long long warps = static_cast<long long>(gridDim.x) * (THREADS / 32);
+    const long long groups = (prm.rows + NB - 1) / NB;
+    for (long long grp = static_cast<long long>(blockIdx.x) * (THREADS / 32) + (threadIdx.x >> 5);
+         grp < groups; grp += warps) {
+        const long long row0 = grp * NB;
+        const int nrows = prm.rows - row0 < NB ? static_cast<int>(prm.rows - row0) : NB;
+
+        // pass A: sum and sum of squares of each row (dp4a, warp reduction)
+        int sum[NB], sq[NB];
+#pragma unroll
+        for (int r = 0; r < NB; ++r) {
+            sum[r] = 0;
+            sq[r] = 0;
+            if (r < nrows) {
+                const int8_t *xr = prm.x + (row0 + r) * D;
+#pragma unroll
+                for (int j = 0; j < C; ++j) {
+                    const uint4 s = __ldg(reinterpret_cast<const uint4 *>(xr + j * 512 + lane * 16));
+                    const uint32_t w[4] = {s.x, s.y, s.z, s.w};
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) {
+                        sum[r] = __dp4a(static_cast<int>(w[i]), 0x01010101, sum[r]);
+                        sq[r] = __dp4a(static_cast<int>(w[i]), static_cast<int>(w[i]), sq[r]);
+                    }
+                }
+            }
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1)
+#pragma unroll
+            for (int r = 0; r < NB; ++r) {
+                sum[r] += __shfl_xor_sync(0xffffffffu, sum[r], o);
+                sq[r] += __shfl_xor_sync(0xffffffffu, sq[r], o);
+            }
+
+        // lane r: floor(sum c^2 / d) = d sum q^2 - (sum q)^2 of row r (exact,
+        // c = d q - sum), sigma and f
+        long long ms = 0;
+        int sum_own = 0;
+#pragma unroll
+        for (int r = 0; r < NB; ++r)
+            if (lane == r) {
+                ms = static_cast<long long>(D) * sq[r] - static_cast<long long>(sum[r]) * sum[r];
+                sum_own = sum[r];
+            }
+        unsigned long long sigma = isqrt_u42(static_cast<unsigned long long>(ms + prm.eps_c));
+        sigma = sigma < 1 ? 1 : sigma;
+        // f = floor(2^31 / sigma), held as a signed 32-bit value: f = 2^31 only
+        // for sigma = 1, where sum c^2 < 4 d gives |c| < 2^7 and round(c (2^31 -
+        // 1) / 2^16) = round(c 2^31 / 2^16), so 2^31 - 1 stands in exactly
+        uint32_t f_own = recip_2pow31(sigma);
+        f_own = f_own > 0x7fffffffu ? 0x7fffffffu : f_own;
+
+        // pass B: normalise and requantise, row by row
+#pragma unroll 1
+        for (int r = 0; r < nrows; ++r) {
+            const int f = static_cast<int>(__shfl_sync(0xffffffffu, f_own, r));
+            const int sm = __shfl_sync(0xffffffffu, sum_own, r);
+            const int8_t *xr = prm.x + (row0 + r) * D;
+            int8_t *yr = prm.y + (row0 + r) * D;
+#pragma unroll
+            for (int j = 0; j < C; ++j) {
+                const uint4 s = __ldcs(reinterpret_cast<const uint4 *>(xr + j * 512 + lane * 16));
+                const uint32_t w[4] = {s.x, s.y, s.z, s.w};
+                uint32_t o[4] = {0u, 0u, 0u, 0u};
+#pragma unroll
+                for (int e = 0; e < 16; ++e) {
+                    const uint4 rec = cst[(j * 16 + e) * 32 + lane];
+                    const long long b = static_cast<long long>((static_cast<unsigned long long>(rec.y) << 32) | rec.x);
+                    const int cc = D * sbyte_at(w[e >> 2], e & 3) - sm;   // |c| < 2^20
+                    // n = round(c f / 2^16): |c f| < 2^51 and |n| < 2^23, so the
+                    // low word of (c f + 2^15) >> 16 is n
+                    const long long u = static_cast<long long>(cc) * f + (1ll << 15);
+                    const int n = static_cast<int>(__funnelshift_r(static_cast<uint32_t>(u),
+                                                                   static_cast<uint32_t>(u >> 32), 16));
+                    // floor(v / 2^E) = floor(floor(v / 2^31) / 2^(E - 31)); |v| < 2^62
+                    // makes floor(v / 2^31) a 32-bit value
+                    const long long v = static_cast<long long>(static_cast<int>(rec.z)) * n + b;
+                    const int h = static_cast<int>(__funnelshift_r(static_cast<uint32_t>(v),
+                                                                   static_cast<uint32_t>(v >> 32), 31));
+                    const int t = h >> static_cast<int>(rec.w);
+                    const int y8 = t > 127 ? 127 : (t < -127 ? -127 : t);
+                    o[e >> 2] |= (static_cast<uint32_t>(y8) & 0xffu) << (8 * (e & 3));
+                }
+                __stcs(reinterpret_cast<uint4 *>(yr + j * 512 + lane * 16), make_uint4(o[0], o[1], o[2], o[3]));
+            }
+        }
+    }
+}
+
+}  // namespace ipn

@@ -281,3 +281,33 @@ def linear(B: int, T: int, K: int, N: int, seed: int, *, groups: int = 1,
     s_y = np.array([max(np.abs(yr[:, gi * per:(gi + 1) * per]).max(), 1e-30) / 127.0
                     for gi in range(groups)])
     return LinearCase(x, w, bq, float(s_x), s_w, s_y, groups)
+
+
+# ------------------------------------------------------------ LayerNorm
+
+@dataclass
+class NormCase:
+    """Inputs of one integer LayerNorm: int8 frames x [rows, d] on grid S_x
+    (the residual stream), real per-channel gamma and beta, the output grid
+    S_y and epsilon."""
+    x: np.ndarray
+    gamma: np.ndarray
+    beta: np.ndarray
+    s_x: float
+    s_y: float
+    eps: float = 1e-5
+
+
+def norm(rows: int, d: int, seed: int, eps: float = 1e-5) -> NormCase:
+    """Seeded LayerNorm case: each frame round(N(mu_r, 35^2)) clipped to
+    +-127 with a per-frame offset mu_r ~ N(0, 10^2); gamma ~ U[0.3, 2] with
+    10 % negative, beta ~ N(0, 0.5^2); S_x = alpha/127, alpha ~ U[2, 6];
+    S_y = alpha_y/127, alpha_y ~ U[3, 8] (a normalised output stays within
+    a few units)."""
+    g = np.random.Generator(np.random.PCG64(np.random.SeedSequence(seed)))
+    mu = g.normal(0.0, 10.0, size=(rows, 1)).astype(np.float32)
+    xf = g.standard_normal((rows, d), dtype=np.float32) * np.float32(35.0) + mu
+    x = np.clip(np.rint(xf), -127, 127).astype(np.int8)
+    gamma = g.uniform(0.3, 2.0, size=d) * g.choice([-1.0, 1.0], size=d, p=[0.1, 0.9])
+    beta = g.normal(0.0, 0.5, size=d)
+    return NormCase(x, gamma, beta, g.uniform(2.0, 6.0) / 127, g.uniform(3.0, 8.0) / 127, eps)

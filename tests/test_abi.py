@@ -18,7 +18,8 @@ HEADER = os.path.join(ROOT, "include", "ip_mhsa.h")
 CSRC = os.path.join(ROOT, "paper_2609_30846_gb300", "csrc")
 KERNELS = os.path.join(CSRC, "ip_mhsa_kernels.cuh")
 DEVICE_SOURCES = [os.path.join(CSRC, f) for f in
-                  ("ip_mhsa_kernels.cuh", "ip_linear_kernels.cuh", "ip_ptx.cuh")]
+                  ("ip_mhsa_kernels.cuh", "ip_linear_kernels.cuh", "ip_norm_kernels.cuh",
+                   "ip_ptx.cuh")]
 
 
 def declared_functions():
@@ -134,7 +135,7 @@ def test_kernel_source_is_integer_only(path):
     # the remaining operators divide by compile-time powers of two.
     if path == KERNELS:
         assert "div_2pow32" in code and "iexp_neg" in code
-    allowed = {"NSTAGE", "NK", "MROWS", "DH", "BK", "BM", "BN", "STAGES",
+    allowed = {"NSTAGE", "NK", "MROWS", "DH", "BK", "BM", "BN", "STAGES", "D", "NB",
                "16", "2", "4", "8", "32", "256"}
     for m in re.finditer(r"[^/*](/|%)\s*\(?\s*([A-Za-z_0-9]+)", code):
         if m.group(0).startswith("<") or m.group(1) == "/" and code[m.start(1) + 1] in "/*":
@@ -206,3 +207,36 @@ def test_swish_validation(lib):
                                   fake, P(1 << 21), 256, None) == -7
     assert lib.ip_linear_swish_i8(fake, fake, None, fake, fake, None, 1, 4, 128, 128,
                                   fake, P(1 << 21), 256, None) == -1
+
+
+@pytest.mark.parametrize("seed", [0, 1])
+def test_layernorm_constants_match_oracle(lib, seed):
+    import oracle
+    rng = np.random.default_rng(seed)
+    d = 1024
+    gamma = rng.uniform(0.2, 2.0, d) * rng.choice([-1.0, 1.0], d)
+    gamma[5] = 0.0
+    beta = rng.normal(0, 0.5, d)
+    s_x, s_y = rng.uniform(2, 6) / 127, rng.uniform(3, 8) / 127
+    want = oracle.layernorm_constants(s_x, gamma, beta, s_y, 1e-5)
+    got = ip.layernorm_constants(s_x, gamma, beta, s_y, 1e-5)
+    assert got.eps_c == want.eps_c
+    np.testing.assert_array_equal(got.M, want.M)
+    np.testing.assert_array_equal(got.B, want.B)
+    np.testing.assert_array_equal(got.E, want.E)
+
+
+def test_layernorm_validation(lib):
+    P = ctypes.c_void_p
+    fake, ws = P(1 << 20), P(1 << 21)
+
+    def call(rows=4, d=1024, eps=0, x=fake, M=fake, B=fake, E=fake, y=fake, wsp=ws, wsb=256):
+        return lib.ip_layernorm_i8(x, rows, d, eps, M, B, E, y, wsp, wsb, None)
+
+    assert call(d=80) == -4
+    assert call(rows=-1) == -2
+    assert call(eps=-1) == -7
+    assert call(rows=0, x=None, y=None) == 0
+    assert call(M=None) == -1
+    assert call(B=P((1 << 20) + 4)) == -3
+    assert call(wsb=16) == -8

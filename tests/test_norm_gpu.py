@@ -1,0 +1,90 @@
+"""Parity of the integer LayerNorm on the GPU (through the C ABI) with the
+CPU oracle: bit-exact on every output."""
+import numpy as np
+import pytest
+
+pytestmark = pytest.mark.gpu
+
+torch = pytest.importorskip("torch")
+
+
+@pytest.fixture(scope="module")
+def ip():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import paper_2609_30846_gb300 as mod
+    mod.load()
+    return mod
+
+
+@pytest.fixture(scope="module")
+def orc():
+    import oracle
+    oracle.build()
+    return oracle
+
+
+def _d(a):
+    return torch.from_numpy(np.ascontiguousarray(a)).cuda()
+
+
+def case(rows, d, seed, eps=1e-5, spread=35.0):
+    rng = np.random.default_rng(seed)
+    x = np.clip(np.rint(rng.normal(rng.normal(0, 10), spread, size=(rows, d))), -127, 127).astype(np.int8)
+    gamma = rng.uniform(0.3, 2.0, size=d) * rng.choice([-1.0, 1.0], size=d, p=[0.1, 0.9])
+    beta = rng.normal(0.0, 0.5, size=d)
+    s_x, s_y = rng.uniform(2.0, 6.0) / 127, rng.uniform(3.0, 8.0) / 127
+    return x, gamma, beta, s_x, s_y, eps
+
+
+def run_both(ip, orc, x, gamma, beta, s_x, s_y, eps):
+    c = orc.layernorm_constants(s_x, gamma, beta, s_y, eps)
+    ws = torch.zeros(256, dtype=torch.uint8, device="cuda")
+    got = ip.layernorm_i8(_d(x), _d(c.M), _d(c.B), _d(c.E), c.eps_c, workspace=ws)
+    assert ip.status(ws) == 0
+    return got.cpu().numpy(), orc.layernorm(x, c)
+
+
+def assert_same(got, want):
+    bad = got != want
+    if bad.any():
+        idx = np.argwhere(bad)[:5]
+        raise AssertionError(f"{int(bad.sum())} of {got.size} differ; first at {idx.tolist()}: "
+                             f"gpu {got[tuple(idx[0])]} oracle {want[tuple(idx[0])]}")
+
+
+@pytest.mark.parametrize("d", [512, 1024, 1536, 2048])
+@pytest.mark.parametrize("rows", [1, 7, 300])
+def test_shapes(ip, orc, d, rows):
+    assert_same(*run_both(ip, orc, *case(rows, d, seed=d + rows)))
+
+
+def test_special_rows(ip, orc):
+    d = 1024
+    x, gamma, beta, s_x, s_y, _ = case(8, d, seed=5)
+    x[0] = 0                                   # constant rows: sigma from epsilon only
+    x[1] = -127
+    x[2] = np.where(np.arange(d) % 2 == 0, 127, -127)
+    x[3] = np.where(np.arange(d) == 0, 127, -127)   # one outlier
+    x[4] = np.where(np.arange(d) % 2 == 0, 1, 0)
+    for eps in (0.0, 1e-5, 1e-2):
+        assert_same(*run_both(ip, orc, x, gamma, beta, s_x, s_y, eps))
+
+
+def test_small_variance_rows(ip, orc):
+    assert_same(*run_both(ip, orc, *case(64, 1024, seed=6, eps=2e-4, spread=0.6)))
+
+
+def test_encoder_frames_full_size(ip, orc):
+    # the LayerNorm before the attention of one block: B=32 x T=375 frames
+    assert_same(*run_both(ip, orc, *case(32 * 375, 1024, seed=7)))
+
+
+def test_constant_out_of_domain_is_reported(ip, orc):
+    x, gamma, beta, s_x, s_y, eps = case(4, 512, seed=8)
+    c = orc.layernorm_constants(s_x, gamma, beta, s_y, eps)
+    E = c.E.copy()
+    E[3] = 70
+    ws = torch.zeros(256, dtype=torch.uint8, device="cuda")
+    ip.layernorm_i8(_d(x), _d(c.M), _d(c.B), _d(E), c.eps_c, workspace=ws)
+    assert ip.status(ws) == -7
