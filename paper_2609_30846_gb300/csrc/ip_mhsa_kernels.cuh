@@ -9,11 +9,11 @@
 // memory accelerator (TMA) stages with the 128-byte swizzle.
 //
 // One CTA owns 64 query rows of one (b, h): four consumer warps of 16 rows
-// and one producer warp.  The producer issues the TMA loads and prepares each
-// staged chunk for the consumers: for the score pass it computes the bias
-// vectors K u and P v of the chunk (the exact rank-1 split of (Q + 1u^T)K^T
-// and (Q + 1v^T)P^T, since Q + u does not fit an int8 operand), for the
-// attn.V pass it transposes the V tile into the operand layout of the MMA.
+// and one producer warp.  The producer issues the TMA loads and, for the
+// score pass, computes the bias vectors K u and P v of each staged chunk (the
+// exact rank-1 split of (Q + 1u^T)K^T and (Q + 1v^T)P^T, since Q + u does not
+// fit an int8 operand).  The attn.V pass reads the V tile as TMA stages it:
+// transposed ldmatrix loads and byte selects build the MMA operand.
 // The consumers, per CTA:
 //   pass 1  for each chunk of 64 keys: the content MMAs Q K^T, the MMAs of
 //           the position band Q P_band^T for the next chunk (issued before
@@ -24,7 +24,7 @@
 //   pass 2  integer exponentials (a 256-entry table, one copy per row
 //           group to spread the banks) and row sums;
 //   pass 3  probabilities on the grid 2^-8 as the u8 operand of the A.V
-//           MMA, then the output requantisation and 16-byte stores.
+//           MMA, then the output requantisation and 4-byte stores.
 #pragma once
 
 #include <cuda.h>
@@ -136,14 +136,24 @@ __device__ __forceinline__ uint32_t lut_addr(uint32_t lut_g, int d) {
     return lut_g + (static_cast<uint32_t>(d) & 0xffu) * (LUT_COPIES * 4);
 }
 
-// Transposed V tile of one chunk: for each 32-key k step ks, half hf (keys
-// 16 hf .. 16 hf + 15 of the step) and MMA n8 tile nt, one 8 x 16-byte
-// matrix whose row r holds d = nt + 16 r and whose byte 4t + i holds key
-// 32 ks + 16 hf + 2t + (i & 1) + 8 (i >> 1) (the k order of the A operand).
-// Rows are placed at slot r ^ 2((nt >> 2) & 3) to spread the banks.
-__device__ __forceinline__ uint32_t vt_row(int ks, int hf, int nt, int r) {
-    return static_cast<uint32_t>((((ks * 2 + hf) * 16 + nt) << 7) +
-                                 ((r ^ (((nt >> 2) & 3) << 1)) << 4));
+// B fragments of the attn.V MMA for keys 32 ks .. 32 ks + 31 of the staged
+// V tile (keys as rows, 128-byte swizzle) and the 16 values of d in chunk c,
+// with no transposed copy of V: ldmatrix.trans on 16-bit elements hands
+// thread (g, t) the byte pairs (d = 16c + 2g, 16c + 2g + 1) of keys 2t, 2t + 1
+// (r0), 8 + 2t, 9 + 2t (r1) and the same + 16 (r2, r3); byte selects split
+// them into the fragment of the even d (n-tile 2c) and of the odd d (n-tile
+// 2c + 1).  The k order, keys 2t, 2t + 1, 8 + 2t, 9 + 2t then + 16, is the one
+// of the probability operand (prob_operand).  N-tile 2c + p holds d =
+// 16c + 2n + p in its column n.
+__device__ __forceinline__ void vfrag(uint32_t vtile, int ks, int c, int lane, uint32_t &b0e,
+                                      uint32_t &b1e, uint32_t &b0o, uint32_t &b1o) {
+    const int key = 32 * ks + 8 * (lane >> 3) + (lane & 7);
+    uint32_t r0, r1, r2, r3;
+    ldsm_x4_trans(vtile + swz(key, c), r0, r1, r2, r3);
+    b0e = __byte_perm(r0, r1, 0x6420);
+    b1e = __byte_perm(r2, r3, 0x6420);
+    b0o = __byte_perm(r0, r1, 0x7531);
+    b1o = __byte_perm(r2, r3, 0x7531);
 }
 
 // floor(2^32 / s) for s >= 2 by restoring binary long division (the
@@ -414,9 +424,9 @@ __device__ __forceinline__ void send_partial(const int (&oacc)[16][4], uint32_t 
             sts32(xo + ((i * 4 + e) * 32 + lane) * 4, static_cast<uint32_t>(oacc[8 * (1 - HK) + i][e]));
 }
 
-// Adds the partner's partial sums of this warp's n-tiles 8 HK .. 8 HK + 7,
-// requantises them (Eq. 7) and stores two 8-byte runs per row: d =
-// nt + 32 t + 16 hh for nt in 8 HK .. 8 HK + 7.
+// Adds the partner's partial sums of this warp's n-tiles 8 HK .. 8 HK + 7
+// (d = 64 HK .. 64 HK + 63), requantises them (Eq. 7) and stores four bytes
+// per row and d chunk: d = 16c + 4t .. 16c + 4t + 3 for c in 4 HK .. 4 HK + 3.
 template <int HK>
 __device__ __forceinline__ void finish_half(int (&oacc)[16][4], uint32_t pxo, int lane, int wrow0,
                                             int T, int len, size_t bh, long long m_o,
@@ -431,22 +441,18 @@ __device__ __forceinline__ void finish_half(int (&oacc)[16][4], uint32_t pxo, in
     for (int rr = 0; rr < 2; ++rr) {
         const int row = wrow0 + g + 8 * rr;
         if (row >= T) continue;
-        int8_t *dst = out + (bh * T + row) * DH + 32 * t4 + 8 * HK;
+        int8_t *dst = out + (bh * T + row) * DH + 4 * t4;
 #pragma unroll
-        for (int hh = 0; hh < 2; ++hh) {
-            uint32_t wv[2];
+        for (int c = 4 * HK; c < 4 * HK + 4; ++c) {
+            uint32_t w = 0;
 #pragma unroll
-            for (int wq = 0; wq < 2; ++wq) {
-                uint32_t w = 0;
-#pragma unroll
-                for (int e = 0; e < 4; ++e) {
-                    const long long x = m_o * oacc[8 * HK + 4 * wq + e][2 * rr + hh] + half_o;
-                    const int o = row < len ? clamp127(x >> sh_o) : 0;
-                    w |= (static_cast<uint32_t>(o) & 0xffu) << (8 * e);
-                }
-                wv[wq] = w;
+            for (int e = 0; e < 4; ++e) {
+                // byte e: d = 16c + 4t + e = n-tile 2c + (e & 1), column 2t + (e >> 1)
+                const long long x = m_o * oacc[2 * c + (e & 1)][2 * rr + (e >> 1)] + half_o;
+                const int o = row < len ? clamp127(x >> sh_o) : 0;
+                w |= (static_cast<uint32_t>(o) & 0xffu) << (8 * e);
             }
-            *reinterpret_cast<uint2 *>(dst + 16 * hh) = make_uint2(wv[0], wv[1]);
+            *reinterpret_cast<uint32_t *>(dst + 16 * c) = w;
         }
     }
 }
@@ -485,35 +491,6 @@ __device__ __forceinline__ void prep_bias(uint32_t ktile, uint32_t ptile, uint32
             acc = __dp4a(static_cast<int>(x.w), static_cast<int>(vw[4 * ch + 3]), acc);
         }
         sts32(pv + row * 4, static_cast<uint32_t>(acc));
-    }
-}
-
-// Transposes the staged V tile (rows = keys, 128-byte swizzle) into the
-// MMA operand layout of vt_row.  Work unit: 4 keys x 4 d; lane l, round k:
-// t = l & 3, 4-d block db = (l >> 2) + 8 (k & 3), half hf = (k >> 2) & 1,
-// k step ks = k >> 3.
-__device__ __forceinline__ void prep_vt(uint32_t vtile, uint32_t vt, int lane) {
-    const int t4 = lane & 3;
-#pragma unroll 4
-    for (int k = 0; k < 16; ++k) {
-        const int db = (lane >> 2) + 8 * (k & 3);
-        const int hf = (k >> 2) & 1;
-        const int ks = k >> 3;
-        const int d0 = 4 * db;
-        const int kb = 32 * ks + 16 * hf + 2 * t4;
-        uint32_t x[4];
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            const int key = kb + (i & 1) + 8 * (i >> 1);
-            x[i] = lds32(vtile + swz(key, d0 >> 4) + (d0 & 15));
-        }
-        uint32_t y[4];
-        transpose4(x[0], x[1], x[2], x[3], y[0], y[1], y[2], y[3]);
-#pragma unroll
-        for (int c = 0; c < 4; ++c) {
-            const int d = d0 + c;
-            sts32(vt + vt_row(ks, hf, d & 15, d >> 4) + 4 * t4, y[c]);
-        }
     }
 }
 
@@ -652,25 +629,27 @@ __global__ void __launch_bounds__(NTHREADS, 2)
         }
         for (int it = 0; it < total; ++it) {
             const int s = it & 1;
-            if (!warp_wait(full_bar(s), (it >> 1) & 1, prm.timeout_cycles)) {
-                if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_FULL);
-                ok = false;
-                break;
-            }
-            landed = it + 1;
-            if (it < nchunks)
+            if (it < nchunks) {
+                // score pass: the bias vectors of the staged chunk
+                if (!warp_wait(full_bar(s), (it >> 1) & 1, prm.timeout_cycles)) {
+                    if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_FULL);
+                    ok = false;
+                    break;
+                }
+                landed = it + 1;
                 prep_bias(stage_addr(s), stage_addr(s) + K_TILE_BYTES, stage_addr(s) + KU_OFF,
                           stage_addr(s) + PV_OFF, uw, vw, lane);
-            else
-                prep_vt(stage_addr(s), stage_addr(s) + K_TILE_BYTES, lane);
-            __syncwarp();
-            if (lane == 0) mbar_arrive(ready_bar(s));
+                __syncwarp();
+                if (lane == 0) mbar_arrive(ready_bar(s));
+            }
+            // (attn.V pass: the consumers read the V tile as TMA left it)
             if (it + 2 < total) {
                 if (!warp_wait(empty_bar(s), (it >> 1) & 1, prm.timeout_cycles)) {
                     if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_EMPTY);
                     ok = false;
                     break;
                 }
+                landed = it + 1;   // released by the consumers, so it had landed
                 if (lane == 0) issue(it + 2);
                 issued = it + 3;
             }
@@ -820,7 +799,6 @@ __global__ void __launch_bounds__(NTHREADS, 2)
 #pragma unroll
         for (int nt = 0; nt < 16; ++nt) oacc[nt][0] = oacc[nt][1] = oacc[nt][2] = oacc[nt][3] = 0;
         const int kvalid_last = len - (nchunks - 1) * NK;
-        const int lm_row = lane & 7, lm_mat = lane >> 3;
         for (int c = 0; c < nchunks; ++c) {
             const uint4 sv = lds128(scores + c * CHUNK_SCORE_BYTES + hk * 512 + lane * 16);
             uint32_t pw[4] = {prob_word(sv.x, lut_g, mx0, mx1, f0, f1),
@@ -835,18 +813,17 @@ __global__ void __launch_bounds__(NTHREADS, 2)
             prob_operand(pw, af);
             const int it = nchunks + c;
             const int s = it & 1;
-            if (!warp_wait(ready_bar(s), (it >> 1) & 1, prm.timeout_cycles)) {
-                if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_READY);
+            if (!warp_wait(full_bar(s), (it >> 1) & 1, prm.timeout_cycles)) {
+                if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_FULL);
                 return;
             }
-            const uint32_t vt = stage_addr(s) + K_TILE_BYTES;
+            const uint32_t vtile = stage_addr(s);
 #pragma unroll
             for (int grp = 0; grp < 4; ++grp) {
                 uint32_t bv[2][4];
 #pragma unroll
                 for (int i = 0; i < 2; ++i)
-                    ldsm_x4(vt + vt_row(hk, lm_mat & 1, 4 * grp + 2 * i + (lm_mat >> 1), lm_row),
-                            bv[i][0], bv[i][1], bv[i][2], bv[i][3]);
+                    vfrag(vtile, hk, 2 * grp + i, lane, bv[i][0], bv[i][1], bv[i][2], bv[i][3]);
 #pragma unroll
                 for (int i = 0; i < 2; ++i) {
                     mma_u8s8(oacc[4 * grp + 2 * i], af, bv[i][0], bv[i][1]);
@@ -1000,11 +977,11 @@ __global__ void __launch_bounds__(NTHREADS, 2)
     for (int c = 0; c < nchunks; ++c) {
         const int it = nchunks + c;
         const int s = it & 1;
-        if (!warp_wait(ready_bar(s), (it >> 1) & 1, prm.timeout_cycles)) {
-            if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_READY);
+        if (!warp_wait(full_bar(s), (it >> 1) & 1, prm.timeout_cycles)) {
+            if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_FULL);
             return;
         }
-        const uint32_t vt = stage_addr(s) + K_TILE_BYTES;
+        const uint32_t vtile = stage_addr(s);
 #pragma unroll
         for (int ks = 0; ks < 2; ++ks) {
             const int nxt = min(2 * c + ks + 1, nsteps - 1);
@@ -1015,11 +992,8 @@ __global__ void __launch_bounds__(NTHREADS, 2)
             for (int grp = 0; grp < 4; ++grp) {
                 uint32_t b[2][4];
 #pragma unroll
-                for (int i = 0; i < 2; ++i) {
-                    // matrix m = lm_mat: tile nt = 4 grp + 2 i + (m >> 1), half hf = m & 1
-                    ldsm_x4(vt + vt_row(ks, lm_mat & 1, 4 * grp + 2 * i + (lm_mat >> 1), lm_row),
-                            b[i][0], b[i][1], b[i][2], b[i][3]);
-                }
+                for (int i = 0; i < 2; ++i)   // d chunk 2 grp + i: n-tiles 4 grp + 2 i, + 1
+                    vfrag(vtile, ks, 2 * grp + i, lane, b[i][0], b[i][1], b[i][2], b[i][3]);
 #pragma unroll
                 for (int i = 0; i < 2; ++i) {
                     mma_u8s8(oacc[4 * grp + 2 * i], af, b[i][0], b[i][1]);
@@ -1038,32 +1012,26 @@ __global__ void __launch_bounds__(NTHREADS, 2)
         if (lane == 0) mbar_arrive(empty_bar(s));
     }
 
-    // ---- output requantisation (Eq. 7) and 16-byte stores
+    // ---- output requantisation (Eq. 7): per row and d chunk c, four bytes
+    // d = 16c + 4t .. 16c + 4t + 3 (n-tiles 2c, 2c + 1, columns 2t, 2t + 1)
     const long long m_o = prm.m_o;
     const long long half_o = 1ll << (prm.sh_o - 1);
 #pragma unroll
     for (int rr = 0; rr < 2; ++rr) {
         const int row = wrow0 + g + 8 * rr;
         if (row >= T) continue;
-        uint32_t wout[8];
+        int8_t *dst = prm.out + (static_cast<size_t>(bh) * T + row) * DH + 4 * t4;
 #pragma unroll
-        for (int hh = 0; hh < 2; ++hh) {
+        for (int c = 0; c < 8; ++c) {
+            uint32_t w = 0;
 #pragma unroll
-            for (int wq = 0; wq < 4; ++wq) {
-                uint32_t w = 0;
-#pragma unroll
-                for (int e = 0; e < 4; ++e) {
-                    const int nt = wq * 4 + e;
-                    const long long x = m_o * oacc[nt][2 * rr + hh] + half_o;
-                    const int o = row < len ? clamp127(x >> prm.sh_o) : 0;
-                    w |= (static_cast<uint32_t>(o) & 0xffu) << (8 * e);
-                }
-                wout[hh * 4 + wq] = w;
+            for (int e = 0; e < 4; ++e) {
+                const long long x = m_o * oacc[2 * c + (e & 1)][2 * rr + (e >> 1)] + half_o;
+                const int o = row < len ? clamp127(x >> prm.sh_o) : 0;
+                w |= (static_cast<uint32_t>(o) & 0xffu) << (8 * e);
             }
+            *reinterpret_cast<uint32_t *>(dst + 16 * c) = w;
         }
-        int8_t *dst = prm.out + (static_cast<size_t>(bh) * T + row) * DH + 32 * t4;
-        *reinterpret_cast<uint4 *>(dst) = make_uint4(wout[0], wout[1], wout[2], wout[3]);
-        *reinterpret_cast<uint4 *>(dst + 16) = make_uint4(wout[4], wout[5], wout[6], wout[7]);
     }
 }
 
