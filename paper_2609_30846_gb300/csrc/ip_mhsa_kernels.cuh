@@ -9,8 +9,8 @@
 // memory accelerator (TMA) stages with the 128-byte swizzle.
 //
 // One CTA owns 64 query rows of one (b, h): four consumer warps of 16 rows
-// and one producer warp.  The producer issues the TMA loads and, for the
-// score pass, computes the bias vectors K u and P v of each staged chunk (the
+// and two producer warps.  The first issues the TMA loads; for the score
+// pass both compute the bias vectors K u and P v of each staged chunk (the
 // exact rank-1 split of (Q + 1u^T)K^T and (Q + 1v^T)P^T, since Q + u does not
 // fit an int8 operand).  The attn.V pass reads the V tile as TMA stages it:
 // transposed ldmatrix loads and byte selects build the MMA operand.
@@ -37,7 +37,8 @@ namespace ipk {
 constexpr int DH = 128;
 constexpr int MROWS = 64;                 // query rows per CTA
 constexpr int NCWARPS = 4;                // consumer warps, 16 rows each
-constexpr int NTHREADS = (NCWARPS + 1) * 32;
+constexpr int NPWARPS = 2;                // producer warps: TMA + bias vectors, bias vectors
+constexpr int NTHREADS = (NCWARPS + NPWARPS) * 32;
 constexpr int NK = 64;                    // keys per chunk
 constexpr int NSTAGE = 2;
 constexpr int BAND_ROWS = 128;            // P rows staged per chunk (NK + MROWS - 1, padded)
@@ -459,38 +460,36 @@ __device__ __forceinline__ void finish_half(int (&oacc)[16][4], uint32_t pxo, in
 
 // ---------------------------------------------------------- producer parts --
 
-// K u for the chunk's 64 keys and P v for the 128 staged band rows; lane l
-// takes keys l, l+32 and band rows l, l+32, l+64, l+96.
-__device__ __forceinline__ void prep_bias(uint32_t ktile, uint32_t ptile, uint32_t ku, uint32_t pv,
-                                          const uint32_t (&uw)[32], const uint32_t (&vw)[32],
-                                          int lane) {
+// Dot product of one staged 128-byte row (128-byte swizzle) with a vector
+// held as 32 packed words: the bias K u of a key or P v of a band row.
+__device__ __forceinline__ void bias_row(uint32_t tile, uint32_t dst, const uint32_t (&w)[32],
+                                         int row) {
+    int acc = 0;
 #pragma unroll
-    for (int k = 0; k < 2; ++k) {
-        const int row = lane + 32 * k;
-        int acc = 0;
-#pragma unroll
-        for (int ch = 0; ch < 8; ++ch) {
-            const uint4 x = lds128(ktile + swz(row, ch));
-            acc = __dp4a(static_cast<int>(x.x), static_cast<int>(uw[4 * ch + 0]), acc);
-            acc = __dp4a(static_cast<int>(x.y), static_cast<int>(uw[4 * ch + 1]), acc);
-            acc = __dp4a(static_cast<int>(x.z), static_cast<int>(uw[4 * ch + 2]), acc);
-            acc = __dp4a(static_cast<int>(x.w), static_cast<int>(uw[4 * ch + 3]), acc);
-        }
-        sts32(ku + row * 4, static_cast<uint32_t>(acc));
+    for (int ch = 0; ch < 8; ++ch) {
+        const uint4 x = lds128(tile + swz(row, ch));
+        acc = __dp4a(static_cast<int>(x.x), static_cast<int>(w[4 * ch + 0]), acc);
+        acc = __dp4a(static_cast<int>(x.y), static_cast<int>(w[4 * ch + 1]), acc);
+        acc = __dp4a(static_cast<int>(x.z), static_cast<int>(w[4 * ch + 2]), acc);
+        acc = __dp4a(static_cast<int>(x.w), static_cast<int>(w[4 * ch + 3]), acc);
     }
-#pragma unroll
-    for (int k = 0; k < 4; ++k) {
-        const int row = lane + 32 * k;
-        int acc = 0;
-#pragma unroll
-        for (int ch = 0; ch < 8; ++ch) {
-            const uint4 x = lds128(ptile + swz(row, ch));
-            acc = __dp4a(static_cast<int>(x.x), static_cast<int>(vw[4 * ch + 0]), acc);
-            acc = __dp4a(static_cast<int>(x.y), static_cast<int>(vw[4 * ch + 1]), acc);
-            acc = __dp4a(static_cast<int>(x.z), static_cast<int>(vw[4 * ch + 2]), acc);
-            acc = __dp4a(static_cast<int>(x.w), static_cast<int>(vw[4 * ch + 3]), acc);
-        }
-        sts32(pv + row * 4, static_cast<uint32_t>(acc));
+    sts32(dst + row * 4, static_cast<uint32_t>(acc));
+}
+
+// The two producer warps share the bias vectors of a staged chunk (192 dot
+// products): warp 0 takes K u of keys l, l + 32 and P v of band row l, warp
+// 1 P v of band rows 32 + l, 64 + l, 96 + l.
+__device__ __forceinline__ void prep_bias(int pw, uint32_t ktile, uint32_t ptile, uint32_t ku,
+                                          uint32_t pv, const uint32_t (&uw)[32],
+                                          const uint32_t (&vw)[32], int lane) {
+    if (pw == 0) {
+        bias_row(ktile, ku, uw, lane);
+        bias_row(ktile, ku, uw, lane + 32);
+        bias_row(ptile, pv, vw, lane);
+    } else {
+        bias_row(ptile, pv, vw, lane + 32);
+        bias_row(ptile, pv, vw, lane + 64);
+        bias_row(ptile, pv, vw, lane + 96);
     }
 }
 
@@ -571,7 +570,7 @@ __global__ void __launch_bounds__(NTHREADS, 2)
     if (threadIdx.x == 0) {
         for (int s = 0; s < NSTAGE; ++s) {
             mbar_init(full_bar(s), 1);
-            mbar_init(ready_bar(s), 1);
+            mbar_init(ready_bar(s), NPWARPS);
             mbar_init(empty_bar(s), NCWARPS);
         }
         mbar_init(never_bar, 1);
@@ -594,7 +593,8 @@ __global__ void __launch_bounds__(NTHREADS, 2)
     // Use `it` of the stage ring (stage it & 1, phase it >> 1): TMA lands
     // (full), the producer prepares it (ready), the consumers release it
     // (empty), and the stage is refilled with use it + 2.
-    if (warp == NCWARPS) {
+    if (warp >= NCWARPS) {
+        const int pw = warp - NCWARPS;   // 0: TMA and its share of the biases; 1: its share
         uint32_t uw[32], vw[32];
         {
             const uint4 *u4 = reinterpret_cast<const uint4 *>(prm.u + static_cast<size_t>(h) * DH);
@@ -621,6 +621,22 @@ __global__ void __launch_bounds__(NTHREADS, 2)
                 tma_load_3d(dst, &tm_v, 0, j0, bh, full_bar(s));
             }
         };
+        if (pw == 1) {
+            // second producer warp: its share of the bias vectors of each
+            // staged score-pass chunk
+            for (int it = 0; it < nchunks; ++it) {
+                const int s = it & 1;
+                if (!warp_wait(full_bar(s), (it >> 1) & 1, prm.timeout_cycles)) {
+                    if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_FULL);
+                    return;
+                }
+                prep_bias(1, stage_addr(s), stage_addr(s) + K_TILE_BYTES, stage_addr(s) + KU_OFF,
+                          stage_addr(s) + PV_OFF, uw, vw, lane);
+                __syncwarp();
+                if (lane == 0) mbar_arrive(ready_bar(s));
+            }
+            return;
+        }
         int issued = total > 1 ? 2 : 1, landed = 0;
         bool ok = true;
         if (lane == 0) {
@@ -637,7 +653,7 @@ __global__ void __launch_bounds__(NTHREADS, 2)
                     break;
                 }
                 landed = it + 1;
-                prep_bias(stage_addr(s), stage_addr(s) + K_TILE_BYTES, stage_addr(s) + KU_OFF,
+                prep_bias(0, stage_addr(s), stage_addr(s) + K_TILE_BYTES, stage_addr(s) + KU_OFF,
                           stage_addr(s) + PV_OFF, uw, vw, lane);
                 __syncwarp();
                 if (lane == 0) mbar_arrive(ready_bar(s));
