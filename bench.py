@@ -256,11 +256,12 @@ def run_reference(args):
 
 # The projections around the attention of one encoder block (B=32, T=375,
 # d=1024): Q/K/V stacked and written head-split, the output projection from
-# the heads, and the feed-forward pair with the fused minimax Swish.
+# the attention's row-major output, and the feed-forward pair with the fused
+# minimax Swish.
 NEXT_ROWS = [
     # name, K, N, groups, x_layout, y_layout, swish
     ("linear_qkv_1024x3072_heads", 1024, 3072, 3, 0, 1, False),
-    ("linear_out_heads_1024x1024", 1024, 1024, 1, 1, 0, False),
+    ("linear_out_1024x1024", 1024, 1024, 1, 0, 0, False),   # reads the attention's row-major O
     ("ffn1_swish_1024x4096", 1024, 4096, 1, 0, 0, True),
     ("ffn2_4096x1024", 4096, 1024, 1, 0, 0, False),
 ]

@@ -255,6 +255,18 @@ int ip_layernorm_constants(double S_x, const double *gamma, const double *beta, 
                            double S_y, double eps, long long *eps_c, int32_t *M, long long *B,
                            int32_t *E);
 
+/* ip_relpos_mhsa_i8 with a choice of output layout: out_layout =
+ * IP_LAYOUT_HEADS writes [B][H][T][dh] (as ip_relpos_mhsa_i8), IP_LAYOUT_ROWS
+ * writes [B][T][H][dh], i.e. [B][T][H dh] row-major, the frames' rows that
+ * the output projection (ip_linear_i8 with a row-major input) reads.  Other
+ * values: IP_ERR_PARAM.  Everything else as ip_relpos_mhsa_i8. */
+int ip_relpos_mhsa_i8_ex(const int8_t *q, const int8_t *k, const int8_t *v, const int8_t *p,
+                         const int8_t *u, const int8_t *v_bias, const int32_t *multipliers,
+                         const int32_t *shifts, const ip_isoftmax_params *sm,
+                         const int32_t *lengths, int B, int H, int T, int dh, int8_t *out,
+                         int out_layout, void *workspace, size_t workspace_bytes,
+                         ip_stream_t stream);
+
 /* Text of an IP_* code. */
 const char *ip_strerror(int code);
 

@@ -31,7 +31,7 @@ EXPORTS = (
     "ip_dyadic_pair",
     "ip_isoftmax_params_from_scale", "ip_probe_int8_mma", "ip_relpos_mhsa_i8_noalloc",
     "ip_debug_set_split_mode", "ip_linear_i8", "ip_linear_swish_i8", "ip_swish_params_from_scales",
-    "ip_layernorm_i8", "ip_layernorm_constants",
+    "ip_layernorm_i8", "ip_layernorm_constants", "ip_relpos_mhsa_i8_ex",
 )
 
 ROWS = 0    # IP_LAYOUT_ROWS:  [B][T][C]
@@ -109,6 +109,9 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
         lib.ip_dyadic_pair.restype = I
         lib.ip_isoftmax_params_from_scale.argtypes = [ctypes.c_double, ctypes.POINTER(SoftmaxParams)]
         lib.ip_isoftmax_params_from_scale.restype = I
+        lib.ip_relpos_mhsa_i8_ex.argtypes = [P] * 6 + [P, P, ctypes.POINTER(SoftmaxParams), P] + [
+            I] * 4 + [P, I, P, ctypes.c_size_t, P]
+        lib.ip_relpos_mhsa_i8_ex.restype = I
         lib.ip_linear_i8.argtypes = [P, I, P, P, P, P, I, I, I, I, I, P, I, P, ctypes.c_size_t, P]
         lib.ip_linear_i8.restype = I
         lib.ip_linear_swish_i8.argtypes = [P, P, P, P, P, ctypes.POINTER(SwishParams), I, I, I, I,
@@ -234,28 +237,30 @@ def _dev_ptr(t, name, dtype, shape):
 
 
 def relpos_mhsa_i8(q, k, v, p, u, v_bias, consts: LayerConstants, lengths=None, out=None,
-                   workspace=None, stream=None):
+                   workspace=None, stream=None, out_layout: int = HEADS):
     """Whole layer on the GPU.  q, k, v: int8 [B, H, T, 128] CUDA tensors;
     p: int8 [H, 2T-1, 128]; u, v_bias: int8 [H, 128]; lengths: int32 [B]
-    CUDA tensor or None.  Returns out (int8 [B, H, T, 128]).  Asynchronous on
-    `stream` (default: torch's current stream)."""
+    CUDA tensor or None.  Returns out: int8 [B, H, T, 128] (HEADS) or
+    [B, T, H, 128] (ROWS, the frames' rows of the output projection).
+    Asynchronous on `stream` (default: torch's current stream)."""
     import torch
     B, H, T, dh = q.shape
     shp = (B, H, T, dh)
+    oshp = shp if out_layout == HEADS else (B, T, H, dh)
     args = [_dev_ptr(q, "q", torch.int8, shp), _dev_ptr(k, "k", torch.int8, shp),
             _dev_ptr(v, "v", torch.int8, shp), _dev_ptr(p, "p", torch.int8, (H, 2 * T - 1, dh)),
             _dev_ptr(u, "u", torch.int8, (H, dh)), _dev_ptr(v_bias, "v_bias", torch.int8, (H, dh))]
     if out is None:
-        out = torch.empty(shp, dtype=torch.int8, device=q.device)
+        out = torch.empty(oshp, dtype=torch.int8, device=q.device)
     lens = None if lengths is None else _dev_ptr(lengths, "lengths", torch.int32, (B,))
     if workspace is None:
         workspace = torch.zeros(workspace_bytes(B, H, T, dh), dtype=torch.uint8, device=q.device)
     sm = SoftmaxParams(*consts.softmax)
-    rc = load().ip_relpos_mhsa_i8(
+    rc = load().ip_relpos_mhsa_i8_ex(
         *args, _arr(consts.multipliers, ctypes.c_int32), _arr(consts.shifts, ctypes.c_int32),
-        ctypes.byref(sm), lens, B, H, T, dh, _dev_ptr(out, "out", torch.int8, shp),
+        ctypes.byref(sm), lens, B, H, T, dh, _dev_ptr(out, "out", torch.int8, oshp), out_layout,
         ctypes.c_void_p(workspace.data_ptr()), workspace.numel(), _stream_handle(stream))
-    _check("ip_relpos_mhsa_i8", rc)
+    _check("ip_relpos_mhsa_i8_ex", rc)
     return out
 
 

@@ -161,6 +161,17 @@ int ip_relpos_mhsa_i8(const int8_t *q, const int8_t *k, const int8_t *v, const i
                       const int32_t *shifts, const ip_isoftmax_params *sm,
                       const int32_t *lengths, int B, int H, int T, int dh, int8_t *out,
                       void *workspace, size_t workspace_bytes, ip_stream_t stream) {
+    return ip_relpos_mhsa_i8_ex(q, k, v, p, u, v_bias, multipliers, shifts, sm, lengths, B, H, T,
+                                dh, out, IP_LAYOUT_HEADS, workspace, workspace_bytes, stream);
+}
+
+int ip_relpos_mhsa_i8_ex(const int8_t *q, const int8_t *k, const int8_t *v, const int8_t *p,
+                         const int8_t *u, const int8_t *v_bias, const int32_t *multipliers,
+                         const int32_t *shifts, const ip_isoftmax_params *sm,
+                         const int32_t *lengths, int B, int H, int T, int dh, int8_t *out,
+                         int out_layout, void *workspace, size_t workspace_bytes,
+                         ip_stream_t stream) {
+    if (out_layout != IP_LAYOUT_ROWS && out_layout != IP_LAYOUT_HEADS) return IP_ERR_PARAM;
     int rc = check_shape(B, H, T, dh);
     if (rc != IP_OK) return rc;
     if (B == 0 || H == 0) return IP_OK;   // empty problem: nothing to read or write
@@ -224,6 +235,7 @@ int ip_relpos_mhsa_i8(const int8_t *q, const int8_t *k, const int8_t *v, const i
     prm.split_h0 = sp.h0;
     prm.split_tile0 = sp.tile0;
     prm.first_split = sp.first;
+    prm.out_rows = out_layout == IP_LAYOUT_ROWS ? 1 : 0;
     const dim3 grid1(ntiles, H, B + sp.extra);
     ipk::relpos_mhsa_fused_kernel<<<grid1, ipk::NTHREADS, smem, st>>>(tm_k, tm_v, tm_p, prm);
     if (cudaGetLastError() != cudaSuccess) return IP_ERR_CUDA;

@@ -91,7 +91,14 @@ struct FusedParams {
     // 32 rows each by the CTAs of the grid slices z >= B (dispatched last).
     int nsplit, split_b0, split_h0, split_tile0;
     long long first_split;    // linear index of the first split tile
+    int out_rows;             // output [B][T][H][DH] instead of [B][H][T][DH]
 };
+
+// Offset of output row `row` of (b, h).
+__device__ __forceinline__ size_t out_offset(const FusedParams &p, int b, int h, int row) {
+    return p.out_rows ? ((static_cast<size_t>(b) * p.T + row) * p.H + h) * DH
+                      : ((static_cast<size_t>(b) * p.H + h) * p.T + row) * DH;
+}
 
 constexpr int ERR_TIMEOUT_FULL = 1;
 constexpr int ERR_TIMEOUT_EMPTY = 2;
@@ -430,8 +437,9 @@ __device__ __forceinline__ void send_partial(const int (&oacc)[16][4], uint32_t 
 // per row and d chunk: d = 16c + 4t .. 16c + 4t + 3 for c in 4 HK .. 4 HK + 3.
 template <int HK>
 __device__ __forceinline__ void finish_half(int (&oacc)[16][4], uint32_t pxo, int lane, int wrow0,
-                                            int T, int len, size_t bh, long long m_o,
-                                            long long half_o, int sh_o, int8_t *out) {
+                                            int len, const FusedParams &prm, int b, int h,
+                                            long long m_o, long long half_o) {
+    const int T = prm.T, sh_o = prm.sh_o;
     const int g = lane >> 2, t4 = lane & 3;
 #pragma unroll
     for (int i = 0; i < 8; ++i)
@@ -442,7 +450,7 @@ __device__ __forceinline__ void finish_half(int (&oacc)[16][4], uint32_t pxo, in
     for (int rr = 0; rr < 2; ++rr) {
         const int row = wrow0 + g + 8 * rr;
         if (row >= T) continue;
-        int8_t *dst = out + (bh * T + row) * DH + 4 * t4;
+        int8_t *dst = prm.out + out_offset(prm, b, h, row) + 4 * t4;
 #pragma unroll
         for (int c = 4 * HK; c < 4 * HK + 4; ++c) {
             uint32_t w = 0;
@@ -550,9 +558,9 @@ __global__ void __launch_bounds__(NTHREADS, 2)
         if (r0 >= len) {
             // Every row of this tile (half) is padding: write zeros.
             const int rows = (T - r0) < nrows ? (T - r0) : nrows;
-            int4 *dst = reinterpret_cast<int4 *>(prm.out + (static_cast<size_t>(bh) * T + r0) * DH);
             for (int c = threadIdx.x; c < rows * (DH / 16); c += NTHREADS)
-                dst[c] = make_int4(0, 0, 0, 0);
+                *reinterpret_cast<int4 *>(prm.out + out_offset(prm, b, h, r0 + (c >> 3)) +
+                                          16 * (c & 7)) = make_int4(0, 0, 0, 0);
             return;
         }
     }
@@ -862,11 +870,9 @@ __global__ void __launch_bounds__(NTHREADS, 2)
         const long long m_o = prm.m_o;
         const long long half_o = 1ll << (prm.sh_o - 1);
         if (hk == 0)
-            finish_half<0>(oacc, xpart + XO_OFF, lane, wrow0, T, len, bh, m_o, half_o, prm.sh_o,
-                           prm.out);
+            finish_half<0>(oacc, xpart + XO_OFF, lane, wrow0, len, prm, b, h, m_o, half_o);
         else
-            finish_half<1>(oacc, xpart + XO_OFF, lane, wrow0, T, len, bh, m_o, half_o, prm.sh_o,
-                           prm.out);
+            finish_half<1>(oacc, xpart + XO_OFF, lane, wrow0, len, prm, b, h, m_o, half_o);
         return;
     }
 
@@ -1036,7 +1042,7 @@ __global__ void __launch_bounds__(NTHREADS, 2)
     for (int rr = 0; rr < 2; ++rr) {
         const int row = wrow0 + g + 8 * rr;
         if (row >= T) continue;
-        int8_t *dst = prm.out + (static_cast<size_t>(bh) * T + row) * DH + 4 * t4;
+        int8_t *dst = prm.out + out_offset(prm, b, h, row) + 4 * t4;
 #pragma unroll
         for (int c = 0; c < 8; ++c) {
             uint32_t w = 0;

@@ -81,3 +81,20 @@ def test_modes_agree_on_the_encoder_layer(ip):
     ip.set_split_mode(-1)
     assert_same(outs[1], outs[0])
     assert_same(outs[2], outs[0])
+
+
+@pytest.mark.parametrize("T,masked", [(75, False), (150, True), (375, False)])
+def test_row_major_output_is_the_transpose(ip, orc, mode, T, masked):
+    # the frames' rows [B, T, H, 128] for the output projection, every tile
+    # path (whole, split, padding rows)
+    lengths = np.array([T, max(1, T // 3), T // 2 + 1], np.int32) if masked else None
+    lay = synth.draw(3, 8, T, 128, seed=970 + T, p_mode="sinusoid", masked=masked, lengths=lengths)
+    c = ip.layer_constants(lay.scales)
+    want = oracle_out(orc, lay, c, lay.lengths)
+    d = lambda a: torch.from_numpy(np.ascontiguousarray(a)).cuda()
+    ws = torch.zeros(ip.workspace_bytes(3, 8, T, 128), dtype=torch.uint8, device="cuda")
+    lens = None if lay.lengths is None else d(lay.lengths.astype(np.int32))
+    got = ip.relpos_mhsa_i8(d(lay.q), d(lay.k), d(lay.v), d(lay.p), d(lay.u), d(lay.vb), c,
+                            lengths=lens, workspace=ws, out_layout=ip.ROWS)
+    assert ip.status(ws) == 0
+    assert_same(got.cpu().numpy(), np.ascontiguousarray(want.transpose(0, 2, 1, 3)))
