@@ -24,11 +24,12 @@ import numpy as np
 from .consts import (IBERT_A, IBERT_B, IBERT_C, LayerConstants, dyadic,
                      dyadic_pair, isoftmax_params, layer_constants, linear_constants,
                      SWISH_A, SWISH_C, SwishParams, swish_params, NormConstants,
-                     layernorm_constants)
+                     layernorm_constants, residual_params, glu_params, Swish16Params,
+                     swish16_params)
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
-_SRCS = [os.path.join(_HERE, f) for f in ("ipo_mhsa.c", "ipo_linear.c", "ipo_norm.c")]
-_HDRS = [os.path.join(_HERE, f) for f in ("ipo_mhsa.h", "ipo_linear.h", "ipo_norm.h")]
+_SRCS = [os.path.join(_HERE, f) for f in ("ipo_mhsa.c", "ipo_linear.c", "ipo_norm.c", "ipo_block.c")]
+_HDRS = [os.path.join(_HERE, f) for f in ("ipo_mhsa.h", "ipo_linear.h", "ipo_norm.h", "ipo_block.h")]
 _LIB = os.path.join(_HERE, "libipo_mhsa.so")
 _lock = threading.Lock()
 _lib = None
@@ -72,6 +73,14 @@ def _load():
             lib.ipo_linear_i8.restype = ctypes.c_int
             lib.ipo_swish_i8.argtypes = [P, ctypes.c_longlong, P, P]
             lib.ipo_swish_i8.restype = ctypes.c_int
+            LL = ctypes.c_longlong
+            lib.ipo_residual_i8.argtypes = [P, P, LL, i32, i32, i32, P]
+            lib.ipo_glu_i8.argtypes = [P, LL, ctypes.c_int, P, P]
+            lib.ipo_dwconv_i16.argtypes = [P, ctypes.c_int, ctypes.c_int, ctypes.c_int, P,
+                                           ctypes.c_int, P, P, P, P]
+            lib.ipo_swish_i16.argtypes = [P, LL, P, P]
+            for f in (lib.ipo_residual_i8, lib.ipo_glu_i8, lib.ipo_dwconv_i16, lib.ipo_swish_i16):
+                f.restype = ctypes.c_int
             lib.ipo_isqrt.argtypes = [ctypes.c_int64]
             lib.ipo_isqrt.restype = ctypes.c_int64
             lib.ipo_layernorm_i8.argtypes = [P, ctypes.c_longlong, ctypes.c_int, ctypes.c_int64,
@@ -221,6 +230,60 @@ def swish(z, p: SwishParams) -> np.ndarray:
     return y
 
 
+class _Swish16(ctypes.Structure):
+    _fields_ = [("q_c", ctypes.c_int32), ("q_one", ctypes.c_int64), ("m", ctypes.c_int32),
+                ("s", ctypes.c_int32)]
+
+
+def residual(x, y, m_x: int, m_y: int, s: int) -> np.ndarray:
+    """Residual addition of two int8 tensors onto one int8 grid (Eqs. 1-4)."""
+    x = np.ascontiguousarray(x, dtype=np.int8)
+    y = np.ascontiguousarray(y, dtype=np.int8)
+    assert x.shape == y.shape
+    z = np.empty_like(x)
+    _check(_load().ipo_residual_i8(_ptr(x), _ptr(y), x.size, m_x, m_y, s, _ptr(z)),
+           "ipo_residual_i8")
+    return z
+
+
+def glu(ab, p: SwishParams) -> np.ndarray:
+    """Gated linear unit a sigma(b) over the last axis [a | b] of int8 ab."""
+    ab = np.ascontiguousarray(ab, dtype=np.int8)
+    C2 = ab.shape[-1]
+    rows = ab.size // C2
+    y = np.empty(ab.shape[:-1] + (C2 // 2,), dtype=np.int8)
+    prm = _Swish(p.q_c, p.q_one, p.m, p.s)
+    _check(_load().ipo_glu_i8(_ptr(ab), rows, C2 // 2, ctypes.addressof(prm), _ptr(y)),
+           "ipo_glu_i8")
+    return y
+
+
+def dwconv(x, w, bias, m, s) -> np.ndarray:
+    """Depthwise convolution over time with folded BatchNorm onto INT16,
+    x int8 [B, T, C], w int8 [C, K]."""
+    x = np.ascontiguousarray(x, dtype=np.int8)
+    w = np.ascontiguousarray(w, dtype=np.int8)
+    B, T, C = x.shape
+    K = w.shape[1]
+    y = np.empty((B, T, C), dtype=np.int16)
+    b = np.ascontiguousarray(bias, dtype=np.int32)
+    m = np.ascontiguousarray(m, dtype=np.int32)
+    s = np.ascontiguousarray(s, dtype=np.int32)
+    _check(_load().ipo_dwconv_i16(_ptr(x), B, T, C, _ptr(w), K, _ptr(b), _ptr(m), _ptr(s),
+                                  _ptr(y)), "ipo_dwconv_i16")
+    return y
+
+
+def swish16(z, p: "Swish16Params") -> np.ndarray:
+    """Integer Swish of INT16 values onto int8."""
+    z = np.ascontiguousarray(z, dtype=np.int16)
+    y = np.empty(z.shape, dtype=np.int8)
+    prm = _Swish16(p.q_c, p.q_one, p.m, p.s)
+    _check(_load().ipo_swish_i16(_ptr(z), z.size, ctypes.addressof(prm), _ptr(y)),
+           "ipo_swish_i16")
+    return y
+
+
 def isqrt(n: int) -> int:
     """floor(sqrt(n)) of the oracle's integer Newton iteration, 0 <= n < 2^62."""
     return int(_load().ipo_isqrt(int(n)))
@@ -242,7 +305,8 @@ def layernorm(x, c: "NormConstants") -> np.ndarray:
 
 
 __all__ = ["build", "linear", "swish", "isqrt", "layernorm", "layernorm_constants",
-           "NormConstants", "swish_params", "SwishParams", "SWISH_A", "SWISH_C", "linear_constants", "ROWS", "HEADS", "relpos_mhsa", "content_scores", "position_scores",
+           "NormConstants", "residual", "glu", "dwconv", "swish16", "residual_params",
+           "glu_params", "swish16_params", "Swish16Params", "swish_params", "SwishParams", "SWISH_A", "SWISH_C", "linear_constants", "ROWS", "HEADS", "relpos_mhsa", "content_scores", "position_scores",
            "fused_scores", "iexp", "isoftmax", "set_threads", "dyadic",
            "dyadic_pair", "isoftmax_params", "layer_constants", "LayerConstants",
            "IBERT_A", "IBERT_B", "IBERT_C", "OracleError"]

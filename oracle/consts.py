@@ -166,3 +166,38 @@ def layernorm_constants(s_x: float, gamma, beta, s_y: float, eps: float = 1e-5) 
         B[i] = b
     eps_c = int(math.floor(eps * d * d / (s_x * s_x) + 0.5))
     return NormConstants(eps_c, M, B, E)
+
+
+def residual_params(s_x: float, s_y: float, s_z: float, alpha: float = 1.0) -> tuple[int, int, int]:
+    """(m_x, m_y, s) of the residual addition z = x + alpha y (Eqs. 1-4) onto
+    S_z: the dyadic pair of S_x / S_z and alpha S_y / S_z on one shift."""
+    return dyadic_pair(s_x / s_z, alpha * s_y / s_z)
+
+
+def glu_params(s_a: float, s_b: float, s_y: float, a: float = SWISH_A,
+               c: float = SWISH_C) -> SwishParams:
+    """Constants of GLU(a, b) = a sigma(b), sigma(b) = (1 + tanh(b/2)) / 2
+    with the minimax tanh: q_c, q_one on the grid of b, and the dyadic of
+    S_a S_t / (2 S_y), S_t = |a| (S_b/2)^2."""
+    s_t = abs(a) * (s_b / 2.0) ** 2
+    q_c = int(math.floor(2.0 * c / s_b + 0.5))
+    q_one = int(math.floor(1.0 / s_t + 0.5))
+    m, s = dyadic(s_a * s_t / (2.0 * s_y))
+    return SwishParams(q_c, q_one, m, s)
+
+
+@dataclass(frozen=True)
+class Swish16Params:
+    q_c: int
+    q_one: int
+    m: int
+    s: int
+
+
+def swish16_params(s_z: float, s_y: float, a: float = SWISH_A, c: float = SWISH_C) -> Swish16Params:
+    """Swish constants for an INT16 input grid S_z (the BatchNorm output of
+    Sec. 3.3) onto an int8 grid S_y; as swish_params."""
+    p = swish_params(s_z, s_y, a, c)
+    if not (1 <= p.q_c < 2 ** 16 and 1 <= p.q_one < 2 ** 31 and p.q_one >= p.q_c ** 2):
+        raise ValueError(f"INT16 grid {s_z!r} outside the Swish domain (q_c={p.q_c}, q_one={p.q_one})")
+    return Swish16Params(p.q_c, p.q_one, p.m, p.s)

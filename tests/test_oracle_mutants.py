@@ -98,6 +98,27 @@ NORM_MUTANTS = {
 
 NORM_PINS = ["tests/test_oracle_norm.py"]
 
+# mistakes planted in the block oracle (residual, GLU, depthwise conv, INT16 Swish)
+BLOCK_MUTANTS = {
+    "res_drop_y": ("int64_t v = (int64_t)m_x * x[i] + (int64_t)m_y * y[i];",
+                   "int64_t v = (int64_t)m_x * x[i];"),
+    "glu_swap": ("int64_t a = ab[(size_t)r * 2 * C + c];\n            int64_t b = ab[(size_t)r * 2 * C + C + c];",
+                 "int64_t b = ab[(size_t)r * 2 * C + c];\n            int64_t a = ab[(size_t)r * 2 * C + C + c];"),
+    "glu_sign": ("int64_t t = (int64_t)p->q_one + sg * L;                   /* 1 + tanh */",
+                 "int64_t t = (int64_t)p->q_one - sg * L;                   /* 1 + tanh */"),
+    "dw_wrap": ("if (tt < 0 || tt >= T) continue;               /* zero padding */",
+                "tt = (tt + T) % T;"),
+    "dw_flip": ("acc += (int64_t)w[(size_t)c * K + k] * x",
+                "acc += (int64_t)w[(size_t)c * K + (K - 1 - k)] * x"),
+    "dw_no_bias": ("int64_t acc = bias[c];", "int64_t acc = 0;"),
+    "sw16_clip": ("int64_t dclip = (mag < p->q_c ? mag : p->q_c) - p->q_c;\n        int64_t L = p->q_one",
+                  "int64_t dclip = mag - p->q_c;\n        int64_t L = p->q_one"),
+    "sw16_overflow": ("__int128 v = (__int128)p->m * (__int128)(q * t)",
+                      "__int128 v = (__int128)(int64_t)((uint64_t)p->m * (uint64_t)(q * t))"),
+}
+
+BLOCK_PINS = ["tests/test_oracle_block.py"]
+
 PINS = [
     "tests/test_oracle_relshift.py",
     "tests/test_oracle_scores.py",
@@ -118,7 +139,7 @@ def _copy_tree(dst):
 
 
 GROUPS = [(MUTANTS, PINS, "ipo_mhsa.c"), (LINEAR_MUTANTS, LINEAR_PINS, "ipo_linear.c"),
-          (NORM_MUTANTS, NORM_PINS, "ipo_norm.c")]
+          (NORM_MUTANTS, NORM_PINS, "ipo_norm.c"), (BLOCK_MUTANTS, BLOCK_PINS, "ipo_block.c")]
 
 
 @pytest.mark.slow
