@@ -255,6 +255,70 @@ int ip_layernorm_constants(double S_x, const double *gamma, const double *beta, 
                            double S_y, double eps, long long *eps_c, int32_t *M, long long *B,
                            int32_t *E);
 
+/* ---- rest of the Conformer block (Sec. 2.1 Eqs. 1-5, Sec. 3.3) ---------- */
+
+/* Residual addition of two int8 tensors of n elements on grids S_x, S_y onto
+ * S_z (Eqs. 1-4; the feed-forward branches enter with alpha = 1/2):
+ *   z = clamp(round(2^-(31+s) (m_x x + m_y y)), -127, 127)
+ * (m_x, m_y, s) from ip_residual_params (one shared shift, as Eq. 11).
+ * x, y, z: device, 16-byte aligned; m_x, m_y in [0, 2^31), s in [0, 31].
+ * n == 0 returns IP_OK without touching any pointer.  Asynchronous on
+ * `stream`.  Returns IP_OK or IP_ERR_*. */
+int ip_residual_i8(const int8_t *x, const int8_t *y, long long n, int32_t m_x, int32_t m_y,
+                   int32_t s, int8_t *z, ip_stream_t stream);
+
+/* (m_x, m_y, s) of z = x + alpha y onto S_z (host, float64). */
+int ip_residual_params(double S_x, double S_y, double S_z, double alpha, int32_t *m_x,
+                       int32_t *m_y, int32_t *s);
+
+/* The ConvBlock's first pointwise convolution with the gated linear unit of
+ * Eq. 5 fused: the projection x W^T onto the int8 grids of a and b (m, s per
+ * row of w), then GLU(a, b) = a sigma(b), sigma(b) = (1 + tanh(b/2)) / 2 with
+ * the minimax tanh:
+ *   D = min(|b|, q_c) - q_c;  t = q_one + sgn(b) (q_one - D^2)
+ *   y = clamp(round(2^-(31+s) m a t), -127, 127)
+ * w: device int8 [N][K] with the rows of a and b interleaved (row 2c is a_c,
+ * row 2c + 1 is b_c; N even, output channels N/2); bias, m, s per row as
+ * ip_linear_i8; glu: host constants (ip_glu_params), q_c and q_one from S_b.
+ * x: [B][T][K] row-major; y: [B][T][N/2] row-major.  Other arguments and
+ * errors as ip_linear_i8. */
+int ip_linear_glu_i8(const int8_t *x, const int8_t *w, const int32_t *bias, const int32_t *m,
+                     const int32_t *s, const ip_swish_params *glu, int B, int T, int K, int N,
+                     int8_t *y, void *workspace, size_t workspace_bytes, ip_stream_t stream);
+
+/* GLU constants for the grids S_a, S_b of the two halves and S_y of the
+ * output (host, float64): q_c = round(2c / S_b), q_one = round(1 / S_t),
+ * S_t = |a| (S_b/2)^2, m 2^-(31+s) = S_a S_t / (2 S_y). */
+int ip_glu_params(double S_a, double S_b, double S_y, ip_swish_params *out);
+
+/* Swish constants for an INT16 input (the BatchNorm output, Sec. 3.3):
+ * q_c in [1, 2^16), q_one in [1, 2^31) with q_one >= q_c^2, m, s. */
+typedef struct {
+    int32_t q_c;
+    long long q_one;
+    int32_t m, s;
+} ip_swish16_params;
+
+/* Depthwise convolution over time with BatchNorm folded into w and bias
+ * (Sec. 2.2), onto the INT16 grid (Sec. 3.3), then the minimax Swish onto
+ * int8 (the INT16 tensor never reaches memory):
+ *   acc = sum_k w[c][k] x[b][t + k - K/2][c] + bias[c]   (zero padding)
+ *   z   = clamp(round(2^-(31+s[c]) m[c] acc), -32767, 32767)
+ *   y   = Swish(z) with the steps of ip_linear_swish_i8 on z's grid; the
+ *         product m z t (up to 78 bits) is formed exactly.
+ * x, y: device int8 [B][T][C] row-major; w: device int8 [C][K], K odd in
+ * [1, 15]; bias, m, s: device int32 [C] (|bias| < 2^30, m >= 0, s in
+ * [0, 31]; out-of-domain values are clamped and reported as IP_ERR_PARAM by
+ * ip_relpos_mhsa_status); sw: host (IP_ERR_PARAM outside its domain).
+ * Workspace as ip_relpos_mhsa_i8.  Returns IP_OK or IP_ERR_*. */
+int ip_dwconv_swish_i8(const int8_t *x, int B, int T, int C, const int8_t *w, int K,
+                       const int32_t *bias, const int32_t *m, const int32_t *s,
+                       const ip_swish16_params *sw, int8_t *y, void *workspace,
+                       size_t workspace_bytes, ip_stream_t stream);
+
+/* Swish constants of an INT16 input grid S_z and int8 output grid S_y. */
+int ip_swish16_params_from_scales(double S_z, double S_y, ip_swish16_params *out);
+
 /* ip_relpos_mhsa_i8 with a choice of output layout: out_layout =
  * IP_LAYOUT_HEADS writes [B][H][T][dh] (as ip_relpos_mhsa_i8), IP_LAYOUT_ROWS
  * writes [B][T][H][dh], i.e. [B][T][H dh] row-major, the frames' rows that

@@ -31,7 +31,9 @@ EXPORTS = (
     "ip_dyadic_pair",
     "ip_isoftmax_params_from_scale", "ip_probe_int8_mma", "ip_relpos_mhsa_i8_noalloc",
     "ip_debug_set_split_mode", "ip_linear_i8", "ip_linear_swish_i8", "ip_swish_params_from_scales",
-    "ip_layernorm_i8", "ip_layernorm_constants", "ip_relpos_mhsa_i8_ex",
+    "ip_layernorm_i8", "ip_layernorm_constants", "ip_relpos_mhsa_i8_ex", "ip_residual_i8",
+    "ip_residual_params", "ip_linear_glu_i8", "ip_glu_params", "ip_dwconv_swish_i8",
+    "ip_swish16_params_from_scales",
 )
 
 ROWS = 0    # IP_LAYOUT_ROWS:  [B][T][C]
@@ -52,6 +54,11 @@ class IpError(RuntimeError):
 
 class SwishParams(ctypes.Structure):
     _fields_ = [("q_c", ctypes.c_int32), ("q_one", ctypes.c_int32), ("m", ctypes.c_int32),
+                ("s", ctypes.c_int32)]
+
+
+class Swish16Params(ctypes.Structure):
+    _fields_ = [("q_c", ctypes.c_int32), ("q_one", ctypes.c_longlong), ("m", ctypes.c_int32),
                 ("s", ctypes.c_int32)]
 
 
@@ -126,6 +133,21 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
         D = ctypes.c_double
         lib.ip_layernorm_constants.argtypes = [D, P, P, I, D, D, ctypes.POINTER(LL), P, P, P]
         lib.ip_layernorm_constants.restype = I
+        i32p_ = ctypes.POINTER(ctypes.c_int32)
+        lib.ip_residual_i8.argtypes = [P, P, ctypes.c_longlong, I, I, I, P, P]
+        lib.ip_residual_i8.restype = I
+        lib.ip_residual_params.argtypes = [D, D, D, D, i32p_, i32p_, i32p_]
+        lib.ip_residual_params.restype = I
+        lib.ip_linear_glu_i8.argtypes = [P, P, P, P, P, ctypes.POINTER(SwishParams), I, I, I, I, P,
+                                         P, ctypes.c_size_t, P]
+        lib.ip_linear_glu_i8.restype = I
+        lib.ip_glu_params.argtypes = [D, D, D, ctypes.POINTER(SwishParams)]
+        lib.ip_glu_params.restype = I
+        lib.ip_dwconv_swish_i8.argtypes = [P, I, I, I, P, I, P, P, P, ctypes.POINTER(Swish16Params),
+                                           P, P, ctypes.c_size_t, P]
+        lib.ip_dwconv_swish_i8.restype = I
+        lib.ip_swish16_params_from_scales.argtypes = [D, D, ctypes.POINTER(Swish16Params)]
+        lib.ip_swish16_params_from_scales.restype = I
         lib.ip_probe_int8_mma.argtypes = [I, I, P, P]
         lib.ip_probe_int8_mma.restype = ctypes.c_longlong
         _lib = lib
@@ -414,6 +436,89 @@ def layernorm_i8(x, M, B, E, eps_c: int, *, out=None, workspace=None, stream=Non
     return out
 
 
+def residual_params(s_x: float, s_y: float, s_z: float, alpha: float = 1.0):
+    """(m_x, m_y, s) of z = x + alpha y onto S_z (Eqs. 1-4)."""
+    a, b, s = ctypes.c_int32(), ctypes.c_int32(), ctypes.c_int32()
+    _check("ip_residual_params", load().ip_residual_params(s_x, s_y, s_z, alpha, ctypes.byref(a),
+                                                          ctypes.byref(b), ctypes.byref(s)))
+    return a.value, b.value, s.value
+
+
+def residual_i8(x, y, m_x: int, m_y: int, s: int, *, out=None, stream=None):
+    """Residual addition of two int8 CUDA tensors of one shape."""
+    import torch
+    if out is None:
+        out = torch.empty_like(x)
+    n = x.numel()
+    rc = load().ip_residual_i8(_dev_ptr(x, "x", torch.int8, tuple(x.shape)),
+                               _dev_ptr(y, "y", torch.int8, tuple(x.shape)), n, m_x, m_y, s,
+                               _dev_ptr(out, "out", torch.int8, tuple(x.shape)),
+                               _stream_handle(stream))
+    _check("ip_residual_i8", rc)
+    return out
+
+
+def glu_params(s_a: float, s_b: float, s_y: float) -> tuple[int, int, int, int]:
+    """(q_c, q_one, m, s) of GLU(a, b) = a sigma(b) (Eq. 5, minimax tanh)."""
+    prm = SwishParams()
+    _check("ip_glu_params", load().ip_glu_params(s_a, s_b, s_y, ctypes.byref(prm)))
+    return prm.q_c, prm.q_one, prm.m, prm.s
+
+
+def linear_glu_i8(x, w_interleaved, bias, m, s, glu: tuple[int, int, int, int], *, out=None,
+                  workspace=None, stream=None):
+    """Pointwise convolution with the GLU fused: x int8 [B, T, K]; w int8 [N, K]
+    with rows (a_c, b_c) interleaved; bias, m, s int32 [N]; returns int8
+    [B, T, N/2]."""
+    import torch
+    N, K = w_interleaved.shape
+    B, T, _ = x.shape
+    if out is None:
+        out = torch.empty((B, T, N // 2), dtype=torch.int8, device=x.device)
+    if workspace is None:
+        workspace = torch.zeros(256, dtype=torch.uint8, device=x.device)
+    bp = None if bias is None else _dev_ptr(bias, "bias", torch.int32, (N,))
+    g = SwishParams(*glu)
+    rc = load().ip_linear_glu_i8(
+        _dev_ptr(x, "x", torch.int8, (B, T, K)), _dev_ptr(w_interleaved, "w", torch.int8, (N, K)), bp,
+        _dev_ptr(m, "m", torch.int32, (N,)), _dev_ptr(s, "s", torch.int32, (N,)), ctypes.byref(g),
+        B, T, K, N, _dev_ptr(out, "out", torch.int8, (B, T, N // 2)),
+        ctypes.c_void_p(workspace.data_ptr()), workspace.numel(), _stream_handle(stream))
+    _check("ip_linear_glu_i8", rc)
+    return out
+
+
+def swish16_params(s_z: float, s_y: float) -> tuple[int, int, int, int]:
+    """(q_c, q_one, m, s) of the Swish of an INT16 input grid."""
+    prm = Swish16Params()
+    _check("ip_swish16_params_from_scales",
+           load().ip_swish16_params_from_scales(s_z, s_y, ctypes.byref(prm)))
+    return prm.q_c, prm.q_one, prm.m, prm.s
+
+
+def dwconv_swish_i8(x, w, bias, m, s, sw16: tuple[int, int, int, int], *, out=None,
+                    workspace=None, stream=None):
+    """Depthwise convolution over time (folded BatchNorm, INT16) + Swish:
+    x int8 [B, T, C]; w int8 [C, K]; bias, m, s int32 [C]; returns int8
+    [B, T, C]."""
+    import torch
+    B, T, C = x.shape
+    K = w.shape[1]
+    if out is None:
+        out = torch.empty_like(x)
+    if workspace is None:
+        workspace = torch.zeros(256, dtype=torch.uint8, device=x.device)
+    p = Swish16Params(*sw16)
+    rc = load().ip_dwconv_swish_i8(
+        _dev_ptr(x, "x", torch.int8, (B, T, C)), B, T, C, _dev_ptr(w, "w", torch.int8, (C, K)), K,
+        _dev_ptr(bias, "bias", torch.int32, (C,)), _dev_ptr(m, "m", torch.int32, (C,)),
+        _dev_ptr(s, "s", torch.int32, (C,)), ctypes.byref(p),
+        _dev_ptr(out, "out", torch.int8, (B, T, C)), ctypes.c_void_p(workspace.data_ptr()),
+        workspace.numel(), _stream_handle(stream))
+    _check("ip_dwconv_swish_i8", rc)
+    return out
+
+
 def relpos_mhsa_i8_host(q, k, v, p, u, v_bias, consts: LayerConstants, lengths, out, arena,
                         stream=None):
     """Whole layer from host buffers (torch CPU tensors, ideally pinned):
@@ -444,5 +549,6 @@ __all__ = ["build", "load", "relpos_mhsa_i8", "relpos_mhsa_i8_host", "status", "
            "dyadic_pair", "isoftmax_params_from_scale", "set_timeout_cycles", "strerror",
            "int8_mma_peak_tops", "set_stall_injection", "set_split_mode", "linear_i8",
            "linear_constants", "ROWS", "HEADS", "linear_swish_i8", "swish_params_from_scales",
-           "layernorm_i8", "layernorm_constants", "NormConstants",
+           "layernorm_i8", "layernorm_constants", "NormConstants", "residual_i8",
+           "residual_params", "linear_glu_i8", "glu_params", "dwconv_swish_i8", "swish16_params",
            "IpError", "LibraryError", "EXPORTS"]

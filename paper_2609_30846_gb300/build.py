@@ -14,9 +14,11 @@ ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 LIB = os.path.join(PKG, "libipmhsa.so")
-SOURCES = [os.path.join(CSRC, f) for f in ("ip_mhsa.cu", "ip_linear.cu", "ip_norm.cu")]
+SOURCES = [os.path.join(CSRC, f) for f in ("ip_mhsa.cu", "ip_linear.cu", "ip_norm.cu",
+                                           "ip_block.cu")]
 DEPS = SOURCES + [os.path.join(CSRC, f) for f in ("ip_mhsa_kernels.cuh", "ip_linear_kernels.cuh",
-                                                  "ip_norm_kernels.cuh", "ip_ptx.cuh",
+                                                  "ip_norm_kernels.cuh", "ip_block_kernels.cuh",
+                                                  "ip_ptx.cuh",
                                                   "ip_probe.cuh")] + [
     os.path.join(INCLUDE, "ip_mhsa.h")]
 ARCH = "-gencode=arch=compute_103a,code=sm_103a"

@@ -1,0 +1,150 @@
+// Host side of the remaining Conformer-block parts of the C ABI
+// (include/ip_mhsa.h): residual additions, the depthwise convolution with
+// folded BatchNorm and Swish, and their offline constants.  Device code:
+// ip_block_kernels.cuh.
+#include "ip_mhsa.h"
+#include "ip_block_kernels.cuh"
+
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <mutex>
+
+namespace {
+
+bool aligned(const void *p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+std::mutex g_mu;
+int g_sms[64] = {0};
+
+int sm_count() {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
+    std::lock_guard<std::mutex> lock(g_mu);
+    if (g_sms[dev] == 0) {
+        int n = 0;
+        if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
+        g_sms[dev] = n;
+    }
+    return g_sms[dev];
+}
+
+int check_swish16(const ip_swish16_params *p) {
+    if (p->q_c < 1 || p->q_c >= (1 << 16) || p->q_one < 1 || p->q_one >= (1ll << 31) ||
+        p->q_one < static_cast<long long>(p->q_c) * p->q_c || p->m < 0 || p->s < 0 || p->s > 31)
+        return IP_ERR_PARAM;
+    return IP_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int ip_residual_i8(const int8_t *x, const int8_t *y, long long n, int32_t m_x, int32_t m_y,
+                   int32_t s, int8_t *z, ip_stream_t stream) {
+    if (n < 0) return IP_ERR_SHAPE;
+    if (m_x < 0 || m_y < 0 || s < 0 || s > 31) return IP_ERR_PARAM;
+    if (n == 0) return IP_OK;
+    if (!x || !y || !z) return IP_ERR_NULL;
+    if (!aligned(x, 16) || !aligned(y, 16) || !aligned(z, 16)) return IP_ERR_ALIGN;
+    const int nsm = sm_count();
+    if (nsm <= 0) return IP_ERR_CUDA;
+    ipb::ResidualParams p;
+    p.x = x;
+    p.y = y;
+    p.z = z;
+    p.n = n;
+    p.m_x = m_x;
+    p.m_y = m_y;
+    p.s = s;
+    const long long vec = (n >> 4) + 1;
+    long long blocks = (vec + ipb::RES_THREADS - 1) / ipb::RES_THREADS;
+    const long long cap = static_cast<long long>(nsm) * 8;
+    blocks = blocks < cap ? blocks : cap;
+    ipb::residual_i8_kernel<<<static_cast<unsigned>(blocks), ipb::RES_THREADS, 0,
+                              reinterpret_cast<cudaStream_t>(stream)>>>(p);
+    return cudaGetLastError() == cudaSuccess ? IP_OK : IP_ERR_CUDA;
+}
+
+int ip_dwconv_swish_i8(const int8_t *x, int B, int T, int C, const int8_t *w, int K,
+                       const int32_t *bias, const int32_t *m, const int32_t *s,
+                       const ip_swish16_params *sw, int8_t *y, void *workspace,
+                       size_t workspace_bytes, ip_stream_t stream) {
+    if (B < 0 || B > IP_MAX_B || T < 1 || C < 1 || K < 1 || K % 2 == 0 || K > ipb::DW_KMAX)
+        return IP_ERR_SHAPE;
+    if ((T + ipb::DW_FRAMES - 1) / ipb::DW_FRAMES > 65535) return IP_ERR_SHAPE;
+    if (!sw) return IP_ERR_NULL;
+    int rc = check_swish16(sw);
+    if (rc != IP_OK) return rc;
+    if (B == 0) return IP_OK;
+    if (!x || !w || !bias || !m || !s || !y || !workspace) return IP_ERR_NULL;
+    if (!aligned(bias, 4) || !aligned(m, 4) || !aligned(s, 4) || !aligned(workspace, 256))
+        return IP_ERR_ALIGN;
+    if (workspace_bytes < 256) return IP_ERR_WORKSPACE;
+    ipb::DwParams p;
+    p.x = x;
+    p.w = w;
+    p.bias = bias;
+    p.m = m;
+    p.s = s;
+    p.y = y;
+    p.B = B;
+    p.T = T;
+    p.C = C;
+    p.K = K;
+    p.sw_qc = sw->q_c;
+    p.sw_qone = sw->q_one;
+    p.sw_m = sw->m;
+    p.sw_s = sw->s;
+    p.err = static_cast<int *>(workspace);
+    const dim3 grid((C + ipb::DW_THREADS - 1) / ipb::DW_THREADS,
+                    (T + ipb::DW_FRAMES - 1) / ipb::DW_FRAMES, B);
+    ipb::dwconv_swish_kernel<<<grid, ipb::DW_THREADS, 0, reinterpret_cast<cudaStream_t>(stream)>>>(p);
+    return cudaGetLastError() == cudaSuccess ? IP_OK : IP_ERR_CUDA;
+}
+
+int ip_residual_params(double S_x, double S_y, double S_z, double alpha, int32_t *m_x,
+                       int32_t *m_y, int32_t *s) {
+    if (!m_x || !m_y || !s) return IP_ERR_NULL;
+    if (!(S_x > 0.0) || !(S_y > 0.0) || !(S_z > 0.0) || !(alpha > 0.0)) return IP_ERR_PARAM;
+    return ip_dyadic_pair(S_x / S_z, alpha * S_y / S_z, m_x, m_y, s);
+}
+
+int ip_glu_params(double S_a, double S_b, double S_y, ip_swish_params *out) {
+    if (!out) return IP_ERR_NULL;
+    if (!(S_a > 0.0) || !(S_b > 0.0) || !(S_y > 0.0) || !std::isfinite(S_a) ||
+        !std::isfinite(S_b) || !std::isfinite(S_y))
+        return IP_ERR_PARAM;
+    const double s_t = -IP_SWISH_A * (S_b / 2.0) * (S_b / 2.0);
+    const double qc = std::floor(2.0 * IP_SWISH_C / S_b + 0.5);
+    const double qone = std::floor(1.0 / s_t + 0.5);
+    if (qc < 1.0 || qc >= 32768.0 || qone < 1.0 || qone >= 8388608.0 || qone < qc * qc)
+        return IP_ERR_PARAM;
+    ip_swish_params p;
+    p.q_c = static_cast<int32_t>(qc);
+    p.q_one = static_cast<int32_t>(qone);
+    const int rc = ip_dyadic_multiplier(S_a * s_t / (2.0 * S_y), &p.m, &p.s);
+    if (rc != IP_OK) return rc;
+    *out = p;
+    return IP_OK;
+}
+
+int ip_swish16_params_from_scales(double S_z, double S_y, ip_swish16_params *out) {
+    if (!out) return IP_ERR_NULL;
+    if (!(S_z > 0.0) || !(S_y > 0.0) || !std::isfinite(S_z) || !std::isfinite(S_y))
+        return IP_ERR_PARAM;
+    const double s_t = -IP_SWISH_A * (S_z / 2.0) * (S_z / 2.0);
+    const double qc = std::floor(2.0 * IP_SWISH_C / S_z + 0.5);
+    const double qone = std::floor(1.0 / s_t + 0.5);
+    if (qc < 1.0 || qc >= 65536.0 || qone < 1.0 || qone >= 2147483648.0 || qone < qc * qc)
+        return IP_ERR_PARAM;
+    ip_swish16_params p;
+    p.q_c = static_cast<int32_t>(qc);
+    p.q_one = static_cast<long long>(qone);
+    const int rc = ip_dyadic_multiplier(S_z * s_t / (2.0 * S_y), &p.m, &p.s);
+    if (rc != IP_OK) return rc;
+    *out = p;
+    return IP_OK;
+}
+
+}  // extern "C"

@@ -76,10 +76,13 @@ int ensure_smem() {
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return IP_ERR_CUDA;
     std::lock_guard<std::mutex> lock(g_mu);
     if (g_smem_set[dev]) return IP_OK;
-    if (cudaFuncSetAttribute(ipl::linear_i8_kernel<false>,
+    if (cudaFuncSetAttribute(ipl::linear_i8_kernel<ipl::EPI_PLAIN>,
                              cudaFuncAttributeMaxDynamicSharedMemorySize,
                              ipl::SMEM_LAUNCH) != cudaSuccess ||
-        cudaFuncSetAttribute(ipl::linear_i8_kernel<true>,
+        cudaFuncSetAttribute(ipl::linear_i8_kernel<ipl::EPI_SWISH>,
+                             cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             ipl::SMEM_LAUNCH) != cudaSuccess ||
+        cudaFuncSetAttribute(ipl::linear_i8_kernel<ipl::EPI_GLU>,
                              cudaFuncAttributeMaxDynamicSharedMemorySize,
                              ipl::SMEM_LAUNCH) != cudaSuccess)
         return IP_ERR_CUDA;
@@ -96,8 +99,8 @@ int check_swish(const ip_swish_params *p) {
 }
 
 int linear_launch(const int8_t *x, int x_layout, const int8_t *w, const int32_t *bias,
-                  const int32_t *m, const int32_t *s, const ip_swish_params *sw, int B, int T,
-                  int K, int N, int G, int8_t *y, int y_layout, void *workspace,
+                  const int32_t *m, const int32_t *s, const ip_swish_params *sw, int epi, int B,
+                  int T, int K, int N, int G, int8_t *y, int y_layout, void *workspace,
                   size_t workspace_bytes, ip_stream_t stream) {
     if ((x_layout != IP_LAYOUT_ROWS && x_layout != IP_LAYOUT_HEADS) ||
         (y_layout != IP_LAYOUT_ROWS && y_layout != IP_LAYOUT_HEADS))
@@ -166,10 +169,12 @@ int linear_launch(const int8_t *x, int x_layout, const int8_t *w, const int32_t 
     const unsigned grid = prm.ntiles < static_cast<unsigned>(nsm) ? prm.ntiles
                                                                   : static_cast<unsigned>(nsm);
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-    if (sw)
-        ipl::linear_i8_kernel<true><<<grid, ipl::THREADS, ipl::SMEM_LAUNCH, st>>>(tm_x, tm_w, prm);
+    if (epi == ipl::EPI_SWISH)
+        ipl::linear_i8_kernel<ipl::EPI_SWISH><<<grid, ipl::THREADS, ipl::SMEM_LAUNCH, st>>>(tm_x, tm_w, prm);
+    else if (epi == ipl::EPI_GLU)
+        ipl::linear_i8_kernel<ipl::EPI_GLU><<<grid, ipl::THREADS, ipl::SMEM_LAUNCH, st>>>(tm_x, tm_w, prm);
     else
-        ipl::linear_i8_kernel<false><<<grid, ipl::THREADS, ipl::SMEM_LAUNCH, st>>>(tm_x, tm_w, prm);
+        ipl::linear_i8_kernel<ipl::EPI_PLAIN><<<grid, ipl::THREADS, ipl::SMEM_LAUNCH, st>>>(tm_x, tm_w, prm);
     if (cudaGetLastError() != cudaSuccess) return IP_ERR_CUDA;
     return IP_OK;
 }
@@ -182,8 +187,8 @@ int ip_linear_i8(const int8_t *x, int x_layout, const int8_t *w, const int32_t *
                  const int32_t *m, const int32_t *s, int B, int T, int K, int N, int G,
                  int8_t *y, int y_layout, void *workspace, size_t workspace_bytes,
                  ip_stream_t stream) {
-    return linear_launch(x, x_layout, w, bias, m, s, nullptr, B, T, K, N, G, y, y_layout,
-                         workspace, workspace_bytes, stream);
+    return linear_launch(x, x_layout, w, bias, m, s, nullptr, ipl::EPI_PLAIN, B, T, K, N, G, y,
+                         y_layout, workspace, workspace_bytes, stream);
 }
 
 int ip_linear_swish_i8(const int8_t *x, const int8_t *w, const int32_t *bias, const int32_t *m,
@@ -192,8 +197,18 @@ int ip_linear_swish_i8(const int8_t *x, const int8_t *w, const int32_t *bias, co
     if (!sw) return IP_ERR_NULL;
     const int rc = check_swish(sw);
     if (rc != IP_OK) return rc;
-    return linear_launch(x, IP_LAYOUT_ROWS, w, bias, m, s, sw, B, T, K, N, 1, y, IP_LAYOUT_ROWS,
-                         workspace, workspace_bytes, stream);
+    return linear_launch(x, IP_LAYOUT_ROWS, w, bias, m, s, sw, ipl::EPI_SWISH, B, T, K, N, 1, y,
+                         IP_LAYOUT_ROWS, workspace, workspace_bytes, stream);
+}
+
+int ip_linear_glu_i8(const int8_t *x, const int8_t *w, const int32_t *bias, const int32_t *m,
+                     const int32_t *s, const ip_swish_params *glu, int B, int T, int K, int N,
+                     int8_t *y, void *workspace, size_t workspace_bytes, ip_stream_t stream) {
+    if (!glu) return IP_ERR_NULL;
+    const int rc = check_swish(glu);
+    if (rc != IP_OK) return rc;
+    return linear_launch(x, IP_LAYOUT_ROWS, w, bias, m, s, glu, ipl::EPI_GLU, B, T, K, N, 1, y,
+                         IP_LAYOUT_ROWS, workspace, workspace_bytes, stream);
 }
 
 int ip_swish_params_from_scales(double S_z, double S_y, ip_swish_params *out) {

@@ -106,7 +106,23 @@ __device__ __forceinline__ int swish_i8(int z, const LinearParams &p) {
     return clamp127(v >> p.sw_e);
 }
 
-template <bool SWISH>
+// Gated linear unit of Eq. 5 on two requantised int8 values: a sigma(b)
+// with sigma(b) = (1 + tanh(b/2)) / 2 and the minimax tanh on b's grid;
+// |a t| < 2^31 (t <= 2 q_one < 2^24).
+__device__ __forceinline__ int glu_i8(int a, int b, const LinearParams &p) {
+    const int mag = b < 0 ? -b : b;
+    const int dc = (mag < p.sw_qc ? mag : p.sw_qc) - p.sw_qc;
+    const int L = p.sw_qone - dc * dc;
+    const int t = b > 0 ? p.sw_qone + L : (b < 0 ? p.sw_qone - L : p.sw_qone);
+    const long long v = static_cast<long long>(p.sw_m) * (a * t) + (1ll << (p.sw_e - 1));
+    return clamp127(v >> p.sw_e);
+}
+
+constexpr int EPI_PLAIN = 0;   // requantised int8
+constexpr int EPI_SWISH = 1;   // + minimax Swish
+constexpr int EPI_GLU = 2;     // interleaved pairs (a_c, b_c) -> a_c sigma(b_c)
+
+template <int EPI>
 __global__ void __launch_bounds__(THREADS, 1)
     linear_i8_kernel(const __grid_constant__ CUtensorMap tm_x,
                      const __grid_constant__ CUtensorMap tm_w, const LinearParams prm) {
@@ -133,7 +149,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
     }
-    if (SWISH && threadIdx.x < 256) {
+    if (EPI == EPI_SWISH && threadIdx.x < 256) {
         // the Swish of every int8 input, entry at the byte value of z
         const int z = static_cast<int>(static_cast<int8_t>(static_cast<uint8_t>(threadIdx.x)));
         const uint32_t y = static_cast<uint32_t>(swish_i8(z, prm)) & 0xffu;
@@ -249,6 +265,46 @@ __global__ void __launch_bounds__(THREADS, 1)
             }
         if (bad) atomicOr(prm.err, ERR_PARAM);
 
+        if (EPI == EPI_GLU) {
+            // pairs (a_c, b_c) in columns (2t, 2t + 1) of each n8 tile: output
+            // channel 4j + t of this warp's 16 (row of 16 bytes)
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+#pragma unroll
+                for (int j = 0; j < 4; ++j)
+#pragma unroll
+                    for (int rr = 0; rr < 2; ++rr) {
+                        int z[2];
+#pragma unroll
+                        for (int q = 0; q < 2; ++q) {
+                            const int cix = 2 * j + q;
+                            const long long v = static_cast<long long>(cm[cix]) *
+                                                    (acc[i][j][2 * rr + q] + cb[cix]) +
+                                                (1ll << (ce[cix] - 1));
+                            z[q] = clamp127(v >> ce[cix]);
+                        }
+                        const uint32_t o = static_cast<uint32_t>(glu_i8(z[0], z[1], prm)) & 0xffu;
+                        const int r = 16 * i + g + 8 * rr;
+                        asm volatile("st.shared.u8 [%0], %1;" ::"r"(ob + r * OUT_ROW + 4 * j + t4),
+                                     "r"(o)
+                                     : "memory");
+                    }
+            __syncwarp();
+            // 64 rows x 16 bytes: lane -> rows lane, lane + 32
+            const int Nout = prm.N >> 1;
+#pragma unroll
+            for (int it = 0; it < 2; ++it) {
+                const int r = 32 * it + lane;
+                const uint4 v = lds128(ob + r * OUT_ROW);
+                if (L.m0 + 64 * wm + r < frames) {
+                    const size_t off = static_cast<size_t>(L.m0 + 64 * wm + r) * Nout + (n0 >> 1) + 16 * wn;
+                    *reinterpret_cast<uint4 *>(prm.y + off) = v;
+                }
+            }
+            __syncwarp();
+            continue;
+        }
+
 #pragma unroll
         for (int i = 0; i < 4; ++i)
 #pragma unroll
@@ -263,7 +319,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                                                 (acc[i][j][2 * rr + q] + cb[c]) +
                                             (1ll << (ce[c] - 1));
                         uint32_t o = static_cast<uint32_t>(clamp127(v >> ce[c])) & 0xffu;
-                        if (SWISH) o = swish_lut[o];
+                        if (EPI == EPI_SWISH) o = swish_lut[o];
                         two |= o << (8 * q);
                     }
                     const int r = 16 * i + g + 8 * rr;

@@ -240,3 +240,33 @@ def test_layernorm_validation(lib):
     assert call(M=None) == -1
     assert call(B=P((1 << 20) + 4)) == -3
     assert call(wsb=16) == -8
+
+
+def test_block_constants_match_oracle(lib):
+    import oracle
+    for args in [(0.05, 0.04, 0.06, 0.5), (0.03, 0.03, 0.04, 1.0)]:
+        assert ip.residual_params(*args) == oracle.residual_params(*args)
+    for args in [(0.05, 0.06, 0.03), (0.02, 0.08, 0.01)]:
+        want = oracle.glu_params(*args)
+        assert ip.glu_params(*args) == (want.q_c, want.q_one, want.m, want.s)
+    for args in [(8 / 32767, 8 / 127), (20 / 32767, 5 / 127)]:
+        want = oracle.swish16_params(*args)
+        assert ip.swish16_params(*args) == (want.q_c, want.q_one, want.m, want.s)
+    with pytest.raises(ip.IpError):
+        ip.swish16_params(3 / 32767, 3 / 127)
+
+
+def test_block_validation(lib):
+    P = ctypes.c_void_p
+    fake, ws = P(1 << 20), P(1 << 21)
+    assert lib.ip_residual_i8(fake, fake, -1, 1, 1, 0, fake, None) == -2
+    assert lib.ip_residual_i8(fake, fake, 16, -1, 1, 0, fake, None) == -7
+    assert lib.ip_residual_i8(fake, fake, 16, 1, 1, 32, fake, None) == -7
+    assert lib.ip_residual_i8(None, None, 0, 1, 1, 0, None, None) == 0
+    assert lib.ip_residual_i8(P((1 << 20) + 8), fake, 16, 1, 1, 0, fake, None) == -3
+    sw = ip.Swish16Params(100, 20000, 2 ** 30, 3)
+    assert lib.ip_dwconv_swish_i8(fake, 1, 8, 64, fake, 8, fake, fake, fake, ctypes.byref(sw),
+                                  fake, ws, 256, None) == -2      # even kernel
+    bad = ip.Swish16Params(200, 20000, 2 ** 30, 3)               # q_one < q_c^2
+    assert lib.ip_dwconv_swish_i8(fake, 1, 8, 64, fake, 9, fake, fake, fake, ctypes.byref(bad),
+                                  fake, ws, 256, None) == -7

@@ -1,0 +1,111 @@
+"""Parity of the remaining Conformer-block kernels with the oracle (bit-exact):
+residual additions, the GLU projection, the depthwise convolution with
+folded BatchNorm on INT16 followed by the Swish."""
+import numpy as np
+import pytest
+
+import synth
+
+pytestmark = pytest.mark.gpu
+
+torch = pytest.importorskip("torch")
+
+
+@pytest.fixture(scope="module")
+def ip():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import paper_2609_30846_gb300 as mod
+    mod.load()
+    return mod
+
+
+@pytest.fixture(scope="module")
+def orc():
+    import oracle
+    oracle.build()
+    return oracle
+
+
+def _d(a):
+    return torch.from_numpy(np.ascontiguousarray(a)).cuda()
+
+
+def assert_same(got, want):
+    bad = got != want
+    if bad.any():
+        idx = np.argwhere(bad)[:5]
+        raise AssertionError(f"{int(bad.sum())} of {got.size} differ; first at {idx.tolist()}: "
+                             f"gpu {got[tuple(idx[0])]} oracle {want[tuple(idx[0])]}")
+
+
+@pytest.mark.parametrize("n,alpha", [(16, 1.0), (1000, 0.5), (12000 * 1024 + 7, 0.5), (3, 1.0)])
+def test_residual(ip, orc, n, alpha):
+    rng = np.random.default_rng(n)
+    x = rng.integers(-127, 128, size=n).astype(np.int8)
+    y = rng.integers(-127, 128, size=n).astype(np.int8)
+    m_x, m_y, s = orc.residual_params(0.05, 0.03, 0.06, alpha)
+    got = ip.residual_i8(_d(x), _d(y), m_x, m_y, s).cpu().numpy()
+    assert_same(got, orc.residual(x, y, m_x, m_y, s))
+
+
+def interleave(w):
+    N2 = w.shape[0]
+    C = N2 // 2
+    out = np.empty_like(w)
+    out[0::2] = w[:C]
+    out[1::2] = w[C:]
+    return out
+
+
+@pytest.mark.parametrize("B,T,K,C", [(1, 5, 128, 64), (2, 130, 256, 192), (32, 375, 1024, 1024)])
+def test_glu_projection(ip, orc, B, T, K, C):
+    # the ConvBlock's first pointwise convolution, 2C outputs [a | b] -> C
+    lc = synth.linear(B, T, K, 2 * C, seed=500 + T, groups=2)
+    m, s = orc.linear_constants(lc.s_x, lc.s_w, lc.s_y_per_channel())
+    g = orc.glu_params(float(lc.s_y[0]), float(lc.s_y[1]), 0.8 * float(lc.s_y[0]))
+    ab = orc.linear(lc.x, lc.w, lc.bias, m, s)
+    want = orc.glu(ab, g)
+    perm = np.empty(2 * C, np.int64)
+    perm[0::2] = np.arange(C)
+    perm[1::2] = np.arange(C) + C
+    ws = torch.zeros(256, dtype=torch.uint8, device="cuda")
+    got = ip.linear_glu_i8(_d(lc.x), _d(interleave(lc.w)), _d(lc.bias[perm]), _d(m[perm]),
+                           _d(s[perm]), (g.q_c, g.q_one, g.m, g.s), workspace=ws)
+    assert ip.status(ws) == 0
+    assert_same(got.cpu().numpy(), want)
+
+
+@pytest.mark.parametrize("B,T,C,K", [(1, 1, 256, 9), (2, 33, 256, 9), (3, 100, 512, 5),
+                                     (32, 375, 1024, 9), (1, 70, 300, 15)])
+def test_dwconv_swish(ip, orc, B, T, C, K):
+    rng = np.random.default_rng(T * C + K)
+    x = rng.integers(-127, 128, size=(B, T, C)).astype(np.int8)
+    w = rng.integers(-127, 128, size=(C, K)).astype(np.int8)
+    bias = rng.integers(-20000, 20000, size=C).astype(np.int32)
+    s_x, s_w = 0.04, rng.uniform(0.001, 0.01, C)
+    s_bn = 40.0 / 32767                      # INT16 grid of the folded BatchNorm output
+    m, s = orc.linear_constants(s_x, s_w, np.full(C, s_bn))
+    p16 = orc.swish16_params(s_bn, 5.0 / 127)
+    want = orc.swish16(orc.dwconv(x, w, bias, m, s), p16)
+    ws = torch.zeros(256, dtype=torch.uint8, device="cuda")
+    got = ip.dwconv_swish_i8(_d(x), _d(w), _d(bias), _d(m), _d(s),
+                             (p16.q_c, p16.q_one, p16.m, p16.s), workspace=ws)
+    assert ip.status(ws) == 0
+    assert_same(got.cpu().numpy(), want)
+
+
+def test_dwconv_saturating_int16(ip, orc):
+    # accumulators far beyond the INT16 grid: clamped before the Swish
+    B, T, C, K = 1, 40, 256, 9
+    x = np.full((B, T, C), 127, np.int8)
+    x[:, ::2] = -127
+    w = np.full((C, K), 127, np.int8)
+    bias = np.zeros(C, np.int32)
+    m = np.full(C, 2 ** 31 - 1, np.int32)
+    s = np.zeros(C, np.int32)
+    p16 = orc.swish16_params(40.0 / 32767, 5.0 / 127)
+    want = orc.swish16(orc.dwconv(x, w, bias, m, s), p16)
+    got = ip.dwconv_swish_i8(_d(x), _d(w), _d(bias), _d(m), _d(s),
+                             (p16.q_c, p16.q_one, p16.m, p16.s))
+    assert_same(got.cpu().numpy(), want)
