@@ -399,7 +399,49 @@ def measure_next_rows(dev, peak, steps: int, cpu: bool):
                                "cores": os.cpu_count() or 1, "kind": "oracle",
                                "sample": f"{n} frames of {B * T}, {dt:.2f} s"}
     rows["layernorm_1024"] = row
-    del x, out, flush_w, flush_r
+    del x, out
+
+    # one whole integer Conformer block (Eqs. 1-5): 19 launches
+    import synth.block as sblock
+    from paper_2609_30846_gb300.block import GPU_LAUNCHES, ConformerBlock
+    case = sblock.conformer_block(B, T, seed=7300)
+    blk = ConformerBlock(case, B, T, dev)
+    x = torch.from_numpy(case.x).to(dev)
+    for _ in range(3):
+        blk(x, stream=stream)
+    times = []
+    for _ in range(steps):
+        flush()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        blk(x, stream=stream)
+        e1.record(stream)
+        e1.synchronize()
+        times.append(e0.elapsed_time(e1) * 1e-3)
+    if ip.status(blk.ws, stream) != 0:
+        raise SystemExit("conformer block: a kernel reported an error")
+    t = statistics.median(times)
+    ops = blk.useful_ops()
+    row = {"value": ops / t / 1e12, "unit": "TOPS", "us_per_block": t * 1e6,
+           "frames_per_s": B * T / t, "shape": {"B": B, "T": T, "d": 1024, "ff": 4096, "heads": 8},
+           "roofline": {"bound": "tensor", "achieved": ops / t / 1e12, "peak": peak,
+                        "unit": "TOPS", "frac": ops / t / 1e12 / peak, "traffic": None},
+           "kernel": "19 launches: layernorm x5, linear x8 (2 with Swish, 1 with GLU), "
+                     "relpos_mhsa_fused, dwconv_swish, residual x4",
+           "gpu_launches": GPU_LAUNCHES}
+    if cpu:
+        import oracle
+        from oracle.block import conformer_block as oracle_block
+        oracle.build()
+        one = sblock.BlockCase(**{**case.__dict__, "x": np.ascontiguousarray(case.x[:1])})
+        t0 = time.perf_counter()
+        oracle_block(one)
+        dt = time.perf_counter() - t0
+        row["cpu_baseline"] = {"value": ops / B / dt / 1e12, "unit": "TOPS",
+                               "cores": os.cpu_count() or 1, "kind": "oracle",
+                               "sample": f"1 of {B} utterances (T={T}), {dt:.1f} s"}
+    rows["conformer_block"] = row
+    del x, blk, flush_w, flush_r
     return rows
 
 

@@ -1,0 +1,135 @@
+"""One integer Conformer block (Sec. 2.1 Eqs. 1-5) as a sequence of the
+library's kernels, every integer constant derived by the library's own
+offline helpers from the declared grids:
+
+  Z1 = X  + 1/2 FFN1(LN1(X))              (Eq. 1)  LayerNorm, linear + Swish, linear, residual
+  Z2 = Z1 + MHSA(LN2(Z1))                 (Eq. 2)  LayerNorm, Q/K/V head-split, rel-pos MHSA
+                                                   (row-major output), output projection, residual
+  Z3 = Z2 + Conv(LN3(Z2))                 (Eqs. 3, 5) LayerNorm, pointwise + GLU, depthwise
+                                                   + BatchNorm (INT16) + Swish, pointwise, residual
+  H  = LN5(Z3 + 1/2 FFN2(LN4(Z3)))        (Eq. 4)
+
+Nineteen launches on one stream, all of them CUDA kernels of this library.
+The parameter object carries int8 weights with per-channel grids, real
+LayerNorm parameters and the activation grids (attributes as
+`synth.block.BlockCase`).
+"""
+from __future__ import annotations
+
+import numpy as np
+
+from . import (HEADS, ROWS, dwconv_swish_i8, glu_params, layer_constants, layernorm_constants,
+               layernorm_i8, linear_constants, linear_glu_i8, linear_i8, linear_swish_i8,
+               relpos_mhsa_i8, residual_i8, residual_params, swish16_params,
+               swish_params_from_scales, workspace_bytes)
+
+GPU_LAUNCHES = 19
+
+
+class ConformerBlock:
+    """Device-resident constants and buffers of one block for a batch shape."""
+
+    def __init__(self, params, B: int, T: int, device):
+        import torch
+        self.B, self.T = B, T
+        S = params.s
+        D = params.x.shape[-1] if params.x is not None else 1024
+        self.D = D
+        d = lambda a: torch.from_numpy(np.ascontiguousarray(a)).to(device)
+
+        def lnc(name):
+            q = params.ln[name]
+            k = layernorm_constants(q.s_in, q.gamma, q.beta, q.s_out, q.eps)
+            return (d(k.M), d(k.B), d(k.E), k.eps_c)
+
+        def linc(name, perm=None):
+            L = params.lin[name]
+            m, s = linear_constants(L.s_in, L.s_w, L.s_out)
+            w, b = L.w, L.bias
+            if perm is not None:
+                w, b, m, s = w[perm], b[perm], m[perm], s[perm]
+            return (d(w), d(b), d(m), d(s))
+
+        self.ln = {n: lnc(n) for n in ("ln1", "ln2", "ln3", "ln4", "ln5")}
+        self.lin = {n: linc(n) for n in ("ff1a", "ff1b", "ff2a", "ff2b", "qkv", "out", "pw2")}
+        perm = np.empty(2 * D, np.int64)            # rows (a_c, b_c) interleaved for the GLU
+        perm[0::2] = np.arange(D)
+        perm[1::2] = np.arange(D) + D
+        self.lin["pw1"] = linc("pw1", perm)
+        self.sw1 = swish_params_from_scales(S["ff1z"], S["ff1h"])
+        self.sw2 = swish_params_from_scales(S["ff2z"], S["ff2h"])
+        self.glu = glu_params(S["pw1a"], S["pw1b"], S["glu"])
+        m, s = linear_constants(S["glu"], params.dw_sw, np.full(D, S["bn"]))
+        self.dw = (d(params.dw_w), d(params.dw_bias), d(m), d(s))
+        self.sw16 = swish16_params(S["bn"], S["convsw"])
+        self.res = [residual_params(S["x"], S["ff1o"], S["z1"], 0.5),
+                    residual_params(S["z1"], S["mhsa"], S["z2"], 1.0),
+                    residual_params(S["z2"], S["conv"], S["z3"], 1.0),
+                    residual_params(S["z3"], S["ff2o"], S["z4"], 0.5)]
+        self.attn = layer_constants(params.attn_scales)
+        self.p, self.u, self.vb = d(params.p), d(params.u), d(params.vb)
+        H = params.u.shape[0]
+        e = lambda *shape: torch.empty(shape, dtype=torch.int8, device=device)
+        self.a = e(B, T, D)
+        self.h = e(B, T, 4 * D)
+        self.f = e(B, T, D)
+        self.z = [e(B, T, D) for _ in range(4)]
+        self.qkv = e(3, B, H, T, D // H)
+        self.o = e(B, T, H, D // H)
+        self.g = e(B, T, D)
+        self.out = e(B, T, D)
+        self.ws = torch.zeros(max(256, workspace_bytes(B, H, T)), dtype=torch.uint8, device=device)
+
+    def __call__(self, x, stream=None):
+        """x: int8 [B, T, D] CUDA tensor on the input grid; returns the block's
+        int8 output (a buffer owned by this object).  Asynchronous on `stream`."""
+        ws, st = self.ws, stream
+        a, h, f, z = self.a, self.h, self.f, self.z
+
+        def ln(name, src, dst):
+            M, Bc, E, eps = self.ln[name]
+            layernorm_i8(src, M, Bc, E, eps, out=dst, workspace=ws, stream=st)
+
+        def lin(name, src, dst, **kw):
+            w, b, m, s = self.lin[name]
+            linear_i8(src, w, b, m, s, out=dst, workspace=ws, stream=st, **kw)
+
+        def ffn(pre, sw, src):
+            w, b, m, s = self.lin[pre + "a"]
+            linear_swish_i8(src, w, b, m, s, sw, out=h, workspace=ws, stream=st)
+            lin(pre + "b", h, f)
+
+        # Eq. 1
+        ln("ln1", x, a)
+        ffn("ff1", self.sw1, a)
+        residual_i8(x, f, *self.res[0], out=z[0], stream=st)
+        # Eq. 2
+        ln("ln2", z[0], a)
+        lin("qkv", a, self.qkv, y_layout=HEADS, groups=3)
+        relpos_mhsa_i8(self.qkv[0], self.qkv[1], self.qkv[2], self.p, self.u, self.vb, self.attn,
+                       out=self.o, workspace=ws, stream=st, out_layout=ROWS)
+        lin("out", self.o.view(self.B, self.T, self.D), f)
+        residual_i8(z[0], f, *self.res[1], out=z[1], stream=st)
+        # Eqs. 3, 5
+        ln("ln3", z[1], a)
+        w, b, m, s = self.lin["pw1"]
+        linear_glu_i8(a, w, b, m, s, self.glu, out=self.g, workspace=ws, stream=st)
+        dwconv_swish_i8(self.g, *self.dw, self.sw16, out=a, workspace=ws, stream=st)
+        lin("pw2", a, f)
+        residual_i8(z[1], f, *self.res[2], out=z[2], stream=st)
+        # Eq. 4
+        ln("ln4", z[2], a)
+        ffn("ff2", self.sw2, a)
+        residual_i8(z[2], f, *self.res[3], out=z[3], stream=st)
+        ln("ln5", z[3], self.out)
+        return self.out
+
+    def useful_ops(self) -> float:
+        """Integer multiply-adds x 2 of the block's contractions (projections,
+        feed-forward, pointwise and depthwise convolutions, attention)."""
+        B, T, D = self.B, self.T, self.D
+        frames = B * T
+        gemm = 2.0 * frames * D * (4 * D + 4 * D + 3 * D + D + 2 * D + D + 4 * D + 4 * D)
+        attn = 6.0 * 128 * T * T * B * (D // 128)
+        dw = 2.0 * frames * D * 9
+        return gemm + attn + dw
