@@ -583,12 +583,20 @@ def run_ours(args):
         pin = lambda a: torch.from_numpy(np.ascontiguousarray(a)).pin_memory()
         hl = [dict(q=pin(l.q), k=pin(l.k), v=pin(l.v), p=pin(l.p), u=pin(l.u), vb=pin(l.vb),
                    out=torch.empty((B, H, T, dh), dtype=torch.int8).pin_memory()) for l in layers]
-        arena = torch.empty(ip.host_arena_bytes(B, H, T, dh), dtype=torch.uint8, device=dev)
+        # two arenas on two streams: one layer's uploads and download overlap
+        # the neighbouring layer's kernel (asynchronous host-buffer calls)
+        arenas = [torch.empty(ip.host_arena_bytes(B, H, T, dh), dtype=torch.uint8, device=dev)
+                  for _ in range(2)]
+        streams = [stream, torch.cuda.Stream(dev)]
 
         def e2e_step():
-            for h_, c in zip(hl, consts):
+            for li, (h_, c) in enumerate(zip(hl, consts)):
                 ip.relpos_mhsa_i8_host(h_["q"], h_["k"], h_["v"], h_["p"], h_["u"], h_["vb"], c,
-                                       None, h_["out"], arena, stream=stream)
+                                       None, h_["out"], arenas[li & 1], stream=streams[li & 1],
+                                       wait=False)
+            for j in range(2):
+                if ip.host_status(arenas[j], B, H, T, dh, stream=streams[j]) != 0:
+                    raise SystemExit("end-to-end: a kernel reported an error")
         e2e_step()
         torch.cuda.synchronize(dev)
         if dist:

@@ -331,6 +331,26 @@ int ip_relpos_mhsa_i8_ex(const int8_t *q, const int8_t *k, const int8_t *v, cons
                          int out_layout, void *workspace, size_t workspace_bytes,
                          ip_stream_t stream);
 
+/* ip_relpos_mhsa_i8_host without the final wait: enqueues the uploads, the
+ * kernel and the download on `stream` and returns.  The output in `out` (and
+ * the inputs' host buffers, which stay in use until the uploads are done) is
+ * valid once the stream has synchronised; ip_relpos_mhsa_host_status then
+ * reports device-side errors.  Calls on different streams with different
+ * arenas overlap one call's copies with another's kernel.  Pinned host
+ * buffers make the copies asynchronous. */
+int ip_relpos_mhsa_i8_host_async(const int8_t *q, const int8_t *k, const int8_t *v,
+                                 const int8_t *p, const int8_t *u, const int8_t *v_bias,
+                                 const int32_t *multipliers, const int32_t *shifts,
+                                 const ip_isoftmax_params *sm, const int32_t *lengths, int B,
+                                 int H, int T, int dh, int8_t *out, void *arena,
+                                 size_t arena_bytes, ip_stream_t stream);
+
+/* Status of the last ip_relpos_mhsa_i8_host_async call that used `arena`
+ * (same shape arguments): synchronises `stream`, returns IP_OK,
+ * IP_ERR_TIMEOUT or IP_ERR_PARAM, and clears the status word. */
+int ip_relpos_mhsa_host_status(const void *arena, int B, int H, int T, int dh,
+                               ip_stream_t stream);
+
 /* Text of an IP_* code. */
 const char *ip_strerror(int code);
 

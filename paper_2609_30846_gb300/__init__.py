@@ -33,7 +33,7 @@ EXPORTS = (
     "ip_debug_set_split_mode", "ip_linear_i8", "ip_linear_swish_i8", "ip_swish_params_from_scales",
     "ip_layernorm_i8", "ip_layernorm_constants", "ip_relpos_mhsa_i8_ex", "ip_residual_i8",
     "ip_residual_params", "ip_linear_glu_i8", "ip_glu_params", "ip_dwconv_swish_i8",
-    "ip_swish16_params_from_scales",
+    "ip_swish16_params_from_scales", "ip_relpos_mhsa_i8_host_async", "ip_relpos_mhsa_host_status",
 )
 
 ROWS = 0    # IP_LAYOUT_ROWS:  [B][T][C]
@@ -119,6 +119,10 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
         lib.ip_relpos_mhsa_i8_ex.argtypes = [P] * 6 + [P, P, ctypes.POINTER(SoftmaxParams), P] + [
             I] * 4 + [P, I, P, ctypes.c_size_t, P]
         lib.ip_relpos_mhsa_i8_ex.restype = I
+        lib.ip_relpos_mhsa_i8_host_async.argtypes = lib.ip_relpos_mhsa_i8_host.argtypes
+        lib.ip_relpos_mhsa_i8_host_async.restype = I
+        lib.ip_relpos_mhsa_host_status.argtypes = [P, I, I, I, I, P]
+        lib.ip_relpos_mhsa_host_status.restype = I
         lib.ip_linear_i8.argtypes = [P, I, P, P, P, P, I, I, I, I, I, P, I, P, ctypes.c_size_t, P]
         lib.ip_linear_i8.restype = I
         lib.ip_linear_swish_i8.argtypes = [P, P, P, P, P, ctypes.POINTER(SwishParams), I, I, I, I,
@@ -520,9 +524,12 @@ def dwconv_swish_i8(x, w, bias, m, s, sw16: tuple[int, int, int, int], *, out=No
 
 
 def relpos_mhsa_i8_host(q, k, v, p, u, v_bias, consts: LayerConstants, lengths, out, arena,
-                        stream=None):
+                        stream=None, wait: bool = True):
     """Whole layer from host buffers (torch CPU tensors, ideally pinned):
-    copies in, runs, copies the result into `out` and synchronises."""
+    copies in, runs, copies the result into `out` and synchronises.  With
+    wait=False the call only enqueues (ip_relpos_mhsa_i8_host_async): `out`
+    is valid after the stream synchronises, and host_status() reports
+    errors."""
     import torch
     B, H, T, dh = q.shape
     for name, t in (("q", q), ("k", k), ("v", v), ("p", p), ("u", u), ("v_bias", v_bias), ("out", out)):
@@ -535,13 +542,20 @@ def relpos_mhsa_i8_host(q, k, v, p, u, v_bias, consts: LayerConstants, lengths, 
         lens = ctypes.c_void_p(lengths.data_ptr())
     sm = SoftmaxParams(*consts.softmax)
     ptr = lambda t: ctypes.c_void_p(t.data_ptr())
-    rc = load().ip_relpos_mhsa_i8_host(
-        ptr(q), ptr(k), ptr(v), ptr(p), ptr(u), ptr(v_bias),
-        _arr(consts.multipliers, ctypes.c_int32), _arr(consts.shifts, ctypes.c_int32),
-        ctypes.byref(sm), lens, B, H, T, dh, ptr(out), ctypes.c_void_p(arena.data_ptr()),
-        arena.numel(), _stream_handle(stream))
-    _check("ip_relpos_mhsa_i8_host", rc)
+    fn = load().ip_relpos_mhsa_i8_host if wait else load().ip_relpos_mhsa_i8_host_async
+    rc = fn(ptr(q), ptr(k), ptr(v), ptr(p), ptr(u), ptr(v_bias),
+            _arr(consts.multipliers, ctypes.c_int32), _arr(consts.shifts, ctypes.c_int32),
+            ctypes.byref(sm), lens, B, H, T, dh, ptr(out), ctypes.c_void_p(arena.data_ptr()),
+            arena.numel(), _stream_handle(stream))
+    _check("ip_relpos_mhsa_i8_host" if wait else "ip_relpos_mhsa_i8_host_async", rc)
     return out
+
+
+def host_status(arena, B: int, H: int, T: int, dh: int = IP_DH, stream=None) -> int:
+    """Synchronises `stream` and returns the status of the last asynchronous
+    host-buffer call that used `arena` (0 = ok)."""
+    return load().ip_relpos_mhsa_host_status(ctypes.c_void_p(arena.data_ptr()), B, H, T, dh,
+                                             _stream_handle(stream))
 
 
 __all__ = ["build", "load", "relpos_mhsa_i8", "relpos_mhsa_i8_host", "status", "workspace_bytes",
@@ -551,4 +565,5 @@ __all__ = ["build", "load", "relpos_mhsa_i8", "relpos_mhsa_i8_host", "status", "
            "linear_constants", "ROWS", "HEADS", "linear_swish_i8", "swish_params_from_scales",
            "layernorm_i8", "layernorm_constants", "NormConstants", "residual_i8",
            "residual_params", "linear_glu_i8", "glu_params", "dwconv_swish_i8", "swish16_params",
+           "host_status",
            "IpError", "LibraryError", "EXPORTS"]

@@ -264,18 +264,17 @@ size_t ip_relpos_mhsa_host_arena_bytes(int B, int H, int T, int dh) {
     return 4 * act + pb + 2 * bias + lens + ws_bytes();
 }
 
-int ip_relpos_mhsa_i8_host(const int8_t *q, const int8_t *k, const int8_t *v, const int8_t *p,
-                           const int8_t *u, const int8_t *v_bias, const int32_t *multipliers,
-                           const int32_t *shifts, const ip_isoftmax_params *sm,
-                           const int32_t *lengths, int B, int H, int T, int dh, int8_t *out,
-                           void *arena, size_t arena_bytes, ip_stream_t stream) {
-    int rc = check_shape(B, H, T, dh);
-    if (rc != IP_OK) return rc;
-    if (B == 0 || H == 0) return IP_OK;
-    if (!q || !k || !v || !p || !u || !v_bias || !out || !arena) return IP_ERR_NULL;
-    if (!aligned(arena, 256)) return IP_ERR_ALIGN;
-    if (arena_bytes < ip_relpos_mhsa_host_arena_bytes(B, H, T, dh)) return IP_ERR_WORKSPACE;
-    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+namespace {
+
+// Arena of the host-buffer entry points: inputs, output, lengths and the
+// status word, each 256-byte aligned, in this order.
+struct HostArena {
+    int8_t *q, *k, *v, *out, *p, *u, *vb;
+    int32_t *len;
+    void *ws;
+};
+
+HostArena host_arena(void *arena, int B, int H, int T, int dh) {
     const size_t nact = static_cast<size_t>(B) * H * T * dh;
     const size_t np = static_cast<size_t>(H) * (2ull * T - 1) * dh;
     const size_t nb = static_cast<size_t>(H) * dh;
@@ -286,31 +285,88 @@ int ip_relpos_mhsa_i8_host(const int8_t *q, const int8_t *k, const int8_t *v, co
         off += align_up(bytes, 256);
         return r;
     };
-    int8_t *dq = reinterpret_cast<int8_t *>(take(nact));
-    int8_t *dk = reinterpret_cast<int8_t *>(take(nact));
-    int8_t *dv = reinterpret_cast<int8_t *>(take(nact));
-    int8_t *dout = reinterpret_cast<int8_t *>(take(nact));
-    int8_t *dp = reinterpret_cast<int8_t *>(take(np));
-    int8_t *du = reinterpret_cast<int8_t *>(take(nb));
-    int8_t *dvb = reinterpret_cast<int8_t *>(take(nb));
-    int32_t *dlen = reinterpret_cast<int32_t *>(take(4ull * (B > 0 ? B : 1)));
-    void *ws = take(ws_bytes());
-    if (cudaMemsetAsync(ws, 0, ws_bytes(), st) != cudaSuccess) return IP_ERR_CUDA;
+    HostArena h;
+    h.q = reinterpret_cast<int8_t *>(take(nact));
+    h.k = reinterpret_cast<int8_t *>(take(nact));
+    h.v = reinterpret_cast<int8_t *>(take(nact));
+    h.out = reinterpret_cast<int8_t *>(take(nact));
+    h.p = reinterpret_cast<int8_t *>(take(np));
+    h.u = reinterpret_cast<int8_t *>(take(nb));
+    h.vb = reinterpret_cast<int8_t *>(take(nb));
+    h.len = reinterpret_cast<int32_t *>(take(4ull * (B > 0 ? B : 1)));
+    h.ws = take(ws_bytes());
+    return h;
+}
+
+// Enqueues zeroing of the status word, the uploads, the kernel and the
+// download on `stream`; nothing waits.
+int host_enqueue(const int8_t *q, const int8_t *k, const int8_t *v, const int8_t *p,
+                 const int8_t *u, const int8_t *v_bias, const int32_t *multipliers,
+                 const int32_t *shifts, const ip_isoftmax_params *sm, const int32_t *lengths,
+                 int B, int H, int T, int dh, int8_t *out, void *arena, size_t arena_bytes,
+                 ip_stream_t stream, HostArena *where) {
+    int rc = check_shape(B, H, T, dh);
+    if (rc != IP_OK) return rc;
+    if (B == 0 || H == 0) return IP_OK;
+    if (!q || !k || !v || !p || !u || !v_bias || !out || !arena) return IP_ERR_NULL;
+    if (!aligned(arena, 256)) return IP_ERR_ALIGN;
+    if (arena_bytes < ip_relpos_mhsa_host_arena_bytes(B, H, T, dh)) return IP_ERR_WORKSPACE;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    const size_t nact = static_cast<size_t>(B) * H * T * dh;
+    const size_t np = static_cast<size_t>(H) * (2ull * T - 1) * dh;
+    const size_t nb = static_cast<size_t>(H) * dh;
+    const HostArena h = host_arena(arena, B, H, T, dh);
+    *where = h;
+    if (cudaMemsetAsync(h.ws, 0, ws_bytes(), st) != cudaSuccess) return IP_ERR_CUDA;
     struct Copy {
         void *dst;
         const void *src;
         size_t n;
-    } copies[] = {{dq, q, nact}, {dk, k, nact}, {dv, v, nact}, {dp, p, np},
-                  {du, u, nb},   {dvb, v_bias, nb}, {dlen, lengths, lengths ? 4ull * B : 0}};
+    } copies[] = {{h.q, q, nact}, {h.k, k, nact}, {h.v, v, nact}, {h.p, p, np},
+                  {h.u, u, nb},   {h.vb, v_bias, nb}, {h.len, lengths, lengths ? 4ull * B : 0}};
     for (const Copy &c : copies)
         if (c.n && cudaMemcpyAsync(c.dst, c.src, c.n, cudaMemcpyHostToDevice, st) != cudaSuccess)
             return IP_ERR_CUDA;
-    rc = ip_relpos_mhsa_i8(dq, dk, dv, dp, du, dvb, multipliers, shifts, sm,
-                           lengths ? dlen : nullptr, B, H, T, dh, dout, ws, ws_bytes(), stream);
+    rc = ip_relpos_mhsa_i8(h.q, h.k, h.v, h.p, h.u, h.vb, multipliers, shifts, sm,
+                           lengths ? h.len : nullptr, B, H, T, dh, h.out, h.ws, ws_bytes(),
+                           stream);
     if (rc != IP_OK) return rc;
-    if (nact && cudaMemcpyAsync(out, dout, nact, cudaMemcpyDeviceToHost, st) != cudaSuccess)
+    if (nact && cudaMemcpyAsync(out, h.out, nact, cudaMemcpyDeviceToHost, st) != cudaSuccess)
         return IP_ERR_CUDA;
-    return ip_relpos_mhsa_status(ws, stream);
+    return IP_OK;
+}
+
+}  // namespace
+
+int ip_relpos_mhsa_i8_host(const int8_t *q, const int8_t *k, const int8_t *v, const int8_t *p,
+                           const int8_t *u, const int8_t *v_bias, const int32_t *multipliers,
+                           const int32_t *shifts, const ip_isoftmax_params *sm,
+                           const int32_t *lengths, int B, int H, int T, int dh, int8_t *out,
+                           void *arena, size_t arena_bytes, ip_stream_t stream) {
+    HostArena h;
+    const int rc = host_enqueue(q, k, v, p, u, v_bias, multipliers, shifts, sm, lengths, B, H, T,
+                                dh, out, arena, arena_bytes, stream, &h);
+    if (rc != IP_OK || B == 0 || H == 0) return rc;
+    return ip_relpos_mhsa_status(h.ws, stream);
+}
+
+int ip_relpos_mhsa_i8_host_async(const int8_t *q, const int8_t *k, const int8_t *v,
+                                 const int8_t *p, const int8_t *u, const int8_t *v_bias,
+                                 const int32_t *multipliers, const int32_t *shifts,
+                                 const ip_isoftmax_params *sm, const int32_t *lengths, int B,
+                                 int H, int T, int dh, int8_t *out, void *arena,
+                                 size_t arena_bytes, ip_stream_t stream) {
+    HostArena h;
+    return host_enqueue(q, k, v, p, u, v_bias, multipliers, shifts, sm, lengths, B, H, T, dh,
+                        out, arena, arena_bytes, stream, &h);
+}
+
+int ip_relpos_mhsa_host_status(const void *arena, int B, int H, int T, int dh,
+                               ip_stream_t stream) {
+    if (!arena) return IP_ERR_NULL;
+    const int rc = check_shape(B, H, T, dh);
+    if (rc != IP_OK) return rc;
+    return ip_relpos_mhsa_status(host_arena(const_cast<void *>(arena), B, H, T, dh).ws, stream);
 }
 
 const char *ip_strerror(int code) {

@@ -160,3 +160,26 @@ def test_repeated_calls_share_workspace(ip, orc):
                                 _dev(lay.vb), c, workspace=ws)
         assert ip.status(ws) == 0
         assert_same(out.cpu().numpy(), oracle_out(orc, lay, c))
+
+
+def test_async_host_calls_overlap_on_two_streams(ip, orc):
+    # three layers from host buffers, issued without waiting on alternating
+    # streams and arenas, each output checked against the oracle
+    B, H, T = 2, 8, 100
+    lays = [synth.draw(B, H, T, 128, seed=990 + i, p_mode="sinusoid") for i in range(3)]
+    pin = lambda a: torch.from_numpy(np.ascontiguousarray(a)).pin_memory()
+    arenas = [torch.empty(ip.host_arena_bytes(B, H, T), dtype=torch.uint8, device="cuda")
+              for _ in range(2)]
+    streams = [torch.cuda.Stream(), torch.cuda.Stream()]
+    outs = []
+    for i, lay in enumerate(lays):
+        c = ip.layer_constants(lay.scales)
+        out = torch.empty((B, H, T, 128), dtype=torch.int8).pin_memory()
+        ip.relpos_mhsa_i8_host(pin(lay.q), pin(lay.k), pin(lay.v), pin(lay.p), pin(lay.u),
+                               pin(lay.vb), c, None, out, arenas[i & 1], stream=streams[i & 1],
+                               wait=False)
+        outs.append((out, c))
+    for j in range(2):
+        assert ip.host_status(arenas[j], B, H, T, stream=streams[j]) == 0
+    for (out, c), lay in zip(outs, lays):
+        assert_same(out.numpy(), oracle_out(orc, lay, c))
