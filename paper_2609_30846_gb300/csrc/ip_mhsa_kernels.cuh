@@ -17,7 +17,8 @@
 // The consumers, per CTA:
 //   pass 1  for each chunk of 64 keys: the content MMAs Q K^T, the MMAs of
 //           the position band Q P_band^T for the next chunk (issued before
-//           this chunk's epilogue so that the tensor pipe stays busy), the
+//           this chunk's epilogue so that the tensor pipe stays busy; the 16
+//           band columns it shares with this chunk are carried over), the
 //           relative shift as an index remap through shared memory, the
 //           fused requantisation of Eq. 11 and the key mask; int8 scores
 //           stay in shared memory, row maxima in registers;
@@ -48,6 +49,7 @@ constexpr int KU_OFF = K_TILE_BYTES + P_TILE_BYTES;   // int32 K u of the chunk'
 constexpr int PV_OFF = KU_OFF + NK * 4;                // int32 P v of the band rows
 constexpr int STAGE_BYTES = 25600;        // PV_OFF + BAND_ROWS * 4, rounded to 1024
 constexpr int BAND_TILES = 10;            // n8 tiles of one warp's band: 16 + NK - 1 -> 80
+constexpr int CARRY_TILES = BAND_TILES - NK / 8;   // band tiles shared by consecutive chunks
 constexpr int REMAP_STRIDE = 88;          // int32 words per band row in the remap buffer
 constexpr int REMAP_BYTES = 16 * REMAP_STRIDE * 4;
 constexpr int LUT_ENTRIES = 256;
@@ -56,6 +58,7 @@ constexpr int CHUNK_SCORE_BYTES = 16 * NK;   // one warp's int8 scores of one ch
 
 static_assert(PV_OFF + BAND_ROWS * 4 <= STAGE_BYTES, "stage layout");
 static_assert(STAGE_BYTES % 1024 == 0, "the 128-byte swizzle needs 1024-byte aligned tiles");
+static_assert(CARRY_TILES == 2 && (BAND_TILES - CARRY_TILES) % 4 == 0, "band tiling");
 
 struct SmemLayout {
     int stages, scores, remap, lut, bars, total;
@@ -908,8 +911,16 @@ __global__ void __launch_bounds__(NTHREADS, 2)
             }
             const uint32_t ptile = stage_addr(s ^ 1) + K_TILE_BYTES + band_row0 * 128;
             const uint32_t pvs = stage_addr(s ^ 1) + PV_OFF + band_row0 * 4;
+            // The band of chunk c + 1 starts NK positions after that of chunk
+            // c: its first CARRY_TILES tiles are the last ones of chunk c
+            // (the same rows of Q against the same rows of P), kept in
+            // registers; only the other NK columns are new MMAs.
 #pragma unroll
-            for (int nt = 0; nt < BAND_TILES; ++nt) {
+            for (int nt = 0; nt < CARRY_TILES; ++nt)
+#pragma unroll
+                for (int e = 0; e < 4; ++e) bacc[nt][e] = bacc[NK / 8 + nt][e];
+#pragma unroll
+            for (int nt = CARRY_TILES; nt < BAND_TILES; ++nt) {
                 const int2 v = lds64(pvs + (nt * 8 + 2 * t4) * 4);
                 bacc[nt][0] = v.x;
                 bacc[nt][1] = v.y;
@@ -920,18 +931,18 @@ __global__ void __launch_bounds__(NTHREADS, 2)
             uint32_t packed[8];
 #pragma unroll
             for (int m = 0; m < 4; ++m) {
-                const int kh = m >> 1, t0 = (m & 1) * 5;
-                uint32_t b[5][4];
+                const int kh = m >> 1, t0 = CARRY_TILES + (m & 1) * 4;
+                uint32_t b[4][4];
 #pragma unroll
-                for (int i = 0; i < 5; ++i)
+                for (int i = 0; i < 4; ++i)
                     ldsm_x4(ptile + swz((t0 + i) * 8 + lm_row, kh * 4 + lm_mat), b[i][0], b[i][1],
                             b[i][2], b[i][3]);
 #pragma unroll
-                for (int i = 0; i < 5; ++i) mma_s8s8(bacc[t0 + i], qa[2 * kh], b[i][0], b[i][1]);
+                for (int i = 0; i < 4; ++i) mma_s8s8(bacc[t0 + i], qa[2 * kh], b[i][0], b[i][1]);
                 packed[2 * m] = score_tile<false>(cacc[2 * m], 2 * m, remap, lane, m_c, m_p, half_s,
                                                   s_s, NK, mx0, mx1);
 #pragma unroll
-                for (int i = 0; i < 5; ++i) mma_s8s8(bacc[t0 + i], qa[2 * kh + 1], b[i][2], b[i][3]);
+                for (int i = 0; i < 4; ++i) mma_s8s8(bacc[t0 + i], qa[2 * kh + 1], b[i][2], b[i][3]);
                 packed[2 * m + 1] = score_tile<false>(cacc[2 * m + 1], 2 * m + 1, remap, lane, m_c,
                                                       m_p, half_s, s_s, NK, mx0, mx1);
             }
