@@ -19,7 +19,7 @@ SOURCES = [os.path.join(CSRC, f) for f in ("ip_mhsa.cu", "ip_linear.cu", "ip_nor
 DEPS = SOURCES + [os.path.join(CSRC, f) for f in ("ip_mhsa_kernels.cuh", "ip_linear_kernels.cuh",
                                                   "ip_norm_kernels.cuh", "ip_block_kernels.cuh",
                                                   "ip_ptx.cuh",
-                                                  "ip_probe.cuh")] + [
+                                                  "ip_probe.cuh", "ip_host_util.h")] + [
     os.path.join(INCLUDE, "ip_mhsa.h")]
 ARCH = "-gencode=arch=compute_103a,code=sm_103a"
 

@@ -3,6 +3,7 @@
 // ip_linear_kernels.cuh.
 #include "ip_mhsa.h"
 #include "ip_linear_kernels.cuh"
+#include "ip_host_util.h"
 
 #include <cuda.h>
 #include <cuda_runtime.h>
@@ -62,13 +63,6 @@ int sm_count() {
         g_sms[dev] = n;
     }
     return g_sms[dev];
-}
-
-// Constant of udiv_magic: floor(2^64 / d) + 1, or 0 for d = 1.
-unsigned long long div_magic(unsigned long long d) {
-    if (d <= 1) return 0;
-    const unsigned __int128 one = static_cast<unsigned __int128>(1) << 64;
-    return static_cast<unsigned long long>(one / d) + 1;
 }
 
 int ensure_smem() {
@@ -157,9 +151,9 @@ int linear_launch(const int8_t *x, int x_layout, const int8_t *w, const int32_t 
                                       ? (static_cast<long long>(B) * T + ipl::BM - 1) / ipl::BM
                                       : static_cast<long long>(B) * prm.tpu;
     prm.ntiles = static_cast<unsigned>(frame_tiles * prm.ntn);
-    prm.magic_ntn = div_magic(prm.ntn);
-    prm.magic_T = div_magic(T);
-    prm.magic_tpu = div_magic(prm.tpu);
+    prm.magic_ntn = iph::div_magic(prm.ntn);
+    prm.magic_T = iph::div_magic(T);
+    prm.magic_tpu = iph::div_magic(prm.tpu);
     prm.sw_qc = sw ? sw->q_c : 0;
     prm.sw_qone = sw ? sw->q_one : 0;
     prm.sw_m = sw ? sw->m : 0;

@@ -236,8 +236,7 @@ __global__ void __launch_bounds__(THREADS, 1)
 #pragma unroll
                     for (int j = 0; j < 4; ++j) mma_s8s8(acc[i][j], af[i], bf[j][0], bf[j][1]);
             }
-            __syncwarp();
-            if (lane == 0) mbar_arrive(empty_bar(s));
+            release_stage(empty_bar(s), lane);
         }
 
         // ------------------------------------------------------ epilogue

@@ -4,6 +4,7 @@
 #include "ip_mhsa.h"
 #include "ip_mhsa_kernels.cuh"
 #include "ip_probe.cuh"
+#include "ip_host_util.h"
 
 #include <cuda.h>
 #include <cuda_runtime.h>
@@ -227,6 +228,7 @@ int ip_relpos_mhsa_i8_ex(const int8_t *q, const int8_t *k, const int8_t *v, cons
     prm.q_ln2 = sm->q_ln2;
     prm.q_b = sm->q_b;
     prm.q_c = sm->q_c;
+    prm.ln2_magic = iph::div_magic(static_cast<unsigned long long>(sm->q_ln2));
     prm.timeout_cycles = g_timeout_cycles;
     prm.stall_injection = g_stall_injection;
     const SplitPlan sp = plan_split(B, H, ntiles, resident_ctas(smem));

@@ -87,6 +87,7 @@ struct FusedParams {
     int32_t m_c, m_p, m_o;
     int32_t sh_s, sh_o;       // total right shifts, 31 + s
     int32_t q_ln2, q_b, q_c;
+    unsigned long long ln2_magic;   // udiv_magic constant of q_ln2
     long long timeout_cycles; // bound of every barrier wait
     int stall_injection;      // test hook: consumers first wait on a barrier nobody arrives on
     // Tail split: the last nsplit tiles of the (b, h, tile) order, from
@@ -168,13 +169,15 @@ __device__ __forceinline__ void vfrag(uint32_t vtile, int ks, int c, int lane, u
 }
 
 // floor(2^32 / s) for s >= 2 by restoring binary long division (the
-// quotient is at most 2^31).
+// quotient is at most 2^31).  With 2^(L-1) <= s < 2^L the quotient is at
+// most 2^(33-L), so the digits start at bit 33 - L.
 __device__ __forceinline__ uint32_t div_2pow32(unsigned long long s) {
     if (s > (1ull << 32)) return 0u;
     unsigned long long rem = 1ull << 32;
     uint32_t quo = 0;
+    const int top = __clzll(static_cast<long long>(s)) - 31;   // 33 - L
 #pragma unroll 1
-    for (int bit = 31; bit >= 0; --bit) {
+    for (int bit = top < 31 ? top : 31; bit >= 0; --bit) {
         const unsigned long long t = s << bit;
         if (t <= rem) {
             rem -= t;
@@ -185,17 +188,11 @@ __device__ __forceinline__ uint32_t div_2pow32(unsigned long long s) {
 }
 
 // I-BERT integer exponential of d = -nd (0 <= nd < 512): z = floor(nd /
-// q_ln2) by long division, p = -nd + z q_ln2, ((p + q_b)^2 + q_c) >> z.
-__device__ __forceinline__ uint32_t iexp_neg(int nd, int q_ln2, int q_b, int q_c) {
-    int rem = nd, z = 0;
-#pragma unroll 1
-    for (int bit = 8; bit >= 0; --bit) {
-        const int t = q_ln2 << bit;
-        if (q_ln2 <= (nd >> bit) && t <= rem) {
-            rem -= t;
-            z |= 1 << bit;
-        }
-    }
+// q_ln2) (exact multiply-high by the constant of q_ln2), p = -nd + z q_ln2,
+// ((p + q_b)^2 + q_c) >> z.
+__device__ __forceinline__ uint32_t iexp_neg(int nd, int q_ln2, int q_b, int q_c,
+                                             unsigned long long ln2_magic) {
+    const int z = static_cast<int>(udiv_magic(static_cast<uint32_t>(nd), ln2_magic));
     const long long p = -static_cast<long long>(nd) + static_cast<long long>(z) * q_ln2;
     const long long t = p + q_b;
     const long long L = t * t + q_c;
@@ -578,7 +575,31 @@ __global__ void __launch_bounds__(NTHREADS, 2)
     const uint32_t never_bar = bar_base + 8u * (3 * NSTAGE);   // test hook only
     auto pair_bar = [&](int strip2) { return bar_base + 8u * (3 * NSTAGE + 1 + strip2); };
 
-    if (threadIdx.x == 0) {
+    const uint32_t stage_base = smem_u32(smem + L.stages);
+    auto stage_addr = [&](int s) { return stage_base + s * STAGE_BYTES; };
+    // Use `it` of the stage ring (stage it & 1, phase it >> 1): TMA lands
+    // (full), the producers prepare it (ready), the consumers release it
+    // (empty), and the stage is refilled with use it + 2.
+    auto issue = [&](int it) {
+        const int s = it & 1;
+        const uint32_t dst = stage_addr(s);
+        if (it < nchunks) {
+            const int j0 = it * NK;
+            mbar_expect_tx(full_bar(s), K_TILE_BYTES + P_TILE_BYTES);
+            tma_load_3d(dst, &tm_k, 0, j0, bh, full_bar(s));
+            tma_load_3d(dst + K_TILE_BYTES, &tm_p, 0, j0 - i0 - (MROWS - 1) + T - 1, h,
+                        full_bar(s));
+        } else {
+            const int j0 = (it - nchunks) * NK;
+            mbar_expect_tx(full_bar(s), K_TILE_BYTES);
+            tma_load_3d(dst, &tm_v, 0, j0, bh, full_bar(s));
+        }
+    };
+
+    // The thread that issues the copies initialises the barriers and sends
+    // the first two chunks off at once; the exponential table and the Q
+    // fragments are built while they travel.
+    if (threadIdx.x == NCWARPS * 32) {
         for (int s = 0; s < NSTAGE; ++s) {
             mbar_init(full_bar(s), 1);
             mbar_init(ready_bar(s), NPWARPS);
@@ -589,21 +610,38 @@ __global__ void __launch_bounds__(NTHREADS, 2)
         mbar_init(pair_bar(1), 2);
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        issue(0);
+        if (total > 1) issue(1);
+    }
+
+    // Consumers: row strip of 16 rows, one per warp in a whole tile; in a
+    // split tile strips 2 part, 2 part + 1, each shared by warps 2s', 2s' + 1.
+    // Q fragments (A operand) for the four 32-wide k steps, rows >= T zero.
+    const int g = lane >> 2;       // row group of the MMA fragments
+    const int t4 = lane & 3;       // thread in group
+    const int strip = part < 0 ? warp : 2 * part + (warp >> 1);
+    const int wrow0 = i0 + strip * 16;
+    uint32_t qa[4][4];
+    if (warp < NCWARPS) {
+        const int8_t *qbase = prm.q + static_cast<size_t>(bh) * T * DH;
+        const int r0 = wrow0 + g, r1 = wrow0 + g + 8;
+#pragma unroll
+        for (int ks = 0; ks < 4; ++ks) {
+            const int c0 = ks * 32 + 4 * t4;
+            qa[ks][0] = r0 < T ? *reinterpret_cast<const uint32_t *>(qbase + static_cast<size_t>(r0) * DH + c0) : 0u;
+            qa[ks][1] = r1 < T ? *reinterpret_cast<const uint32_t *>(qbase + static_cast<size_t>(r1) * DH + c0) : 0u;
+            qa[ks][2] = r0 < T ? *reinterpret_cast<const uint32_t *>(qbase + static_cast<size_t>(r0) * DH + c0 + 16) : 0u;
+            qa[ks][3] = r1 < T ? *reinterpret_cast<const uint32_t *>(qbase + static_cast<size_t>(r1) * DH + c0 + 16) : 0u;
+        }
     }
     for (int d = threadIdx.x; d < LUT_ENTRIES; d += NTHREADS) {
-        const uint32_t e = iexp_neg(d, prm.q_ln2, prm.q_b, prm.q_c);
+        const uint32_t e = iexp_neg(d, prm.q_ln2, prm.q_b, prm.q_c, prm.ln2_magic);
 #pragma unroll
         for (int c = 0; c < LUT_COPIES; ++c) sts32(lut + (d * LUT_COPIES + c) * 4, e);
     }
     __syncthreads();
 
-    const uint32_t stage_base = smem_u32(smem + L.stages);
-    auto stage_addr = [&](int s) { return stage_base + s * STAGE_BYTES; };
-
     // ------------------------------------------------------------ producer
-    // Use `it` of the stage ring (stage it & 1, phase it >> 1): TMA lands
-    // (full), the producer prepares it (ready), the consumers release it
-    // (empty), and the stage is refilled with use it + 2.
     if (warp >= NCWARPS) {
         const int pw = warp - NCWARPS;   // 0: TMA and its share of the biases; 1: its share
         uint32_t uw[32], vw[32];
@@ -617,21 +655,6 @@ __global__ void __launch_bounds__(NTHREADS, 2)
                 vw[4 * c] = bq.x; vw[4 * c + 1] = bq.y; vw[4 * c + 2] = bq.z; vw[4 * c + 3] = bq.w;
             }
         }
-        auto issue = [&](int it) {
-            const int s = it & 1;
-            const uint32_t dst = stage_addr(s);
-            if (it < nchunks) {
-                const int j0 = it * NK;
-                mbar_expect_tx(full_bar(s), K_TILE_BYTES + P_TILE_BYTES);
-                tma_load_3d(dst, &tm_k, 0, j0, bh, full_bar(s));
-                tma_load_3d(dst + K_TILE_BYTES, &tm_p, 0, j0 - i0 - (MROWS - 1) + T - 1, h,
-                            full_bar(s));
-            } else {
-                const int j0 = (it - nchunks) * NK;
-                mbar_expect_tx(full_bar(s), K_TILE_BYTES);
-                tma_load_3d(dst, &tm_v, 0, j0, bh, full_bar(s));
-            }
-        };
         if (pw == 1) {
             // second producer warp: its share of the bias vectors of each
             // staged score-pass chunk
@@ -643,17 +666,12 @@ __global__ void __launch_bounds__(NTHREADS, 2)
                 }
                 prep_bias(1, stage_addr(s), stage_addr(s) + K_TILE_BYTES, stage_addr(s) + KU_OFF,
                           stage_addr(s) + PV_OFF, uw, vw, lane);
-                __syncwarp();
-                if (lane == 0) mbar_arrive(ready_bar(s));
+                release_stage(ready_bar(s), lane);
             }
             return;
         }
-        int issued = total > 1 ? 2 : 1, landed = 0;
+        int issued = total > 1 ? 2 : 1, landed = 0;   // chunks 0 and 1 left at the start
         bool ok = true;
-        if (lane == 0) {
-            issue(0);
-            if (total > 1) issue(1);
-        }
         for (int it = 0; it < total; ++it) {
             const int s = it & 1;
             if (it < nchunks) {
@@ -666,8 +684,7 @@ __global__ void __launch_bounds__(NTHREADS, 2)
                 landed = it + 1;
                 prep_bias(0, stage_addr(s), stage_addr(s) + K_TILE_BYTES, stage_addr(s) + KU_OFF,
                           stage_addr(s) + PV_OFF, uw, vw, lane);
-                __syncwarp();
-                if (lane == 0) mbar_arrive(ready_bar(s));
+                release_stage(ready_bar(s), lane);
             }
             // (attn.V pass: the consumers read the V tile as TMA left it)
             if (it + 2 < total) {
@@ -691,28 +708,6 @@ __global__ void __launch_bounds__(NTHREADS, 2)
     }
 
     // ------------------------------------------------------------ consumers
-    const int g = lane >> 2;       // row group of the MMA fragments
-    const int t4 = lane & 3;       // thread in group
-    // Row strip of 16 rows: one per warp in a whole tile; in a split tile
-    // strips 2 part, 2 part + 1, each shared by warps 2s', 2s' + 1.
-    const int strip = part < 0 ? warp : 2 * part + (warp >> 1);
-    const int wrow0 = i0 + strip * 16;
-    const int8_t *qbase = prm.q + static_cast<size_t>(bh) * T * DH;
-
-    // Q fragments (A operand) for the four 32-wide k steps, rows >= T zero.
-    uint32_t qa[4][4];
-    {
-        const int r0 = wrow0 + g, r1 = wrow0 + g + 8;
-#pragma unroll
-        for (int ks = 0; ks < 4; ++ks) {
-            const int c0 = ks * 32 + 4 * t4;
-            qa[ks][0] = r0 < T ? *reinterpret_cast<const uint32_t *>(qbase + static_cast<size_t>(r0) * DH + c0) : 0u;
-            qa[ks][1] = r1 < T ? *reinterpret_cast<const uint32_t *>(qbase + static_cast<size_t>(r1) * DH + c0) : 0u;
-            qa[ks][2] = r0 < T ? *reinterpret_cast<const uint32_t *>(qbase + static_cast<size_t>(r0) * DH + c0 + 16) : 0u;
-            qa[ks][3] = r1 < T ? *reinterpret_cast<const uint32_t *>(qbase + static_cast<size_t>(r1) * DH + c0 + 16) : 0u;
-        }
-    }
-
     const uint32_t remap = smem_u32(smem + L.remap) + warp * REMAP_BYTES;
     const uint32_t scores = smem_u32(smem + L.scores) + warp * (prm.nchunk_max * CHUNK_SCORE_BYTES);
     const long long m_c = prm.m_c, m_p = prm.m_p;
@@ -745,8 +740,7 @@ __global__ void __launch_bounds__(NTHREADS, 2)
             half_chunk_mma(hb, hc, qa, stage_addr(s) + K_TILE_BYTES + band_row0 * 128,
                            stage_addr(s) + PV_OFF + band_row0 * 4, stage_addr(s),
                            stage_addr(s) + KU_OFF, nt0, lane);
-            __syncwarp();
-            if (lane == 0) mbar_arrive(empty_bar(s));
+            release_stage(empty_bar(s), lane);
 #pragma unroll
             for (int i = 0; i < 6; ++i) {
                 sts64(remap + (g * REMAP_STRIDE + (nt0 + i) * 8 + 2 * t4) * 4, hb[i][0], hb[i][1]);
@@ -857,8 +851,7 @@ __global__ void __launch_bounds__(NTHREADS, 2)
                     mma_u8s8(oacc[4 * grp + 2 * i + 1], af, bv[i][2], bv[i][3]);
                 }
             }
-            __syncwarp();
-            if (lane == 0) mbar_arrive(empty_bar(s));
+            release_stage(empty_bar(s), lane);
         }
 
         // the partner finishes the other half of the output columns
@@ -901,8 +894,7 @@ __global__ void __launch_bounds__(NTHREADS, 2)
         }
         int cacc[8][4];
         content_mma(cacc, qa, stage_addr(s), stage_addr(s) + KU_OFF, lane);
-        __syncwarp();
-        if (lane == 0) mbar_arrive(empty_bar(s));
+        release_stage(empty_bar(s), lane);
         const uint32_t sdst = scores + c * CHUNK_SCORE_BYTES;
         if (c + 1 < nchunks) {
             if (!warp_wait(ready_bar(s ^ 1), ((c + 1) >> 1) & 1, prm.timeout_cycles)) {
@@ -1041,8 +1033,7 @@ __global__ void __launch_bounds__(NTHREADS, 2)
             }
             prob_operand(pw, af);
         }
-        __syncwarp();
-        if (lane == 0) mbar_arrive(empty_bar(s));
+        release_stage(empty_bar(s), lane);
     }
 
     // ---- output requantisation (Eq. 7): per row and d chunk c, four bytes

@@ -36,6 +36,17 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
     return ok != 0;
 }
 
+// Hands a shared-memory stage that this warp has read with generic loads
+// (ldmatrix, ld.shared) back to the warp that refills it by TMA: the proxy
+// fence orders those reads before the async-proxy writes of the refill
+// (without it a refill could land before a read was performed), then lane 0
+// arrives on `bar`.
+__device__ __forceinline__ void release_stage(uint32_t bar, int lane) {
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    __syncwarp();
+    if (lane == 0) mbar_arrive(bar);
+}
+
 // Waits for the phase of `parity` to complete; gives up after `limit` clock
 // cycles and returns false.
 __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, long long limit) {
