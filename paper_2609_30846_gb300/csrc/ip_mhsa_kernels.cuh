@@ -341,8 +341,9 @@ __device__ __forceinline__ uint32_t prob_word(uint32_t wv, uint32_t lut_g, int m
         const int mx = e < 2 ? mx0 : mx1;
         const uint32_t f = e < 2 ? f0 : f1;
         const uint32_t ev = lds32(lut_addr(lut_g, mx - sc[e]));
-        const unsigned long long y = (static_cast<unsigned long long>(ev) * f) >> 24;
-        a[e] = static_cast<uint32_t>(min(y, 255ull));
+        // min(floor(ev f / 2^24), 255) with ev f = hi 2^32 + lo: 255 when
+        // hi > 0, else lo >> 24 (at most 255)
+        a[e] = __umulhi(ev, f) != 0u ? 255u : (ev * f) >> 24;
     }
     return pack4(a[0], a[1], a[2], a[3]);
 }
