@@ -69,10 +69,16 @@ typedef struct {
 #define IP_MAX_T 2048   /* frames; the int8 scores of a 64-row tile stay in shared memory */
 #define IP_MAX_B 65535
 #define IP_MAX_H 65535
+/* B H ceil(T / 64) (the 64-row query tiles of a call) must stay below this:
+ * the kernel's work items are numbered with 31 bits. */
+#define IP_MAX_TILES (1ll << 30)
 
 /* Bytes of device workspace a call needs: the device-side status word of
  * the calls that use it.  The caller zero-fills the workspace once before
- * its first use; ip_relpos_mhsa_status reads and clears it.  0 if the shape
+ * its first use; ip_relpos_mhsa_status reads and clears it.  The workspace
+ * also holds the work-item counters of the attention kernel (its CTAs claim
+ * query tiles from them), which every call returns to zero when it ends;
+ * calls that share a workspace must not overlap on the GPU.  0 if the shape
  * is invalid. */
 size_t ip_relpos_mhsa_workspace_bytes(int B, int H, int T, int dh);
 
@@ -88,7 +94,8 @@ size_t ip_relpos_mhsa_workspace_bytes(int B, int H, int T, int dh);
  *                 256-byte aligned, owned by the caller; one call at a time
  *                 per workspace.
  * The call validates its arguments on the host and then enqueues one
- * kernel on `stream`.  B == 0 or H == 0 is an empty problem: the call
+ * kernel on `stream` (a persistent grid of one CTA per resident slot that
+ * walks the 64-row query tiles of all (b, h)).  B == 0 or H == 0 is an empty problem: the call
  * returns IP_OK without touching any pointer.  A kernel-side barrier timeout is reported later by
  * ip_relpos_mhsa_status. */
 int ip_relpos_mhsa_i8(const int8_t *q, const int8_t *k, const int8_t *v,

@@ -25,7 +25,9 @@ size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 bool aligned(const void *p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 
-// The workspace holds the device error word of the calls that use it.
+// The workspace holds the device error word of the calls that use it (byte
+// 0) and the attention kernel's item counters (bytes 64 and 128), which the
+// last CTA of every launch returns to zero.
 size_t ws_bytes() { return WS_HEADER; }
 
 int check_shape(int B, int H, int T, int dh) {
@@ -114,38 +116,31 @@ int resident_ctas(int smem) {
     return g_occ_slots;
 }
 
-// Tail split.  The N tiles run in waves of `slots` CTAs; when the last wave
-// is at most half full (r = N mod slots tiles, 2 r <= slots), its r tiles
-// are done as 2 r halves of 32 rows whose warps split the keys of every
-// chunk, so the last wave takes about half as long.  The halves live in
-// grid slices after the B batch slices, which the block scheduler
-// dispatches last.
-struct SplitPlan {
-    int nsplit = 0, extra = 0, b0 = 0, h0 = 0, tile0 = 0;
-    long long first = 0;
+// Work items of the persistent kernel.  The N whole tiles run on G resident
+// CTAs in rounds; when the last round is at most half full (r = N mod G
+// tiles, 2 r <= G), its r tiles become 2 r halves of 32 rows whose warps
+// split the keys of every chunk, so the last round takes about half as long.
+struct ItemPlan {
+    uint32_t nwhole = 0, nitems = 0, grid = 0;
 };
 
-SplitPlan plan_split(int B, int H, int ntiles, int slots) {
-    SplitPlan sp;
-    const long long N = static_cast<long long>(B) * H * ntiles;
-    long long ns = 0;
+ItemPlan plan_items(long long N, int slots) {
+    ItemPlan ip;
+    long long nwhole = N, nitems = N;
     if (g_split_mode == 1) {
-        ns = N;
+        nwhole = 0;
+        nitems = 2 * N;
     } else if (g_split_mode < 0 && slots > 0) {
         const long long r = N % slots;
-        if (r > 0 && 2 * r <= slots) ns = r;
+        if (r > 0 && 2 * r <= slots) {
+            nwhole = N - r;
+            nitems = N + r;
+        }
     }
-    const long long per_slice = static_cast<long long>(ntiles) * H;
-    const long long extra = (2 * ns + per_slice - 1) / per_slice;
-    if (ns == 0 || B + extra > IP_MAX_B) return sp;
-    sp.nsplit = static_cast<int>(ns);
-    sp.extra = static_cast<int>(extra);
-    sp.first = N - ns;
-    sp.tile0 = static_cast<int>(sp.first % ntiles);
-    const long long bh = sp.first / ntiles;
-    sp.h0 = static_cast<int>(bh % H);
-    sp.b0 = static_cast<int>(bh / H);
-    return sp;
+    ip.nwhole = static_cast<uint32_t>(nwhole);
+    ip.nitems = static_cast<uint32_t>(nitems);
+    ip.grid = static_cast<uint32_t>(nitems < slots ? nitems : slots);
+    return ip;
 }
 
 }  // namespace
@@ -197,25 +192,27 @@ int ip_relpos_mhsa_i8_ex(const int8_t *q, const int8_t *k, const int8_t *v, cons
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
     int *err = static_cast<int *>(workspace);
 
-    CUtensorMap tm_k, tm_v, tm_p;
+    CUtensorMap tm_q, tm_k, tm_v, tm_p;
     const unsigned long long bh = static_cast<unsigned long long>(B) * H;
-    if (!make_map(&tm_k, k, T, bh, ipk::NK) || !make_map(&tm_v, v, T, bh, ipk::NK) ||
+    if (!make_map(&tm_q, q, T, bh, ipk::MROWS) || !make_map(&tm_k, k, T, bh, ipk::NK) || !make_map(&tm_v, v, T, bh, ipk::NK) ||
         !make_map(&tm_p, p, 2ull * T - 1, H, ipk::BAND_ROWS))
         return IP_ERR_CUDA;
 
     const int ntiles = (T + ipk::MROWS - 1) / ipk::MROWS;
+    const long long N = static_cast<long long>(B) * H * ntiles;   // whole tiles
+    if (N >= IP_MAX_TILES) return IP_ERR_SHAPE;   // item indices stay below 2^31
     const int nchunk_max = (T + ipk::NK - 1) / ipk::NK;
     const int smem = ipk::smem_layout(nchunk_max).total + 1024;
     rc = ensure_smem(smem);
     if (rc != IP_OK) return rc;
 
     ipk::FusedParams prm;
-    prm.q = q;
     prm.u = u;
     prm.vb = v_bias;
     prm.out = out;
     prm.lengths = lengths;
     prm.err = err;
+    prm.sched = reinterpret_cast<unsigned int *>(static_cast<char *>(workspace) + 64);
     prm.B = B;
     prm.H = H;
     prm.T = T;
@@ -231,15 +228,17 @@ int ip_relpos_mhsa_i8_ex(const int8_t *q, const int8_t *k, const int8_t *v, cons
     prm.ln2_magic = iph::div_magic(static_cast<unsigned long long>(sm->q_ln2));
     prm.timeout_cycles = g_timeout_cycles;
     prm.stall_injection = g_stall_injection;
-    const SplitPlan sp = plan_split(B, H, ntiles, resident_ctas(smem));
-    prm.nsplit = sp.nsplit;
-    prm.split_b0 = sp.b0;
-    prm.split_h0 = sp.h0;
-    prm.split_tile0 = sp.tile0;
-    prm.first_split = sp.first;
+    const int slots = resident_ctas(smem);
+    if (slots < 1) return IP_ERR_CUDA;
+    const ItemPlan ip = plan_items(N, slots);
+    prm.ntiles = ntiles;
+    prm.tiles_magic = iph::div_magic(static_cast<unsigned long long>(ntiles));
+    prm.heads_magic = iph::div_magic(static_cast<unsigned long long>(H));
+    prm.nwhole = ip.nwhole;
+    prm.nitems = ip.nitems;
     prm.out_rows = out_layout == IP_LAYOUT_ROWS ? 1 : 0;
-    const dim3 grid1(ntiles, H, B + sp.extra);
-    ipk::relpos_mhsa_fused_kernel<<<grid1, ipk::NTHREADS, smem, st>>>(tm_k, tm_v, tm_p, prm);
+    ipk::relpos_mhsa_fused_kernel<<<ip.grid, ipk::NTHREADS, smem, st>>>(tm_q, tm_k, tm_v, tm_p,
+                                                                         prm);
     if (cudaGetLastError() != cudaSuccess) return IP_ERR_CUDA;
     return IP_OK;
 }
@@ -250,7 +249,7 @@ int ip_relpos_mhsa_status(const void *workspace, ip_stream_t stream) {
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
     if (cudaMemcpyAsync(&word, workspace, sizeof(int), cudaMemcpyDeviceToHost, st) != cudaSuccess)
         return IP_ERR_CUDA;
-    if (cudaMemsetAsync(const_cast<void *>(workspace), 0, sizeof(int), st) != cudaSuccess)
+    if (cudaMemsetAsync(const_cast<void *>(workspace), 0, ws_bytes(), st) != cudaSuccess)
         return IP_ERR_CUDA;
     if (cudaStreamSynchronize(st) != cudaSuccess) return IP_ERR_CUDA;
     if (word & 15) return IP_ERR_TIMEOUT;   // a bounded barrier wait ran out

@@ -8,13 +8,17 @@
 // runs on the tensor pipe), fed from shared-memory tiles that the tensor
 // memory accelerator (TMA) stages with the 128-byte swizzle.
 //
-// One CTA owns 64 query rows of one (b, h): four consumer warps of 16 rows
-// and two producer warps.  The first issues the TMA loads; for the score
-// pass both compute the bias vectors K u and P v of each staged chunk (the
-// exact rank-1 split of (Q + 1u^T)K^T and (Q + 1v^T)P^T, since Q + u does not
-// fit an int8 operand).  The attn.V pass reads the V tile as TMA stages it:
-// transposed ldmatrix loads and byte selects build the MMA operand.
-// The consumers, per CTA:
+// The CTAs are persistent (one per resident slot) and take work items in
+// turn: a whole 64-row tile of one (b, h), or, for the tail of the work, a
+// 32-row half of one.  Four consumer warps of 16 rows and two producer
+// warps: the copy warp issues the TMA loads through a two-stage ring that
+// runs on across items (the next item's first chunks are in flight while
+// the current one finishes), and the bias warp computes the bias vectors
+// K u and P v of each staged score-pass chunk (the exact rank-1 split of
+// (Q + 1u^T)K^T and (Q + 1v^T)P^T, since Q + u does not fit an int8
+// operand).  The attn.V pass reads the V tile as TMA stages it: transposed
+// ldmatrix loads and byte selects build the MMA operand.
+// The consumers, per item:
 //   pass 1  for each chunk of 64 keys: the content MMAs Q K^T, the MMAs of
 //           the position band Q P_band^T for the next chunk (issued before
 //           this chunk's epilogue so that the tensor pipe stays busy; the 16
@@ -38,7 +42,7 @@ namespace ipk {
 constexpr int DH = 128;
 constexpr int MROWS = 64;                 // query rows per CTA
 constexpr int NCWARPS = 4;                // consumer warps, 16 rows each
-constexpr int NPWARPS = 2;                // producer warps: TMA + bias vectors, bias vectors
+constexpr int NPWARPS = 2;                // producer warps: the copy warp and the bias warp
 constexpr int NTHREADS = (NCWARPS + NPWARPS) * 32;
 constexpr int NK = 64;                    // keys per chunk
 constexpr int NSTAGE = 2;
@@ -53,22 +57,24 @@ constexpr int CARRY_TILES = BAND_TILES - NK / 8;   // band tiles shared by conse
 constexpr int REMAP_STRIDE = 88;          // int32 words per band row in the remap buffer
 constexpr int REMAP_BYTES = 16 * REMAP_STRIDE * 4;
 constexpr int LUT_ENTRIES = 256;
-constexpr int LUT_COPIES = 8;             // one per MMA row group
+constexpr int LUT_COPIES = 4;             // row groups g and g + 4 share one
 constexpr int CHUNK_SCORE_BYTES = 16 * NK;   // one warp's int8 scores of one chunk
+constexpr int Q_TILE_BYTES = MROWS * DH;  // the Q rows of the current item
 
 static_assert(PV_OFF + BAND_ROWS * 4 <= STAGE_BYTES, "stage layout");
 static_assert(STAGE_BYTES % 1024 == 0, "the 128-byte swizzle needs 1024-byte aligned tiles");
 static_assert(CARRY_TILES == 2 && (BAND_TILES - CARRY_TILES) % 4 == 0, "band tiling");
 
 struct SmemLayout {
-    int stages, scores, remap, lut, bars, total;
+    int stages, qtile, scores, remap, lut, bars, total;
 };
 
 // Offsets from a 1024-byte aligned base.
 __host__ __device__ inline SmemLayout smem_layout(int nchunk_max) {
     SmemLayout L;
     L.stages = 0;
-    L.scores = NSTAGE * STAGE_BYTES;
+    L.qtile = NSTAGE * STAGE_BYTES;   // 1024-byte aligned (128-byte swizzle); Ring::qtile
+    L.scores = L.qtile + Q_TILE_BYTES;
     L.remap = L.scores + NCWARPS * nchunk_max * CHUNK_SCORE_BYTES;
     L.lut = L.remap + NCWARPS * REMAP_BYTES;
     L.bars = L.lut + LUT_ENTRIES * LUT_COPIES * 4;
@@ -77,7 +83,6 @@ __host__ __device__ inline SmemLayout smem_layout(int nchunk_max) {
 }
 
 struct FusedParams {
-    const int8_t *q;
     const int8_t *u;          // [H][DH]
     const int8_t *vb;         // [H][DH]
     int8_t *out;
@@ -90,11 +95,14 @@ struct FusedParams {
     unsigned long long ln2_magic;   // udiv_magic constant of q_ln2
     long long timeout_cycles; // bound of every barrier wait
     int stall_injection;      // test hook: consumers first wait on a barrier nobody arrives on
-    // Tail split: the last nsplit tiles of the (b, h, tile) order, from
-    // tile split_tile0 of (split_b0, split_h0) on, are done as two halves of
-    // 32 rows each by the CTAs of the grid slices z >= B (dispatched last).
-    int nsplit, split_b0, split_h0, split_tile0;
-    long long first_split;    // linear index of the first split tile
+    // Work items, claimed in order by the persistent CTAs: items [0, nwhole)
+    // are whole 64-row tiles in (b, h, tile) order, items [nwhole, nitems)
+    // the two 32-row halves of the tiles from nwhole on.
+    unsigned int *sched;      // workspace words: [0] next item, [16] CTAs done claiming
+    int ntiles;                        // 64-row tiles per (b, h)
+    unsigned long long tiles_magic;    // udiv_magic constant of ntiles
+    unsigned long long heads_magic;    // udiv_magic constant of H
+    uint32_t nwhole, nitems;           // nitems < 2^31
     int out_rows;             // output [B][T][H][DH] instead of [B][H][T][DH]
 };
 
@@ -104,6 +112,7 @@ __device__ __forceinline__ size_t out_offset(const FusedParams &p, int b, int h,
                       : ((static_cast<size_t>(b) * p.H + h) * p.T + row) * DH;
 }
 
+constexpr uint32_t NO_ITEM = 0xffffffffu;
 constexpr int ERR_TIMEOUT_FULL = 1;
 constexpr int ERR_TIMEOUT_EMPTY = 2;
 constexpr int ERR_TIMEOUT_READY = 4;
@@ -485,408 +494,121 @@ __device__ __forceinline__ void bias_row(uint32_t tile, uint32_t dst, const uint
     sts32(dst + row * 4, static_cast<uint32_t>(acc));
 }
 
-// The two producer warps share the bias vectors of a staged chunk (192 dot
-// products): warp 0 takes K u of keys l, l + 32 and P v of band row l, warp
-// 1 P v of band rows 32 + l, 64 + l, 96 + l.
-__device__ __forceinline__ void prep_bias(int pw, uint32_t ktile, uint32_t ptile, uint32_t ku,
-                                          uint32_t pv, const uint32_t (&uw)[32],
-                                          const uint32_t (&vw)[32], int lane) {
-    if (pw == 0) {
-        bias_row(ktile, ku, uw, lane);
-        bias_row(ktile, ku, uw, lane + 32);
-        bias_row(ptile, pv, vw, lane);
-    } else {
-        bias_row(ptile, pv, vw, lane + 32);
-        bias_row(ptile, pv, vw, lane + 64);
-        bias_row(ptile, pv, vw, lane + 96);
-    }
+// The bias warp's work on a staged score-pass chunk: K u of the 64 keys
+// (rows l, l + 32) and P v of the 128 band rows (l, l + 32, l + 64, l + 96).
+__device__ __forceinline__ void prep_bias(uint32_t ktile, uint32_t ptile, uint32_t ku, uint32_t pv,
+                                          const uint32_t (&uw)[32], const uint32_t (&vw)[32],
+                                          int lane) {
+    bias_row(ktile, ku, uw, lane);
+    bias_row(ktile, ku, uw, lane + 32);
+#pragma unroll
+    for (int r = 0; r < 4; ++r) bias_row(ptile, pv, vw, lane + 32 * r);
 }
 
-// ------------------------------------------------------------ fused kernel --
+// ------------------------------------------------------------- work items --
 
-__global__ void __launch_bounds__(NTHREADS, 2)
-    relpos_mhsa_fused_kernel(const __grid_constant__ CUtensorMap tm_k,
-                             const __grid_constant__ CUtensorMap tm_v,
-                             const __grid_constant__ CUtensorMap tm_p, const FusedParams prm) {
-    extern __shared__ uint8_t smem_raw[];
-    uint8_t *smem = reinterpret_cast<uint8_t *>(
-        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-    const SmemLayout L = smem_layout(prm.nchunk_max);
+// One work item: a whole 64-row tile of (b, h) (part < 0) or the 32-row half
+// `part` of one.  Items are decoded without a division instruction (exact
+// multiply-high by the constants of ntiles and H).
+struct Item {
+    int b, h, bh, i0, part, len, nchunks;
+    bool pad;   // every row of the tile (half) is padding
+};
 
-    // Grid (ntiles, H, B + extra): slices z < B hold one CTA per tile, the
-    // slices after them the halves of the split tiles.  No run-time
-    // division anywhere in the kernel.
-    const int T = prm.T;
-    const int ntiles = static_cast<int>(gridDim.x);
-    int tile = blockIdx.x;
-    int h = blockIdx.y;
-    int b = blockIdx.z;
-    int part = -1;                 // -1: whole tile; 0, 1: half of a split tile
-    if (b >= prm.B) {
-        const long long t = blockIdx.x + static_cast<long long>(ntiles) *
-                                             (blockIdx.y + static_cast<long long>(prm.H) * (b - prm.B));
-        if (t >= 2ll * prm.nsplit) return;
-        part = static_cast<int>(t & 1);
-        tile = prm.split_tile0 + static_cast<int>(t >> 1);
-        h = prm.split_h0;
-        b = prm.split_b0;
-        while (tile >= ntiles) {   // at most nsplit / ntiles + 1 steps
-            tile -= ntiles;
-            ++h;
-        }
-        while (h >= prm.H) {
-            h -= prm.H;
-            ++b;
-        }
-    } else if (prm.nsplit > 0) {
-        const long long lin = blockIdx.x + static_cast<long long>(ntiles) *
-                                               (blockIdx.y + static_cast<long long>(prm.H) * b);
-        if (lin >= prm.first_split) return;   // done by the two halves
+__device__ __forceinline__ Item decode_item(const FusedParams &p, uint32_t item) {
+    Item it;
+    uint32_t lin = item;
+    it.part = -1;
+    if (item >= p.nwhole) {
+        const uint32_t t = item - p.nwhole;
+        lin = p.nwhole + (t >> 1);
+        it.part = static_cast<int>(t & 1u);
     }
-    const int bh = b * prm.H + h;
-    const int i0 = tile * MROWS;
-    int len = T;
-    if (prm.lengths != nullptr) {
-        len = prm.lengths[b];
-        len = len < 0 ? 0 : (len > T ? T : len);
+    const uint32_t bh = udiv_magic(lin, p.tiles_magic);
+    const int tile = static_cast<int>(lin - bh * static_cast<uint32_t>(p.ntiles));
+    it.b = static_cast<int>(udiv_magic(bh, p.heads_magic));
+    it.h = static_cast<int>(bh) - it.b * p.H;
+    it.bh = static_cast<int>(bh);
+    it.i0 = tile * MROWS;
+    int len = p.T;
+    if (p.lengths != nullptr) {
+        len = p.lengths[it.b];
+        len = len < 0 ? 0 : (len > p.T ? p.T : len);
     }
-    const int warp = threadIdx.x >> 5;
-    const int lane = threadIdx.x & 31;
+    it.len = len;
+    it.nchunks = (len + NK - 1) / NK;
+    it.pad = (it.part < 0 ? it.i0 : it.i0 + 32 * it.part) >= len;
+    return it;
+}
 
-    {
-        const int r0 = part < 0 ? i0 : i0 + 32 * part;
-        const int nrows = part < 0 ? MROWS : 32;
-        if (r0 >= len) {
-            // Every row of this tile (half) is padding: write zeros.
-            const int rows = (T - r0) < nrows ? (T - r0) : nrows;
-            for (int c = threadIdx.x; c < rows * (DH / 16); c += NTHREADS)
-                *reinterpret_cast<int4 *>(prm.out + out_offset(prm, b, h, r0 + (c >> 3)) +
-                                          16 * (c & 7)) = make_int4(0, 0, 0, 0);
-            return;
-        }
-    }
-    const int nchunks = (len + NK - 1) / NK;
-    const int total = 2 * nchunks;   // uses of the stage ring: pass-1 chunks, then pass-3 chunks
-
-    const uint32_t lut = smem_u32(smem + L.lut);
-    const uint32_t bar_base = smem_u32(smem + L.bars);
-    auto full_bar = [&](int s) { return bar_base + 8u * s; };
-    auto ready_bar = [&](int s) { return bar_base + 8u * (NSTAGE + s); };
-    auto empty_bar = [&](int s) { return bar_base + 8u * (2 * NSTAGE + s); };
-    const uint32_t never_bar = bar_base + 8u * (3 * NSTAGE);   // test hook only
-    auto pair_bar = [&](int strip2) { return bar_base + 8u * (3 * NSTAGE + 1 + strip2); };
-
-    const uint32_t stage_base = smem_u32(smem + L.stages);
-    auto stage_addr = [&](int s) { return stage_base + s * STAGE_BYTES; };
-    // Use `it` of the stage ring (stage it & 1, phase it >> 1): TMA lands
-    // (full), the producers prepare it (ready), the consumers release it
-    // (empty), and the stage is refilled with use it + 2.
-    auto issue = [&](int it) {
-        const int s = it & 1;
-        const uint32_t dst = stage_addr(s);
-        if (it < nchunks) {
-            const int j0 = it * NK;
-            mbar_expect_tx(full_bar(s), K_TILE_BYTES + P_TILE_BYTES);
-            tma_load_3d(dst, &tm_k, 0, j0, bh, full_bar(s));
-            tma_load_3d(dst + K_TILE_BYTES, &tm_p, 0, j0 - i0 - (MROWS - 1) + T - 1, h,
-                        full_bar(s));
-        } else {
-            const int j0 = (it - nchunks) * NK;
-            mbar_expect_tx(full_bar(s), K_TILE_BYTES);
-            tma_load_3d(dst, &tm_v, 0, j0, bh, full_bar(s));
-        }
-    };
-
-    // The thread that issues the copies initialises the barriers and sends
-    // the first two chunks off at once; the exponential table and the Q
-    // fragments are built while they travel.
-    if (threadIdx.x == NCWARPS * 32) {
-        for (int s = 0; s < NSTAGE; ++s) {
-            mbar_init(full_bar(s), 1);
-            mbar_init(ready_bar(s), NPWARPS);
-            mbar_init(empty_bar(s), NCWARPS);
-        }
-        mbar_init(never_bar, 1);
-        mbar_init(pair_bar(0), 2);
-        mbar_init(pair_bar(1), 2);
-        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-        issue(0);
-        if (total > 1) issue(1);
-    }
-
-    // Consumers: row strip of 16 rows, one per warp in a whole tile; in a
-    // split tile strips 2 part, 2 part + 1, each shared by warps 2s', 2s' + 1.
-    // Q fragments (A operand) for the four 32-wide k steps, rows >= T zero.
-    const int g = lane >> 2;       // row group of the MMA fragments
-    const int t4 = lane & 3;       // thread in group
-    const int strip = part < 0 ? warp : 2 * part + (warp >> 1);
-    const int wrow0 = i0 + strip * 16;
-    uint32_t qa[4][4];
-    if (warp < NCWARPS) {
-        const int8_t *qbase = prm.q + static_cast<size_t>(bh) * T * DH;
-        const int r0 = wrow0 + g, r1 = wrow0 + g + 8;
+// Q fragments (A operand) of 16-row strip `strip` of the staged Q tile for
+// the four 32-wide k steps (ldmatrix: matrices rows 0-7 / 8-15 x the two
+// 16-byte halves of k step ks, the m16n8k32 A layout); rows >= T were
+// filled with zeros by the copy.
+__device__ __forceinline__ void load_q(uint32_t qtile, int strip, int lane, uint32_t (&qa)[4][4]) {
+    const int m = lane >> 3;
+    const int row = strip * 16 + ((m & 1) << 3) + (lane & 7);
 #pragma unroll
-        for (int ks = 0; ks < 4; ++ks) {
-            const int c0 = ks * 32 + 4 * t4;
-            qa[ks][0] = r0 < T ? *reinterpret_cast<const uint32_t *>(qbase + static_cast<size_t>(r0) * DH + c0) : 0u;
-            qa[ks][1] = r1 < T ? *reinterpret_cast<const uint32_t *>(qbase + static_cast<size_t>(r1) * DH + c0) : 0u;
-            qa[ks][2] = r0 < T ? *reinterpret_cast<const uint32_t *>(qbase + static_cast<size_t>(r0) * DH + c0 + 16) : 0u;
-            qa[ks][3] = r1 < T ? *reinterpret_cast<const uint32_t *>(qbase + static_cast<size_t>(r1) * DH + c0 + 16) : 0u;
-        }
-    }
-    for (int d = threadIdx.x; d < LUT_ENTRIES; d += NTHREADS) {
-        const uint32_t e = iexp_neg(d, prm.q_ln2, prm.q_b, prm.q_c, prm.ln2_magic);
-#pragma unroll
-        for (int c = 0; c < LUT_COPIES; ++c) sts32(lut + (d * LUT_COPIES + c) * 4, e);
-    }
-    __syncthreads();
+    for (int ks = 0; ks < 4; ++ks)
+        ldsm_x4(qtile + swz(row, 2 * ks + (m >> 1)), qa[ks][0], qa[ks][1], qa[ks][2], qa[ks][3]);
+}
 
-    // ------------------------------------------------------------ producer
-    if (warp >= NCWARPS) {
-        const int pw = warp - NCWARPS;   // 0: TMA and its share of the biases; 1: its share
-        uint32_t uw[32], vw[32];
-        {
-            const uint4 *u4 = reinterpret_cast<const uint4 *>(prm.u + static_cast<size_t>(h) * DH);
-            const uint4 *v4 = reinterpret_cast<const uint4 *>(prm.vb + static_cast<size_t>(h) * DH);
-#pragma unroll
-            for (int c = 0; c < 8; ++c) {
-                const uint4 a = __ldg(u4 + c), bq = __ldg(v4 + c);
-                uw[4 * c] = a.x; uw[4 * c + 1] = a.y; uw[4 * c + 2] = a.z; uw[4 * c + 3] = a.w;
-                vw[4 * c] = bq.x; vw[4 * c + 1] = bq.y; vw[4 * c + 2] = bq.z; vw[4 * c + 3] = bq.w;
-            }
-        }
-        if (pw == 1) {
-            // second producer warp: its share of the bias vectors of each
-            // staged score-pass chunk
-            for (int it = 0; it < nchunks; ++it) {
-                const int s = it & 1;
-                if (!warp_wait(full_bar(s), (it >> 1) & 1, prm.timeout_cycles)) {
-                    if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_FULL);
-                    return;
-                }
-                prep_bias(1, stage_addr(s), stage_addr(s) + K_TILE_BYTES, stage_addr(s) + KU_OFF,
-                          stage_addr(s) + PV_OFF, uw, vw, lane);
-                release_stage(ready_bar(s), lane);
-            }
-            return;
-        }
-        int issued = total > 1 ? 2 : 1, landed = 0;   // chunks 0 and 1 left at the start
-        bool ok = true;
-        for (int it = 0; it < total; ++it) {
-            const int s = it & 1;
-            if (it < nchunks) {
-                // score pass: the bias vectors of the staged chunk
-                if (!warp_wait(full_bar(s), (it >> 1) & 1, prm.timeout_cycles)) {
-                    if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_FULL);
-                    ok = false;
-                    break;
-                }
-                landed = it + 1;
-                prep_bias(0, stage_addr(s), stage_addr(s) + K_TILE_BYTES, stage_addr(s) + KU_OFF,
-                          stage_addr(s) + PV_OFF, uw, vw, lane);
-                release_stage(ready_bar(s), lane);
-            }
-            // (attn.V pass: the consumers read the V tile as TMA left it)
-            if (it + 2 < total) {
-                if (!warp_wait(empty_bar(s), (it >> 1) & 1, prm.timeout_cycles)) {
-                    if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_EMPTY);
-                    ok = false;
-                    break;
-                }
-                landed = it + 1;   // released by the consumers, so it had landed
-                if (lane == 0) issue(it + 2);
-                issued = it + 3;
-            }
-        }
-        if (!ok) {
-            // Let the copies already issued land before the CTA exits
-            // (bounded by a fixed budget independent of the caller's).
-            for (int it = landed; it < issued; ++it)
-                mbar_wait(full_bar(it & 1), (it >> 1) & 1, DRAIN_CYCLES);
-        }
-        return;
-    }
+// Shared-memory stage ring: use u of the ring (all items of a CTA in order;
+// an item takes nchunks score-pass uses, then nchunks attn.V uses) sits in
+// stage u & 1 with barrier phase (u >> 1) & 1.  TMA lands (full), the bias
+// warp prepares a score-pass chunk or passes an attn.V chunk on (ready),
+// the consumers release it (empty), and the stage is refilled with use
+// u + 2.  Every barrier completes one phase per use of its stage and every
+// waiter waits on each phase in order, so a parity names one phase.
+struct Ring {
+    uint32_t stage_base, bar_base;   // the Q tile follows the stages
+    __device__ __forceinline__ uint32_t stage(int u) const { return stage_base + (u & 1) * STAGE_BYTES; }
+    __device__ __forceinline__ uint32_t full(int u) const { return bar_base + 8u * (u & 1); }
+    __device__ __forceinline__ uint32_t ready(int u) const { return bar_base + 8u * (NSTAGE + (u & 1)); }
+    __device__ __forceinline__ uint32_t empty(int u) const { return bar_base + 8u * (2 * NSTAGE + (u & 1)); }
+    __device__ __forceinline__ static uint32_t parity(int u) { return (static_cast<uint32_t>(u) >> 1) & 1u; }
+    // The Q tile of live item k: landed (qfull phase k), read by all
+    // consumer warps (qempty phase k); refilled with item k + 1 after that.
+    __device__ __forceinline__ uint32_t qtile() const { return stage_base + NSTAGE * STAGE_BYTES; }
+    __device__ __forceinline__ uint32_t qfull() const { return bar_base + 8u * (3 * NSTAGE + 3); }
+    __device__ __forceinline__ uint32_t qempty() const { return bar_base + 8u * (3 * NSTAGE + 4); }
+    // Item number of the CTA's live item k (written by the copy warp before
+    // it arrives on that item's barriers), or NO_ITEM after the last.
+    __device__ __forceinline__ uint32_t slot(int k) const { return bar_base + 96u + 4u * (k & 3); }
+};
 
-    // ------------------------------------------------------------ consumers
-    const uint32_t remap = smem_u32(smem + L.remap) + warp * REMAP_BYTES;
-    const uint32_t scores = smem_u32(smem + L.scores) + warp * (prm.nchunk_max * CHUNK_SCORE_BYTES);
+// ------------------------------------------------------ consumer: whole tile --
+// Passes 1-3 and the output of one whole 64-row tile by one consumer warp
+// (its 16-row strip), with ring uses u0 .. u0 + 2 nchunks - 1; the item's
+// Q tile has landed.  Returns false after a barrier wait ran out.
+__device__ __forceinline__ bool consume_whole(const FusedParams &prm, const Item &it, int u0,
+                                              const Ring &R, uint32_t remap, uint32_t scores,
+                                              uint32_t lut, int warp, int lane) {
+    const int T = prm.T, len = it.len, nchunks = it.nchunks;
+    const int g = lane >> 2, t4 = lane & 3;
+    const int wrow0 = it.i0 + warp * 16;
     const long long m_c = prm.m_c, m_p = prm.m_p;
     const long long half_s = 1ll << (prm.sh_s - 1);
     const int s_s = prm.sh_s - 31;
-    const int band_row0 = 48 - 16 * strip;     // this warp's first row in the staged band
+    const int band_row0 = 48 - 16 * warp;      // this warp's first row in the staged band
     int mx0 = -128, mx1 = -128;                // running maxima of rows g and g + 8
-    if (prm.stall_injection && !warp_wait(never_bar, 0, prm.timeout_cycles)) {
-        if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_INJECTED);
-        return;
-    }
-
-    if (part >= 0) {
-        // ---------------------------------------------- split tile (tail)
-        const int hk = warp & 1;                   // key half of every chunk
-        const int nt0 = 4 * hk;
-        const uint32_t pair = pair_bar(warp >> 1);
-        const uint32_t xown = remap;
-        const uint32_t xpart = smem_u32(smem + L.remap) + (warp ^ 1) * REMAP_BYTES;
-        const uint32_t lut_g = lut + 4 * g;
-
-        // pass 1: scores of this warp's key half of every chunk
-        for (int c = 0; c < nchunks; ++c) {
-            const int s = c & 1;
-            if (!warp_wait(ready_bar(s), (c >> 1) & 1, prm.timeout_cycles)) {
-                if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_READY);
-                return;
-            }
-            int hb[6][4], hc[4][4];
-            half_chunk_mma(hb, hc, qa, stage_addr(s) + K_TILE_BYTES + band_row0 * 128,
-                           stage_addr(s) + PV_OFF + band_row0 * 4, stage_addr(s),
-                           stage_addr(s) + KU_OFF, nt0, lane);
-            release_stage(empty_bar(s), lane);
-#pragma unroll
-            for (int i = 0; i < 6; ++i) {
-                sts64(remap + (g * REMAP_STRIDE + (nt0 + i) * 8 + 2 * t4) * 4, hb[i][0], hb[i][1]);
-                sts64(remap + ((g + 8) * REMAP_STRIDE + (nt0 + i) * 8 + 2 * t4) * 4, hb[i][2],
-                      hb[i][3]);
-            }
-            __syncwarp();
-            const int kvalid = len - c * NK;
-            uint32_t pk[4];
-            if (kvalid < NK) {
-#pragma unroll
-                for (int i = 0; i < 4; ++i)
-                    pk[i] = score_tile<true>(hc[i], nt0 + i, remap, lane, m_c, m_p, half_s, s_s,
-                                             kvalid, mx0, mx1);
-            } else {
-#pragma unroll
-                for (int i = 0; i < 4; ++i)
-                    pk[i] = score_tile<false>(hc[i], nt0 + i, remap, lane, m_c, m_p, half_s, s_s,
-                                              kvalid, mx0, mx1);
-            }
-            sts128(scores + c * CHUNK_SCORE_BYTES + hk * 512 + lane * 16, pk[0], pk[1], pk[2],
-                   pk[3]);
-        }
-        mx0 = max(mx0, __shfl_xor_sync(0xffffffffu, mx0, 1));
-        mx0 = max(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
-        mx1 = max(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
-        mx1 = max(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
-        __syncwarp();   // the remap reads of the last chunk are done
-        sts64(xown + XMAX_OFF + lane * 8, mx0, mx1);
-        __syncwarp();
-        if (lane == 0) mbar_arrive(pair);
-        if (!warp_wait(pair, 0, prm.timeout_cycles)) {
-            if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_READY);
-            return;
-        }
-        {
-            const int2 pm = lds64(xpart + XMAX_OFF + lane * 8);
-            mx0 = max(mx0, pm.x);
-            mx1 = max(mx1, pm.y);
-        }
-
-        // pass 2: exponential sums of the key half, then of the whole row
-        unsigned long long sum0 = 0, sum1 = 0;
-        for (int c = 0; c < nchunks; ++c) {
-            const int kvalid = len - c * NK;
-            const uint4 sv = lds128(scores + c * CHUNK_SCORE_BYTES + hk * 512 + lane * 16);
-            if (kvalid < NK)
-                exp_sums<true>(sv, lut_g, mx0, mx1, t4, 32 * hk, kvalid, sum0, sum1);
-            else
-                exp_sums<false>(sv, lut_g, mx0, mx1, t4, 32 * hk, kvalid, sum0, sum1);
-        }
-        sum0 += __shfl_xor_sync(0xffffffffu, sum0, 1);
-        sum0 += __shfl_xor_sync(0xffffffffu, sum0, 2);
-        sum1 += __shfl_xor_sync(0xffffffffu, sum1, 1);
-        sum1 += __shfl_xor_sync(0xffffffffu, sum1, 2);
-        sts64(xown + XSUM_OFF + lane * 16, static_cast<int>(sum0), static_cast<int>(sum0 >> 32));
-        sts64(xown + XSUM_OFF + lane * 16 + 8, static_cast<int>(sum1), static_cast<int>(sum1 >> 32));
-        __syncwarp();
-        if (lane == 0) mbar_arrive(pair);
-        if (!warp_wait(pair, 1, prm.timeout_cycles)) {
-            if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_READY);
-            return;
-        }
-        {
-            const int2 a = lds64(xpart + XSUM_OFF + lane * 16);
-            const int2 bq = lds64(xpart + XSUM_OFF + lane * 16 + 8);
-            sum0 += (static_cast<unsigned long long>(static_cast<uint32_t>(a.y)) << 32) |
-                    static_cast<uint32_t>(a.x);
-            sum1 += (static_cast<unsigned long long>(static_cast<uint32_t>(bq.y)) << 32) |
-                    static_cast<uint32_t>(bq.x);
-        }
-        const uint32_t f0 = div_2pow32(sum0);
-        const uint32_t f1 = div_2pow32(sum1);
-
-        // pass 3: probabilities of the key half x V (k step hk of every chunk)
-        int oacc[16][4];
-#pragma unroll
-        for (int nt = 0; nt < 16; ++nt) oacc[nt][0] = oacc[nt][1] = oacc[nt][2] = oacc[nt][3] = 0;
-        const int kvalid_last = len - (nchunks - 1) * NK;
-        for (int c = 0; c < nchunks; ++c) {
-            const uint4 sv = lds128(scores + c * CHUNK_SCORE_BYTES + hk * 512 + lane * 16);
-            uint32_t pw[4] = {prob_word(sv.x, lut_g, mx0, mx1, f0, f1),
-                              prob_word(sv.y, lut_g, mx0, mx1, f0, f1),
-                              prob_word(sv.z, lut_g, mx0, mx1, f0, f1),
-                              prob_word(sv.w, lut_g, mx0, mx1, f0, f1)};
-            if (c == nchunks - 1 && kvalid_last < NK) {
-#pragma unroll
-                for (int q = 0; q < 4; ++q) pw[q] &= key_mask(32 * hk, q, t4, kvalid_last);
-            }
-            uint32_t af[4];
-            prob_operand(pw, af);
-            const int it = nchunks + c;
-            const int s = it & 1;
-            if (!warp_wait(full_bar(s), (it >> 1) & 1, prm.timeout_cycles)) {
-                if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_FULL);
-                return;
-            }
-            const uint32_t vtile = stage_addr(s);
-#pragma unroll
-            for (int grp = 0; grp < 4; ++grp) {
-                uint32_t bv[2][4];
-#pragma unroll
-                for (int i = 0; i < 2; ++i)
-                    vfrag(vtile, hk, 2 * grp + i, lane, bv[i][0], bv[i][1], bv[i][2], bv[i][3]);
-#pragma unroll
-                for (int i = 0; i < 2; ++i) {
-                    mma_u8s8(oacc[4 * grp + 2 * i], af, bv[i][0], bv[i][1]);
-                    mma_u8s8(oacc[4 * grp + 2 * i + 1], af, bv[i][2], bv[i][3]);
-                }
-            }
-            release_stage(empty_bar(s), lane);
-        }
-
-        // the partner finishes the other half of the output columns
-        if (hk == 0) send_partial<0>(oacc, xown + XO_OFF, lane);
-        else send_partial<1>(oacc, xown + XO_OFF, lane);
-        __syncwarp();
-        if (lane == 0) mbar_arrive(pair);
-        if (!warp_wait(pair, 0, prm.timeout_cycles)) {
-            if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_READY);
-            return;
-        }
-        const long long m_o = prm.m_o;
-        const long long half_o = 1ll << (prm.sh_o - 1);
-        if (hk == 0)
-            finish_half<0>(oacc, xpart + XO_OFF, lane, wrow0, len, prm, b, h, m_o, half_o);
-        else
-            finish_half<1>(oacc, xpart + XO_OFF, lane, wrow0, len, prm, b, h, m_o, half_o);
-        return;
-    }
+    uint32_t qa[4][4];
+    load_q(R.qtile(), warp, lane, qa);
 
     // ---- pass 1: scores.  A warp that issues an integer MMA waits until the
     // tensor pipe accepts it, so the band MMAs of chunk c+1 are issued in
     // groups with the epilogue of chunk c between them: the epilogue runs
     // while the pipe works through the band.
     int bacc[BAND_TILES][4];
-    if (!warp_wait(ready_bar(0), 0, prm.timeout_cycles)) {
+    if (!warp_wait(R.ready(u0), Ring::parity(u0), prm.timeout_cycles)) {
         if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_READY);
-        return;
+        return false;
     }
-    band_mma(bacc, qa, stage_addr(0) + K_TILE_BYTES + band_row0 * 128,
-             stage_addr(0) + PV_OFF + band_row0 * 4, lane);
+    band_mma(bacc, qa, R.stage(u0) + K_TILE_BYTES + band_row0 * 128,
+             R.stage(u0) + PV_OFF + band_row0 * 4, lane);
     const int lm_row = lane & 7, lm_mat = lane >> 3;
     for (int c = 0; c < nchunks; ++c) {
-        const int s = c & 1;
+        const int u = u0 + c;
         __syncwarp();
 #pragma unroll
         for (int nt = 0; nt < BAND_TILES; ++nt) {
@@ -894,16 +616,16 @@ __global__ void __launch_bounds__(NTHREADS, 2)
             sts64(remap + ((g + 8) * REMAP_STRIDE + nt * 8 + 2 * t4) * 4, bacc[nt][2], bacc[nt][3]);
         }
         int cacc[8][4];
-        content_mma(cacc, qa, stage_addr(s), stage_addr(s) + KU_OFF, lane);
-        release_stage(empty_bar(s), lane);
+        content_mma(cacc, qa, R.stage(u), R.stage(u) + KU_OFF, lane);
+        release_stage(R.empty(u), lane);
         const uint32_t sdst = scores + c * CHUNK_SCORE_BYTES;
         if (c + 1 < nchunks) {
-            if (!warp_wait(ready_bar(s ^ 1), ((c + 1) >> 1) & 1, prm.timeout_cycles)) {
+            if (!warp_wait(R.ready(u + 1), Ring::parity(u + 1), prm.timeout_cycles)) {
                 if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_READY);
-                return;
+                return false;
             }
-            const uint32_t ptile = stage_addr(s ^ 1) + K_TILE_BYTES + band_row0 * 128;
-            const uint32_t pvs = stage_addr(s ^ 1) + PV_OFF + band_row0 * 4;
+            const uint32_t ptile = R.stage(u + 1) + K_TILE_BYTES + band_row0 * 128;
+            const uint32_t pvs = R.stage(u + 1) + PV_OFF + band_row0 * 4;
             // The band of chunk c + 1 starts NK positions after that of chunk
             // c: its first CARRY_TILES tiles are the last ones of chunk c
             // (the same rows of Q against the same rows of P), kept in
@@ -953,6 +675,8 @@ __global__ void __launch_bounds__(NTHREADS, 2)
         }
     }
 
+    release_stage(R.qempty(), lane);   // done with the Q tile
+
     // ---- row maxima across the quad
     mx0 = max(mx0, __shfl_xor_sync(0xffffffffu, mx0, 1));
     mx0 = max(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
@@ -960,7 +684,7 @@ __global__ void __launch_bounds__(NTHREADS, 2)
     mx1 = max(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
 
     // ---- pass 2: sums of the integer exponentials
-    const uint32_t lut_g = lut + 4 * g;
+    const uint32_t lut_g = lut + 4 * (g & (LUT_COPIES - 1));
     unsigned long long sum0 = 0, sum1 = 0;
     for (int c = 0; c < nchunks; ++c) {
         const int kvalid = len - c * NK;
@@ -1001,13 +725,12 @@ __global__ void __launch_bounds__(NTHREADS, 2)
         prob_operand(pw, af);
     }
     for (int c = 0; c < nchunks; ++c) {
-        const int it = nchunks + c;
-        const int s = it & 1;
-        if (!warp_wait(full_bar(s), (it >> 1) & 1, prm.timeout_cycles)) {
-            if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_FULL);
-            return;
+        const int u = u0 + nchunks + c;
+        if (!warp_wait(R.ready(u), Ring::parity(u), prm.timeout_cycles)) {
+            if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_READY);
+            return false;
         }
-        const uint32_t vtile = stage_addr(s);
+        const uint32_t vtile = R.stage(u);
 #pragma unroll
         for (int ks = 0; ks < 2; ++ks) {
             const int nxt = min(2 * c + ks + 1, nsteps - 1);
@@ -1034,20 +757,20 @@ __global__ void __launch_bounds__(NTHREADS, 2)
             }
             prob_operand(pw, af);
         }
-        release_stage(empty_bar(s), lane);
+        release_stage(R.empty(u), lane);
     }
 
-    // ---- output requantisation (Eq. 7): per row and d chunk c, four bytes
-    // d = 16c + 4t .. 16c + 4t + 3 (n-tiles 2c, 2c + 1, columns 2t, 2t + 1)
+    // ---- output requantisation (Eq. 7): per d chunk c and row, four bytes
+    // d = 16c + 4t .. 16c + 4t + 3 (n-tiles 2c, 2c + 1, columns 2t, 2t + 1).
+    // The d chunks go in the order their last MMAs were issued, so the
+    // first ones are requantised while the pipe finishes the others.
     const long long m_o = prm.m_o;
     const long long half_o = 1ll << (prm.sh_o - 1);
 #pragma unroll
-    for (int rr = 0; rr < 2; ++rr) {
-        const int row = wrow0 + g + 8 * rr;
-        if (row >= T) continue;
-        int8_t *dst = prm.out + out_offset(prm, b, h, row) + 4 * t4;
+    for (int c = 0; c < 8; ++c) {
 #pragma unroll
-        for (int c = 0; c < 8; ++c) {
+        for (int rr = 0; rr < 2; ++rr) {
+            const int row = wrow0 + g + 8 * rr;
             uint32_t w = 0;
 #pragma unroll
             for (int e = 0; e < 4; ++e) {
@@ -1055,8 +778,438 @@ __global__ void __launch_bounds__(NTHREADS, 2)
                 const int o = row < len ? clamp127(x >> prm.sh_o) : 0;
                 w |= (static_cast<uint32_t>(o) & 0xffu) << (8 * e);
             }
-            *reinterpret_cast<uint32_t *>(dst + 16 * c) = w;
+            if (row < T)
+                *reinterpret_cast<uint32_t *>(prm.out + out_offset(prm, it.b, it.h, row) + 4 * t4 +
+                                              16 * c) = w;
         }
+    }
+    return true;
+}
+
+// -------------------------------------------------------- consumer: half tile --
+// One 32-row half of a tile: the two warps of a 16-row strip take the key
+// halves [0, 32) and [32, 64) of every chunk and combine row maxima,
+// exponential sums and attn.V partial sums through their exchange areas
+// behind the strip pair's barrier (four phases per half: maxima, sums,
+// partials, and the partner done reading before the areas are reused).
+__device__ __forceinline__ bool consume_half(const FusedParams &prm, const Item &it, int u0,
+                                             const Ring &R, uint32_t remap,
+                                             uint32_t scores, uint32_t lut, uint32_t pair,
+                                             int warp, int lane) {
+    const int len = it.len, nchunks = it.nchunks;
+    const int g = lane >> 2, t4 = lane & 3;
+    const int strip = 2 * it.part + (warp >> 1);
+    const int wrow0 = it.i0 + strip * 16;
+    const long long m_c = prm.m_c, m_p = prm.m_p;
+    const long long half_s = 1ll << (prm.sh_s - 1);
+    const int s_s = prm.sh_s - 31;
+    const int band_row0 = 48 - 16 * strip;
+    int mx0 = -128, mx1 = -128;
+    const int hk = warp & 1;                   // key half of every chunk
+    const int nt0 = 4 * hk;
+    const uint32_t xown = remap;
+    const uint32_t xpart = hk ? remap - REMAP_BYTES : remap + REMAP_BYTES;   // warp ^ 1
+    const uint32_t lut_g = lut + 4 * (g & (LUT_COPIES - 1));
+    uint32_t qa[4][4];
+    load_q(R.qtile(), strip, lane, qa);
+
+    // pass 1: scores of this warp's key half of every chunk
+    for (int c = 0; c < nchunks; ++c) {
+        const int u = u0 + c;
+        if (!warp_wait(R.ready(u), Ring::parity(u), prm.timeout_cycles)) {
+            if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_READY);
+            return false;
+        }
+        int hb[6][4], hc[4][4];
+        half_chunk_mma(hb, hc, qa, R.stage(u) + K_TILE_BYTES + band_row0 * 128,
+                       R.stage(u) + PV_OFF + band_row0 * 4, R.stage(u), R.stage(u) + KU_OFF, nt0,
+                       lane);
+        release_stage(R.empty(u), lane);
+        __syncwarp();   // the remap reads of the previous chunk are done
+#pragma unroll
+        for (int i = 0; i < 6; ++i) {
+            sts64(remap + (g * REMAP_STRIDE + (nt0 + i) * 8 + 2 * t4) * 4, hb[i][0], hb[i][1]);
+            sts64(remap + ((g + 8) * REMAP_STRIDE + (nt0 + i) * 8 + 2 * t4) * 4, hb[i][2],
+                  hb[i][3]);
+        }
+        __syncwarp();
+        const int kvalid = len - c * NK;
+        uint32_t pk[4];
+        if (kvalid < NK) {
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+                pk[i] = score_tile<true>(hc[i], nt0 + i, remap, lane, m_c, m_p, half_s, s_s,
+                                         kvalid, mx0, mx1);
+        } else {
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+                pk[i] = score_tile<false>(hc[i], nt0 + i, remap, lane, m_c, m_p, half_s, s_s,
+                                          kvalid, mx0, mx1);
+        }
+        sts128(scores + c * CHUNK_SCORE_BYTES + hk * 512 + lane * 16, pk[0], pk[1], pk[2], pk[3]);
+    }
+    release_stage(R.qempty(), lane);   // done with the Q tile
+    mx0 = max(mx0, __shfl_xor_sync(0xffffffffu, mx0, 1));
+    mx0 = max(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
+    mx1 = max(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
+    mx1 = max(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
+    __syncwarp();   // the remap reads of the last chunk are done
+    sts64(xown + XMAX_OFF + lane * 8, mx0, mx1);
+    __syncwarp();
+    if (lane == 0) mbar_arrive(pair);
+    if (!warp_wait(pair, 0, prm.timeout_cycles)) {
+        if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_READY);
+        return false;
+    }
+    {
+        const int2 pm = lds64(xpart + XMAX_OFF + lane * 8);
+        mx0 = max(mx0, pm.x);
+        mx1 = max(mx1, pm.y);
+    }
+
+    // pass 2: exponential sums of the key half, then of the whole row
+    unsigned long long sum0 = 0, sum1 = 0;
+    for (int c = 0; c < nchunks; ++c) {
+        const int kvalid = len - c * NK;
+        const uint4 sv = lds128(scores + c * CHUNK_SCORE_BYTES + hk * 512 + lane * 16);
+        if (kvalid < NK)
+            exp_sums<true>(sv, lut_g, mx0, mx1, t4, 32 * hk, kvalid, sum0, sum1);
+        else
+            exp_sums<false>(sv, lut_g, mx0, mx1, t4, 32 * hk, kvalid, sum0, sum1);
+    }
+    sum0 += __shfl_xor_sync(0xffffffffu, sum0, 1);
+    sum0 += __shfl_xor_sync(0xffffffffu, sum0, 2);
+    sum1 += __shfl_xor_sync(0xffffffffu, sum1, 1);
+    sum1 += __shfl_xor_sync(0xffffffffu, sum1, 2);
+    sts64(xown + XSUM_OFF + lane * 16, static_cast<int>(sum0), static_cast<int>(sum0 >> 32));
+    sts64(xown + XSUM_OFF + lane * 16 + 8, static_cast<int>(sum1), static_cast<int>(sum1 >> 32));
+    __syncwarp();
+    if (lane == 0) mbar_arrive(pair);
+    if (!warp_wait(pair, 1, prm.timeout_cycles)) {
+        if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_READY);
+        return false;
+    }
+    {
+        const int2 a = lds64(xpart + XSUM_OFF + lane * 16);
+        const int2 bq = lds64(xpart + XSUM_OFF + lane * 16 + 8);
+        sum0 += (static_cast<unsigned long long>(static_cast<uint32_t>(a.y)) << 32) |
+                static_cast<uint32_t>(a.x);
+        sum1 += (static_cast<unsigned long long>(static_cast<uint32_t>(bq.y)) << 32) |
+                static_cast<uint32_t>(bq.x);
+    }
+    const uint32_t f0 = div_2pow32(sum0);
+    const uint32_t f1 = div_2pow32(sum1);
+
+    // pass 3: probabilities of the key half x V (k step hk of every chunk)
+    int oacc[16][4];
+#pragma unroll
+    for (int nt = 0; nt < 16; ++nt) oacc[nt][0] = oacc[nt][1] = oacc[nt][2] = oacc[nt][3] = 0;
+    const int kvalid_last = len - (nchunks - 1) * NK;
+    for (int c = 0; c < nchunks; ++c) {
+        const uint4 sv = lds128(scores + c * CHUNK_SCORE_BYTES + hk * 512 + lane * 16);
+        uint32_t pw[4] = {prob_word(sv.x, lut_g, mx0, mx1, f0, f1),
+                          prob_word(sv.y, lut_g, mx0, mx1, f0, f1),
+                          prob_word(sv.z, lut_g, mx0, mx1, f0, f1),
+                          prob_word(sv.w, lut_g, mx0, mx1, f0, f1)};
+        if (c == nchunks - 1 && kvalid_last < NK) {
+#pragma unroll
+            for (int q = 0; q < 4; ++q) pw[q] &= key_mask(32 * hk, q, t4, kvalid_last);
+        }
+        uint32_t af[4];
+        prob_operand(pw, af);
+        const int u = u0 + nchunks + c;
+        if (!warp_wait(R.ready(u), Ring::parity(u), prm.timeout_cycles)) {
+            if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_READY);
+            return false;
+        }
+        const uint32_t vtile = R.stage(u);
+#pragma unroll
+        for (int grp = 0; grp < 4; ++grp) {
+            uint32_t bv[2][4];
+#pragma unroll
+            for (int i = 0; i < 2; ++i)
+                vfrag(vtile, hk, 2 * grp + i, lane, bv[i][0], bv[i][1], bv[i][2], bv[i][3]);
+#pragma unroll
+            for (int i = 0; i < 2; ++i) {
+                mma_u8s8(oacc[4 * grp + 2 * i], af, bv[i][0], bv[i][1]);
+                mma_u8s8(oacc[4 * grp + 2 * i + 1], af, bv[i][2], bv[i][3]);
+            }
+        }
+        release_stage(R.empty(u), lane);
+    }
+
+    // the partner finishes the other half of the output columns
+    if (hk == 0) send_partial<0>(oacc, xown + XO_OFF, lane);
+    else send_partial<1>(oacc, xown + XO_OFF, lane);
+    __syncwarp();
+    if (lane == 0) mbar_arrive(pair);
+    if (!warp_wait(pair, 0, prm.timeout_cycles)) {
+        if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_READY);
+        return false;
+    }
+    const long long m_o = prm.m_o;
+    const long long half_o = 1ll << (prm.sh_o - 1);
+    if (hk == 0)
+        finish_half<0>(oacc, xpart + XO_OFF, lane, wrow0, len, prm, it.b, it.h, m_o, half_o);
+    else
+        finish_half<1>(oacc, xpart + XO_OFF, lane, wrow0, len, prm, it.b, it.h, m_o, half_o);
+    // both warps are done reading the partner's area before either reuses its own
+    __syncwarp();
+    if (lane == 0) mbar_arrive(pair);
+    if (!warp_wait(pair, 1, prm.timeout_cycles)) {
+        if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_READY);
+        return false;
+    }
+    return true;
+}
+
+// ------------------------------------------------------------ fused kernel --
+// Persistent: one CTA per resident slot.  The copy warp claims the items in
+// order from a counter in the workspace, so the last items (the halves of
+// the tail) go to the CTAs that finish first; it writes the zeros of
+// padding items itself and publishes each live item to the other warps
+// through a shared-memory slot.  The stage ring runs on across items, so
+// the copies and bias vectors of the next item's first chunks overlap the
+// end of the current one.
+
+// Zero output rows of a padding item (every row is at or beyond its length).
+__device__ __forceinline__ void zero_rows(const FusedParams &p, const Item &it, int lane) {
+    const int r0 = it.part < 0 ? it.i0 : it.i0 + 32 * it.part;
+    const int nrows = it.part < 0 ? MROWS : 32;
+    const int rows = (p.T - r0) < nrows ? (p.T - r0) : nrows;
+    for (int c = lane; c < rows * (DH / 16); c += 32)
+        *reinterpret_cast<int4 *>(p.out + out_offset(p, it.b, it.h, r0 + (c >> 3)) + 16 * (c & 7)) =
+            make_int4(0, 0, 0, 0);
+}
+
+__global__ void __launch_bounds__(NTHREADS, 2)
+    relpos_mhsa_fused_kernel(const __grid_constant__ CUtensorMap tm_q,
+                             const __grid_constant__ CUtensorMap tm_k,
+                             const __grid_constant__ CUtensorMap tm_v,
+                             const __grid_constant__ CUtensorMap tm_p, const FusedParams prm) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+    const SmemLayout L = smem_layout(prm.nchunk_max);
+    const int T = prm.T;
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+
+    const uint32_t lut = smem_u32(smem + L.lut);
+    Ring R;
+    R.stage_base = smem_u32(smem + L.stages);
+    R.bar_base = smem_u32(smem + L.bars);
+    const uint32_t never_bar = R.bar_base + 8u * (3 * NSTAGE);   // test hook only
+    auto pair_bar = [&](int strip2) { return R.bar_base + 8u * (3 * NSTAGE + 1 + strip2); };
+
+    // Copy of ring use `pos` of item `it` (pos < nchunks: K chunk and the
+    // P band of the tile's rows; else V chunk pos - nchunks) into stage s.
+    auto issue = [&](const Item &it, int pos, int u) {
+        const uint32_t dst = R.stage(u);
+        const uint32_t full = R.full(u);
+        if (pos < it.nchunks) {
+            const int j0 = pos * NK;
+            mbar_expect_tx(full, K_TILE_BYTES + P_TILE_BYTES);
+            tma_load_3d(dst, &tm_k, 0, j0, it.bh, full);
+            tma_load_3d(dst + K_TILE_BYTES, &tm_p, 0, j0 - it.i0 - (MROWS - 1) + T - 1, it.h, full);
+        } else {
+            const int j0 = (pos - it.nchunks) * NK;
+            mbar_expect_tx(full, K_TILE_BYTES);
+            tma_load_3d(dst, &tm_v, 0, j0, it.bh, full);
+        }
+    };
+
+    // Copy warp: the item being issued, its next ring use, and the item
+    // claims.  claim() takes items from the counter until a live one (the
+    // padding ones get their zeros here); false once the work is gone.
+    Item iss{};
+    int iss_pos = 0, issued = 0;
+    int kq = 0;   // live items published (slots written, Q tiles sent)
+    auto claim = [&](uint32_t &item) -> bool {
+        for (;;) {
+            uint32_t x = 0;
+            if (lane == 0) x = atomicAdd(prm.sched, 1u);
+            item = __shfl_sync(0xffffffffu, x, 0);
+            if (item >= prm.nitems) return false;
+            iss = decode_item(prm, item);
+            if (!iss.pad) return true;
+            zero_rows(prm, iss, lane);
+        }
+    };
+    // Publishes the claimed item as live item kq: its slot, then its Q tile
+    // (the arrive on qfull releases the slot write).
+    auto publish = [&](uint32_t item) {
+        if (lane == 0) {
+            sts32(R.slot(kq), item);
+            mbar_expect_tx(R.qfull(), Q_TILE_BYTES);
+            tma_load_3d(R.qtile(), &tm_q, 0, iss.i0, iss.bh, R.qfull());
+        }
+        ++kq;
+        iss_pos = 0;
+    };
+    // No more work: the slot of live item kq says so, and the barriers the
+    // consumers (qfull) and the bias warp (full of ring use u) wait on next
+    // complete without a copy.  The counters are reset by the last CTA.
+    auto finish = [&](int u) {
+        if (lane == 0) {
+            sts32(R.slot(kq), NO_ITEM);
+            mbar_arrive(R.qfull());
+            mbar_arrive(R.full(u));
+        }
+    };
+    auto done_claiming = [&]() {
+        if (lane == 0 && atomicAdd(prm.sched + 16, 1u) == gridDim.x - 1) {
+            atomicExch(prm.sched, 0u);
+            atomicExch(prm.sched + 16, 0u);
+        }
+    };
+
+    // The copy warp initialises the barriers, claims its first item and
+    // sends its first two uses off at once; the exponential table is built
+    // while they travel.
+    bool live0 = false;
+    if (warp == NCWARPS) {
+        if (lane == 0) {
+            for (int s = 0; s < NSTAGE; ++s) {
+                mbar_init(R.full(s), 1);
+                mbar_init(R.ready(s), 1);
+                mbar_init(R.empty(s), NCWARPS);
+            }
+            mbar_init(never_bar, 1);
+            mbar_init(pair_bar(0), 2);
+            mbar_init(pair_bar(1), 2);
+            mbar_init(R.qfull(), 1);
+            mbar_init(R.qempty(), NCWARPS);
+            asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        }
+        __syncwarp();
+        uint32_t item = 0;
+        live0 = claim(item);
+        if (live0) {
+            publish(item);
+            for (int u = 0; u < NSTAGE; ++u) {   // an item has at least two uses
+                if (lane == 0) issue(iss, iss_pos, u);
+                ++iss_pos;
+                ++issued;
+            }
+        } else {
+            finish(0);
+            done_claiming();
+        }
+    }
+    for (int d = threadIdx.x; d < LUT_ENTRIES; d += NTHREADS) {
+        const uint32_t e = iexp_neg(d, prm.q_ln2, prm.q_b, prm.q_c, prm.ln2_magic);
+#pragma unroll
+        for (int c = 0; c < LUT_COPIES; ++c) sts32(lut + (d * LUT_COPIES + c) * 4, e);
+    }
+    __syncthreads();
+
+    // ------------------------------------------------------------ producers
+    if (warp == NCWARPS) {
+        // copy warp: refills the stage of use u with use u + 2 once every
+        // consumer warp has released u
+        if (!live0) return;
+        int landed = 0;
+        bool ok = true;
+        for (int u = 0;; ++u) {
+            if (!warp_wait(R.empty(u), Ring::parity(u), prm.timeout_cycles)) {
+                if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_EMPTY);
+                ok = false;
+                break;
+            }
+            landed = u + 1;   // released by the consumers, so it had landed
+            if (iss_pos == 2 * iss.nchunks) {
+                // the next use starts a new item, whose Q tile replaces the
+                // previous one once every consumer warp is done with that
+                if (!warp_wait(R.qempty(), static_cast<uint32_t>(kq - 1) & 1u, prm.timeout_cycles)) {
+                    if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_EMPTY);
+                    ok = false;
+                    break;
+                }
+                uint32_t item = 0;
+                if (!claim(item)) {
+                    finish(u + 2);
+                    break;
+                }
+                publish(item);
+            }
+            if (lane == 0) issue(iss, iss_pos, u + 2);
+            ++iss_pos;
+            issued = u + 3;
+        }
+        done_claiming();
+        if (!ok) {
+            // Let the copies already issued land before the CTA exits
+            // (bounded by a fixed budget independent of the caller's).
+            for (int u = landed; u < issued; ++u)
+                mbar_wait(R.full(u), Ring::parity(u), DRAIN_CYCLES);
+            mbar_wait(R.qfull(), static_cast<uint32_t>(kq - 1) & 1u, DRAIN_CYCLES);
+        }
+        return;
+    }
+    if (warp == NCWARPS + 1) {
+        // bias warp: K u and P v of every staged score-pass chunk, off the
+        // consumers' path (a chunk lands one use ahead of its consumers).
+        // Every use is acknowledged on `ready` (an attn.V use with no work),
+        // so that each barrier's phases follow the ring uses.
+        uint32_t uw[32], vw[32];
+        int cur_h = -1;
+        int u = 0;
+        for (int kb = 0;; ++kb) {
+            if (!warp_wait(R.full(u), Ring::parity(u), prm.timeout_cycles)) {
+                if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_FULL);
+                return;
+            }
+            const uint32_t item = lds32(R.slot(kb));
+            if (item == NO_ITEM) return;
+            const Item it = decode_item(prm, item);
+            if (it.h != cur_h) {
+                cur_h = it.h;
+                const uint4 *u4 = reinterpret_cast<const uint4 *>(prm.u + static_cast<size_t>(cur_h) * DH);
+                const uint4 *v4 = reinterpret_cast<const uint4 *>(prm.vb + static_cast<size_t>(cur_h) * DH);
+#pragma unroll
+                for (int c = 0; c < 8; ++c) {
+                    const uint4 a = __ldg(u4 + c), bq = __ldg(v4 + c);
+                    uw[4 * c] = a.x; uw[4 * c + 1] = a.y; uw[4 * c + 2] = a.z; uw[4 * c + 3] = a.w;
+                    vw[4 * c] = bq.x; vw[4 * c + 1] = bq.y; vw[4 * c + 2] = bq.z; vw[4 * c + 3] = bq.w;
+                }
+            }
+            for (int pos = 0; pos < 2 * it.nchunks; ++pos, ++u) {
+                if (pos > 0 && !warp_wait(R.full(u), Ring::parity(u), prm.timeout_cycles)) {
+                    if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_FULL);
+                    return;
+                }
+                if (pos < it.nchunks)
+                    prep_bias(R.stage(u), R.stage(u) + K_TILE_BYTES, R.stage(u) + KU_OFF,
+                              R.stage(u) + PV_OFF, uw, vw, lane);
+                release_stage(R.ready(u), lane);
+            }
+        }
+    }
+
+    // ------------------------------------------------------------ consumers
+    const uint32_t remap = smem_u32(smem + L.remap) + warp * REMAP_BYTES;
+    const uint32_t scores = smem_u32(smem + L.scores) + warp * (prm.nchunk_max * CHUNK_SCORE_BYTES);
+    if (prm.stall_injection && !warp_wait(never_bar, 0, prm.timeout_cycles)) {
+        if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_INJECTED);
+        return;
+    }
+    int u0 = 0;
+    for (int k = 0;; ++k) {
+        if (!warp_wait(R.qfull(), static_cast<uint32_t>(k) & 1u, prm.timeout_cycles)) {
+            if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_FULL);
+            return;
+        }
+        const uint32_t item = lds32(R.slot(k));
+        if (item == NO_ITEM) return;
+        const Item it = decode_item(prm, item);
+        const bool ok = it.part < 0
+                            ? consume_whole(prm, it, u0, R, remap, scores, lut, warp, lane)
+                            : consume_half(prm, it, u0, R, remap, scores, lut,
+                                           pair_bar(warp >> 1), warp, lane);
+        if (!ok) return;
+        u0 += 2 * it.nchunks;
     }
 }
 

@@ -183,3 +183,22 @@ def test_async_host_calls_overlap_on_two_streams(ip, orc):
         assert ip.host_status(arenas[j], B, H, T, stream=streams[j]) == 0
     for (out, c), lay in zip(outs, lays):
         assert_same(out.numpy(), oracle_out(orc, lay, c))
+
+
+def test_work_counters_return_to_zero(ip, orc):
+    # The kernel's CTAs claim query tiles from counters in the workspace
+    # (bytes 64 and 128); the last CTA of every call sets them back to zero,
+    # so calls in a row on one workspace each see all the work.
+    lay = synth.layer(3, 2)
+    c = ip.layer_constants(lay.scales)
+    B, H, T, dh = lay.q.shape
+    ws = torch.zeros(ip.workspace_bytes(B, H, T, dh), dtype=torch.uint8, device="cuda")
+    want = oracle_out(orc, lay, c)
+    args = [_dev(a) for a in (lay.q, lay.k, lay.v, lay.p, lay.u, lay.vb)]
+    for _ in range(3):
+        out = ip.relpos_mhsa_i8(*args, c, workspace=ws)
+        torch.cuda.synchronize()
+        counters = ws[64:256].cpu().numpy()
+        assert not counters.any(), counters.nonzero()
+        assert_same(out.cpu().numpy(), want)
+    assert ip.status(ws) == 0
