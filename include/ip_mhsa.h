@@ -385,6 +385,13 @@ int ip_debug_set_stall_injection(int on);
  * it).  The outputs are the same bit for bit in every mode. */
 int ip_debug_set_split_mode(int mode);
 
+/* Test hook: nonzero makes the attention kernel add the exponentials of
+ * its softmax rows in 64-bit partial sums even where the host has shown
+ * that 32-bit partial sums cannot wrap (exp(0) x 16 ceil(T/64) < 2^32, the
+ * faster path); 0 restores the choice.  Both give the same sums, so the
+ * outputs are the same bit for bit. */
+int ip_debug_set_wide_sums(int on);
+
 /* Diagnostic: enqueues a throughput probe of the integer warp MMA
  * (mma.sync m16n8k32 s8 x s8 -> s32, eight independent accumulators per
  * warp, `iters` rounds) on `stream`; sink is a device int array of

@@ -30,7 +30,7 @@ EXPORTS = (
     "ip_debug_set_timeout_cycles", "ip_debug_set_stall_injection", "ip_dyadic_multiplier",
     "ip_dyadic_pair",
     "ip_isoftmax_params_from_scale", "ip_probe_int8_mma", "ip_relpos_mhsa_i8_noalloc",
-    "ip_debug_set_split_mode", "ip_linear_i8", "ip_linear_swish_i8", "ip_swish_params_from_scales",
+    "ip_debug_set_split_mode", "ip_debug_set_wide_sums", "ip_linear_i8", "ip_linear_swish_i8", "ip_swish_params_from_scales",
     "ip_layernorm_i8", "ip_layernorm_constants", "ip_relpos_mhsa_i8_ex", "ip_residual_i8",
     "ip_residual_params", "ip_linear_glu_i8", "ip_glu_params", "ip_dwconv_swish_i8",
     "ip_swish16_params_from_scales", "ip_relpos_mhsa_i8_host_async", "ip_relpos_mhsa_host_status",
@@ -110,6 +110,8 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
         lib.ip_debug_set_stall_injection.restype = I
         lib.ip_debug_set_split_mode.argtypes = [I]
         lib.ip_debug_set_split_mode.restype = I
+        lib.ip_debug_set_wide_sums.argtypes = [I]
+        lib.ip_debug_set_wide_sums.restype = I
         lib.ip_dyadic_multiplier.argtypes = [ctypes.c_double, i32p, i32p]
         lib.ip_dyadic_multiplier.restype = I
         lib.ip_dyadic_pair.argtypes = [ctypes.c_double, ctypes.c_double, i32p, i32p, i32p]
@@ -236,6 +238,12 @@ def set_split_mode(mode: int) -> None:
     """Test hook: -1 planned tail split (default), 0 never split, 1 split
     every 64-row tile into two key-split halves."""
     load().ip_debug_set_split_mode(int(mode))
+
+
+def set_wide_sums(on: bool) -> None:
+    """Test hook: always add the softmax exponentials in 64-bit partial sums
+    (False: 32-bit partial sums where they provably cannot wrap)."""
+    load().ip_debug_set_wide_sums(1 if on else 0)
 
 
 def _arr(vals, ctype):

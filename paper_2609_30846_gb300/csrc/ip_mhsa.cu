@@ -20,6 +20,7 @@ constexpr long long DEFAULT_TIMEOUT = 4000000000ll;   // ~2 s at 2 GHz
 long long g_timeout_cycles = DEFAULT_TIMEOUT;
 int g_stall_injection = 0;
 int g_split_mode = -1;   // -1 planned, 0 never, 1 every tile (test hook)
+int g_wide_sums = 0;     // 1: 64-bit exponential sums always (test hook)
 
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
@@ -226,6 +227,12 @@ int ip_relpos_mhsa_i8_ex(const int8_t *q, const int8_t *k, const int8_t *v, cons
     prm.q_b = sm->q_b;
     prm.q_c = sm->q_c;
     prm.ln2_magic = iph::div_magic(static_cast<unsigned long long>(sm->q_ln2));
+    // exp(0) = q_b^2 + q_c bounds every table entry; a thread adds 16 of
+    // them per row and chunk
+    const unsigned long long e0 =
+        static_cast<unsigned long long>(sm->q_b) * sm->q_b + static_cast<unsigned long long>(sm->q_c);
+    prm.sum32 =
+        !g_wide_sums && e0 * 16ull * static_cast<unsigned long long>(nchunk_max) < (1ull << 32) ? 1 : 0;
     prm.timeout_cycles = g_timeout_cycles;
     prm.stall_injection = g_stall_injection;
     const int slots = resident_ctas(smem);
@@ -501,6 +508,11 @@ int ip_debug_set_timeout_cycles(long long cycles) {
 
 int ip_debug_set_split_mode(int mode) {
     g_split_mode = mode < 0 ? -1 : (mode > 0 ? 1 : 0);
+    return IP_OK;
+}
+
+int ip_debug_set_wide_sums(int on) {
+    g_wide_sums = on ? 1 : 0;
     return IP_OK;
 }
 

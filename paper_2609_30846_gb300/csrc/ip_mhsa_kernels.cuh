@@ -95,6 +95,7 @@ struct FusedParams {
     unsigned long long ln2_magic;   // udiv_magic constant of q_ln2
     long long timeout_cycles; // bound of every barrier wait
     int stall_injection;      // test hook: consumers first wait on a barrier nobody arrives on
+    int sum32;                // exp(0) x 16 nchunk_max < 2^32: 32-bit partial sums in pass 2
     // Work items, claimed in order by the persistent CTAs: items [0, nwhole)
     // are whole 64-row tiles in (b, h, tile) order, items [nwhole, nitems)
     // the two 32-row halves of the tiles from nwhole on.
@@ -135,26 +136,30 @@ __device__ __forceinline__ void transpose4(uint32_t x0, uint32_t x1, uint32_t x2
     y3 = __byte_perm(t1, t3, 0x7632);
 }
 
-// Sign-extended byte I of w (prmt with the sign-replicate bit set in the
-// three upper selector nibbles).
-template <int I>
-__device__ __forceinline__ int sbyte(uint32_t w) {
-    constexpr uint32_t s = 8u | I;
-    constexpr uint32_t sel = (s << 12) | (s << 8) | (s << 4) | I;
-    uint32_t r;
-    asm("prmt.b32 %0, %1, 0, %2;" : "=r"(r) : "r"(w), "n"(sel));
-    return static_cast<int>(r);
-}
-
 // Packs the low bytes of four values: [a.b0, b.b0, c.b0, d.b0].
 __device__ __forceinline__ uint32_t pack4(uint32_t a, uint32_t b, uint32_t c, uint32_t d) {
     return __byte_perm(__byte_perm(a, b, 0x0040), __byte_perm(c, d, 0x0040), 0x5410);
 }
 
-// Address of exp table entry d (0 <= d <= 255 by construction: the row
-// maximum minus a score of the row; the mask keeps it inside the table).
-__device__ __forceinline__ uint32_t lut_addr(uint32_t lut_g, int d) {
-    return lut_g + (static_cast<uint32_t>(d) & 0xffu) * (LUT_COPIES * 4);
+// Table indices of the four scores of a packed word (rows g, g, g + 8,
+// g + 8): the row maximum minus the score, 0 .. 255 since the maximum is
+// at least every score of its row (masked keys, -128, included).  With
+// every byte offset by 128 no byte difference borrows from the next, so
+// one 32-bit subtraction gives all four.  mx4h: the maxima of the word's
+// rows, offset by 128, in the word's byte order.
+__device__ __forceinline__ uint32_t exp_index4(uint32_t w, uint32_t mx4h) {
+    return mx4h - (w ^ 0x80808080u);
+}
+
+__device__ __forceinline__ uint32_t max4h(int mx0, int mx1) {
+    const uint32_t a = static_cast<uint32_t>(mx0 + 128) & 0xffu;
+    const uint32_t b = static_cast<uint32_t>(mx1 + 128) & 0xffu;
+    return a | (a << 8) | (b << 16) | (b << 24);
+}
+
+// Address of the exp table entry of byte e of an index word.
+__device__ __forceinline__ uint32_t lut_at(uint32_t lut_g, uint32_t d4, int e) {
+    return lut_g + ((d4 >> (8 * e)) & 0xffu) * (LUT_COPIES * 4);
 }
 
 // B fragments of the attn.V MMA for keys 32 ks .. 32 ks + 31 of the staged
@@ -319,19 +324,18 @@ __device__ __forceinline__ void score_epilogue(const int (&cacc)[8][4], uint32_t
 }
 
 // Sum of the integer exponentials of one stored half chunk (16 scores per
-// thread: rows g and g+8, 8 keys each).
+// thread: rows g and g+8, 8 keys each), in 64 bits.
 template <bool MASK>
-__device__ __forceinline__ void exp_sums(uint4 sv, uint32_t lut_g, int mx0, int mx1, int t4,
+__device__ __forceinline__ void exp_sums(uint4 sv, uint32_t lut_g, uint32_t mx4h, int t4,
                                          int kbase, int kvalid, unsigned long long &s0,
                                          unsigned long long &s1) {
     const uint32_t wv[4] = {sv.x, sv.y, sv.z, sv.w};
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
-        const int sc[4] = {sbyte<0>(wv[q]), sbyte<1>(wv[q]), sbyte<2>(wv[q]), sbyte<3>(wv[q])};
+        const uint32_t d4 = exp_index4(wv[q], mx4h);
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
-            const int mx = e < 2 ? mx0 : mx1;
-            uint32_t ev = lds32(lut_addr(lut_g, mx - sc[e]));
+            uint32_t ev = lds32(lut_at(lut_g, d4, e));
             if (MASK && kbase + q * 8 + 2 * t4 + (e & 1) >= kvalid) ev = 0u;
             if (e < 2) s0 += ev;
             else s1 += ev;
@@ -339,17 +343,35 @@ __device__ __forceinline__ void exp_sums(uint4 sv, uint32_t lut_g, int mx0, int 
     }
 }
 
+// The same in four 32-bit partial sums (a[0], a[1]: row g; a[2], a[3]: row
+// g + 8), for calls whose exp(0) times the terms a thread adds per row
+// stays below 2^32 (the host checks it), so no partial sum wraps.
+template <bool MASK>
+__device__ __forceinline__ void exp_sums32(uint4 sv, uint32_t lut_g, uint32_t mx4h, int t4,
+                                           int kbase, int kvalid, uint32_t (&a)[4]) {
+    const uint32_t wv[4] = {sv.x, sv.y, sv.z, sv.w};
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        const uint32_t d4 = exp_index4(wv[q], mx4h);
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            uint32_t ev = lds32(lut_at(lut_g, d4, e));
+            if (MASK && kbase + q * 8 + 2 * t4 + (e & 1) >= kvalid) ev = 0u;
+            a[(e >> 1) * 2 + (q & 1)] += ev;
+        }
+    }
+}
+
 // Probabilities of one packed score word (rows g, g+8 x two keys) on the
 // grid 2^-8.  Masked keys (score -128) are zeroed by the caller.
-__device__ __forceinline__ uint32_t prob_word(uint32_t wv, uint32_t lut_g, int mx0, int mx1,
+__device__ __forceinline__ uint32_t prob_word(uint32_t wv, uint32_t lut_g, uint32_t mx4h,
                                               uint32_t f0, uint32_t f1) {
-    const int sc[4] = {sbyte<0>(wv), sbyte<1>(wv), sbyte<2>(wv), sbyte<3>(wv)};
+    const uint32_t d4 = exp_index4(wv, mx4h);
     uint32_t a[4];
 #pragma unroll
     for (int e = 0; e < 4; ++e) {
-        const int mx = e < 2 ? mx0 : mx1;
         const uint32_t f = e < 2 ? f0 : f1;
-        const uint32_t ev = lds32(lut_addr(lut_g, mx - sc[e]));
+        const uint32_t ev = lds32(lut_at(lut_g, d4, e));
         // min(floor(ev f / 2^24), 255) with ev f = hi 2^32 + lo: 255 when
         // hi > 0, else lo >> 24 (at most 255)
         a[e] = __umulhi(ev, f) != 0u ? 255u : (ev * f) >> 24;
@@ -685,16 +707,34 @@ __device__ __forceinline__ bool consume_whole(const FusedParams &prm, const Item
 
     // ---- pass 2: sums of the integer exponentials
     const uint32_t lut_g = lut + 4 * (g & (LUT_COPIES - 1));
+    const uint32_t mx4h = max4h(mx0, mx1);
     unsigned long long sum0 = 0, sum1 = 0;
-    for (int c = 0; c < nchunks; ++c) {
-        const int kvalid = len - c * NK;
+    if (prm.sum32) {
+        uint32_t a[4] = {0u, 0u, 0u, 0u};
+        for (int c = 0; c < nchunks; ++c) {
+            const int kvalid = len - c * NK;
 #pragma unroll
-        for (int hf = 0; hf < 2; ++hf) {
-            const uint4 sv = lds128(scores + c * CHUNK_SCORE_BYTES + hf * 512 + lane * 16);
-            if (kvalid < NK)
-                exp_sums<true>(sv, lut_g, mx0, mx1, t4, 32 * hf, kvalid, sum0, sum1);
-            else
-                exp_sums<false>(sv, lut_g, mx0, mx1, t4, 32 * hf, kvalid, sum0, sum1);
+            for (int hf = 0; hf < 2; ++hf) {
+                const uint4 sv = lds128(scores + c * CHUNK_SCORE_BYTES + hf * 512 + lane * 16);
+                if (kvalid < NK)
+                    exp_sums32<true>(sv, lut_g, mx4h, t4, 32 * hf, kvalid, a);
+                else
+                    exp_sums32<false>(sv, lut_g, mx4h, t4, 32 * hf, kvalid, a);
+            }
+        }
+        sum0 = static_cast<unsigned long long>(a[0]) + a[1];
+        sum1 = static_cast<unsigned long long>(a[2]) + a[3];
+    } else {
+        for (int c = 0; c < nchunks; ++c) {
+            const int kvalid = len - c * NK;
+#pragma unroll
+            for (int hf = 0; hf < 2; ++hf) {
+                const uint4 sv = lds128(scores + c * CHUNK_SCORE_BYTES + hf * 512 + lane * 16);
+                if (kvalid < NK)
+                    exp_sums<true>(sv, lut_g, mx4h, t4, 32 * hf, kvalid, sum0, sum1);
+                else
+                    exp_sums<false>(sv, lut_g, mx4h, t4, 32 * hf, kvalid, sum0, sum1);
+            }
         }
     }
     sum0 += __shfl_xor_sync(0xffffffffu, sum0, 1);
@@ -714,10 +754,10 @@ __device__ __forceinline__ bool consume_whole(const FusedParams &prm, const Item
     const int kvalid_last = len - (nchunks - 1) * NK;   // valid keys of the last chunk
     {
         const uint4 sv = lds128(scores + lane * 16);
-        uint32_t pw[4] = {prob_word(sv.x, lut_g, mx0, mx1, f0, f1),
-                          prob_word(sv.y, lut_g, mx0, mx1, f0, f1),
-                          prob_word(sv.z, lut_g, mx0, mx1, f0, f1),
-                          prob_word(sv.w, lut_g, mx0, mx1, f0, f1)};
+        uint32_t pw[4] = {prob_word(sv.x, lut_g, mx4h, f0, f1),
+                          prob_word(sv.y, lut_g, mx4h, f0, f1),
+                          prob_word(sv.z, lut_g, mx4h, f0, f1),
+                          prob_word(sv.w, lut_g, mx4h, f0, f1)};
         if (nchunks == 1 && kvalid_last < NK) {
 #pragma unroll
             for (int q = 0; q < 4; ++q) pw[q] &= key_mask(0, q, t4, kvalid_last);
@@ -748,7 +788,7 @@ __device__ __forceinline__ bool consume_whole(const FusedParams &prm, const Item
                     mma_u8s8(oacc[4 * grp + 2 * i], af, b[i][0], b[i][1]);
                     mma_u8s8(oacc[4 * grp + 2 * i + 1], af, b[i][2], b[i][3]);
                 }
-                pw[grp] = prob_word(wn[grp], lut_g, mx0, mx1, f0, f1);
+                pw[grp] = prob_word(wn[grp], lut_g, mx4h, f0, f1);
             }
             if ((nxt >> 1) == nchunks - 1 && kvalid_last < NK) {
                 const int kbase = (nxt & 1) * 32;
@@ -868,14 +908,15 @@ __device__ __forceinline__ bool consume_half(const FusedParams &prm, const Item 
     }
 
     // pass 2: exponential sums of the key half, then of the whole row
+    const uint32_t mx4h = max4h(mx0, mx1);
     unsigned long long sum0 = 0, sum1 = 0;
     for (int c = 0; c < nchunks; ++c) {
         const int kvalid = len - c * NK;
         const uint4 sv = lds128(scores + c * CHUNK_SCORE_BYTES + hk * 512 + lane * 16);
         if (kvalid < NK)
-            exp_sums<true>(sv, lut_g, mx0, mx1, t4, 32 * hk, kvalid, sum0, sum1);
+            exp_sums<true>(sv, lut_g, mx4h, t4, 32 * hk, kvalid, sum0, sum1);
         else
-            exp_sums<false>(sv, lut_g, mx0, mx1, t4, 32 * hk, kvalid, sum0, sum1);
+            exp_sums<false>(sv, lut_g, mx4h, t4, 32 * hk, kvalid, sum0, sum1);
     }
     sum0 += __shfl_xor_sync(0xffffffffu, sum0, 1);
     sum0 += __shfl_xor_sync(0xffffffffu, sum0, 2);
@@ -907,10 +948,10 @@ __device__ __forceinline__ bool consume_half(const FusedParams &prm, const Item 
     const int kvalid_last = len - (nchunks - 1) * NK;
     for (int c = 0; c < nchunks; ++c) {
         const uint4 sv = lds128(scores + c * CHUNK_SCORE_BYTES + hk * 512 + lane * 16);
-        uint32_t pw[4] = {prob_word(sv.x, lut_g, mx0, mx1, f0, f1),
-                          prob_word(sv.y, lut_g, mx0, mx1, f0, f1),
-                          prob_word(sv.z, lut_g, mx0, mx1, f0, f1),
-                          prob_word(sv.w, lut_g, mx0, mx1, f0, f1)};
+        uint32_t pw[4] = {prob_word(sv.x, lut_g, mx4h, f0, f1),
+                          prob_word(sv.y, lut_g, mx4h, f0, f1),
+                          prob_word(sv.z, lut_g, mx4h, f0, f1),
+                          prob_word(sv.w, lut_g, mx4h, f0, f1)};
         if (c == nchunks - 1 && kvalid_last < NK) {
 #pragma unroll
             for (int q = 0; q < 4; ++q) pw[q] &= key_mask(32 * hk, q, t4, kvalid_last);
