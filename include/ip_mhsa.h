@@ -385,11 +385,14 @@ int ip_debug_set_stall_injection(int on);
  * it).  The outputs are the same bit for bit in every mode. */
 int ip_debug_set_split_mode(int mode);
 
-/* Test hook: nonzero makes the attention kernel add the exponentials of
- * its softmax rows in 64-bit partial sums even where the host has shown
- * that 32-bit partial sums cannot wrap (exp(0) x 16 ceil(T/64) < 2^32, the
- * faster path); 0 restores the choice.  Both give the same sums, so the
- * outputs are the same bit for bit. */
+/* Test hook: nonzero makes the attention kernel take its general softmax
+ * arithmetic everywhere: 64-bit partial row sums even where the host has
+ * shown that 32-bit partial sums cannot wrap (exp(0) x 16 ceil(T/64) <
+ * 2^32), and the probability as min(floor(e f / 2^24), 255) from the full
+ * 64-bit product even where every row sum exceeds 2^8 (exp(0) > 2^8, so
+ * f < 2^24 and one multiply-high gives it); 0 restores the choice.  Both
+ * paths compute the same integers, so the outputs are the same bit for
+ * bit. */
 int ip_debug_set_wide_sums(int on);
 
 /* Diagnostic: enqueues a throughput probe of the integer warp MMA

@@ -241,8 +241,9 @@ def set_split_mode(mode: int) -> None:
 
 
 def set_wide_sums(on: bool) -> None:
-    """Test hook: always add the softmax exponentials in 64-bit partial sums
-    (False: 32-bit partial sums where they provably cannot wrap)."""
+    """Test hook: always take the general softmax arithmetic (64-bit partial
+    row sums, probabilities from the full 64-bit product); False: the fast
+    paths where the host has shown they give the same integers."""
     load().ip_debug_set_wide_sums(1 if on else 0)
 
 

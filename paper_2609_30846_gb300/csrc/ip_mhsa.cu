@@ -20,7 +20,7 @@ constexpr long long DEFAULT_TIMEOUT = 4000000000ll;   // ~2 s at 2 GHz
 long long g_timeout_cycles = DEFAULT_TIMEOUT;
 int g_stall_injection = 0;
 int g_split_mode = -1;   // -1 planned, 0 never, 1 every tile (test hook)
-int g_wide_sums = 0;     // 1: 64-bit exponential sums always (test hook)
+int g_wide_sums = 0;     // 1: general softmax arithmetic always (test hook)
 
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
@@ -233,6 +233,8 @@ int ip_relpos_mhsa_i8_ex(const int8_t *q, const int8_t *k, const int8_t *v, cons
         static_cast<unsigned long long>(sm->q_b) * sm->q_b + static_cast<unsigned long long>(sm->q_c);
     prm.sum32 =
         !g_wide_sums && e0 * 16ull * static_cast<unsigned long long>(nchunk_max) < (1ull << 32) ? 1 : 0;
+    // a row's sum includes exp(0) (its maximum's own term)
+    prm.f24 = !g_wide_sums && e0 > 256ull ? 1 : 0;
     prm.timeout_cycles = g_timeout_cycles;
     prm.stall_injection = g_stall_injection;
     const int slots = resident_ctas(smem);

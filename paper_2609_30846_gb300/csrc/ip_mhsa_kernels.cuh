@@ -96,6 +96,7 @@ struct FusedParams {
     long long timeout_cycles; // bound of every barrier wait
     int stall_injection;      // test hook: consumers first wait on a barrier nobody arrives on
     int sum32;                // exp(0) x 16 nchunk_max < 2^32: 32-bit partial sums in pass 2
+    int f24;                  // exp(0) > 2^8: every row sum exceeds 2^8, so f = 2^32 / sum < 2^24
     // Work items, claimed in order by the persistent CTAs: items [0, nwhole)
     // are whole 64-row tiles in (b, h, tile) order, items [nwhole, nitems)
     // the two 32-row halves of the tiles from nwhole on.
@@ -362,8 +363,17 @@ __device__ __forceinline__ void exp_sums32(uint4 sv, uint32_t lut_g, uint32_t mx
     }
 }
 
+template <bool B> struct BoolTag {
+    static constexpr bool value = B;
+};
+
 // Probabilities of one packed score word (rows g, g+8 x two keys) on the
-// grid 2^-8.  Masked keys (score -128) are zeroed by the caller.
+// grid 2^-8: min(floor(ev f / 2^24), 255).  Masked keys (score -128) are
+// zeroed by the caller.  F24: every row sum exceeds 2^8, so f < 2^24 and
+// the callers pass f0, f1 times 2^8: the floor is then the high word of
+// ev (f 2^8).  Otherwise, with ev f = hi 2^32 + lo, it is 255 when hi > 0,
+// else lo >> 24 (at most 255).
+template <bool F24>
 __device__ __forceinline__ uint32_t prob_word(uint32_t wv, uint32_t lut_g, uint32_t mx4h,
                                               uint32_t f0, uint32_t f1) {
     const uint32_t d4 = exp_index4(wv, mx4h);
@@ -372,9 +382,10 @@ __device__ __forceinline__ uint32_t prob_word(uint32_t wv, uint32_t lut_g, uint3
     for (int e = 0; e < 4; ++e) {
         const uint32_t f = e < 2 ? f0 : f1;
         const uint32_t ev = lds32(lut_at(lut_g, d4, e));
-        // min(floor(ev f / 2^24), 255) with ev f = hi 2^32 + lo: 255 when
-        // hi > 0, else lo >> 24 (at most 255)
-        a[e] = __umulhi(ev, f) != 0u ? 255u : (ev * f) >> 24;
+        if (F24)
+            a[e] = min(__umulhi(ev, f), 255u);
+        else
+            a[e] = __umulhi(ev, f) != 0u ? 255u : (ev * f) >> 24;
     }
     return pack4(a[0], a[1], a[2], a[3]);
 }
@@ -749,56 +760,64 @@ __device__ __forceinline__ bool consume_whole(const FusedParams &prm, const Item
     int oacc[16][4];
 #pragma unroll
     for (int nt = 0; nt < 16; ++nt) oacc[nt][0] = oacc[nt][1] = oacc[nt][2] = oacc[nt][3] = 0;
-    const int nsteps = 2 * nchunks;
-    uint32_t af[4];
-    const int kvalid_last = len - (nchunks - 1) * NK;   // valid keys of the last chunk
-    {
-        const uint4 sv = lds128(scores + lane * 16);
-        uint32_t pw[4] = {prob_word(sv.x, lut_g, mx4h, f0, f1),
-                          prob_word(sv.y, lut_g, mx4h, f0, f1),
-                          prob_word(sv.z, lut_g, mx4h, f0, f1),
-                          prob_word(sv.w, lut_g, mx4h, f0, f1)};
-        if (nchunks == 1 && kvalid_last < NK) {
+    auto pass3 = [&](auto f24_tag, uint32_t fa, uint32_t fb) -> bool {
+        constexpr bool F24 = decltype(f24_tag)::value;
+        const int nsteps = 2 * nchunks;
+        uint32_t af[4];
+        const int kvalid_last = len - (nchunks - 1) * NK;   // valid keys of the last chunk
+        {
+            const uint4 sv = lds128(scores + lane * 16);
+            uint32_t pw[4] = {prob_word<F24>(sv.x, lut_g, mx4h, fa, fb),
+                              prob_word<F24>(sv.y, lut_g, mx4h, fa, fb),
+                              prob_word<F24>(sv.z, lut_g, mx4h, fa, fb),
+                              prob_word<F24>(sv.w, lut_g, mx4h, fa, fb)};
+            if (nchunks == 1 && kvalid_last < NK) {
 #pragma unroll
-            for (int q = 0; q < 4; ++q) pw[q] &= key_mask(0, q, t4, kvalid_last);
-        }
-        prob_operand(pw, af);
-    }
-    for (int c = 0; c < nchunks; ++c) {
-        const int u = u0 + nchunks + c;
-        if (!warp_wait(R.ready(u), Ring::parity(u), prm.timeout_cycles)) {
-            if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_READY);
-            return false;
-        }
-        const uint32_t vtile = R.stage(u);
-#pragma unroll
-        for (int ks = 0; ks < 2; ++ks) {
-            const int nxt = min(2 * c + ks + 1, nsteps - 1);
-            const uint4 svn = lds128(scores + (nxt >> 1) * CHUNK_SCORE_BYTES + (nxt & 1) * 512 + lane * 16);
-            const uint32_t wn[4] = {svn.x, svn.y, svn.z, svn.w};
-            uint32_t pw[4];
-#pragma unroll
-            for (int grp = 0; grp < 4; ++grp) {
-                uint32_t b[2][4];
-#pragma unroll
-                for (int i = 0; i < 2; ++i)   // d chunk 2 grp + i: n-tiles 4 grp + 2 i, + 1
-                    vfrag(vtile, ks, 2 * grp + i, lane, b[i][0], b[i][1], b[i][2], b[i][3]);
-#pragma unroll
-                for (int i = 0; i < 2; ++i) {
-                    mma_u8s8(oacc[4 * grp + 2 * i], af, b[i][0], b[i][1]);
-                    mma_u8s8(oacc[4 * grp + 2 * i + 1], af, b[i][2], b[i][3]);
-                }
-                pw[grp] = prob_word(wn[grp], lut_g, mx4h, f0, f1);
-            }
-            if ((nxt >> 1) == nchunks - 1 && kvalid_last < NK) {
-                const int kbase = (nxt & 1) * 32;
-#pragma unroll
-                for (int q = 0; q < 4; ++q) pw[q] &= key_mask(kbase, q, t4, kvalid_last);
+                for (int q = 0; q < 4; ++q) pw[q] &= key_mask(0, q, t4, kvalid_last);
             }
             prob_operand(pw, af);
         }
-        release_stage(R.empty(u), lane);
-    }
+        for (int c = 0; c < nchunks; ++c) {
+            const int u = u0 + nchunks + c;
+            if (!warp_wait(R.ready(u), Ring::parity(u), prm.timeout_cycles)) {
+                if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_READY);
+                return false;
+            }
+            const uint32_t vtile = R.stage(u);
+#pragma unroll
+            for (int ks = 0; ks < 2; ++ks) {
+                const int nxt = min(2 * c + ks + 1, nsteps - 1);
+                const uint4 svn =
+                    lds128(scores + (nxt >> 1) * CHUNK_SCORE_BYTES + (nxt & 1) * 512 + lane * 16);
+                const uint32_t wn[4] = {svn.x, svn.y, svn.z, svn.w};
+                uint32_t pw[4];
+#pragma unroll
+                for (int grp = 0; grp < 4; ++grp) {
+                    uint32_t b[2][4];
+#pragma unroll
+                    for (int i = 0; i < 2; ++i)   // d chunk 2 grp + i: n-tiles 4 grp + 2 i, + 1
+                        vfrag(vtile, ks, 2 * grp + i, lane, b[i][0], b[i][1], b[i][2], b[i][3]);
+#pragma unroll
+                    for (int i = 0; i < 2; ++i) {
+                        mma_u8s8(oacc[4 * grp + 2 * i], af, b[i][0], b[i][1]);
+                        mma_u8s8(oacc[4 * grp + 2 * i + 1], af, b[i][2], b[i][3]);
+                    }
+                    pw[grp] = prob_word<F24>(wn[grp], lut_g, mx4h, fa, fb);
+                }
+                if ((nxt >> 1) == nchunks - 1 && kvalid_last < NK) {
+                    const int kbase = (nxt & 1) * 32;
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) pw[q] &= key_mask(kbase, q, t4, kvalid_last);
+                }
+                prob_operand(pw, af);
+            }
+            release_stage(R.empty(u), lane);
+        }
+        return true;
+    };
+    const bool ok3 = prm.f24 ? pass3(BoolTag<true>(), f0 << 8, f1 << 8)
+                             : pass3(BoolTag<false>(), f0, f1);
+    if (!ok3) return false;
 
     // ---- output requantisation (Eq. 7): per d chunk c and row, four bytes
     // d = 16c + 4t .. 16c + 4t + 3 (n-tiles 2c, 2c + 1, columns 2t, 2t + 1).
@@ -948,10 +967,10 @@ __device__ __forceinline__ bool consume_half(const FusedParams &prm, const Item 
     const int kvalid_last = len - (nchunks - 1) * NK;
     for (int c = 0; c < nchunks; ++c) {
         const uint4 sv = lds128(scores + c * CHUNK_SCORE_BYTES + hk * 512 + lane * 16);
-        uint32_t pw[4] = {prob_word(sv.x, lut_g, mx4h, f0, f1),
-                          prob_word(sv.y, lut_g, mx4h, f0, f1),
-                          prob_word(sv.z, lut_g, mx4h, f0, f1),
-                          prob_word(sv.w, lut_g, mx4h, f0, f1)};
+        uint32_t pw[4] = {prob_word<false>(sv.x, lut_g, mx4h, f0, f1),
+                          prob_word<false>(sv.y, lut_g, mx4h, f0, f1),
+                          prob_word<false>(sv.z, lut_g, mx4h, f0, f1),
+                          prob_word<false>(sv.w, lut_g, mx4h, f0, f1)};
         if (c == nchunks - 1 && kvalid_last < NK) {
 #pragma unroll
             for (int q = 0; q < 4; ++q) pw[q] &= key_mask(32 * hk, q, t4, kvalid_last);

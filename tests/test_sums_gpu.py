@@ -1,10 +1,13 @@
-"""Parity of the softmax row sums in both widths.
+"""Parity of the softmax arithmetic on its general and its fast paths.
 
 The kernel adds the integer exponentials of a row in 32-bit partial sums
-when exp(0) times the terms one thread adds per row stays below 2^32 (the
-host checks the bound per call), else in 64 bits.  Both must give the same
-sums, so each case here runs with the 64-bit path forced and must match the
-oracle bit for bit; the other parity tests take the planned path.
+when exp(0) times the terms one thread adds per row stays below 2^32, else
+in 64 bits; and it takes each probability min(floor(e f / 2^24), 255) as
+one multiply-high of e and f 2^8 when exp(0) > 2^8 (every row sum then
+exceeds 2^8, so f < 2^24), else from the full 64-bit product.  The host
+checks both bounds per call.  The paths compute the same integers, so each
+case here runs with the general paths forced and must match the oracle bit
+for bit; the other parity tests take the planned (mostly fast) paths.
 """
 import numpy as np
 import pytest
@@ -42,6 +45,20 @@ def test_workloads_with_wide_sums(ip, orc, w):
     assert_same(run_gpu(ip, lay, c, lay.lengths), oracle_out(orc, lay, c, lay.lengths))
 
 
+def test_small_exponentials_take_the_general_path(ip, orc):
+    # exp(0) = q_b^2 + q_c <= 2^8: a row sum can be as small as exp(0), so
+    # the planned probabilities take the full 64-bit product as well
+    lay = synth.draw(3, 2, 130, 128, seed=1760, p_mode="sinusoid")
+    base = ip.layer_constants(lay.scales)
+    ip.set_wide_sums(False)
+    try:
+        for sm in ((3, 6, 10), (1, 2, 0), (5, 16, 0), (2, 10, 156)):
+            c = ip.LayerConstants(base.multipliers, base.shifts, sm)
+            assert_same(run_gpu(ip, lay, c), oracle_out(orc, lay, c))
+    finally:
+        ip.set_wide_sums(True)
+
+
 def test_encoder_layer_with_wide_sums(ip, orc):
     lay = synth.layer(3, 7)
     c = ip.layer_constants(lay.scales)
@@ -63,7 +80,8 @@ def test_masks_and_halves_with_wide_sums(ip, orc, split):
 
 def test_large_exponentials_take_the_wide_path(ip, orc):
     # exp(0) = q_b^2 + q_c near 2^27: 16 terms per thread and chunk would
-    # wrap 32 bits, so the planned path is the 64-bit one as well
+    # wrap 32 bits, so the planned sums are the 64-bit ones as well (and the
+    # probabilities take the one multiply-high path)
     lay = synth.draw(2, 2, 96, 128, seed=1750, p_mode="sinusoid")
     base = ip.layer_constants(lay.scales)
     c = ip.LayerConstants(base.multipliers, base.shifts, (20, 100, 1 << 27))
