@@ -640,16 +640,25 @@ __device__ __forceinline__ bool consume_whole(const FusedParams &prm, const Item
     band_mma(bacc, qa, R.stage(u0) + K_TILE_BYTES + band_row0 * 128,
              R.stage(u0) + PV_OFF + band_row0 * 4, lane);
     const int lm_row = lane & 7, lm_mat = lane >> 3;
+    uint32_t packed[8];   // int8 scores of the previous chunk, stored late
     for (int c = 0; c < nchunks; ++c) {
         const int u = u0 + c;
+        // The content MMAs go first: they do not need the band, whose last
+        // MMAs are still in the pipe, nor the previous chunk's scores, whose
+        // stores would otherwise hold back their loads.
+        int cacc[8][4];
+        content_mma(cacc, qa, R.stage(u), R.stage(u) + KU_OFF, lane);
+        if (c > 0) {
+            const uint32_t sprev = scores + (c - 1) * CHUNK_SCORE_BYTES;
+            sts128(sprev + lane * 16, packed[0], packed[1], packed[2], packed[3]);
+            sts128(sprev + 512 + lane * 16, packed[4], packed[5], packed[6], packed[7]);
+        }
         __syncwarp();
 #pragma unroll
         for (int nt = 0; nt < BAND_TILES; ++nt) {
             sts64(remap + (g * REMAP_STRIDE + nt * 8 + 2 * t4) * 4, bacc[nt][0], bacc[nt][1]);
             sts64(remap + ((g + 8) * REMAP_STRIDE + nt * 8 + 2 * t4) * 4, bacc[nt][2], bacc[nt][3]);
         }
-        int cacc[8][4];
-        content_mma(cacc, qa, R.stage(u), R.stage(u) + KU_OFF, lane);
         release_stage(R.empty(u), lane);
         const uint32_t sdst = scores + c * CHUNK_SCORE_BYTES;
         if (c + 1 < nchunks) {
@@ -676,7 +685,6 @@ __device__ __forceinline__ bool consume_whole(const FusedParams &prm, const Item
                 bacc[nt][3] = v.y;
             }
             __syncwarp();
-            uint32_t packed[8];
 #pragma unroll
             for (int m = 0; m < 4; ++m) {
                 const int kh = m >> 1, t0 = CARRY_TILES + (m & 1) * 4;
@@ -694,8 +702,6 @@ __device__ __forceinline__ bool consume_whole(const FusedParams &prm, const Item
                 packed[2 * m + 1] = score_tile<false>(cacc[2 * m + 1], 2 * m + 1, remap, lane, m_c,
                                                       m_p, half_s, s_s, NK, mx0, mx1);
             }
-            sts128(sdst + lane * 16, packed[0], packed[1], packed[2], packed[3]);
-            sts128(sdst + 512 + lane * 16, packed[4], packed[5], packed[6], packed[7]);
         } else {
             __syncwarp();
             const int kvalid = len - c * NK;
