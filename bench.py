@@ -283,9 +283,13 @@ def measure_next_rows(dev, peak, steps: int, cpu: bool):
 
     def flush():
         # write a buffer larger than L2, then read another one, so that the
-        # timed launch finds L2 full of clean lines (no write-back inside it)
+        # timed launch finds L2 full of clean lines (no write-back inside it);
+        # then keep the GPU busy for about 100 us, so that the start event
+        # and the timed launches are queued before it goes idle (the host
+        # time of issuing them stays out of the measurement)
         flush_w.zero_()
         flush_r.sum()
+        torch.cuda._sleep(200_000)
 
     rows = {}
     for name, K, N, G, xl, yl, sw in NEXT_ROWS:

@@ -48,11 +48,11 @@ long long resident(int nsm) {
 
 template <int C>
 int launch(const ipn::NormParams &prm, int nsm, cudaStream_t st) {
+    // every resident CTA gets batches (dealt warp-major), up to one per CTA
     const long long batches = (prm.rows + ipn::NB - 1) / ipn::NB;
-    const long long need = (batches + ipn::THREADS / 32 - 1) / (ipn::THREADS / 32);
     const long long cap = resident<C>(nsm);
     if (cap <= 0) return IP_ERR_CUDA;
-    const unsigned grid = static_cast<unsigned>(need < cap ? need : cap);
+    const unsigned grid = static_cast<unsigned>(batches < cap ? batches : cap);
     ipn::layernorm_i8_kernel<C><<<grid, ipn::THREADS, C * 8192, st>>>(prm);
     return cudaGetLastError() == cudaSuccess ? IP_OK : IP_ERR_CUDA;
 }

@@ -3,15 +3,16 @@
 // floating-point type, no division by a run-time value (d is a compile-time
 // multiple of 512; the square root and the reciprocal are digit-by-digit).
 //
-// One warp per batch of four rows of d channels, batches dealt round-robin
-// over the warps of the grid.  Per row: the sum and the sum of squares of the
+// One warp per batch of four rows of d channels, batches dealt warp-major
+// over a grid of all resident CTAs.  Per row: the sum and the sum of squares of the
 // int8 values (dp4a, warp reduction), floor(sum c^2 / d) = d sum q^2 -
 // (sum q)^2 exactly for the centred values c_i = d q_i - sum, sigma =
 // isqrt(that + eps_c) (at least 1), f = floor(2^31 / sigma), and per element
 // n = round(c f / 2^16), y = clamp(round((M_i n + B_i) / 2^E_i), -127, 127).
-// Lane l takes the 16-byte segments l, l + 32, ... of the row (coalesced);
-// the per-channel constants (B, M, E) of its channels sit in shared memory
-// in lane-major order, one 16-byte record per channel.
+// Lane l takes the 16-byte segments l, l + 32, ... of the row (coalesced)
+// and keeps them in registers between the two passes; the per-channel
+// constants (B, M, E) of its channels sit in shared memory in lane-major
+// order, one 16-byte record per channel, each read once per batch of rows.
 #pragma once
 
 #include <stdint.h>
@@ -74,11 +75,129 @@ __device__ __forceinline__ int sbyte_at(uint32_t w, int e) {
 }
 
 // C = d / 512 segments of 16 channels per lane.  A warp takes NB rows at a
-// time: it reduces them, lane r computes the square root and the reciprocal
-// of row r (one chain of those scalar steps serves NB rows), then it
-// normalises the rows one after the other, reading each again (from L2, it
-// was just read).  Loops over rows stay rolled so that the code fits the
-// instruction cache.
+// time and keeps their int8 values in registers: it reduces them, lane r
+// computes the square root and the reciprocal of row r (one chain of those
+// scalar steps serves NB rows), then it normalises the rows from registers,
+// each channel record read from shared memory once for the NB rows.  The
+// segment loop stays rolled so that the code fits the instruction cache.
+// Pass A of one batch of NB rows (rows past the end read as zero): the rows
+// into registers, sum and sum of squares of each row (dp4a, warp
+// reduction); lane r then computes floor(sum c^2 / d) = d sum q^2 -
+// (sum q)^2 of row r (exact, c = d q - sum), sigma and f = floor(2^31 /
+// sigma), which every lane receives for every row.
+template <int C>
+struct Batch {
+    uint4 xv[NB][C];
+    int sum[NB], f[NB];
+};
+
+template <int C>
+__device__ __forceinline__ void pass_a(const NormParams &prm, long long row0, int nrows, int lane,
+                                       Batch<C> &bt) {
+    constexpr int D = 512 * C;
+    int sq[NB];
+#pragma unroll
+    for (int r = 0; r < NB; ++r) {
+        const int8_t *xr = prm.x + (row0 + (r < nrows ? r : 0)) * D;
+#pragma unroll
+        for (int j = 0; j < C; ++j)
+            bt.xv[r][j] = r < nrows ? __ldcs(reinterpret_cast<const uint4 *>(xr + j * 512 + lane * 16))
+                                    : make_uint4(0u, 0u, 0u, 0u);
+    }
+#pragma unroll
+    for (int r = 0; r < NB; ++r) {
+        bt.sum[r] = 0;
+        sq[r] = 0;
+#pragma unroll
+        for (int j = 0; j < C; ++j) {
+            const uint32_t w[4] = {bt.xv[r][j].x, bt.xv[r][j].y, bt.xv[r][j].z, bt.xv[r][j].w};
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                bt.sum[r] = __dp4a(static_cast<int>(w[i]), 0x01010101, bt.sum[r]);
+                sq[r] = __dp4a(static_cast<int>(w[i]), static_cast<int>(w[i]), sq[r]);
+            }
+        }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1)
+#pragma unroll
+        for (int r = 0; r < NB; ++r) {
+            bt.sum[r] += __shfl_xor_sync(0xffffffffu, bt.sum[r], o);
+            sq[r] += __shfl_xor_sync(0xffffffffu, sq[r], o);
+        }
+    long long ms = 0;
+#pragma unroll
+    for (int r = 0; r < NB; ++r)
+        if (lane == r) ms = static_cast<long long>(D) * sq[r] - static_cast<long long>(bt.sum[r]) * bt.sum[r];
+    unsigned long long sigma = isqrt_u42(static_cast<unsigned long long>(ms + prm.eps_c));
+    sigma = sigma < 1 ? 1 : sigma;
+    // f = floor(2^31 / sigma), held as a signed 32-bit value: f = 2^31 only
+    // for sigma = 1, where sum c^2 < 4 d gives |c| < 2^7 and round(c (2^31 -
+    // 1) / 2^16) = round(c 2^31 / 2^16), so 2^31 - 1 stands in exactly
+    uint32_t f_own = recip_2pow31(sigma);
+    f_own = f_own > 0x7fffffffu ? 0x7fffffffu : f_own;
+#pragma unroll
+    for (int r = 0; r < NB; ++r) bt.f[r] = static_cast<int>(__shfl_sync(0xffffffffu, f_own, r));
+}
+
+// Pass B of one batch: normalise and requantise the rows from registers;
+// each channel record serves the NB rows.  The segment loop stays rolled so
+// that the code fits the instruction cache.
+template <int C>
+__device__ __forceinline__ void pass_b(const NormParams &prm, const uint4 *cst, long long row0,
+                                       int nrows, int lane, const Batch<C> &bt) {
+    constexpr int D = 512 * C;
+#pragma unroll 1
+    for (int j = 0; j < C; ++j) {
+        uint4 xj[NB];
+#pragma unroll
+        for (int r = 0; r < NB; ++r) xj[r] = bt.xv[r][0];
+#pragma unroll
+        for (int jj = 1; jj < C; ++jj)
+            if (j == jj) {
+#pragma unroll
+                for (int r = 0; r < NB; ++r) xj[r] = bt.xv[r][jj];
+            }
+        uint32_t o[NB][4];
+#pragma unroll
+        for (int r = 0; r < NB; ++r) o[r][0] = o[r][1] = o[r][2] = o[r][3] = 0u;
+#pragma unroll
+        for (int e = 0; e < 16; ++e) {
+            const uint4 rec = cst[(j * 16 + e) * 32 + lane];
+            const long long b = static_cast<long long>((static_cast<unsigned long long>(rec.y) << 32) | rec.x);
+#pragma unroll
+            for (int r = 0; r < NB; ++r) {
+                const uint32_t w[4] = {xj[r].x, xj[r].y, xj[r].z, xj[r].w};
+                const int cc = D * sbyte_at(w[e >> 2], e & 3) - bt.sum[r];   // |c| < 2^20
+                // n = round(c f / 2^16): |c f| < 2^51 and |n| < 2^23, so the
+                // low word of (c f + 2^15) >> 16 is n
+                const long long u = static_cast<long long>(cc) * bt.f[r] + (1ll << 15);
+                const int n = static_cast<int>(__funnelshift_r(static_cast<uint32_t>(u),
+                                                               static_cast<uint32_t>(u >> 32), 16));
+                // floor(v / 2^E) = floor(floor(v / 2^31) / 2^(E - 31)); |v| < 2^62
+                // makes floor(v / 2^31) a 32-bit value
+                const long long v = static_cast<long long>(static_cast<int>(rec.z)) * n + b;
+                const int h = static_cast<int>(__funnelshift_r(static_cast<uint32_t>(v),
+                                                               static_cast<uint32_t>(v >> 32), 31));
+                const int t = h >> static_cast<int>(rec.w);
+                const int y8 = t > 127 ? 127 : (t < -127 ? -127 : t);
+                o[r][e >> 2] |= (static_cast<uint32_t>(y8) & 0xffu) << (8 * (e & 3));
+            }
+        }
+#pragma unroll
+        for (int r = 0; r < NB; ++r)
+            if (r < nrows)
+                __stcs(reinterpret_cast<uint4 *>(prm.y + (row0 + r) * D + j * 512 + lane * 16),
+                       make_uint4(o[r][0], o[r][1], o[r][2], o[r][3]));
+    }
+}
+
+// C = d / 512 segments of 16 channels per lane.  A warp takes NB rows at a
+// time and keeps their int8 values in registers: pass A reduces them (lane
+// r computes the square root and the reciprocal of row r, one chain of
+// those scalar steps for NB rows), pass B normalises them.  The first
+// batch's pass A runs before the channel records are built, so its loads
+// overlap that set-up.
 template <int C>
 __global__ void __launch_bounds__(THREADS)
     layernorm_i8_kernel(const NormParams prm) {
@@ -86,6 +205,19 @@ __global__ void __launch_bounds__(THREADS)
     extern __shared__ uint8_t smem_raw[];
     uint4 *cst = reinterpret_cast<uint4 *>(smem_raw);   // [C * 16][32] records
     const int lane = threadIdx.x & 31;
+    // Batches are dealt warp-major (warp w of CTA c takes batch w G + c, then
+    // that plus 8 G, ...), so that with fewer batches than warps every CTA,
+    // and every SM, keeps about the same number of busy warps.
+    const long long warps = static_cast<long long>(gridDim.x) * (THREADS / 32);
+    const long long groups = (prm.rows + NB - 1) / NB;
+    long long grp = static_cast<long long>(threadIdx.x >> 5) * gridDim.x + blockIdx.x;
+
+    Batch<C> bt;
+    const bool first = grp < groups;
+    if (first) {
+        const long long row0 = grp * NB;
+        pass_a<C>(prm, row0, prm.rows - row0 < NB ? static_cast<int>(prm.rows - row0) : NB, lane, bt);
+    }
 
     // per-channel records {B' lo, B' hi, M, E - 31} with B' = B + 2^(E-1)
     // (the rounding term folded in): channel j 512 + l 16 + e of lane l goes
@@ -107,94 +239,16 @@ __global__ void __launch_bounds__(THREADS)
     }
     if (bad) atomicOr(prm.err, ERR_PARAM);
     __syncthreads();
+    if (!first) return;
 
-    const long long warps = static_cast<long long>(gridDim.x) * (THREADS / 32);
-    const long long groups = (prm.rows + NB - 1) / NB;
-    for (long long grp = static_cast<long long>(blockIdx.x) * (THREADS / 32) + (threadIdx.x >> 5);
-         grp < groups; grp += warps) {
+    for (;;) {
         const long long row0 = grp * NB;
         const int nrows = prm.rows - row0 < NB ? static_cast<int>(prm.rows - row0) : NB;
-
-        // pass A: sum and sum of squares of each row (dp4a, warp reduction)
-        int sum[NB], sq[NB];
-#pragma unroll
-        for (int r = 0; r < NB; ++r) {
-            sum[r] = 0;
-            sq[r] = 0;
-            if (r < nrows) {
-                const int8_t *xr = prm.x + (row0 + r) * D;
-#pragma unroll
-                for (int j = 0; j < C; ++j) {
-                    const uint4 s = __ldg(reinterpret_cast<const uint4 *>(xr + j * 512 + lane * 16));
-                    const uint32_t w[4] = {s.x, s.y, s.z, s.w};
-#pragma unroll
-                    for (int i = 0; i < 4; ++i) {
-                        sum[r] = __dp4a(static_cast<int>(w[i]), 0x01010101, sum[r]);
-                        sq[r] = __dp4a(static_cast<int>(w[i]), static_cast<int>(w[i]), sq[r]);
-                    }
-                }
-            }
-        }
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1)
-#pragma unroll
-            for (int r = 0; r < NB; ++r) {
-                sum[r] += __shfl_xor_sync(0xffffffffu, sum[r], o);
-                sq[r] += __shfl_xor_sync(0xffffffffu, sq[r], o);
-            }
-
-        // lane r: floor(sum c^2 / d) = d sum q^2 - (sum q)^2 of row r (exact,
-        // c = d q - sum), sigma and f
-        long long ms = 0;
-        int sum_own = 0;
-#pragma unroll
-        for (int r = 0; r < NB; ++r)
-            if (lane == r) {
-                ms = static_cast<long long>(D) * sq[r] - static_cast<long long>(sum[r]) * sum[r];
-                sum_own = sum[r];
-            }
-        unsigned long long sigma = isqrt_u42(static_cast<unsigned long long>(ms + prm.eps_c));
-        sigma = sigma < 1 ? 1 : sigma;
-        // f = floor(2^31 / sigma), held as a signed 32-bit value: f = 2^31 only
-        // for sigma = 1, where sum c^2 < 4 d gives |c| < 2^7 and round(c (2^31 -
-        // 1) / 2^16) = round(c 2^31 / 2^16), so 2^31 - 1 stands in exactly
-        uint32_t f_own = recip_2pow31(sigma);
-        f_own = f_own > 0x7fffffffu ? 0x7fffffffu : f_own;
-
-        // pass B: normalise and requantise, row by row
-#pragma unroll 1
-        for (int r = 0; r < nrows; ++r) {
-            const int f = static_cast<int>(__shfl_sync(0xffffffffu, f_own, r));
-            const int sm = __shfl_sync(0xffffffffu, sum_own, r);
-            const int8_t *xr = prm.x + (row0 + r) * D;
-            int8_t *yr = prm.y + (row0 + r) * D;
-#pragma unroll
-            for (int j = 0; j < C; ++j) {
-                const uint4 s = __ldcs(reinterpret_cast<const uint4 *>(xr + j * 512 + lane * 16));
-                const uint32_t w[4] = {s.x, s.y, s.z, s.w};
-                uint32_t o[4] = {0u, 0u, 0u, 0u};
-#pragma unroll
-                for (int e = 0; e < 16; ++e) {
-                    const uint4 rec = cst[(j * 16 + e) * 32 + lane];
-                    const long long b = static_cast<long long>((static_cast<unsigned long long>(rec.y) << 32) | rec.x);
-                    const int cc = D * sbyte_at(w[e >> 2], e & 3) - sm;   // |c| < 2^20
-                    // n = round(c f / 2^16): |c f| < 2^51 and |n| < 2^23, so the
-                    // low word of (c f + 2^15) >> 16 is n
-                    const long long u = static_cast<long long>(cc) * f + (1ll << 15);
-                    const int n = static_cast<int>(__funnelshift_r(static_cast<uint32_t>(u),
-                                                                   static_cast<uint32_t>(u >> 32), 16));
-                    // floor(v / 2^E) = floor(floor(v / 2^31) / 2^(E - 31)); |v| < 2^62
-                    // makes floor(v / 2^31) a 32-bit value
-                    const long long v = static_cast<long long>(static_cast<int>(rec.z)) * n + b;
-                    const int h = static_cast<int>(__funnelshift_r(static_cast<uint32_t>(v),
-                                                                   static_cast<uint32_t>(v >> 32), 31));
-                    const int t = h >> static_cast<int>(rec.w);
-                    const int y8 = t > 127 ? 127 : (t < -127 ? -127 : t);
-                    o[e >> 2] |= (static_cast<uint32_t>(y8) & 0xffu) << (8 * (e & 3));
-                }
-                __stcs(reinterpret_cast<uint4 *>(yr + j * 512 + lane * 16), make_uint4(o[0], o[1], o[2], o[3]));
-            }
-        }
+        pass_b<C>(prm, cst, row0, nrows, lane, bt);
+        grp += warps;
+        if (grp >= groups) break;
+        const long long nrow0 = grp * NB;
+        pass_a<C>(prm, nrow0, prm.rows - nrow0 < NB ? static_cast<int>(prm.rows - nrow0) : NB, lane, bt);
     }
 }
 
