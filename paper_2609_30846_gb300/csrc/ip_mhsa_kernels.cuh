@@ -1130,9 +1130,15 @@ __global__ void __launch_bounds__(NTHREADS, 2)
         }
     };
 
-    // The copy warp initialises the barriers, claims its first item and
-    // sends its first two uses off at once; the exponential table is built
-    // while they travel.
+    // A launch that follows this one on its stream may start now: its CTAs
+    // take the SM slots this grid frees at its end and wait (below) for its
+    // completion before they touch global memory.
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+
+    // The copy warp initialises the barriers, waits for the grid before it
+    // on the stream (its outputs and the reset work counters visible),
+    // claims its first item and sends its first two uses off at once; the
+    // exponential table is built meanwhile.
     bool live0 = false;
     if (warp == NCWARPS) {
         if (lane == 0) {
@@ -1150,6 +1156,7 @@ __global__ void __launch_bounds__(NTHREADS, 2)
             asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
         }
         __syncwarp();
+        asm volatile("griddepcontrol.wait;" ::: "memory");
         uint32_t item = 0;
         live0 = claim(item);
         if (live0) {
@@ -1169,6 +1176,7 @@ __global__ void __launch_bounds__(NTHREADS, 2)
 #pragma unroll
         for (int c = 0; c < LUT_COPIES; ++c) sts32(lut + (d * LUT_COPIES + c) * 4, e);
     }
+    asm volatile("griddepcontrol.wait;" ::: "memory");
     __syncthreads();
 
     // ------------------------------------------------------------ producers
