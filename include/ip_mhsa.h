@@ -70,8 +70,8 @@ typedef struct {
 #define IP_MAX_B 65535
 #define IP_MAX_H 65535
 /* B H ceil(T / 64) (the 64-row query tiles of a call) must stay below this:
- * the kernel's work items are numbered with 31 bits. */
-#define IP_MAX_TILES (1ll << 30)
+ * the kernel's work items (up to four per tile) are numbered with 31 bits. */
+#define IP_MAX_TILES (1ll << 29)
 
 /* Bytes of device workspace a call needs: the device-side status word of
  * the calls that use it.  The caller zero-fills the workspace once before
@@ -378,11 +378,12 @@ int ip_debug_set_stall_injection(int on);
 
 /* Test hook: how the kernels launched afterwards by this process do the
  * tiles of 64 query rows.  Negative (the default): as planned, i.e. when the
- * last wave of CTAs on the GPU would be at most half full, its tiles are
- * done as two halves of 32 rows whose warps split the keys of every chunk
- * and combine their row maxima, exponential sums and attn.V partial sums.
- * 0: no tile is split.  Positive: every tile is split (when the grid allows
- * it).  The outputs are the same bit for bit in every mode. */
+ * last round of work items over the resident CTAs would be at most a
+ * quarter full, its tiles are done as four quarters of 16 rows, when at most
+ * half full as two halves of 32 rows, whose warps split the keys of every
+ * chunk and combine their row maxima, exponential sums and attn.V partial
+ * sums.  0: no tile is split.  1: every tile in halves.  2 (or more): every
+ * tile in quarters.  The outputs are the same bit for bit in every mode. */
 int ip_debug_set_split_mode(int mode);
 
 /* Test hook: nonzero makes the attention kernel take its general softmax

@@ -236,7 +236,8 @@ def set_stall_injection(on: bool) -> None:
 
 def set_split_mode(mode: int) -> None:
     """Test hook: -1 planned tail split (default), 0 never split, 1 split
-    every 64-row tile into two key-split halves."""
+    every 64-row tile into two key-split halves, 2 into four key-split
+    quarters."""
     load().ip_debug_set_split_mode(int(mode))
 
 

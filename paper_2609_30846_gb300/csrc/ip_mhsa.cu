@@ -19,7 +19,7 @@ constexpr size_t WS_HEADER = 256;          // error word and padding
 constexpr long long DEFAULT_TIMEOUT = 4000000000ll;   // ~2 s at 2 GHz
 long long g_timeout_cycles = DEFAULT_TIMEOUT;
 int g_stall_injection = 0;
-int g_split_mode = -1;   // -1 planned, 0 never, 1 every tile (test hook)
+int g_split_mode = -1;   // -1 planned, 0 never, 1 / 2: every tile in halves / quarters (test hook)
 int g_wide_sums = 0;     // 1: general softmax arithmetic always (test hook)
 
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
@@ -118,22 +118,29 @@ int resident_ctas(int smem) {
 }
 
 // Work items of the persistent kernel.  The N whole tiles run on G resident
-// CTAs in rounds; when the last round is at most half full (r = N mod G
-// tiles, 2 r <= G), its r tiles become 2 r halves of 32 rows whose warps
-// split the keys of every chunk, so the last round takes about half as long.
+// CTAs in rounds; when the last round is at most a quarter full (r = N mod G
+// tiles, 4 r <= G) its r tiles become 4 r quarters of 16 rows, when at most
+// half full (2 r <= G) 2 r halves of 32 rows, whose warps split the keys of
+// every chunk, so that the last round takes a fraction of a tile's time.
 struct ItemPlan {
     uint32_t nwhole = 0, nitems = 0, grid = 0;
+    int split_log2 = 1;
 };
 
 ItemPlan plan_items(long long N, int slots) {
     ItemPlan ip;
     long long nwhole = N, nitems = N;
-    if (g_split_mode == 1) {
+    if (g_split_mode == 1 || g_split_mode == 2) {
+        ip.split_log2 = g_split_mode;
         nwhole = 0;
-        nitems = 2 * N;
+        nitems = N << g_split_mode;
     } else if (g_split_mode < 0 && slots > 0) {
         const long long r = N % slots;
-        if (r > 0 && 2 * r <= slots) {
+        if (r > 0 && 4 * r <= slots) {
+            ip.split_log2 = 2;
+            nwhole = N - r;
+            nitems = N + 3 * r;
+        } else if (r > 0 && 2 * r <= slots) {
             nwhole = N - r;
             nitems = N + r;
         }
@@ -244,6 +251,7 @@ int ip_relpos_mhsa_i8_ex(const int8_t *q, const int8_t *k, const int8_t *v, cons
     prm.tiles_magic = iph::div_magic(static_cast<unsigned long long>(ntiles));
     prm.heads_magic = iph::div_magic(static_cast<unsigned long long>(H));
     prm.nwhole = ip.nwhole;
+    prm.split_log2 = ip.split_log2;
     prm.nitems = ip.nitems;
     prm.out_rows = out_layout == IP_LAYOUT_ROWS ? 1 : 0;
     // Programmatic dependent launch: this grid may be scheduled while the
@@ -523,7 +531,7 @@ int ip_debug_set_timeout_cycles(long long cycles) {
 }
 
 int ip_debug_set_split_mode(int mode) {
-    g_split_mode = mode < 0 ? -1 : (mode > 0 ? 1 : 0);
+    g_split_mode = mode < 0 ? -1 : (mode > 2 ? 2 : mode);
     return IP_OK;
 }
 

@@ -99,12 +99,14 @@ struct FusedParams {
     int f24;                  // exp(0) > 2^8: every row sum exceeds 2^8, so f = 2^32 / sum < 2^24
     // Work items, claimed in order by the persistent CTAs: items [0, nwhole)
     // are whole 64-row tiles in (b, h, tile) order, items [nwhole, nitems)
-    // the two 32-row halves of the tiles from nwhole on.
+    // the 2^split_log2 parts (32-row halves or 16-row quarters) of the tiles
+    // from nwhole on.
     unsigned int *sched;      // workspace words: [0] next item, [16] CTAs done claiming
     int ntiles;                        // 64-row tiles per (b, h)
     unsigned long long tiles_magic;    // udiv_magic constant of ntiles
     unsigned long long heads_magic;    // udiv_magic constant of H
     uint32_t nwhole, nitems;           // nitems < 2^31
+    int split_log2;                    // 1: halves, 2: quarters
     int out_rows;             // output [B][T][H][DH] instead of [B][H][T][DH]
 };
 
@@ -540,11 +542,11 @@ __device__ __forceinline__ void prep_bias(uint32_t ktile, uint32_t ptile, uint32
 
 // ------------------------------------------------------------- work items --
 
-// One work item: a whole 64-row tile of (b, h) (part < 0) or the 32-row half
-// `part` of one.  Items are decoded without a division instruction (exact
+// One work item: a whole 64-row tile of (b, h) (part < 0, nparts 1) or part
+// `part` of nparts (2: 32-row halves, 4: 16-row quarters) of one.  Items are decoded without a division instruction (exact
 // multiply-high by the constants of ntiles and H).
 struct Item {
-    int b, h, bh, i0, part, len, nchunks;
+    int b, h, bh, i0, part, nparts, plog2, len, nchunks;
     bool pad;   // every row of the tile (half) is padding
 };
 
@@ -552,10 +554,14 @@ __device__ __forceinline__ Item decode_item(const FusedParams &p, uint32_t item)
     Item it;
     uint32_t lin = item;
     it.part = -1;
+    it.nparts = 1;
+    it.plog2 = 0;
     if (item >= p.nwhole) {
         const uint32_t t = item - p.nwhole;
-        lin = p.nwhole + (t >> 1);
-        it.part = static_cast<int>(t & 1u);
+        lin = p.nwhole + (t >> p.split_log2);
+        it.part = static_cast<int>(t & ((1u << p.split_log2) - 1u));
+        it.nparts = 1 << p.split_log2;
+        it.plog2 = p.split_log2;
     }
     const uint32_t bh = udiv_magic(lin, p.tiles_magic);
     const int tile = static_cast<int>(lin - bh * static_cast<uint32_t>(p.ntiles));
@@ -570,7 +576,7 @@ __device__ __forceinline__ Item decode_item(const FusedParams &p, uint32_t item)
     }
     it.len = len;
     it.nchunks = (len + NK - 1) / NK;
-    it.pad = (it.part < 0 ? it.i0 : it.i0 + 32 * it.part) >= len;
+    it.pad = (it.part < 0 ? it.i0 : it.i0 + (MROWS >> it.plog2) * it.part) >= len;
     return it;
 }
 
@@ -608,6 +614,9 @@ struct Ring {
     // Item number of the CTA's live item k (written by the copy warp before
     // it arrives on that item's barriers), or NO_ITEM after the last.
     __device__ __forceinline__ uint32_t slot(int k) const { return bar_base + 96u + 4u * (k & 3); }
+    // The four consumer warps of a quarter item exchange maxima, sums and
+    // partial sums (one phase per exchange step).
+    __device__ __forceinline__ uint32_t quad() const { return bar_base + 120u; }
 };
 
 // ------------------------------------------------------ consumer: whole tile --
@@ -1029,6 +1038,271 @@ __device__ __forceinline__ bool consume_half(const FusedParams &prm, const Item 
     return true;
 }
 
+// ------------------------------------------------------ consumer: quarter tile --
+// Band n-tiles nt0 .. nt0 + 3 and content n-tiles nt0, nt0 + 1 of one
+// 16-key slice of a chunk (nt0 = 2 w): the band columns of keys 16 w ..
+// 16 w + 15 of 16 rows are 16 w .. 16 w + 30.
+__device__ __forceinline__ void quarter_chunk_mma(int (&bacc)[4][4], int (&cacc)[2][4],
+                                                  const uint32_t (&qa)[4][4], uint32_t ptile,
+                                                  uint32_t pv, uint32_t ktile, uint32_t ku,
+                                                  int nt0, int lane) {
+    const int t4 = lane & 3;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const int2 v = lds64(pv + ((nt0 + i) * 8 + 2 * t4) * 4);
+        bacc[i][0] = v.x;
+        bacc[i][1] = v.y;
+        bacc[i][2] = v.x;
+        bacc[i][3] = v.y;
+    }
+#pragma unroll
+    for (int i = 0; i < 2; ++i) {
+        const int2 v = lds64(ku + ((nt0 + i) * 8 + 2 * t4) * 4);
+        cacc[i][0] = v.x;
+        cacc[i][1] = v.y;
+        cacc[i][2] = v.x;
+        cacc[i][3] = v.y;
+    }
+    const int lm_row = lane & 7, lm_mat = lane >> 3;
+#pragma unroll
+    for (int kh = 0; kh < 2; ++kh) {
+        uint32_t b[4][4], kb[2][4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+            ldsm_x4(ptile + swz((nt0 + i) * 8 + lm_row, kh * 4 + lm_mat), b[i][0], b[i][1],
+                    b[i][2], b[i][3]);
+#pragma unroll
+        for (int i = 0; i < 2; ++i)
+            ldsm_x4(ktile + swz((nt0 + i) * 8 + lm_row, kh * 4 + lm_mat), kb[i][0], kb[i][1],
+                    kb[i][2], kb[i][3]);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) mma_s8s8(bacc[i], qa[2 * kh], b[i][0], b[i][1]);
+#pragma unroll
+        for (int i = 0; i < 2; ++i) mma_s8s8(cacc[i], qa[2 * kh], kb[i][0], kb[i][1]);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) mma_s8s8(bacc[i], qa[2 * kh + 1], b[i][2], b[i][3]);
+#pragma unroll
+        for (int i = 0; i < 2; ++i) mma_s8s8(cacc[i], qa[2 * kh + 1], kb[i][2], kb[i][3]);
+    }
+}
+
+// One 16-row quarter (strip `part`) of a tile, for the tail of the work:
+// the four warps share the strip, warp w taking the keys [16 w, 16 w + 16)
+// of every chunk, and its attn.V product on those keys as m16n8k16 MMAs
+// (k order 2t, 2t + 1, 8 + 2t, 9 + 2t on both operands, as in the 32-key
+// steps).  Row maxima, exponential sums and the attn.V partial sums (warp w
+// finishes d = 32 w .. 32 w + 31) are combined through the warps' exchange
+// areas behind the quad barrier, eight phases per quarter.
+__device__ __forceinline__ bool consume_quarter(const FusedParams &prm, const Item &it, int u0,
+                                                const Ring &R, uint32_t remap, uint32_t remap0,
+                                                uint32_t scores, uint32_t lut, uint32_t quad,
+                                                int warp, int lane) {
+    const int len = it.len, nchunks = it.nchunks;
+    const int g = lane >> 2, t4 = lane & 3;
+    const int strip = it.part;
+    const int wrow0 = it.i0 + strip * 16;
+    const long long m_c = prm.m_c, m_p = prm.m_p;
+    const long long half_s = 1ll << (prm.sh_s - 1);
+    const int s_s = prm.sh_s - 31;
+    const int band_row0 = 48 - 16 * strip;
+    const int nt0 = 2 * warp;                  // this warp's key slice: n-tiles nt0, nt0 + 1
+    int mx0 = -128, mx1 = -128;
+    const uint32_t lut_g = lut + 4 * (g & (LUT_COPIES - 1));
+    int qph = 0;   // phases of the quad barrier used in this quarter
+    auto quad_sync = [&]() -> bool {
+        __syncwarp();
+        if (lane == 0) mbar_arrive(quad);
+        const bool ok = warp_wait(quad, static_cast<uint32_t>(qph) & 1u, prm.timeout_cycles);
+        ++qph;
+        if (!ok && lane == 0) atomicOr(prm.err, ERR_TIMEOUT_READY);
+        return ok;
+    };
+    uint32_t qa[4][4];
+    load_q(R.qtile(), strip, lane, qa);
+
+    // pass 1: scores of this warp's key slice of every chunk
+    for (int c = 0; c < nchunks; ++c) {
+        const int u = u0 + c;
+        if (!warp_wait(R.ready(u), Ring::parity(u), prm.timeout_cycles)) {
+            if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_READY);
+            return false;
+        }
+        int qb[4][4], qc[2][4];
+        quarter_chunk_mma(qb, qc, qa, R.stage(u) + K_TILE_BYTES + band_row0 * 128,
+                          R.stage(u) + PV_OFF + band_row0 * 4, R.stage(u), R.stage(u) + KU_OFF, nt0,
+                          lane);
+        release_stage(R.empty(u), lane);
+        __syncwarp();   // the remap reads of the previous chunk are done
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            sts64(remap + (g * REMAP_STRIDE + i * 8 + 2 * t4) * 4, qb[i][0], qb[i][1]);
+            sts64(remap + ((g + 8) * REMAP_STRIDE + i * 8 + 2 * t4) * 4, qb[i][2], qb[i][3]);
+        }
+        __syncwarp();
+        // band columns stored from the slice's first one: key jj of the slice
+        // and row rho take the band value at jj - rho + 15, as in a chunk
+        const int kvalid = len - c * NK - 16 * warp;   // valid keys of the slice
+        uint32_t pk[2];
+        if (kvalid < 16) {
+#pragma unroll
+            for (int i = 0; i < 2; ++i)
+                pk[i] = score_tile<true>(qc[i], i, remap, lane, m_c, m_p, half_s, s_s, kvalid,
+                                         mx0, mx1);
+        } else {
+#pragma unroll
+            for (int i = 0; i < 2; ++i)
+                pk[i] = score_tile<false>(qc[i], i, remap, lane, m_c, m_p, half_s, s_s, kvalid,
+                                          mx0, mx1);
+        }
+        sts64(scores + c * CHUNK_SCORE_BYTES + lane * 8, static_cast<int>(pk[0]),
+              static_cast<int>(pk[1]));
+    }
+    release_stage(R.qempty(), lane);   // done with the Q tile
+    mx0 = max(mx0, __shfl_xor_sync(0xffffffffu, mx0, 1));
+    mx0 = max(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
+    mx1 = max(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
+    mx1 = max(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
+    __syncwarp();   // the remap reads of the last chunk are done
+    sts64(remap + XMAX_OFF + lane * 8, mx0, mx1);
+    if (!quad_sync()) return false;
+#pragma unroll
+    for (int w = 0; w < NCWARPS; ++w) {
+        const int2 pm = lds64(remap0 + w * REMAP_BYTES + XMAX_OFF + lane * 8);
+        mx0 = max(mx0, pm.x);
+        mx1 = max(mx1, pm.y);
+    }
+    const uint32_t mx4h = max4h(mx0, mx1);
+
+    // pass 2: exponential sums of the slice, then of the whole row
+    unsigned long long sum0 = 0, sum1 = 0;
+    for (int c = 0; c < nchunks; ++c) {
+        const int kvalid = len - c * NK - 16 * warp;
+        const int2 wv = lds64(scores + c * CHUNK_SCORE_BYTES + lane * 8);
+        const uint32_t w2[2] = {static_cast<uint32_t>(wv.x), static_cast<uint32_t>(wv.y)};
+#pragma unroll
+        for (int q = 0; q < 2; ++q) {
+            const uint32_t d4 = exp_index4(w2[q], mx4h);
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                uint32_t ev = lds32(lut_at(lut_g, d4, e));
+                if (q * 8 + 2 * t4 + (e & 1) >= kvalid) ev = 0u;
+                if (e < 2) sum0 += ev;
+                else sum1 += ev;
+            }
+        }
+    }
+    sum0 += __shfl_xor_sync(0xffffffffu, sum0, 1);
+    sum0 += __shfl_xor_sync(0xffffffffu, sum0, 2);
+    sum1 += __shfl_xor_sync(0xffffffffu, sum1, 1);
+    sum1 += __shfl_xor_sync(0xffffffffu, sum1, 2);
+    sts64(remap + XSUM_OFF + lane * 16, static_cast<int>(sum0), static_cast<int>(sum0 >> 32));
+    sts64(remap + XSUM_OFF + lane * 16 + 8, static_cast<int>(sum1), static_cast<int>(sum1 >> 32));
+    if (!quad_sync()) return false;
+    sum0 = 0;
+    sum1 = 0;
+#pragma unroll
+    for (int w = 0; w < NCWARPS; ++w) {
+        const int2 a = lds64(remap0 + w * REMAP_BYTES + XSUM_OFF + lane * 16);
+        const int2 bq = lds64(remap0 + w * REMAP_BYTES + XSUM_OFF + lane * 16 + 8);
+        sum0 += (static_cast<unsigned long long>(static_cast<uint32_t>(a.y)) << 32) |
+                static_cast<uint32_t>(a.x);
+        sum1 += (static_cast<unsigned long long>(static_cast<uint32_t>(bq.y)) << 32) |
+                static_cast<uint32_t>(bq.x);
+    }
+    const uint32_t f0 = div_2pow32(sum0);
+    const uint32_t f1 = div_2pow32(sum1);
+
+    // pass 3: probabilities of the slice x V (m16n8k16, k = the slice's keys)
+    int oacc[16][4];
+#pragma unroll
+    for (int nt = 0; nt < 16; ++nt) oacc[nt][0] = oacc[nt][1] = oacc[nt][2] = oacc[nt][3] = 0;
+    const int vkey = 16 * warp + 8 * ((lane >> 3) & 1) + (lane & 7);
+    for (int c = 0; c < nchunks; ++c) {
+        const int kvalid = len - c * NK - 16 * warp;
+        const int2 wv = lds64(scores + c * CHUNK_SCORE_BYTES + lane * 8);
+        uint32_t pw0 = prob_word<false>(static_cast<uint32_t>(wv.x), lut_g, mx4h, f0, f1);
+        uint32_t pw1 = prob_word<false>(static_cast<uint32_t>(wv.y), lut_g, mx4h, f0, f1);
+        if (kvalid < 16) {
+            pw0 &= key_mask(0, 0, t4, kvalid);
+            pw1 &= key_mask(0, 1, t4, kvalid);
+        }
+        // A: row g, then g + 8, keys 2t, 2t + 1, 8 + 2t, 9 + 2t of the slice
+        const uint32_t a0 = __byte_perm(pw0, pw1, 0x5410);
+        const uint32_t a1 = __byte_perm(pw0, pw1, 0x7632);
+        const int u = u0 + nchunks + c;
+        if (!warp_wait(R.ready(u), Ring::parity(u), prm.timeout_cycles)) {
+            if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_READY);
+            return false;
+        }
+        const uint32_t vtile = R.stage(u);
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            // d chunks 2j, 2j + 1: the slice's keys 0-7 and 8-15 of each
+            uint32_t r0, r1, r2, r3;
+            ldsm_x4_trans(vtile + swz(vkey, 2 * j + (lane >> 4)), r0, r1, r2, r3);
+            mma_u8s8_k16(oacc[4 * j], a0, a1, __byte_perm(r0, r1, 0x6420));
+            mma_u8s8_k16(oacc[4 * j + 1], a0, a1, __byte_perm(r0, r1, 0x7531));
+            mma_u8s8_k16(oacc[4 * j + 2], a0, a1, __byte_perm(r2, r3, 0x6420));
+            mma_u8s8_k16(oacc[4 * j + 3], a0, a1, __byte_perm(r2, r3, 0x7531));
+        }
+        release_stage(R.empty(u), lane);
+    }
+
+    // the partial sums: in round r each warp sends the n-tiles of warp
+    // (w + r) mod 4 and adds those warp (w - r) mod 4 sent it
+    const uint32_t xo = remap + XO_OFF;
+#pragma unroll 1
+    for (int r = 1; r < NCWARPS; ++r) {
+        const int dst = (warp + r) & (NCWARPS - 1);
+        const int src = (warp - r) & (NCWARPS - 1);
+#pragma unroll
+        for (int w = 0; w < NCWARPS; ++w)
+            if (w == dst) {
+#pragma unroll
+                for (int i = 0; i < 4; ++i)
+#pragma unroll
+                    for (int e = 0; e < 4; ++e)
+                        sts32(xo + ((i * 4 + e) * 32 + lane) * 4, static_cast<uint32_t>(oacc[4 * w + i][e]));
+            }
+        if (!quad_sync()) return false;
+        const uint32_t xs = remap0 + src * REMAP_BYTES + XO_OFF;
+#pragma unroll
+        for (int w = 0; w < NCWARPS; ++w)
+            if (w == warp) {
+#pragma unroll
+                for (int i = 0; i < 4; ++i)
+#pragma unroll
+                    for (int e = 0; e < 4; ++e)
+                        oacc[4 * w + i][e] += static_cast<int>(lds32(xs + ((i * 4 + e) * 32 + lane) * 4));
+            }
+        if (!quad_sync()) return false;
+    }
+
+    // Eq. 7 and the stores of d chunks 2w, 2w + 1 (n-tiles 4w .. 4w + 3)
+    const long long m_o = prm.m_o;
+    const long long half_o = 1ll << (prm.sh_o - 1);
+    const int T = prm.T;
+#pragma unroll
+    for (int cc = 0; cc < 8; ++cc) {
+        if ((cc >> 1) != warp) continue;
+#pragma unroll
+        for (int rr = 0; rr < 2; ++rr) {
+            const int row = wrow0 + g + 8 * rr;
+            if (row >= T) continue;
+            uint32_t w = 0;
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const long long x = m_o * oacc[2 * cc + (e & 1)][2 * rr + (e >> 1)] + half_o;
+                const int o = row < len ? clamp127(x >> prm.sh_o) : 0;
+                w |= (static_cast<uint32_t>(o) & 0xffu) << (8 * e);
+            }
+            *reinterpret_cast<uint32_t *>(prm.out + out_offset(prm, it.b, it.h, row) + 4 * t4 +
+                                          16 * cc) = w;
+        }
+    }
+    return true;
+}
+
 // ------------------------------------------------------------ fused kernel --
 // Persistent: one CTA per resident slot.  The copy warp claims the items in
 // order from a counter in the workspace, so the last items (the halves of
@@ -1040,8 +1314,8 @@ __device__ __forceinline__ bool consume_half(const FusedParams &prm, const Item 
 
 // Zero output rows of a padding item (every row is at or beyond its length).
 __device__ __forceinline__ void zero_rows(const FusedParams &p, const Item &it, int lane) {
-    const int r0 = it.part < 0 ? it.i0 : it.i0 + 32 * it.part;
-    const int nrows = it.part < 0 ? MROWS : 32;
+    const int nrows = MROWS >> it.plog2;
+    const int r0 = it.part < 0 ? it.i0 : it.i0 + nrows * it.part;
     const int rows = (p.T - r0) < nrows ? (p.T - r0) : nrows;
     for (int c = lane; c < rows * (DH / 16); c += 32)
         *reinterpret_cast<int4 *>(p.out + out_offset(p, it.b, it.h, r0 + (c >> 3)) + 16 * (c & 7)) =
@@ -1152,6 +1426,7 @@ __global__ void __launch_bounds__(NTHREADS, 2)
             mbar_init(pair_bar(1), 2);
             mbar_init(R.qfull(), 1);
             mbar_init(R.qempty(), NCWARPS);
+            mbar_init(R.quad(), NCWARPS);
             asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
             asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
         }
@@ -1278,10 +1553,12 @@ __global__ void __launch_bounds__(NTHREADS, 2)
         const uint32_t item = lds32(R.slot(k));
         if (item == NO_ITEM) return;
         const Item it = decode_item(prm, item);
-        const bool ok = it.part < 0
-                            ? consume_whole(prm, it, u0, R, remap, scores, lut, warp, lane)
-                            : consume_half(prm, it, u0, R, remap, scores, lut,
-                                           pair_bar(warp >> 1), warp, lane);
+        const bool ok =
+            it.nparts == 1   ? consume_whole(prm, it, u0, R, remap, scores, lut, warp, lane)
+            : it.nparts == 2 ? consume_half(prm, it, u0, R, remap, scores, lut, pair_bar(warp >> 1),
+                                            warp, lane)
+                             : consume_quarter(prm, it, u0, R, remap, smem_u32(smem + L.remap),
+                                               scores, lut, R.quad(), warp, lane);
         if (!ok) return;
         u0 += 2 * it.nchunks;
     }

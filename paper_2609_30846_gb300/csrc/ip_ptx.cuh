@@ -175,6 +175,14 @@ __device__ __forceinline__ void mma_u8s8(int (&d)[4], const uint32_t (&a)[4], ui
         : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
 }
 
+// D += A B with A 16x16 u8 (row), B 16x8 s8 (col), D 16x8 s32.
+__device__ __forceinline__ void mma_u8s8_k16(int (&d)[4], uint32_t a0, uint32_t a1, uint32_t b0) {
+    asm("mma.sync.aligned.m16n8k16.row.col.s32.u8.s8.s32 {%0,%1,%2,%3}, {%4,%5}, {%6},"
+        " {%0,%1,%2,%3};"
+        : "+r"(d[0]), "+r"(d[1]), "+r"(d[2]), "+r"(d[3])
+        : "r"(a0), "r"(a1), "r"(b0));
+}
+
 // Offset of the 16-byte chunk `chunk` of row `row` in a tile written by TMA
 // with the 128-byte swizzle (rows of 128 bytes, 1024-byte aligned).
 __device__ __forceinline__ uint32_t swz(int row, int chunk) {

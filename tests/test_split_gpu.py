@@ -1,11 +1,12 @@
 """Parity of the tail split with the oracle.
 
 The kernel may do a 64-row tile as two halves of 32 rows whose warp pairs
-split the keys of every chunk and combine their row maxima, exponential
-sums and attn.V partial sums.  Integer arithmetic makes the combination
-exact, so every mode must match the oracle bit for bit: here each case runs
-with no tile split and with every tile split (the planned mode, which
-splits only the last wave, runs in the other parity tests).
+split the keys of every chunk, or as four quarters of 16 rows whose four
+warps split them, and combine their row maxima, exponential sums and attn.V
+partial sums.  Integer arithmetic makes the combination exact, so every mode
+must match the oracle bit for bit: here each case runs with no tile split
+and with every tile split both ways (the planned mode, which splits only the
+last round, runs in the other parity tests).
 """
 import numpy as np
 import pytest
@@ -35,7 +36,7 @@ def orc():
     return oracle
 
 
-@pytest.fixture(params=[0, 1], ids=["whole", "split"])
+@pytest.fixture(params=[0, 1, 2], ids=["whole", "halves", "quarters"])
 def mode(request, ip):
     ip.set_split_mode(request.param)
     yield request.param
@@ -71,16 +72,16 @@ def test_workloads(ip, orc, mode, w):
 
 
 def test_modes_agree_on_the_encoder_layer(ip):
-    # one full encoder layer (B=32, T=375) in all three modes
+    # one full encoder layer (B=32, T=375) in all four modes
     lay = synth.layer(3, 7)
     c = ip.layer_constants(lay.scales)
     outs = []
-    for m in (-1, 0, 1):
+    for m in (-1, 0, 1, 2):
         ip.set_split_mode(m)
         outs.append(run_gpu(ip, lay, c))
     ip.set_split_mode(-1)
-    assert_same(outs[1], outs[0])
-    assert_same(outs[2], outs[0])
+    for o in outs[1:]:
+        assert_same(o, outs[0])
 
 
 @pytest.mark.parametrize("T,masked", [(75, False), (150, True), (375, False)])
@@ -105,7 +106,8 @@ def test_every_tile_split_is_repeatable(ip):
     # stage follows its release closely; a refill that overtook the
     # consumers' shared-memory reads showed up as +-1 differences in a few
     # rows of one in twenty runs.  Forty runs of the encoder layer with every
-    # tile split must all equal the unsplit result.
+    # tile split (twenty in halves, twenty in quarters) must all equal the
+    # unsplit result.
     lay = synth.layer(3, 7)
     c = ip.layer_constants(lay.scales)
     d = lambda a: torch.from_numpy(np.ascontiguousarray(a)).cuda()
@@ -114,12 +116,13 @@ def test_every_tile_split_is_repeatable(ip):
                      device="cuda")
     ip.set_split_mode(0)
     want = ip.relpos_mhsa_i8(q, k, v, p, u, vb, c, workspace=ws).clone()
-    ip.set_split_mode(1)
     out = torch.empty_like(want)
     bad = 0
-    for _ in range(40):
-        ip.relpos_mhsa_i8(q, k, v, p, u, vb, c, out=out, workspace=ws)
-        bad += int(not torch.equal(out, want))
+    for m in (1, 2):
+        ip.set_split_mode(m)
+        for _ in range(20):
+            ip.relpos_mhsa_i8(q, k, v, p, u, vb, c, out=out, workspace=ws)
+            bad += int(not torch.equal(out, want))
     ip.set_split_mode(-1)
     assert ip.status(ws) == 0
     assert bad == 0, f"{bad} of 40 runs differ"

@@ -65,7 +65,7 @@ def test_encoder_layer_with_wide_sums(ip, orc):
     assert_same(run_gpu(ip, lay, c), oracle_out(orc, lay, c))
 
 
-@pytest.mark.parametrize("split", [0, 1])
+@pytest.mark.parametrize("split", [0, 1, 2])
 def test_masks_and_halves_with_wide_sums(ip, orc, split):
     T = 150
     lens = np.array([0, 1, 33, 64, 97, 150, 7, 120], np.int32)
