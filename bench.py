@@ -424,9 +424,25 @@ def measure_next_rows(dev, peak, steps: int, cpu: bool):
         times.append(e0.elapsed_time(e1) * 1e-3)
     if ip.status(blk.ws, stream) != 0:
         raise SystemExit("conformer block: a kernel reported an error")
+    t_eager = statistics.median(times)
+    # the same nineteen launches captured once into a CUDA graph and replayed
+    graph = blk.graph(x)
+    times = []
+    for _ in range(steps):
+        flush()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        graph.replay()
+        e1.record(stream)
+        e1.synchronize()
+        times.append(e0.elapsed_time(e1) * 1e-3)
+    torch.cuda.synchronize(dev)
+    if ip.status(blk.ws, stream) != 0:
+        raise SystemExit("conformer block (graph): a kernel reported an error")
     t = statistics.median(times)
     ops = blk.useful_ops()
     row = {"value": ops / t / 1e12, "unit": "TOPS", "us_per_block": t * 1e6,
+           "us_per_block_eager": t_eager * 1e6, "launch": "CUDA graph replay",
            "frames_per_s": B * T / t, "shape": {"B": B, "T": T, "d": 1024, "ff": 4096, "heads": 8},
            "roofline": {"bound": "tensor", "achieved": ops / t / 1e12, "peak": peak,
                         "unit": "TOPS", "frac": ops / t / 1e12 / peak, "traffic": None},

@@ -9,7 +9,9 @@ offline helpers from the declared grids:
                                                    + BatchNorm (INT16) + Swish, pointwise, residual
   H  = LN5(Z3 + 1/2 FFN2(LN4(Z3)))        (Eq. 4)
 
-Nineteen launches on one stream, all of them CUDA kernels of this library.
+Nineteen launches on one stream, all of them CUDA kernels of this library;
+`ConformerBlock.graph` captures them into a CUDA graph that replays with no
+host work per launch.
 The parameter object carries int8 weights with per-channel grids, real
 LayerNorm parameters and the activation grids (attributes as
 `synth.block.BlockCase`).
@@ -123,6 +125,26 @@ class ConformerBlock:
         residual_i8(z[2], f, *self.res[3], out=z[3], stream=st)
         ln("ln5", z[3], self.out)
         return self.out
+
+    def graph(self, x, warmup: int = 2):
+        """Captures the block's nineteen launches on `x` (a fixed int8 [B, T,
+        D] CUDA tensor) into a CUDA graph and returns it: `g.replay()` runs
+        the block again on whatever `x` then holds, with no host work per
+        launch.  The eager call runs `warmup` times first, so that the
+        library's one-time set-up (kernel attributes, occupancy queries) is
+        done outside the capture."""
+        import torch
+        side = torch.cuda.Stream(x.device)
+        side.wait_stream(torch.cuda.current_stream(x.device))
+        with torch.cuda.stream(side):
+            for _ in range(warmup):
+                self(x, stream=side)
+        torch.cuda.current_stream(x.device).wait_stream(side)
+        torch.cuda.synchronize(x.device)
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            self(x, stream=torch.cuda.current_stream(x.device))
+        return g
 
     def useful_ops(self) -> float:
         """Integer multiply-adds x 2 of the block's contractions (projections,

@@ -31,3 +31,26 @@ def test_block_matches_oracle(ip, B, T, seed):
     got = got.cpu().numpy()
     bad = got != want
     assert not bad.any(), f"{int(bad.sum())} of {got.size} outputs differ"
+
+
+def test_block_graph_replay_matches_oracle(ip):
+    # the nineteen launches captured once into a CUDA graph; each replay on a
+    # new input equals the oracle's block on that input
+    import synth.block as sb
+    from oracle.block import conformer_block as oracle_block
+    from paper_2609_30846_gb300.block import ConformerBlock
+    B, T = 2, 100
+    cases = [sb.conformer_block(B, T, seed=s) for s in (11, 12)]
+    blk = ConformerBlock(cases[0], B, T, torch.device("cuda"))
+    x = torch.from_numpy(cases[0].x).cuda()
+    g = blk.graph(x)
+    for case in cases:
+        # same weights and grids, new frames
+        x.copy_(torch.from_numpy(case.x).cuda())
+        g.replay()
+        torch.cuda.synchronize()
+        want = oracle_block(sb.BlockCase(**{**cases[0].__dict__, "x": case.x}))
+        got = blk.out.cpu().numpy()
+        bad = got != want
+        assert not bad.any(), f"{int(bad.sum())} of {got.size} outputs differ"
+    assert ip.status(blk.ws) == 0
