@@ -4,6 +4,7 @@
 // ip_block_kernels.cuh.
 #include "ip_mhsa.h"
 #include "ip_block_kernels.cuh"
+#include "ip_host_util.h"
 
 #include <cuda_runtime.h>
 
@@ -61,8 +62,10 @@ int ip_residual_i8(const int8_t *x, const int8_t *y, long long n, int32_t m_x, i
     long long blocks = (vec + ipb::RES_THREADS - 1) / ipb::RES_THREADS;
     const long long cap = static_cast<long long>(nsm) * 8;
     blocks = blocks < cap ? blocks : cap;
-    ipb::residual_i8_kernel<<<static_cast<unsigned>(blocks), ipb::RES_THREADS, 0,
-                              reinterpret_cast<cudaStream_t>(stream)>>>(p);
+    if (iph::launch_pdl(ipb::residual_i8_kernel, dim3(static_cast<unsigned>(blocks)),
+                        dim3(ipb::RES_THREADS), 0, reinterpret_cast<cudaStream_t>(stream), p) !=
+        cudaSuccess)
+        return IP_ERR_CUDA;
     return cudaGetLastError() == cudaSuccess ? IP_OK : IP_ERR_CUDA;
 }
 
@@ -99,7 +102,9 @@ int ip_dwconv_swish_i8(const int8_t *x, int B, int T, int C, const int8_t *w, in
     p.err = static_cast<int *>(workspace);
     const dim3 grid((C + ipb::DW_THREADS - 1) / ipb::DW_THREADS,
                     (T + ipb::DW_FRAMES - 1) / ipb::DW_FRAMES, B);
-    ipb::dwconv_swish_kernel<<<grid, ipb::DW_THREADS, 0, reinterpret_cast<cudaStream_t>(stream)>>>(p);
+    if (iph::launch_pdl(ipb::dwconv_swish_kernel, grid, dim3(ipb::DW_THREADS), 0,
+                        reinterpret_cast<cudaStream_t>(stream), p) != cudaSuccess)
+        return IP_ERR_CUDA;
     return cudaGetLastError() == cudaSuccess ? IP_OK : IP_ERR_CUDA;
 }
 

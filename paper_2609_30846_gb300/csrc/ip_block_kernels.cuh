@@ -37,6 +37,8 @@ __device__ __forceinline__ int residual_one(int x, int y, const ResidualParams &
 }
 
 __global__ void __launch_bounds__(RES_THREADS) residual_i8_kernel(const ResidualParams p) {
+    pdl_launch_dependents();
+    pdl_wait();   // the grid before this one on the stream: complete, memory visible
     const long long nv = p.n >> 4;   // 16-byte vectors
     const long long stride = static_cast<long long>(gridDim.x) * RES_THREADS;
     for (long long i = static_cast<long long>(blockIdx.x) * RES_THREADS + threadIdx.x; i < nv;
@@ -101,6 +103,8 @@ __device__ __forceinline__ int swish16(int z, const DwParams &p) {
 // the Swish onto int8.  Thread: one channel; CTA: 256 channels x DW_FRAMES
 // frames of one utterance, a sliding window of K input frames in registers.
 __global__ void __launch_bounds__(DW_THREADS) dwconv_swish_kernel(const DwParams p) {
+    pdl_launch_dependents();
+    pdl_wait();   // the grid before this one on the stream: complete, memory visible
     const int c = blockIdx.x * DW_THREADS + threadIdx.x;
     const int t0 = blockIdx.y * DW_FRAMES;
     const int b = blockIdx.z;

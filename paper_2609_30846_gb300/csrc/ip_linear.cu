@@ -163,13 +163,17 @@ int linear_launch(const int8_t *x, int x_layout, const int8_t *w, const int32_t 
     const unsigned grid = prm.ntiles < static_cast<unsigned>(nsm) ? prm.ntiles
                                                                   : static_cast<unsigned>(nsm);
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    cudaError_t lrc;
     if (epi == ipl::EPI_SWISH)
-        ipl::linear_i8_kernel<ipl::EPI_SWISH><<<grid, ipl::THREADS, ipl::SMEM_LAUNCH, st>>>(tm_x, tm_w, prm);
+        lrc = iph::launch_pdl(ipl::linear_i8_kernel<ipl::EPI_SWISH>, dim3(grid), dim3(ipl::THREADS),
+                              ipl::SMEM_LAUNCH, st, tm_x, tm_w, prm);
     else if (epi == ipl::EPI_GLU)
-        ipl::linear_i8_kernel<ipl::EPI_GLU><<<grid, ipl::THREADS, ipl::SMEM_LAUNCH, st>>>(tm_x, tm_w, prm);
+        lrc = iph::launch_pdl(ipl::linear_i8_kernel<ipl::EPI_GLU>, dim3(grid), dim3(ipl::THREADS),
+                              ipl::SMEM_LAUNCH, st, tm_x, tm_w, prm);
     else
-        ipl::linear_i8_kernel<ipl::EPI_PLAIN><<<grid, ipl::THREADS, ipl::SMEM_LAUNCH, st>>>(tm_x, tm_w, prm);
-    if (cudaGetLastError() != cudaSuccess) return IP_ERR_CUDA;
+        lrc = iph::launch_pdl(ipl::linear_i8_kernel<ipl::EPI_PLAIN>, dim3(grid), dim3(ipl::THREADS),
+                              ipl::SMEM_LAUNCH, st, tm_x, tm_w, prm);
+    if (lrc != cudaSuccess || cudaGetLastError() != cudaSuccess) return IP_ERR_CUDA;
     return IP_OK;
 }
 

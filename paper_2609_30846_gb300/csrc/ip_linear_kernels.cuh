@@ -141,6 +141,7 @@ __global__ void __launch_bounds__(THREADS, 1)
 
     const uint32_t lut = base + SMEM_LUT;
     const uint8_t *swish_lut = smem + SMEM_LUT;
+    pdl_launch_dependents();
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
             mbar_init(full_bar(s), 1);
@@ -155,6 +156,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         const uint32_t y = static_cast<uint32_t>(swish_i8(z, prm)) & 0xffu;
         asm volatile("st.shared.u8 [%0], %1;" ::"r"(lut + threadIdx.x), "r"(y) : "memory");
     }
+    pdl_wait();   // the grid before this one on the stream: complete, memory visible
     __syncthreads();
 
     // ---------------------------------------------------------- producer

@@ -257,18 +257,8 @@ int ip_relpos_mhsa_i8_ex(const int8_t *q, const int8_t *k, const int8_t *v, cons
     // Programmatic dependent launch: this grid may be scheduled while the
     // kernel before it on the stream finishes (the kernel waits for that
     // grid before its first global access, so the order of the two is kept).
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(ip.grid);
-    cfg.blockDim = dim3(ipk::NTHREADS);
-    cfg.dynamicSmemBytes = static_cast<size_t>(smem);
-    cfg.stream = st;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[0].val.programmaticStreamSerializationAllowed = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    if (cudaLaunchKernelEx(&cfg, ipk::relpos_mhsa_fused_kernel, tm_q, tm_k, tm_v, tm_p, prm) !=
-        cudaSuccess)
+    if (iph::launch_pdl(ipk::relpos_mhsa_fused_kernel, dim3(ip.grid), dim3(ipk::NTHREADS),
+                        static_cast<size_t>(smem), st, tm_q, tm_k, tm_v, tm_p, prm) != cudaSuccess)
         return IP_ERR_CUDA;
     if (cudaGetLastError() != cudaSuccess) return IP_ERR_CUDA;
     return IP_OK;

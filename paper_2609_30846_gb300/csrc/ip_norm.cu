@@ -3,6 +3,7 @@
 // Device code: ip_norm_kernels.cuh.
 #include "ip_mhsa.h"
 #include "ip_norm_kernels.cuh"
+#include "ip_host_util.h"
 
 #include <cuda_runtime.h>
 
@@ -53,7 +54,9 @@ int launch(const ipn::NormParams &prm, int nsm, cudaStream_t st) {
     const long long cap = resident<C>(nsm);
     if (cap <= 0) return IP_ERR_CUDA;
     const unsigned grid = static_cast<unsigned>(batches < cap ? batches : cap);
-    ipn::layernorm_i8_kernel<C><<<grid, ipn::THREADS, C * 8192, st>>>(prm);
+    if (iph::launch_pdl(ipn::layernorm_i8_kernel<C>, dim3(grid), dim3(ipn::THREADS), C * 8192, st,
+                        prm) != cudaSuccess)
+        return IP_ERR_CUDA;
     return cudaGetLastError() == cudaSuccess ? IP_OK : IP_ERR_CUDA;
 }
 

@@ -214,6 +214,8 @@ __global__ void __launch_bounds__(THREADS)
 
     Batch<C> bt;
     const bool first = grp < groups;
+    pdl_launch_dependents();
+    pdl_wait();   // the grid before this one on the stream: complete, memory visible
     if (first) {
         const long long row0 = grp * NB;
         pass_a<C>(prm, row0, prm.rows - row0 < NB ? static_cast<int>(prm.rows - row0) : NB, lane, bt);

@@ -183,6 +183,15 @@ __device__ __forceinline__ void mma_u8s8_k16(int (&d)[4], uint32_t a0, uint32_t 
         : "r"(a0), "r"(a1), "r"(b0));
 }
 
+// Programmatic dependent launch: let the next launch on the stream be
+// scheduled now (its CTAs take the SM slots this grid frees), and wait for
+// the grid before this one on the stream to complete, with its memory
+// visible, before the first global access.
+__device__ __forceinline__ void pdl_launch_dependents() {
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 // Offset of the 16-byte chunk `chunk` of row `row` in a tile written by TMA
 // with the 128-byte swizzle (rows of 128 bytes, 1024-byte aligned).
 __device__ __forceinline__ uint32_t swz(int row, int chunk) {

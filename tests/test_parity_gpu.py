@@ -202,3 +202,23 @@ def test_work_counters_return_to_zero(ip, orc):
         assert not counters.any(), counters.nonzero()
         assert_same(out.cpu().numpy(), want)
     assert ip.status(ws) == 0
+
+
+def test_back_to_back_launches_see_the_previous_output(ip, orc):
+    # Each launch may be scheduled while the one before it on the stream
+    # finishes (programmatic dependent launch) and must wait for it before
+    # reading memory: a second call that takes the first call's output as
+    # its Q, K and V, issued right behind it, must see that output complete.
+    lay = synth.layer(3, 9)
+    c = ip.layer_constants(lay.scales)
+    B, H, T, dh = lay.q.shape
+    ws = torch.zeros(ip.workspace_bytes(B, H, T, dh), dtype=torch.uint8, device="cuda")
+    first = ip.relpos_mhsa_i8(_dev(lay.q), _dev(lay.k), _dev(lay.v), _dev(lay.p), _dev(lay.u),
+                              _dev(lay.vb), c, workspace=ws)
+    second = ip.relpos_mhsa_i8(first, first, first, _dev(lay.p), _dev(lay.u), _dev(lay.vb), c,
+                               workspace=ws)
+    assert ip.status(ws) == 0
+    want1 = oracle_out(orc, lay, c)
+    assert_same(first.cpu().numpy(), want1)
+    lay2 = synth.Layer(want1, want1, want1, lay.p, lay.u, lay.vb, None, lay.scales)
+    assert_same(second.cpu().numpy(), oracle_out(orc, lay2, c))
