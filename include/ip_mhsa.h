@@ -92,7 +92,9 @@ size_t ip_relpos_mhsa_workspace_bytes(int B, int H, int T, int dh);
  *                 [0, T]), or NULL for all T.
  *   workspace   : device memory of workspace_bytes >= the size above,
  *                 256-byte aligned, owned by the caller; one call at a time
- *                 per workspace.
+ *                 per workspace.  NULL: the workspace registered with
+ *                 ip_set_workspace (IP_ERR_NULL if there is none, or
+ *                 IP_ERR_WORKSPACE if it is smaller than the call needs).
  * The call validates its arguments on the host and then enqueues one
  * kernel on `stream` (a persistent grid of one CTA per resident slot that
  * walks the 64-row query tiles of all (b, h)).  B == 0 or H == 0 is an empty problem: the call
@@ -107,8 +109,19 @@ int ip_relpos_mhsa_i8(const int8_t *q, const int8_t *k, const int8_t *v,
 
 /* Synchronises `stream`, reports the device-side status of the calls that
  * used `workspace` since the previous status call (IP_OK, IP_ERR_TIMEOUT,
- * or IP_ERR_CUDA) and clears it. */
+ * or IP_ERR_CUDA) and clears it.  workspace = NULL: the one registered with
+ * ip_set_workspace (IP_ERR_NULL if there is none). */
 int ip_relpos_mhsa_status(const void *workspace, ip_stream_t stream);
+
+/* Registers a default workspace for the attention calls of this process
+ * that pass a NULL workspace: device memory of `bytes` (at least
+ * ip_relpos_mhsa_workspace_bytes), 256-byte aligned, zero-filled once by the
+ * caller and owned by it until it is replaced or released.  ptr = NULL
+ * releases the registration.  Since calls that share a workspace must not
+ * overlap on the GPU, the default suits callers that issue their attention
+ * calls on one stream.  IP_ERR_ALIGN for a misaligned ptr,
+ * IP_ERR_WORKSPACE if bytes is too small. */
+int ip_set_workspace(void *ptr, size_t bytes);
 
 /* Bytes of device staging memory ip_relpos_mhsa_i8_host needs (inputs,
  * output, lengths and workspace), 0 if the shape is invalid. */

@@ -34,6 +34,7 @@ EXPORTS = (
     "ip_layernorm_i8", "ip_layernorm_constants", "ip_relpos_mhsa_i8_ex", "ip_residual_i8",
     "ip_residual_params", "ip_linear_glu_i8", "ip_glu_params", "ip_dwconv_swish_i8",
     "ip_swish16_params_from_scales", "ip_relpos_mhsa_i8_host_async", "ip_relpos_mhsa_host_status",
+    "ip_set_workspace",
 )
 
 ROWS = 0    # IP_LAYOUT_ROWS:  [B][T][C]
@@ -102,6 +103,8 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
         lib.ip_relpos_mhsa_i8_noalloc.restype = I
         lib.ip_relpos_mhsa_status.argtypes = [P, P]
         lib.ip_relpos_mhsa_status.restype = I
+        lib.ip_set_workspace.argtypes = [P, ctypes.c_size_t]
+        lib.ip_set_workspace.restype = I
         lib.ip_strerror.argtypes = [I]
         lib.ip_strerror.restype = ctypes.c_char_p
         lib.ip_debug_set_timeout_cycles.argtypes = [ctypes.c_longlong]
@@ -289,13 +292,16 @@ def relpos_mhsa_i8(q, k, v, p, u, v_bias, consts: LayerConstants, lengths=None, 
     if out is None:
         out = torch.empty(oshp, dtype=torch.int8, device=q.device)
     lens = None if lengths is None else _dev_ptr(lengths, "lengths", torch.int32, (B,))
-    if workspace is None:
+    if workspace is None and _default_workspace is None:
         workspace = torch.zeros(workspace_bytes(B, H, T, dh), dtype=torch.uint8, device=q.device)
+    # workspace None here: the library uses the registered default workspace
+    ws_ptr = None if workspace is None else ctypes.c_void_p(workspace.data_ptr())
+    ws_len = 0 if workspace is None else workspace.numel()
     sm = SoftmaxParams(*consts.softmax)
     rc = load().ip_relpos_mhsa_i8_ex(
         *args, _arr(consts.multipliers, ctypes.c_int32), _arr(consts.shifts, ctypes.c_int32),
         ctypes.byref(sm), lens, B, H, T, dh, _dev_ptr(out, "out", torch.int8, oshp), out_layout,
-        ctypes.c_void_p(workspace.data_ptr()), workspace.numel(), _stream_handle(stream))
+        ws_ptr, ws_len, _stream_handle(stream))
     _check("ip_relpos_mhsa_i8_ex", rc)
     return out
 
@@ -325,10 +331,34 @@ def int8_mma_peak_tops(iters: int = 4096, repeats: int = 3) -> float:
     return best
 
 
-def status(workspace, stream=None) -> int:
+def status(workspace=None, stream=None) -> int:
     """Synchronises the stream and returns the device-side status code of
-    the last call that used `workspace` (0 = ok)."""
-    return load().ip_relpos_mhsa_status(ctypes.c_void_p(workspace.data_ptr()), _stream_handle(stream))
+    the last call that used `workspace` (0 = ok); None: the default
+    workspace registered by set_workspace."""
+    ptr = None if workspace is None else ctypes.c_void_p(workspace.data_ptr())
+    return load().ip_relpos_mhsa_status(ptr, _stream_handle(stream))
+
+
+_default_workspace = None
+
+
+def set_workspace(workspace) -> None:
+    """Registers `workspace` (a zero-filled uint8 CUDA tensor of at least
+    workspace_bytes(...) bytes) as the default of the attention calls that
+    pass none; None releases it.  The binding keeps the tensor alive while
+    it is registered.  Calls that share it must run on one stream."""
+    global _default_workspace
+    if workspace is None:
+        _check("ip_set_workspace", load().ip_set_workspace(None, 0))
+        _default_workspace = None
+        return
+    import torch
+    if not (isinstance(workspace, torch.Tensor) and workspace.is_cuda and
+            workspace.dtype == torch.uint8 and workspace.is_contiguous()):
+        raise TypeError("workspace: a contiguous uint8 CUDA tensor")
+    _check("ip_set_workspace", load().ip_set_workspace(ctypes.c_void_p(workspace.data_ptr()),
+                                                       workspace.numel()))
+    _default_workspace = workspace
 
 
 def linear_constants(s_x: float, s_w, s_y):
@@ -575,5 +605,5 @@ __all__ = ["build", "load", "relpos_mhsa_i8", "relpos_mhsa_i8_host", "status", "
            "linear_constants", "ROWS", "HEADS", "linear_swish_i8", "swish_params_from_scales",
            "layernorm_i8", "layernorm_constants", "NormConstants", "residual_i8",
            "residual_params", "linear_glu_i8", "glu_params", "dwconv_swish_i8", "swish16_params",
-           "host_status",
+           "host_status", "set_workspace",
            "IpError", "LibraryError", "EXPORTS"]

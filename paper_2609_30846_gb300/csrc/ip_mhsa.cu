@@ -21,6 +21,10 @@ long long g_timeout_cycles = DEFAULT_TIMEOUT;
 int g_stall_injection = 0;
 int g_split_mode = -1;   // -1 planned, 0 never, 1 / 2: every tile in halves / quarters (test hook)
 int g_wide_sums = 0;     // 1: general softmax arithmetic always (test hook)
+// the default workspace registered by ip_set_workspace
+std::mutex g_ws_mu;
+void *g_ws_ptr = nullptr;
+size_t g_ws_bytes = 0;
 
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
@@ -179,6 +183,11 @@ int ip_relpos_mhsa_i8_ex(const int8_t *q, const int8_t *k, const int8_t *v, cons
     int rc = check_shape(B, H, T, dh);
     if (rc != IP_OK) return rc;
     if (B == 0 || H == 0) return IP_OK;   // empty problem: nothing to read or write
+    if (workspace == nullptr) {
+        std::lock_guard<std::mutex> lock(g_ws_mu);
+        workspace = g_ws_ptr;
+        workspace_bytes = g_ws_bytes;
+    }
     if (!q || !k || !v || !p || !u || !v_bias || !multipliers || !shifts || !sm || !out ||
         !workspace)
         return IP_ERR_NULL;
@@ -264,7 +273,22 @@ int ip_relpos_mhsa_i8_ex(const int8_t *q, const int8_t *k, const int8_t *v, cons
     return IP_OK;
 }
 
+int ip_set_workspace(void *ptr, size_t bytes) {
+    if (ptr != nullptr) {
+        if (!aligned(ptr, 256)) return IP_ERR_ALIGN;
+        if (bytes < ws_bytes()) return IP_ERR_WORKSPACE;
+    }
+    std::lock_guard<std::mutex> lock(g_ws_mu);
+    g_ws_ptr = ptr;
+    g_ws_bytes = ptr != nullptr ? bytes : 0;
+    return IP_OK;
+}
+
 int ip_relpos_mhsa_status(const void *workspace, ip_stream_t stream) {
+    if (workspace == nullptr) {
+        std::lock_guard<std::mutex> lock(g_ws_mu);
+        workspace = g_ws_ptr;
+    }
     if (!workspace) return IP_ERR_NULL;
     int word = 0;
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);

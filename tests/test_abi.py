@@ -94,6 +94,29 @@ def test_validation_codes(lib):
     assert _call(lib, H=0, ws=None) == 0
 
 
+def test_default_workspace_registration(lib):
+    # ip_set_workspace validates without touching the device; a call that
+    # passes no workspace takes the registered one (it then fails only on
+    # the bad multiplier below, past every pointer check) and, with none
+    # registered, reports the missing pointer.
+    buf = (ctypes.c_byte * 1024)()
+    base = (ctypes.addressof(buf) + 255) // 256 * 256
+    bad_mult = (ctypes.c_int32 * 3)(-1, 0, 0)
+    try:
+        assert lib.ip_set_workspace(base + 16, 512) == -3
+        assert lib.ip_set_workspace(base, 16) == -8
+        assert _call(lib, ws=None, mult=bad_mult) == -1
+        assert lib.ip_relpos_mhsa_status(None, None) == -1
+        assert lib.ip_set_workspace(base, 512) == 0
+        assert _call(lib, ws=None, mult=bad_mult) == -7
+        assert _call(lib, ws=None, sm=None) == -1
+        # an explicit workspace still wins over the registered one
+        assert _call(lib, ws=base + 16, mult=bad_mult) == -3
+    finally:
+        assert lib.ip_set_workspace(None, 0) == 0
+    assert _call(lib, ws=None, mult=bad_mult) == -1
+
+
 def test_constants_match_oracle(lib):
     import oracle
     rng = np.random.default_rng(0)

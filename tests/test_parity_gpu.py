@@ -204,6 +204,28 @@ def test_work_counters_return_to_zero(ip, orc):
     assert ip.status(ws) == 0
 
 
+def test_default_workspace(ip, orc):
+    # A workspace registered with ip_set_workspace serves the calls that
+    # pass none, its status reads back through a NULL workspace, and its
+    # item counters return to zero like an explicit workspace's.
+    lay = synth.layer(3, 4)
+    c = ip.layer_constants(lay.scales)
+    B, H, T, dh = lay.q.shape
+    ws = torch.zeros(ip.workspace_bytes(B, H, T, dh), dtype=torch.uint8, device="cuda")
+    args = [_dev(a) for a in (lay.q, lay.k, lay.v, lay.p, lay.u, lay.vb)]
+    want = oracle_out(orc, lay, c)
+    ip.set_workspace(ws)
+    try:
+        for _ in range(2):
+            out = ip.relpos_mhsa_i8(*args, c)
+            assert ip.status() == 0
+            assert not ws.cpu().numpy().any()
+            assert_same(out.cpu().numpy(), want)
+    finally:
+        ip.set_workspace(None)
+    assert ip.status() == -1   # IP_ERR_NULL: nothing registered
+
+
 def test_back_to_back_launches_see_the_previous_output(ip, orc):
     # Each launch may be scheduled while the one before it on the stream
     # finishes (programmatic dependent launch) and must wait for it before
