@@ -170,19 +170,38 @@ def job_tops(ops_per_rank: float, world: int, seconds: float) -> float:
     return ops_per_rank * world / seconds / 1e12
 
 
-def traffic_per_launch():
-    """DRAM bytes per fused-kernel launch from the committed ncu summary,
-    if it was taken on the current kernel source (else None)."""
+def _counters():
+    """The committed ncu counters of the fused kernel, if they were taken on
+    the current kernel source (else an empty dict)."""
     if not os.path.exists(TRAFFIC_FILE):
-        return None
+        return {}
     try:
         rec = json.load(open(TRAFFIC_FILE))
         src = hashlib.sha256(open(KERNEL_SRC, "rb").read()).hexdigest()
-        if rec.get("kernel_sha256") != src:
-            return None
-        return rec.get("dram_bytes_per_launch")
+        return rec if rec.get("kernel_sha256") == src else {}
     except (OSError, ValueError):
+        return {}
+
+
+def traffic_per_launch():
+    """DRAM bytes per fused-kernel launch from the committed ncu summary,
+    if it was taken on the current kernel source (else None)."""
+    return _counters().get("dram_bytes_per_launch")
+
+
+def issue_floor(dev, launch_us: float, sm_mhz: float):
+    """The ALU bound of the fused kernel: its issued warp instructions per
+    launch (committed ncu count on the current source) at one instruction
+    per SM sub-partition per cycle (4 per SM) and the SM clock of the run,
+    against the measured launch time."""
+    inst = _counters().get("smsp_inst_executed_per_launch")
+    if not inst or launch_us <= 0 or sm_mhz <= 0:
         return None
+    import torch
+    nsm = torch.cuda.get_device_properties(dev).multi_processor_count
+    floor_us = inst / (nsm * 4 * sm_mhz)
+    return {"inst_per_launch": inst, "floor_us": floor_us, "frac": floor_us / launch_us,
+            "basis": "issued warp instructions / (SMs x 4 sub-partitions x SM clock)"}
 
 
 # ------------------------------------------------------------------- oracle arm
@@ -557,6 +576,7 @@ def run_ours(args):
                 raise ip.IpError("ip_relpos_mhsa_i8", rc, ip.strerror(rc))
 
     peak = ip.int8_mma_peak_tops()
+    pipes = ip.int8_pipe_rates()
     for _ in range(max(args.warmup, 3)):
         step()
     if ip.status(ws, stream) != 0:
@@ -667,6 +687,12 @@ def run_ours(args):
                      "peak_source": "measured in this run: integer warp MMA (mma.sync m16n8k32 "
                                     "s8) probe, CUDA events; sm_103a has no tcgen05 kind::i8",
                      "hbm_floor_frac": (bytes_layer / (HBM_GBS * 1e9)) / (avg_layer_ms * 1e-3),
+                     "alu_floor": issue_floor(dev, avg_layer_ms * 1e3,
+                                              (clk or {}).get("sm_mhz") or 2070.0),
+                     "integer_pipes_tops": pipes,
+                     "integer_pipes_note": "measured in this run: the integer MMA pipe and the "
+                                           "dp4a pipe alone and together (ip_probe_int8_mix); "
+                                           "the fused kernel's contractions use the MMA pipe",
                      "kernel": "relpos_mhsa_fused_kernel (one launch per layer)"},
         "cpu_baseline": cpu,
         "e2e": e2e,

@@ -29,7 +29,9 @@
  *   q, k, v, out : [B][H][T][dh]      p : [H][2T-1][dh]      u, v_bias : [H][dh]
  * Ownership: every buffer belongs to the caller; the library allocates no
  * memory.  Device entry points are asynchronous on `stream`; inputs are not
- * modified.  Return value: IP_OK (0) or a negative IP_ERR_* code
+ * modified.  The attention calls keep the TMA descriptors of the last 32
+ * (pointer, shape) pairs they saw; a descriptor holds nothing but the
+ * address and the shape, so one stays valid for any buffer at that address.  Return value: IP_OK (0) or a negative IP_ERR_* code
  * (ip_strerror gives its text); the library never aborts the process.
  */
 #ifndef IP_MHSA_H
@@ -416,6 +418,14 @@ int ip_debug_set_wide_sums(int on);
  * performs (one multiply-add = 2), or -1 on error.  Timing it with events
  * gives the measured INT8 peak of this GPU. */
 long long ip_probe_int8_mma(int blocks, int iters, int *sink, ip_stream_t stream);
+
+/* Diagnostic: the two integer pipes at once.  In each block of 256 threads
+ * the first mma_warps (0..8) warps run four integer-MMA chains for `iters`
+ * rounds and the other warps eight dp4a chains for 4 iters rounds of four;
+ * sink as above.  Returns the integer ops of the launch (both kinds), or -1
+ * on error.  mma_warps = 0 gives the dp4a rate alone; a launch time close
+ * to that of the MMA warps alone shows the two pipes working concurrently. */
+long long ip_probe_int8_mix(int blocks, int iters, int mma_warps, int *sink, ip_stream_t stream);
 
 /* ---- offline constants (host only, float64, run once per layer) -------- */
 

@@ -34,7 +34,7 @@ EXPORTS = (
     "ip_layernorm_i8", "ip_layernorm_constants", "ip_relpos_mhsa_i8_ex", "ip_residual_i8",
     "ip_residual_params", "ip_linear_glu_i8", "ip_glu_params", "ip_dwconv_swish_i8",
     "ip_swish16_params_from_scales", "ip_relpos_mhsa_i8_host_async", "ip_relpos_mhsa_host_status",
-    "ip_set_workspace",
+    "ip_set_workspace", "ip_probe_int8_mix",
 )
 
 ROWS = 0    # IP_LAYOUT_ROWS:  [B][T][C]
@@ -159,6 +159,8 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
         lib.ip_swish16_params_from_scales.restype = I
         lib.ip_probe_int8_mma.argtypes = [I, I, P, P]
         lib.ip_probe_int8_mma.restype = ctypes.c_longlong
+        lib.ip_probe_int8_mix.argtypes = [I, I, I, P, P]
+        lib.ip_probe_int8_mix.restype = ctypes.c_longlong
         _lib = lib
         return lib
 
@@ -329,6 +331,35 @@ def int8_mma_peak_tops(iters: int = 4096, repeats: int = 3) -> float:
             raise IpError("ip_probe_int8_mma", -5, "launch failed")
         best = max(best, ops / (e0.elapsed_time(e1) * 1e-3) / 1e12)
     return best
+
+
+def int8_pipe_rates(iters: int = 2048, repeats: int = 3) -> dict:
+    """Measured integer throughput (TOPS, best of `repeats` launches, CUDA
+    events) of the integer MMA pipe alone, the dp4a pipe alone, and both at
+    once (half the warps on each)."""
+    import torch
+    props = torch.cuda.get_device_properties(torch.cuda.current_device())
+    blocks = props.multi_processor_count * 2
+    sink = torch.empty(blocks * 256, dtype=torch.int32, device="cuda")
+    st = torch.cuda.current_stream()
+    lib = load()
+    h = ctypes.c_void_p(st.cuda_stream)
+    out = {}
+    for name, mw in (("imma", 8), ("dp4a", 0), ("imma_plus_dp4a", 4)):
+        lib.ip_probe_int8_mix(blocks, iters, mw, ctypes.c_void_p(sink.data_ptr()), h)   # warm-up
+        best = 0.0
+        for _ in range(repeats):
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record(st)
+            ops = lib.ip_probe_int8_mix(blocks, iters, mw, ctypes.c_void_p(sink.data_ptr()), h)
+            e1.record(st)
+            e1.synchronize()
+            if ops < 0:
+                raise IpError("ip_probe_int8_mix", -5, "launch failed")
+            best = max(best, ops / (e0.elapsed_time(e1) * 1e-3) / 1e12)
+        out[name] = best
+    return out
 
 
 def status(workspace=None, stream=None) -> int:
@@ -605,5 +636,5 @@ __all__ = ["build", "load", "relpos_mhsa_i8", "relpos_mhsa_i8_host", "status", "
            "linear_constants", "ROWS", "HEADS", "linear_swish_i8", "swish_params_from_scales",
            "layernorm_i8", "layernorm_constants", "NormConstants", "residual_i8",
            "residual_params", "linear_glu_i8", "glu_params", "dwconv_swish_i8", "swish16_params",
-           "host_status", "set_workspace",
+           "host_status", "set_workspace", "int8_pipe_rates",
            "IpError", "LibraryError", "EXPORTS"]

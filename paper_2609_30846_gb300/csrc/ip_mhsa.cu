@@ -85,6 +85,41 @@ bool make_map(CUtensorMap *m, const void *base, unsigned long long d1, unsigned 
               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// Encoded maps of recent calls, keyed by base pointer and shape (a map
+// depends on nothing else), so that calls on the same buffers skip the
+// encoding; a small table with round-robin replacement.
+struct MapEntry {
+    const void *base;
+    unsigned long long d1, d2;
+    unsigned rows;
+    bool used;
+    CUtensorMap map;
+};
+constexpr int MAP_CACHE = 32;
+std::mutex g_map_mu;
+MapEntry g_maps[MAP_CACHE];
+int g_map_next = 0;
+
+bool cached_map(CUtensorMap *m, const void *base, unsigned long long d1, unsigned long long d2,
+                unsigned rows) {
+    std::lock_guard<std::mutex> lock(g_map_mu);
+    for (const MapEntry &e : g_maps)
+        if (e.used && e.base == base && e.d1 == d1 && e.d2 == d2 && e.rows == rows) {
+            *m = e.map;
+            return true;
+        }
+    if (!make_map(m, base, d1, d2, rows)) return false;
+    MapEntry &e = g_maps[g_map_next];
+    g_map_next = (g_map_next + 1) % MAP_CACHE;
+    e.base = base;
+    e.d1 = d1;
+    e.d2 = d2;
+    e.rows = rows;
+    e.used = true;
+    e.map = *m;
+    return true;
+}
+
 std::mutex g_attr_mu;
 int g_attr_smem[64] = {0};
 
@@ -211,8 +246,8 @@ int ip_relpos_mhsa_i8_ex(const int8_t *q, const int8_t *k, const int8_t *v, cons
 
     CUtensorMap tm_q, tm_k, tm_v, tm_p;
     const unsigned long long bh = static_cast<unsigned long long>(B) * H;
-    if (!make_map(&tm_q, q, T, bh, ipk::MROWS) || !make_map(&tm_k, k, T, bh, ipk::NK) || !make_map(&tm_v, v, T, bh, ipk::NK) ||
-        !make_map(&tm_p, p, 2ull * T - 1, H, ipk::BAND_ROWS))
+    if (!cached_map(&tm_q, q, T, bh, ipk::MROWS) || !cached_map(&tm_k, k, T, bh, ipk::NK) ||
+        !cached_map(&tm_v, v, T, bh, ipk::NK) || !cached_map(&tm_p, p, 2ull * T - 1, H, ipk::BAND_ROWS))
         return IP_ERR_CUDA;
 
     const int ntiles = (T + ipk::MROWS - 1) / ipk::MROWS;
@@ -537,6 +572,20 @@ long long ip_probe_int8_mma(int blocks, int iters, int *sink, ip_stream_t stream
     if (cudaGetLastError() != cudaSuccess) return -1;
     return static_cast<long long>(blocks) * (ipk::PROBE_THREADS / 32) * iters * ipk::PROBE_CHAINS *
            (16ll * 8 * 32 * 2);
+}
+
+long long ip_probe_int8_mix(int blocks, int iters, int mma_warps, int *sink, ip_stream_t stream) {
+    if (blocks < 1 || iters < 1 || mma_warps < 0 || mma_warps > ipk::PROBE_THREADS / 32 || !sink)
+        return -1;
+    ipk::int8_mix_probe_kernel<<<blocks, ipk::PROBE_THREADS, 0,
+                                 reinterpret_cast<cudaStream_t>(stream)>>>(sink, 0x9e3779b9u, iters,
+                                                                           mma_warps);
+    if (cudaGetLastError() != cudaSuccess) return -1;
+    const long long mma = static_cast<long long>(mma_warps) * iters * ipk::MIX_MMA_CHAINS *
+                          (16ll * 8 * 32 * 2);
+    const long long dp4a = static_cast<long long>(ipk::PROBE_THREADS / 32 - mma_warps) * 4 * iters *
+                           4 * ipk::MIX_DP4A_CHAINS * (32ll * 4 * 2);
+    return static_cast<long long>(blocks) * (mma + dp4a);
 }
 
 int ip_debug_set_timeout_cycles(long long cycles) {

@@ -226,6 +226,24 @@ def test_default_workspace(ip, orc):
     assert ip.status() == -1   # IP_ERR_NULL: nothing registered
 
 
+def test_descriptor_cache_across_buffers(ip, orc):
+    # The library keeps the TMA descriptors of recent (pointer, shape)
+    # pairs.  Ten layers on their own buffers (two shapes, 40 descriptors,
+    # more than the table holds), called in an interleaved order twice over,
+    # must each produce their own oracle output.
+    lays = [synth.draw(1 + (i & 1), 2, 70 + 30 * (i & 1), 128, seed=1300 + i, p_mode="sinusoid")
+            for i in range(10)]
+    consts = [ip.layer_constants(l.scales) for l in lays]
+    want = [oracle_out(orc, l, c) for l, c in zip(lays, consts)]
+    dev = [[_dev(a) for a in (l.q, l.k, l.v, l.p, l.u, l.vb)] for l in lays]
+    ws = torch.zeros(256, dtype=torch.uint8, device="cuda")
+    for rnd in range(2):
+        for i in (list(range(10)) if rnd == 0 else [9, 2, 7, 0, 5, 4, 3, 6, 1, 8]):
+            out = ip.relpos_mhsa_i8(*dev[i], consts[i], workspace=ws)
+            assert ip.status(ws) == 0
+            assert_same(out.cpu().numpy(), want[i])
+
+
 def test_back_to_back_launches_see_the_previous_output(ip, orc):
     # Each launch may be scheduled while the one before it on the stream
     # finishes (programmatic dependent launch) and must wait for it before
