@@ -9,6 +9,9 @@
 // (sum q)^2 exactly for the centred values c_i = d q_i - sum, sigma =
 // isqrt(that + eps_c) (at least 1), f = floor(2^31 / sigma), and per element
 // n = round(c f / 2^16), y = clamp(round((M_i n + B_i) / 2^E_i), -127, 127).
+// With d = C 2^9, n is one 32-bit multiply-add and a shift of the int8
+// value q itself: n = floor((q F + G) / 2^7) with F = C f and
+// G = floor((2^15 - sum f) / 2^9), evaluated modulo 2^32 (see pass_a).
 // Lane l takes the 16-byte segments l, l + 32, ... of the row (coalesced)
 // and keeps them in registers between the two passes; the per-channel
 // constants (B, M, E) of its channels sit in shared memory in lane-major
@@ -69,11 +72,6 @@ __device__ __forceinline__ uint32_t recip_2pow31(unsigned long long s) {
     return quo;
 }
 
-// Sign-extended byte e of w.
-__device__ __forceinline__ int sbyte_at(uint32_t w, int e) {
-    return static_cast<int>(static_cast<int8_t>((w >> (8 * e)) & 0xffu));
-}
-
 // C = d / 512 segments of 16 channels per lane.  A warp takes NB rows at a
 // time and keeps their int8 values in registers: it reduces them, lane r
 // computes the square root and the reciprocal of row r (one chain of those
@@ -88,14 +86,14 @@ __device__ __forceinline__ int sbyte_at(uint32_t w, int e) {
 template <int C>
 struct Batch {
     uint4 xv[NB][C];
-    int sum[NB], f[NB];
+    uint32_t F[NB], G[NB];   // n = floor((q F + G) / 2^7) for row r (see pass_a)
 };
 
 template <int C>
 __device__ __forceinline__ void pass_a(const NormParams &prm, long long row0, int nrows, int lane,
                                        Batch<C> &bt) {
     constexpr int D = 512 * C;
-    int sq[NB];
+    int sq[NB], sum[NB];
 #pragma unroll
     for (int r = 0; r < NB; ++r) {
         const int8_t *xr = prm.x + (row0 + (r < nrows ? r : 0)) * D;
@@ -106,14 +104,14 @@ __device__ __forceinline__ void pass_a(const NormParams &prm, long long row0, in
     }
 #pragma unroll
     for (int r = 0; r < NB; ++r) {
-        bt.sum[r] = 0;
+        sum[r] = 0;
         sq[r] = 0;
 #pragma unroll
         for (int j = 0; j < C; ++j) {
             const uint32_t w[4] = {bt.xv[r][j].x, bt.xv[r][j].y, bt.xv[r][j].z, bt.xv[r][j].w};
 #pragma unroll
             for (int i = 0; i < 4; ++i) {
-                bt.sum[r] = __dp4a(static_cast<int>(w[i]), 0x01010101, bt.sum[r]);
+                sum[r] = __dp4a(static_cast<int>(w[i]), 0x01010101, sum[r]);
                 sq[r] = __dp4a(static_cast<int>(w[i]), static_cast<int>(w[i]), sq[r]);
             }
         }
@@ -122,13 +120,13 @@ __device__ __forceinline__ void pass_a(const NormParams &prm, long long row0, in
     for (int o = 16; o > 0; o >>= 1)
 #pragma unroll
         for (int r = 0; r < NB; ++r) {
-            bt.sum[r] += __shfl_xor_sync(0xffffffffu, bt.sum[r], o);
+            sum[r] += __shfl_xor_sync(0xffffffffu, sum[r], o);
             sq[r] += __shfl_xor_sync(0xffffffffu, sq[r], o);
         }
     long long ms = 0;
 #pragma unroll
     for (int r = 0; r < NB; ++r)
-        if (lane == r) ms = static_cast<long long>(D) * sq[r] - static_cast<long long>(bt.sum[r]) * bt.sum[r];
+        if (lane == r) ms = static_cast<long long>(D) * sq[r] - static_cast<long long>(sum[r]) * sum[r];
     unsigned long long sigma = isqrt_u42(static_cast<unsigned long long>(ms + prm.eps_c));
     sigma = sigma < 1 ? 1 : sigma;
     // f = floor(2^31 / sigma), held as a signed 32-bit value: f = 2^31 only
@@ -136,14 +134,26 @@ __device__ __forceinline__ void pass_a(const NormParams &prm, long long row0, in
     // 1) / 2^16) = round(c 2^31 / 2^16), so 2^31 - 1 stands in exactly
     uint32_t f_own = recip_2pow31(sigma);
     f_own = f_own > 0x7fffffffu ? 0x7fffffffu : f_own;
+    // n = floor(u / 2^16) with u = c f + 2^15 and c = D q - sum, D = C 2^9:
+    // u = (q C f + G) 2^9 + l with G = floor((2^15 - sum f) / 2^9) and
+    // 0 <= l < 2^9, so n = floor((q C f + G) / 2^7) (the fraction l / 2^9
+    // never carries an integer quotient over).  With s = sqrt(sum c^2 / d +
+    // eps_c), sigma >= s / 2 when s >= 1 (and every c is 0 when s < 1), and
+    // |c| <= sqrt(d) s, so |c| f <= 2^32 sqrt(d) and |q C f + G| < 2^29:
+    // the 32-bit multiply-add modulo 2^32 gives it exactly.
 #pragma unroll
-    for (int r = 0; r < NB; ++r) bt.f[r] = static_cast<int>(__shfl_sync(0xffffffffu, f_own, r));
+    for (int r = 0; r < NB; ++r) {
+        const uint32_t f = __shfl_sync(0xffffffffu, f_own, r);
+        bt.F[r] = static_cast<uint32_t>(C) * f;
+        const long long g = ((1ll << 15) - static_cast<long long>(sum[r]) * static_cast<long long>(f)) >> 9;
+        bt.G[r] = static_cast<uint32_t>(g);
+    }
 }
 
 // Pass B of one batch: normalise and requantise the rows from registers;
 // each channel record serves the NB rows.  The segment loop stays rolled so
 // that the code fits the instruction cache.
-template <int C>
+template <int C, bool HI>
 __device__ __forceinline__ void pass_b(const NormParams &prm, const uint4 *cst, long long row0,
                                        int nrows, int lane, const Batch<C> &bt) {
     constexpr int D = 512 * C;
@@ -160,35 +170,58 @@ __device__ __forceinline__ void pass_b(const NormParams &prm, const uint4 *cst, 
             }
         uint32_t o[NB][4];
 #pragma unroll
-        for (int r = 0; r < NB; ++r) o[r][0] = o[r][1] = o[r][2] = o[r][3] = 0u;
+        for (int i = 0; i < 4; ++i) {
+          // bytes 3 and 2 first, packed as soon as both are there
+          int t[NB][4];
+          uint32_t hi2[NB];
 #pragma unroll
-        for (int e = 0; e < 16; ++e) {
+          for (int k = 0; k < 4; ++k) {
+            const int ee = 3 - k;
+            const int e = 4 * i + ee;
             const uint4 rec = cst[(j * 16 + e) * 32 + lane];
             const long long b = static_cast<long long>((static_cast<unsigned long long>(rec.y) << 32) | rec.x);
 #pragma unroll
             for (int r = 0; r < NB; ++r) {
                 const uint32_t w[4] = {xj[r].x, xj[r].y, xj[r].z, xj[r].w};
-                const int cc = D * sbyte_at(w[e >> 2], e & 3) - bt.sum[r];   // |c| < 2^20
-                // n = round(c f / 2^16): |c f| < 2^51 and |n| < 2^23, so the
-                // low word of (c f + 2^15) >> 16 is n
-                const long long u = static_cast<long long>(cc) * bt.f[r] + (1ll << 15);
-                const int n = static_cast<int>(__funnelshift_r(static_cast<uint32_t>(u),
-                                                               static_cast<uint32_t>(u >> 32), 16));
-                // floor(v / 2^E) = floor(floor(v / 2^31) / 2^(E - 31)); |v| < 2^62
-                // makes floor(v / 2^31) a 32-bit value
+                const uint32_t q = static_cast<uint32_t>(sbyte(w[i], ee));
+                const int n = static_cast<int>(q * bt.F[r] + bt.G[r]) >> 7;   // |n| < 2^23
+                // floor(v / 2^E), |v| < 2^62: with every E >= 32 the high word
+                // shifted by E - 32 (the record holds E - 32), else
+                // floor(v / 2^31) (a 32-bit value) shifted by E - 31
                 const long long v = static_cast<long long>(static_cast<int>(rec.z)) * n + b;
-                const int h = static_cast<int>(__funnelshift_r(static_cast<uint32_t>(v),
-                                                               static_cast<uint32_t>(v >> 32), 31));
-                const int t = h >> static_cast<int>(rec.w);
-                const int y8 = t > 127 ? 127 : (t < -127 ? -127 : t);
-                o[r][e >> 2] |= (static_cast<uint32_t>(y8) & 0xffu) << (8 * (e & 3));
+                int h;
+                if (HI)
+                    h = static_cast<int>(static_cast<uint32_t>(static_cast<unsigned long long>(v) >> 32));
+                else
+                    h = static_cast<int>(__funnelshift_r(static_cast<uint32_t>(v),
+                                                         static_cast<uint32_t>(v >> 32), 31));
+                t[r][ee] = max(h >> static_cast<int>(rec.w), -127);   // 127 by the saturating pack
+                if (ee == 2) hi2[r] = pack_sat2(t[r][3], t[r][2], 0u);
+                if (ee == 0) o[r][i] = pack_sat2(t[r][1], t[r][0], hi2[r]);
             }
+          }
         }
 #pragma unroll
         for (int r = 0; r < NB; ++r)
             if (r < nrows)
                 __stcs(reinterpret_cast<uint4 *>(prm.y + (row0 + r) * D + j * 512 + lane * 16),
                        make_uint4(o[r][0], o[r][1], o[r][2], o[r][3]));
+    }
+}
+
+// The batches of one warp after the first one's pass A.
+template <int C, bool HI>
+__device__ __forceinline__ void run_batches(const NormParams &prm, const uint4 *cst, long long grp,
+                                            long long warps, long long groups, int lane,
+                                            Batch<C> &bt) {
+    for (;;) {
+        const long long row0 = grp * NB;
+        const int nrows = prm.rows - row0 < NB ? static_cast<int>(prm.rows - row0) : NB;
+        pass_b<C, HI>(prm, cst, row0, nrows, lane, bt);
+        grp += warps;
+        if (grp >= groups) break;
+        const long long nrow0 = grp * NB;
+        pass_a<C>(prm, nrow0, prm.rows - nrow0 < NB ? static_cast<int>(prm.rows - nrow0) : NB, lane, bt);
     }
 }
 
@@ -199,7 +232,7 @@ __device__ __forceinline__ void pass_b(const NormParams &prm, const uint4 *cst, 
 // batch's pass A runs before the channel records are built, so its loads
 // overlap that set-up.
 template <int C>
-__global__ void __launch_bounds__(THREADS)
+__global__ void __launch_bounds__(THREADS, C <= 2 ? 3 : 2)
     layernorm_i8_kernel(const NormParams prm) {
     constexpr int D = 512 * C;
     extern __shared__ uint8_t smem_raw[];
@@ -223,8 +256,9 @@ __global__ void __launch_bounds__(THREADS)
 
     // per-channel records {B' lo, B' hi, M, E - 31} with B' = B + 2^(E-1)
     // (the rounding term folded in): channel j 512 + l 16 + e of lane l goes
-    // to record (j 16 + e) 32 + l
-    bool bad = false;
+    // to record (j 16 + e) 32 + l.  When every E is at least 32 the records
+    // hold E - 32 and pass B shifts the high word of M n + B'.
+    bool bad = false, hi = true;
     for (int k = threadIdx.x; k < D; k += THREADS) {
         const int j = k >> 9, l = (k >> 4) & 31, e = k & 15;
         long long b = prm.B[k];
@@ -235,23 +269,25 @@ __global__ void __launch_bounds__(THREADS)
             b = 0;
         }
         b += 1ll << (ex - 1);
+        hi = hi && ex >= 32;
         cst[(j * 16 + e) * 32 + l] =
             make_uint4(static_cast<uint32_t>(b), static_cast<uint32_t>(static_cast<unsigned long long>(b) >> 32),
                        static_cast<uint32_t>(m), static_cast<uint32_t>(ex - 31));
     }
     if (bad) atomicOr(prm.err, ERR_PARAM);
-    __syncthreads();
-    if (!first) return;
-
-    for (;;) {
-        const long long row0 = grp * NB;
-        const int nrows = prm.rows - row0 < NB ? static_cast<int>(prm.rows - row0) : NB;
-        pass_b<C>(prm, cst, row0, nrows, lane, bt);
-        grp += warps;
-        if (grp >= groups) break;
-        const long long nrow0 = grp * NB;
-        pass_a<C>(prm, nrow0, prm.rows - nrow0 < NB ? static_cast<int>(prm.rows - nrow0) : NB, lane, bt);
+    const bool all_hi = __syncthreads_and(hi) != 0;
+    if (all_hi) {
+        for (int k = threadIdx.x; k < D; k += THREADS) {
+            const int j = k >> 9, l = (k >> 4) & 31, e = k & 15;
+            cst[(j * 16 + e) * 32 + l].w -= 1u;
+        }
+        __syncthreads();
     }
+    if (!first) return;
+    if (all_hi)
+        run_batches<C, true>(prm, cst, grp, warps, groups, lane, bt);
+    else
+        run_batches<C, false>(prm, cst, grp, warps, groups, lane, bt);
 }
 
 }  // namespace ipn

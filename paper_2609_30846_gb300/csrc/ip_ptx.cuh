@@ -202,4 +202,27 @@ __device__ __forceinline__ int clamp127(long long x) {
     return x > 127 ? 127 : (x < -127 ? -127 : static_cast<int>(x));
 }
 
+// (c << 16) | (sat8(a) << 8) | sat8(b): two int32 values saturated to
+// [-128, 127] and packed below the low half of c (cvt.pack.sat).
+__device__ __forceinline__ uint32_t pack_sat2(int a, int b, uint32_t c) {
+    uint32_t w;
+    asm("cvt.pack.sat.s8.s32.b32 %0, %1, %2, %3;" : "=r"(w) : "r"(a), "r"(b), "r"(c));
+    return w;
+}
+
+// Bytes [y0, y1, y2, y3] of four int32 values, each saturated to [-128, 127].
+__device__ __forceinline__ uint32_t pack_sat4(int y0, int y1, int y2, int y3) {
+    return pack_sat2(y1, y0, pack_sat2(y3, y2, 0u));
+}
+
+// Sign-extended byte e (0..3) of w: one prmt, byte e in the low byte and
+// its sign bit replicated in the three above (selector bit 3).
+__device__ __forceinline__ int sbyte(uint32_t w, int e) {
+    const uint32_t s = 0x8u | static_cast<uint32_t>(e);
+    const uint32_t sel = (s << 12) | (s << 8) | (s << 4) | static_cast<uint32_t>(e);
+    uint32_t r;
+    asm("prmt.b32 %0, %1, 0, %2;" : "=r"(r) : "r"(w), "r"(sel));
+    return static_cast<int>(r);
+}
+
 }  // namespace ipk
