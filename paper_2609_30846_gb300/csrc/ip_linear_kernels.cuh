@@ -9,14 +9,19 @@
 // stays inside one utterance.  A producer warp streams K in stages of 128
 // bytes: the 128 x 128 int8 tiles of X and W land through TMA with the
 // 128-byte swizzle in a ring of four stages that runs on across tiles, so
-// the next tile's first stages load during the current tile's epilogue.  Eight consumer warps (2 along the frames x 4
-// along the channels, 64 x 32 each) feed the integer warp MMA (mma.sync
-// m16n8k32 s8 x s8 -> s32) from ldmatrix; sm_103a has no integer tcgen05
-// kind.  The epilogue adds the int32 bias, multiplies by m[n] in int64,
-// shifts right by 31 + s[n] with rounding, clamps to [-127, 127] (and, in
-// the feed-forward variant, applies the minimax integer Swish) and writes
-// each warp's 64 x 32 bytes through shared memory as 16-byte row segments,
-// either row-major [B][T][N] or head-split [G][B][N/G/128][T][128].
+// the next tile's first stages load during the current tile's epilogue.
+// The integer MMA pipe and the dp4a pipe of an SM sub-partition work at the
+// same time, so a tile's channels are split between them: eight MMA warps
+// (2 along the frames x 4 along the channels, 64 x 16 each) take channels
+// 0-63 with the integer warp MMA (mma.sync m16n8k32 s8 x s8 -> s32, from
+// ldmatrix; sm_103a has no integer tcgen05 kind), and eight dp4a warps
+// (16 frames each) take channels 64-127 with dp4a on the same stages.  The
+// epilogue adds the int32 bias, multiplies by m[n] in int64, shifts right by
+// 31 + s[n] with rounding, clamps to [-127, 127] (and, in the feed-forward
+// variant, applies the minimax integer Swish); the MMA warps write their
+// 64 x 16 bytes through shared memory as 16-byte row segments, the dp4a
+// warps their 8-byte row segments directly, either row-major [B][T][N] or
+// head-split [G][B][N/G/128][T][128].
 #pragma once
 
 #include <cuda.h>
@@ -31,8 +36,14 @@ using namespace ipk;
 constexpr int BM = 128;                 // frames per CTA
 constexpr int BN = 128;                 // output channels per CTA
 constexpr int BK = 128;                 // K bytes per stage
-constexpr int NCW = 8;                  // consumer warps: 2 (frames) x 4 (channels)
-constexpr int THREADS = (NCW + 1) * 32;
+constexpr int NCW = 8;                  // MMA warps: 2 (frames) x 4 (channels)
+constexpr int NDW_LOG2 = 3;
+constexpr int NDW = 1 << NDW_LOG2;      // dp4a warps, along the frames (two per SM sub-partition)
+constexpr int DW_ROWS = BM >> NDW_LOG2; // frames of one dp4a warp
+constexpr int RI = DW_ROWS >> 2;        // frames of one dp4a lane (four row groups of lanes)
+constexpr int MMA_COLS = 64;            // channels 0 .. 63 of a tile on the MMA pipe, the rest on dp4a
+constexpr int DW_UNROLL = 2;     // k chunks of a stage unrolled in the dp4a loop
+constexpr int THREADS = (NCW + NDW + 1) * 32;
 constexpr int STAGES = 4;
 constexpr int A_BYTES = BM * BK;
 constexpr int B_BYTES = BN * BK;
@@ -122,6 +133,52 @@ constexpr int EPI_PLAIN = 0;   // requantised int8
 constexpr int EPI_SWISH = 1;   // + minimax Swish
 constexpr int EPI_GLU = 2;     // interleaved pairs (a_c, b_c) -> a_c sigma(b_c)
 
+// Offset in Y of tile row r (0 .. BM - 1) at tile column col, or -1 past the
+// last frame.  Row-major Y [B][T][N] (or [B][T][N / 2] for the gated unit,
+// with `width` its row length) or head-split Y [G][B][N / G / 128][T][128];
+// hh, grp: the tile's head within its group and the group.
+__device__ __forceinline__ long long y_offset(const LinearParams &p, const Tile &L, int r, int col,
+                                              int width, int hh, int grp) {
+    int b = L.b, t = L.t0 + r;
+    if (p.x_layout == LAYOUT_ROWS) {
+        if (L.m0 + r >= p.B * p.T) return -1;
+        if (p.y_layout == LAYOUT_ROWS)
+            return static_cast<long long>(L.m0 + r) * width + col;
+        while (t >= p.T) {   // rows of a flat tile may run into later utterances
+            t -= p.T;
+            ++b;
+        }
+    } else if (t >= p.T) {
+        return -1;
+    }
+    if (p.y_layout == LAYOUT_ROWS) return (static_cast<long long>(b) * p.T + t) * width + col;
+    return (((static_cast<long long>(grp) * p.B + b) * p.heads_per_group + hh) * p.T + t) * 128 + col;
+}
+
+// Per-channel constants of Eq. 7 for channel n, clipped into their domain
+// (bad is set when one was out of it).
+__device__ __forceinline__ void channel_consts(const LinearParams &p, int n, int &cb, int &cm,
+                                               int &ce, bool &bad) {
+    int bi = p.bias != nullptr ? __ldg(p.bias + n) : 0;
+    int mi = __ldg(p.m + n);
+    int si = __ldg(p.s + n);
+    if (mi < 0 || si < 0 || si > 31 || bi >= (1 << 30) || bi <= -(1 << 30)) {
+        bad = true;
+        mi = mi < 0 ? 0 : mi;
+        si = si < 0 ? 0 : (si > 31 ? 31 : si);
+        bi = 0;
+    }
+    cb = bi;
+    cm = mi;
+    ce = 31 + si;
+}
+
+// Eq. 7 for one accumulator: clamp(round(m (acc + bias) / 2^(31 + s))).
+__device__ __forceinline__ int requant(int acc, int cb, int cm, int ce) {
+    const long long v = static_cast<long long>(cm) * (acc + cb) + (1ll << (ce - 1));
+    return clamp127(v >> ce);
+}
+
 template <int EPI>
 __global__ void __launch_bounds__(THREADS, 1)
     linear_i8_kernel(const __grid_constant__ CUtensorMap tm_x,
@@ -145,7 +202,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
             mbar_init(full_bar(s), 1);
-            mbar_init(empty_bar(s), NCW);
+            mbar_init(empty_bar(s), NCW + NDW);
         }
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
@@ -161,7 +218,7 @@ __global__ void __launch_bounds__(THREADS, 1)
 
     // ---------------------------------------------------------- producer
     // Use u of the ring: stage u & 3, phase (u / 4) & 1.
-    if (warp == NCW) {
+    if (warp == NCW + NDW) {
         unsigned u = 0, landed_from = 0;
         bool ok = true;
         for (unsigned idx = blockIdx.x; idx < prm.ntiles && ok; idx += gridDim.x) {
@@ -194,24 +251,123 @@ __global__ void __launch_bounds__(THREADS, 1)
         return;
     }
 
-    // ---------------------------------------------------------- consumers
-    const int wm = warp & 1;        // rows 64 wm .. 64 wm + 63 of the tile
-    const int wn = warp >> 1;       // channels 32 wn .. 32 wn + 31
+    const int frames = prm.B * prm.T;
+
+    // ---------------------------------------------------------- dp4a warps
+    // Channels MMA_COLS .. BN - 1 of every tile, rows DW_ROWS dw .. DW_ROWS dw
+    // + DW_ROWS - 1: lane (rg, cg) = (lane / 8, lane % 8) accumulates rows
+    // DW_ROWS dw + RI rg + i (i < RI) and channels MMA_COLS + 8 cg + j (j < 8)
+    // with dp4a on the same stages the MMA warps read.  Each lane walks the
+    // eight 16-byte k chunks of a stage starting at chunk rg + cg, so that
+    // the 32 lanes of one 16-byte load touch every bank group of the
+    // swizzled tile equally.
+    if (warp >= NCW) {
+        const int dw = warp - NCW;
+        const int rg = lane >> 3, cg = lane & 7;
+        const int r0 = DW_ROWS * dw + RI * rg;
+        const int r7 = r0 & 7;          // 0 or 4: r7 + i = r7 | i for i < RI
+        const int c0 = MMA_COLS + 8 * cg;
+        unsigned u = 0;
+        for (unsigned idx = blockIdx.x; idx < prm.ntiles; idx += gridDim.x) {
+            const Tile L = tile_of(idx, prm);
+            const int n0 = L.nt * BN;
+            int acc[RI][8];
+#pragma unroll
+            for (int i = 0; i < RI; ++i)
+#pragma unroll
+                for (int j = 0; j < 8; ++j) acc[i][j] = 0;
+            for (int it = 0; it < kt; ++it, ++u) {
+                const int s = static_cast<int>(u & (STAGES - 1));
+                if (!warp_wait(full_bar(s), (u / STAGES) & 1, prm.timeout_cycles)) {
+                    if (lane == 0) atomicOr(prm.err, 1);
+                    return;
+                }
+                const uint32_t abase = stage(s) + r0 * 128;
+                const uint32_t bbase = stage(s) + A_BYTES + c0 * 128;
+#pragma unroll (DW_UNROLL)
+                for (int c = 0; c < 8; ++c) {
+                    const int kc = (c + rg + cg) & 7;
+                    uint4 a[RI];
+#pragma unroll
+                    for (int i = 0; i < RI; ++i)
+                        a[i] = lds128(abase + i * 128 + ((kc ^ (r7 | i)) << 4));
+#pragma unroll
+                    for (int j = 0; j < 8; ++j) {
+                        const uint4 b = lds128(bbase + j * 128 + ((kc ^ j) << 4));
+#pragma unroll
+                        for (int i = 0; i < RI; ++i) {
+                            acc[i][j] = __dp4a(static_cast<int>(a[i].x), static_cast<int>(b.x), acc[i][j]);
+                            acc[i][j] = __dp4a(static_cast<int>(a[i].y), static_cast<int>(b.y), acc[i][j]);
+                            acc[i][j] = __dp4a(static_cast<int>(a[i].z), static_cast<int>(b.z), acc[i][j]);
+                            acc[i][j] = __dp4a(static_cast<int>(a[i].w), static_cast<int>(b.w), acc[i][j]);
+                        }
+                    }
+                }
+                release_stage(empty_bar(s), lane);
+            }
+
+            // epilogue: eight channels per lane, one 8-byte (4-byte gated)
+            // segment per row, straight to global memory
+            int cb[8], cm[8], ce[8];
+            bool bad = false;
+#pragma unroll
+            for (int j = 0; j < 8; ++j) channel_consts(prm, n0 + c0 + j, cb[j], cm[j], ce[j], bad);
+            if (bad) atomicOr(prm.err, ERR_PARAM);
+            int hh = L.nt, grp = 0;
+            if (prm.y_layout == LAYOUT_HEADS)
+                while (hh >= prm.heads_per_group) {   // at most G - 1 steps
+                    hh -= prm.heads_per_group;
+                    ++grp;
+                }
+#pragma unroll
+            for (int i = 0; i < RI; ++i) {
+                if (EPI == EPI_GLU) {
+                    uint32_t w = 0;
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) {
+                        const int za = requant(acc[i][2 * q], cb[2 * q], cm[2 * q], ce[2 * q]);
+                        const int zb = requant(acc[i][2 * q + 1], cb[2 * q + 1], cm[2 * q + 1],
+                                               ce[2 * q + 1]);
+                        w |= (static_cast<uint32_t>(glu_i8(za, zb, prm)) & 0xffu) << (8 * q);
+                    }
+                    const long long off = y_offset(prm, L, r0 + i, (n0 + c0) >> 1, prm.N >> 1, hh, grp);
+                    if (off >= 0) *reinterpret_cast<uint32_t *>(prm.y + off) = w;
+                } else {
+                    uint32_t w[2] = {0u, 0u};
+#pragma unroll
+                    for (int j = 0; j < 8; ++j) {
+                        uint32_t o = static_cast<uint32_t>(requant(acc[i][j], cb[j], cm[j], ce[j])) & 0xffu;
+                        if (EPI == EPI_SWISH) o = swish_lut[o];
+                        w[j >> 2] |= o << (8 * (j & 3));
+                    }
+                    const int col = prm.y_layout == LAYOUT_ROWS ? n0 + c0 : c0;
+                    const long long off = y_offset(prm, L, r0 + i, col, prm.N, hh, grp);
+                    if (off >= 0) *reinterpret_cast<uint2 *>(prm.y + off) = make_uint2(w[0], w[1]);
+                }
+            }
+        }
+        return;
+    }
+
+    // ---------------------------------------------------------- MMA warps
+    // Channels 0 .. MMA_COLS - 1: warp (wm, wn) takes rows 64 wm .. 64 wm +
+    // 63 and channels 16 wn .. 16 wn + 15 (two n8 tiles).
+    const int wm = warp & 1;
+    const int wn = warp >> 1;
     const int g = lane >> 2, t4 = lane & 3;
     const int lm_row = lane & 7, lm_mat = lane >> 3;
     const uint32_t ob = base + SMEM_OUT + warp * OUT_WARP_BYTES;
-    const int frames = prm.B * prm.T;
 
     unsigned u = 0;
     for (unsigned idx = blockIdx.x; idx < prm.ntiles; idx += gridDim.x) {
         const Tile L = tile_of(idx, prm);
         const int n0 = L.nt * BN;
 
-        int acc[4][4][4];
+        int acc[4][2][4];
 #pragma unroll
         for (int i = 0; i < 4; ++i)
 #pragma unroll
-            for (int j = 0; j < 4; ++j)
+            for (int j = 0; j < 2; ++j)
                 acc[i][j][0] = acc[i][j][1] = acc[i][j][2] = acc[i][j][3] = 0;
 
         for (int it = 0; it < kt; ++it, ++u) {
@@ -221,85 +377,66 @@ __global__ void __launch_bounds__(THREADS, 1)
                 return;
             }
             const uint32_t at = stage(s) + (64 * wm) * 128;
-            const uint32_t bt = stage(s) + A_BYTES + (32 * wn) * 128;
+            const uint32_t bt = stage(s) + A_BYTES + (16 * wn) * 128;
 #pragma unroll
             for (int ks = 0; ks < 4; ++ks) {
-                uint32_t af[4][4], bf[4][2];
+                uint32_t af[4][4], bf[2][2];
 #pragma unroll
                 for (int i = 0; i < 4; ++i)
                     ldsm_x4(at + swz(16 * i + (lm_mat & 1) * 8 + lm_row, 2 * ks + (lm_mat >> 1)),
                             af[i][0], af[i][1], af[i][2], af[i][3]);
-#pragma unroll
-                for (int jj = 0; jj < 2; ++jj)
-                    ldsm_x4(bt + swz(16 * jj + (lm_mat >> 1) * 8 + lm_row, 2 * ks + (lm_mat & 1)),
-                            bf[2 * jj][0], bf[2 * jj][1], bf[2 * jj + 1][0], bf[2 * jj + 1][1]);
+                ldsm_x4(bt + swz((lm_mat >> 1) * 8 + lm_row, 2 * ks + (lm_mat & 1)), bf[0][0],
+                        bf[0][1], bf[1][0], bf[1][1]);
 #pragma unroll
                 for (int i = 0; i < 4; ++i)
 #pragma unroll
-                    for (int j = 0; j < 4; ++j) mma_s8s8(acc[i][j], af[i], bf[j][0], bf[j][1]);
+                    for (int j = 0; j < 2; ++j) mma_s8s8(acc[i][j], af[i], bf[j][0], bf[j][1]);
             }
             release_stage(empty_bar(s), lane);
         }
 
         // ------------------------------------------------------ epilogue
-        // per-channel constants of this thread's eight channels (Eq. 7), loaded after
-        // the main loop so that they hold no registers during it
-        int cb[8], cm[8], ce[8];
+        // per-channel constants of this thread's four channels (Eq. 7),
+        // loaded after the main loop so that they hold no registers during it
+        int cb[4], cm[4], ce[4];
         bool bad = false;
 #pragma unroll
-        for (int j = 0; j < 4; ++j)
+        for (int j = 0; j < 2; ++j)
 #pragma unroll
-            for (int q = 0; q < 2; ++q) {
-                const int n = n0 + 32 * wn + 8 * j + 2 * t4 + q;
-                int bi = prm.bias != nullptr ? __ldg(prm.bias + n) : 0;
-                int mi = __ldg(prm.m + n);
-                int si = __ldg(prm.s + n);
-                if (mi < 0 || si < 0 || si > 31 || bi >= (1 << 30) || bi <= -(1 << 30)) {
-                    bad = true;
-                    mi = mi < 0 ? 0 : mi;
-                    si = si < 0 ? 0 : (si > 31 ? 31 : si);
-                    bi = 0;
-                }
-                cb[2 * j + q] = bi;
-                cm[2 * j + q] = mi;
-                ce[2 * j + q] = 31 + si;
-            }
+            for (int q = 0; q < 2; ++q)
+                channel_consts(prm, n0 + 16 * wn + 8 * j + 2 * t4 + q, cb[2 * j + q], cm[2 * j + q],
+                               ce[2 * j + q], bad);
         if (bad) atomicOr(prm.err, ERR_PARAM);
 
         if (EPI == EPI_GLU) {
             // pairs (a_c, b_c) in columns (2t, 2t + 1) of each n8 tile: output
-            // channel 4j + t of this warp's 16 (row of 16 bytes)
+            // channel 4j + t of this warp's 8 (row of 8 bytes)
 #pragma unroll
             for (int i = 0; i < 4; ++i)
 #pragma unroll
-                for (int j = 0; j < 4; ++j)
+                for (int j = 0; j < 2; ++j)
 #pragma unroll
                     for (int rr = 0; rr < 2; ++rr) {
-                        int z[2];
-#pragma unroll
-                        for (int q = 0; q < 2; ++q) {
-                            const int cix = 2 * j + q;
-                            const long long v = static_cast<long long>(cm[cix]) *
-                                                    (acc[i][j][2 * rr + q] + cb[cix]) +
-                                                (1ll << (ce[cix] - 1));
-                            z[q] = clamp127(v >> ce[cix]);
-                        }
-                        const uint32_t o = static_cast<uint32_t>(glu_i8(z[0], z[1], prm)) & 0xffu;
+                        const int za = requant(acc[i][j][2 * rr], cb[2 * j], cm[2 * j], ce[2 * j]);
+                        const int zb = requant(acc[i][j][2 * rr + 1], cb[2 * j + 1], cm[2 * j + 1],
+                                               ce[2 * j + 1]);
+                        const uint32_t o = static_cast<uint32_t>(glu_i8(za, zb, prm)) & 0xffu;
                         const int r = 16 * i + g + 8 * rr;
                         asm volatile("st.shared.u8 [%0], %1;" ::"r"(ob + r * OUT_ROW + 4 * j + t4),
                                      "r"(o)
                                      : "memory");
                     }
             __syncwarp();
-            // 64 rows x 16 bytes: lane -> rows lane, lane + 32
-            const int Nout = prm.N >> 1;
+            // 64 rows x 8 bytes: lane -> rows lane, lane + 32
 #pragma unroll
             for (int it = 0; it < 2; ++it) {
                 const int r = 32 * it + lane;
-                const uint4 v = lds128(ob + r * OUT_ROW);
+                const int2 v2 = lds64(ob + r * OUT_ROW);
+                const uint2 v = make_uint2(static_cast<uint32_t>(v2.x), static_cast<uint32_t>(v2.y));
                 if (L.m0 + 64 * wm + r < frames) {
-                    const size_t off = static_cast<size_t>(L.m0 + 64 * wm + r) * Nout + (n0 >> 1) + 16 * wn;
-                    *reinterpret_cast<uint4 *>(prm.y + off) = v;
+                    const size_t off = static_cast<size_t>(L.m0 + 64 * wm + r) * (prm.N >> 1) +
+                                       (n0 >> 1) + 8 * wn;
+                    *reinterpret_cast<uint2 *>(prm.y + off) = v;
                 }
             }
             __syncwarp();
@@ -309,17 +446,15 @@ __global__ void __launch_bounds__(THREADS, 1)
 #pragma unroll
         for (int i = 0; i < 4; ++i)
 #pragma unroll
-            for (int j = 0; j < 4; ++j)
+            for (int j = 0; j < 2; ++j)
 #pragma unroll
                 for (int rr = 0; rr < 2; ++rr) {
                     uint32_t two = 0;
 #pragma unroll
                     for (int q = 0; q < 2; ++q) {
                         const int c = 2 * j + q;
-                        const long long v = static_cast<long long>(cm[c]) *
-                                                (acc[i][j][2 * rr + q] + cb[c]) +
-                                            (1ll << (ce[c] - 1));
-                        uint32_t o = static_cast<uint32_t>(clamp127(v >> ce[c])) & 0xffu;
+                        uint32_t o = static_cast<uint32_t>(requant(acc[i][j][2 * rr + q], cb[c], cm[c],
+                                                                   ce[c])) & 0xffu;
                         if (EPI == EPI_SWISH) o = swish_lut[o];
                         two |= o << (8 * q);
                     }
@@ -331,39 +466,19 @@ __global__ void __launch_bounds__(THREADS, 1)
         __syncwarp();
 
         int hh = L.nt, grp = 0;
-        if (prm.y_layout == LAYOUT_HEADS) {
+        if (prm.y_layout == LAYOUT_HEADS)
             while (hh >= prm.heads_per_group) {   // at most G - 1 steps
                 hh -= prm.heads_per_group;
                 ++grp;
             }
-        }
-        // 64 rows x 32 bytes: lane -> (row 16 it + lane / 2, segment lane & 1)
+        // 64 rows x 16 bytes: lane -> rows lane, lane + 32
 #pragma unroll
-        for (int it = 0; it < 4; ++it) {
-            const int r = 64 * wm + 16 * it + (lane >> 1);
-            const int seg = lane & 1;
-            const uint4 v = lds128(ob + (r - 64 * wm) * OUT_ROW + 16 * seg);
-            int b = L.b, t = L.t0 + r;
-            bool valid;
-            if (prm.x_layout == LAYOUT_ROWS) {
-                valid = L.m0 + r < frames;
-                if (valid && prm.y_layout == LAYOUT_HEADS)
-                    while (t >= prm.T) {   // rows of a flat tile may run into later utterances
-                        t -= prm.T;
-                        ++b;
-                    }
-            } else {
-                valid = t < prm.T;
-            }
-            if (valid) {
-                size_t off;
-                if (prm.y_layout == LAYOUT_ROWS)
-                    off = (static_cast<size_t>(b) * prm.T + t) * prm.N + n0 + 32 * wn + 16 * seg;
-                else
-                    off = (((static_cast<size_t>(grp) * prm.B + b) * prm.heads_per_group + hh) *
-                               prm.T + t) * 128 + 32 * wn + 16 * seg;
-                *reinterpret_cast<uint4 *>(prm.y + off) = v;
-            }
+        for (int it = 0; it < 2; ++it) {
+            const int r = 32 * it + lane;
+            const uint4 v = lds128(ob + r * OUT_ROW);
+            const int col = prm.y_layout == LAYOUT_ROWS ? n0 + 16 * wn : 16 * wn;
+            const long long off = y_offset(prm, L, 64 * wm + r, col, prm.N, hh, grp);
+            if (off >= 0) *reinterpret_cast<uint4 *>(prm.y + off) = v;
         }
         __syncwarp();
     }

@@ -80,6 +80,37 @@ def test_encoder_frames_full_size(ip, orc):
     assert_same(*run_both(ip, orc, *case(32 * 375, 1024, seed=7)))
 
 
+@pytest.mark.parametrize("mode", ["E31", "E32", "E62"])
+def test_requant_shift_paths(ip, orc, mode):
+    # The kernel shifts the high word of M n + B' when every E >= 32 (the
+    # usual constants have E in the high 30s and 40s) and takes
+    # floor(v / 2^31) first when some channel has E = 31.  Constants of
+    # both kinds, at the ends of the domain, against the oracle with the
+    # same constants.
+    x, gamma, beta, s_x, s_y, eps = case(300, 1024, seed=11)
+    c = orc.layernorm_constants(s_x, gamma, beta, s_y, eps)
+    M, B, E = c.M.copy(), c.B.copy(), c.E.copy()
+    ch = np.arange(0, 1024, 61)
+    if mode == "E31":
+        sh = E[ch] - 31
+        M[ch] >>= sh
+        B[ch] >>= sh
+        E[ch] = 31
+    elif mode == "E32":
+        sh = E - 32
+        M >>= sh
+        B >>= sh
+        E[:] = 32
+    else:
+        E[ch] = 62
+        B[ch] = 0
+    c2 = orc.NormConstants(M=M, B=B, E=E, eps_c=c.eps_c)
+    ws = torch.zeros(256, dtype=torch.uint8, device="cuda")
+    got = ip.layernorm_i8(_d(x), _d(M), _d(B), _d(E), c.eps_c, workspace=ws)
+    assert ip.status(ws) == 0
+    assert_same(got.cpu().numpy(), orc.layernorm(x, c2))
+
+
 def test_constant_out_of_domain_is_reported(ip, orc):
     x, gamma, beta, s_x, s_y, eps = case(4, 512, seed=8)
     c = orc.layernorm_constants(s_x, gamma, beta, s_y, eps)
