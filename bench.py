@@ -277,6 +277,8 @@ def run_reference(args):
 # d=1024): Q/K/V stacked and written head-split, the output projection from
 # the attention's row-major output, and the feed-forward pair with the fused
 # minimax Swish.
+NORM_BUFS = 16
+
 NEXT_ROWS = [
     # name, K, N, groups, x_layout, y_layout, swish
     ("linear_qkv_1024x3072_heads", 1024, 3072, 3, 0, 1, False),
@@ -379,26 +381,33 @@ def measure_next_rows(dev, peak, pipes, steps: int, cpu: bool):
         rows[name] = row
         del x, w, b, out
 
-    # integer LayerNorm of the frames before the attention (d = 1024)
+    # integer LayerNorm of the frames before the attention (d = 1024).  One
+    # launch takes under 20 us, close to the event timer's resolution
+    # (about 2 us on this GPU), so a timed group runs NORM_BUFS launches on
+    # as many input/output pairs (393 MB, larger than L2) after the flush.
     d = 1024
     nc = synth.norm(B * T, d, seed=7100)
     k = ip.layernorm_constants(nc.s_x, nc.gamma, nc.beta, nc.s_y, nc.eps)
-    x = torch.from_numpy(nc.x).to(dev)
+    x0 = torch.from_numpy(nc.x).to(dev)
+    xs = [x0] + [x0.clone() for _ in range(NORM_BUFS - 1)]
+    outs = [torch.empty_like(x0) for _ in range(NORM_BUFS)]
     Md, Bd, Ed = (torch.from_numpy(a).to(dev) for a in (k.M, k.B, k.E))
-    out = torch.empty_like(x)
     ws = torch.zeros(256, dtype=torch.uint8, device=dev)
-    call = lambda: ip.layernorm_i8(x, Md, Bd, Ed, k.eps_c, out=out, workspace=ws, stream=stream)
-    for _ in range(3):
-        call()
+    call = lambda i: ip.layernorm_i8(xs[i], Md, Bd, Ed, k.eps_c, out=outs[i], workspace=ws,
+                                     stream=stream)
+    for i in range(NORM_BUFS):
+        call(i)
     times = []
     for _ in range(steps):
         flush()
+        torch.cuda._sleep(1_500_000)   # about 0.7 ms: covers the host issue of the group
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         e0.record(stream)
-        call()
+        for i in range(NORM_BUFS):
+            call(i)
         e1.record(stream)
         e1.synchronize()
-        times.append(e0.elapsed_time(e1) * 1e-3)
+        times.append(e0.elapsed_time(e1) * 1e-3 / NORM_BUFS)
     if ip.status(ws, stream) != 0:
         raise SystemExit("layernorm: kernel reported an error")
     t = statistics.median(times)
@@ -410,7 +419,8 @@ def measure_next_rows(dev, peak, pipes, steps: int, cpu: bool):
            "roofline": {"bound": "alu", "achieved": ops / t / 1e12, "peak": alu_peak,
                         "unit": "Tops/s (int32 lane ops)", "frac": ops / t / 1e12 / alu_peak,
                         "traffic": None, "hbm_frac": elems * 2 / t / 1e9 / HBM_GBS},
-           "kernel": "layernorm_i8_kernel<2>", "gpu_launches": 1}
+           "kernel": "layernorm_i8_kernel<2>", "gpu_launches": NORM_BUFS,
+           "timing": f"{NORM_BUFS} launches on {NORM_BUFS} input/output pairs per event pair"}
     if cpu:
         import oracle
         oracle.build()
@@ -427,7 +437,7 @@ def measure_next_rows(dev, peak, pipes, steps: int, cpu: bool):
                                "cores": os.cpu_count() or 1, "kind": "oracle",
                                "sample": f"{n} frames of {B * T}, {dt:.2f} s"}
     rows["layernorm_1024"] = row
-    del x, out
+    del xs, outs, x0
 
     # one whole integer Conformer block (Eqs. 1-5): 19 launches
     import synth.block as sblock

@@ -29,7 +29,9 @@ int sm_count() {
     return g_sms[dev];
 }
 
-// Resident CTAs of the C-segment kernel on the whole GPU (cached).
+// CTAs of the C-segment kernel on the whole GPU: one per SM, so that its
+// eight warps take two or more batches each and load the next batch's rows
+// while they normalise the current one (cached; 0 if one does not fit).
 template <int C>
 long long resident(int nsm) {
     static int per_sm[64] = {0};
@@ -42,7 +44,7 @@ long long resident(int nsm) {
                                                           ipn::THREADS, C * 8192) != cudaSuccess ||
             n < 1)
             return 0;
-        per_sm[dev] = n;
+        per_sm[dev] = 1;
     }
     return static_cast<long long>(per_sm[dev]) * nsm;
 }

@@ -4,7 +4,8 @@
 // multiple of 512; the square root and the reciprocal are digit-by-digit).
 //
 // One warp per batch of four rows of d channels, batches dealt warp-major
-// over a grid of all resident CTAs.  Per row: the sum and the sum of squares of the
+// over a grid of one CTA per SM, so that every warp takes two or more
+// batches and loads the next one's rows during the current pass B.  Per row: the sum and the sum of squares of the
 // int8 values (dp4a, warp reduction), floor(sum c^2 / d) = d sum q^2 -
 // (sum q)^2 exactly for the centred values c_i = d q_i - sum, sigma =
 // isqrt(that + eps_c) (at least 1), f = floor(2^31 / sigma), and per element
@@ -90,18 +91,23 @@ struct Batch {
 };
 
 template <int C>
-__device__ __forceinline__ void pass_a(const NormParams &prm, long long row0, int nrows, int lane,
-                                       Batch<C> &bt) {
+__device__ __forceinline__ void load_rows(const NormParams &prm, long long row0, int nrows, int lane,
+                                          uint4 (&xv)[NB][C]) {
     constexpr int D = 512 * C;
-    int sq[NB], sum[NB];
 #pragma unroll
     for (int r = 0; r < NB; ++r) {
         const int8_t *xr = prm.x + (row0 + (r < nrows ? r : 0)) * D;
 #pragma unroll
         for (int j = 0; j < C; ++j)
-            bt.xv[r][j] = r < nrows ? __ldcs(reinterpret_cast<const uint4 *>(xr + j * 512 + lane * 16))
-                                    : make_uint4(0u, 0u, 0u, 0u);
+            xv[r][j] = r < nrows ? __ldcs(reinterpret_cast<const uint4 *>(xr + j * 512 + lane * 16))
+                                 : make_uint4(0u, 0u, 0u, 0u);
     }
+}
+
+template <int C>
+__device__ __forceinline__ void pass_a_stats(const NormParams &prm, int lane, Batch<C> &bt) {
+    constexpr int D = 512 * C;
+    int sq[NB], sum[NB];
 #pragma unroll
     for (int r = 0; r < NB; ++r) {
         sum[r] = 0;
@@ -209,7 +215,16 @@ __device__ __forceinline__ void pass_b(const NormParams &prm, const uint4 *cst, 
     }
 }
 
-// The batches of one warp after the first one's pass A.
+template <int C>
+__device__ __forceinline__ void pass_a(const NormParams &prm, long long row0, int nrows, int lane,
+                                       Batch<C> &bt) {
+    load_rows<C>(prm, row0, nrows, lane, bt.xv);
+    pass_a_stats<C>(prm, lane, bt);
+}
+
+// The batches of one warp after the first one's pass A: the next batch's
+// rows are loaded before the current batch's pass B, so their latency
+// hides behind it.
 template <int C, bool HI>
 __device__ __forceinline__ void run_batches(const NormParams &prm, const uint4 *cst, long long grp,
                                             long long warps, long long groups, int lane,
@@ -217,11 +232,21 @@ __device__ __forceinline__ void run_batches(const NormParams &prm, const uint4 *
     for (;;) {
         const long long row0 = grp * NB;
         const int nrows = prm.rows - row0 < NB ? static_cast<int>(prm.rows - row0) : NB;
+        const long long nxt = grp + warps;
+        uint4 xn[NB][C];
+        if (nxt < groups) {
+            const long long nrow0 = nxt * NB;
+            load_rows<C>(prm, nrow0, prm.rows - nrow0 < NB ? static_cast<int>(prm.rows - nrow0) : NB,
+                         lane, xn);
+        }
         pass_b<C, HI>(prm, cst, row0, nrows, lane, bt);
-        grp += warps;
-        if (grp >= groups) break;
-        const long long nrow0 = grp * NB;
-        pass_a<C>(prm, nrow0, prm.rows - nrow0 < NB ? static_cast<int>(prm.rows - nrow0) : NB, lane, bt);
+        if (nxt >= groups) break;
+        grp = nxt;
+#pragma unroll
+        for (int r = 0; r < NB; ++r)
+#pragma unroll
+            for (int j = 0; j < C; ++j) bt.xv[r][j] = xn[r][j];
+        pass_a_stats<C>(prm, lane, bt);
     }
 }
 
@@ -232,7 +257,7 @@ __device__ __forceinline__ void run_batches(const NormParams &prm, const uint4 *
 // batch's pass A runs before the channel records are built, so its loads
 // overlap that set-up.
 template <int C>
-__global__ void __launch_bounds__(THREADS, C <= 2 ? 3 : 2)
+__global__ void __launch_bounds__(THREADS, 1)
     layernorm_i8_kernel(const NormParams prm) {
     constexpr int D = 512 * C;
     extern __shared__ uint8_t smem_raw[];
