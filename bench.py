@@ -226,9 +226,21 @@ def cpu_sample(layers, threads: int, target_s: float):
                            np.ascontiguousarray(lay.v[:nb]), lay.p, lay.u, lay.vb, c)
     dt = time.perf_counter() - t
     ops = useful_ops(nb, w.H, w.T, w.dh, len(layers))
+    # the same oracle on one thread, one 10 s utterance (B=1, T=125)
+    w1 = synth.WORKLOADS[1]
+    l1 = synth.layer(1, 0)
+    c1 = oracle.layer_constants(l1.scales, w1.dh)
+    oracle.set_threads(1)
+    t1 = time.perf_counter()
+    oracle.relpos_mhsa(l1.q, l1.k, l1.v, l1.p, l1.u, l1.vb, c1, l1.lengths)
+    dt1 = time.perf_counter() - t1
+    oracle.set_threads(threads)
     return {"value": ops / dt / 1e12, "unit": "TOPS", "cores": threads, "kind": "oracle",
             "sample": f"{len(layers)} layers x {nb} of {w.B} utterances (T={w.T}, H={w.H}), "
-                      f"{dt:.1f} s, int64 scalar C + OpenMP"}
+                      f"{dt:.1f} s, int64 scalar C + OpenMP",
+            "one_thread": {"value": useful_ops(w1.B, w1.H, w1.T, w1.dh, 1) / dt1 / 1e12,
+                           "unit": "TOPS", "seconds": dt1,
+                           "sample": f"one layer, B={w1.B} H={w1.H} T={w1.T}, 1 thread"}}
 
 
 def run_reference(args):
