@@ -48,7 +48,7 @@ constexpr int STAGES = 4;
 constexpr int A_BYTES = BM * BK;
 constexpr int B_BYTES = BN * BK;
 constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-constexpr int OUT_ROW = 48;             // staged output row of one warp: 32 bytes + pad
+constexpr int OUT_ROW = 48;             // staged output row of an MMA warp: 16 bytes, stride 48 (3 x 16: rows spread over the bank groups)
 constexpr int OUT_WARP_BYTES = 64 * OUT_ROW;
 constexpr int SMEM_OUT = STAGES * STAGE_BYTES;
 constexpr int SMEM_BARS = SMEM_OUT + NCW * OUT_WARP_BYTES;
