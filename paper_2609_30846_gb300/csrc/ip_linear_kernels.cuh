@@ -258,9 +258,10 @@ __global__ void __launch_bounds__(THREADS, 1)
     // + DW_ROWS - 1: lane (rg, cg) = (lane / 8, lane % 8) accumulates rows
     // DW_ROWS dw + RI rg + i (i < RI) and channels MMA_COLS + 8 cg + j (j < 8)
     // with dp4a on the same stages the MMA warps read.  Each lane walks the
-    // eight 16-byte k chunks of a stage starting at chunk rg + cg, so that
-    // the 32 lanes of one 16-byte load touch every bank group of the
-    // swizzled tile equally.
+    // eight 16-byte k chunks of a stage starting at chunk cg: the four lanes
+    // of a channel group then read the same W chunk (one broadcast) and the
+    // eight groups' chunks fall on the eight bank groups of the swizzled
+    // rows, while the X loads of a row group cover every bank group too.
     if (warp >= NCW) {
         const int dw = warp - NCW;
         const int rg = lane >> 3, cg = lane & 7;
@@ -286,7 +287,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                 const uint32_t bbase = stage(s) + A_BYTES + c0 * 128;
 #pragma unroll (DW_UNROLL)
                 for (int c = 0; c < 8; ++c) {
-                    const int kc = (c + rg + cg) & 7;
+                    const int kc = (c + cg) & 7;
                     uint4 a[RI];
 #pragma unroll
                     for (int i = 0; i < RI; ++i)
