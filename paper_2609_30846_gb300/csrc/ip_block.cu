@@ -102,9 +102,19 @@ int ip_dwconv_swish_i8(const int8_t *x, int B, int T, int C, const int8_t *w, in
     p.err = static_cast<int *>(workspace);
     const dim3 grid((C + ipb::DW_THREADS - 1) / ipb::DW_THREADS,
                     (T + ipb::DW_FRAMES - 1) / ipb::DW_FRAMES, B);
-    if (iph::launch_pdl(ipb::dwconv_swish_kernel, grid, dim3(ipb::DW_THREADS), 0,
-                        reinterpret_cast<cudaStream_t>(stream), p) != cudaSuccess)
-        return IP_ERR_CUDA;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    cudaError_t lrc;
+    switch (K) {   // odd, 1 .. DW_KMAX (checked above)
+        case 1: lrc = iph::launch_pdl(ipb::dwconv_swish_kernel<1>, grid, dim3(ipb::DW_THREADS), 0, st, p); break;
+        case 3: lrc = iph::launch_pdl(ipb::dwconv_swish_kernel<3>, grid, dim3(ipb::DW_THREADS), 0, st, p); break;
+        case 5: lrc = iph::launch_pdl(ipb::dwconv_swish_kernel<5>, grid, dim3(ipb::DW_THREADS), 0, st, p); break;
+        case 7: lrc = iph::launch_pdl(ipb::dwconv_swish_kernel<7>, grid, dim3(ipb::DW_THREADS), 0, st, p); break;
+        case 9: lrc = iph::launch_pdl(ipb::dwconv_swish_kernel<9>, grid, dim3(ipb::DW_THREADS), 0, st, p); break;
+        case 11: lrc = iph::launch_pdl(ipb::dwconv_swish_kernel<11>, grid, dim3(ipb::DW_THREADS), 0, st, p); break;
+        case 13: lrc = iph::launch_pdl(ipb::dwconv_swish_kernel<13>, grid, dim3(ipb::DW_THREADS), 0, st, p); break;
+        default: lrc = iph::launch_pdl(ipb::dwconv_swish_kernel<15>, grid, dim3(ipb::DW_THREADS), 0, st, p); break;
+    }
+    if (lrc != cudaSuccess) return IP_ERR_CUDA;
     return cudaGetLastError() == cudaSuccess ? IP_OK : IP_ERR_CUDA;
 }
 

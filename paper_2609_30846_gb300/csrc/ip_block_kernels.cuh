@@ -101,7 +101,9 @@ __device__ __forceinline__ int swish16(int z, const DwParams &p) {
 // Depthwise convolution over time (zero padding at both ends of each
 // utterance), per-channel requantisation onto INT16 (folded BatchNorm), and
 // the Swish onto int8.  Thread: one channel; CTA: 256 channels x DW_FRAMES
-// frames of one utterance, a sliding window of K input frames in registers.
+// frames of one utterance, a sliding window of the K input frames in
+// registers (K, odd, a compile-time constant: no unused taps).
+template <int K>
 __global__ void __launch_bounds__(DW_THREADS) dwconv_swish_kernel(const DwParams p) {
     pdl_launch_dependents();
     pdl_wait();   // the grid before this one on the stream: complete, memory visible
@@ -109,10 +111,10 @@ __global__ void __launch_bounds__(DW_THREADS) dwconv_swish_kernel(const DwParams
     const int t0 = blockIdx.y * DW_FRAMES;
     const int b = blockIdx.z;
     if (c >= p.C) return;
-    const int K = p.K, half = p.K >> 1;
-    int w[DW_KMAX];
+    constexpr int half = K >> 1;
+    int w[K];
 #pragma unroll
-    for (int k = 0; k < DW_KMAX; ++k) w[k] = k < K ? p.w[static_cast<size_t>(c) * K + k] : 0;
+    for (int k = 0; k < K; ++k) w[k] = p.w[static_cast<size_t>(c) * K + k];
     int bias = p.bias[c], mm = p.m[c], ss = p.s[c];
     if (mm < 0 || ss < 0 || ss > 31 || bias >= (1 << 30) || bias <= -(1 << 30)) {
         atomicOr(p.err, ERR_PARAM);
@@ -123,17 +125,17 @@ __global__ void __launch_bounds__(DW_THREADS) dwconv_swish_kernel(const DwParams
     const int8_t *xb = p.x + static_cast<size_t>(b) * p.T * p.C + c;
     int8_t *yb = p.y + static_cast<size_t>(b) * p.T * p.C + c;
     // window[k] holds x[t + k - half] for the current output frame t
-    int win[DW_KMAX];
+    int win[K];
 #pragma unroll
-    for (int k = 0; k < DW_KMAX; ++k) {
+    for (int k = 0; k < K; ++k) {
         const int tt = t0 + k - half;
-        win[k] = (k < K && tt >= 0 && tt < p.T) ? xb[static_cast<size_t>(tt) * p.C] : 0;
+        win[k] = (tt >= 0 && tt < p.T) ? xb[static_cast<size_t>(tt) * p.C] : 0;
     }
     const int tend = t0 + DW_FRAMES < p.T ? t0 + DW_FRAMES : p.T;
     for (int t = t0; t < tend; ++t) {
         int acc = bias;
 #pragma unroll
-        for (int k = 0; k < DW_KMAX; ++k) acc += w[k] * win[k];   // |acc| < 2^30 + 2^18
+        for (int k = 0; k < K; ++k) acc += w[k] * win[k];   // |acc| < 2^30 + 2^18
         // onto INT16: round(m acc / 2^(31+s)); |m acc| < 2^62 + 2^50
         const long long v = static_cast<long long>(mm) * acc + (1ll << (30 + ss));
         const long long h = v >> (31 + ss);
@@ -141,11 +143,9 @@ __global__ void __launch_bounds__(DW_THREADS) dwconv_swish_kernel(const DwParams
         yb[static_cast<size_t>(t) * p.C] = static_cast<int8_t>(swish16(z16, p));
         // slide the window by one frame
 #pragma unroll
-        for (int k = 0; k < DW_KMAX - 1; ++k) win[k] = win[k + 1];
+        for (int k = 0; k < K - 1; ++k) win[k] = win[k + 1];
         const int tn = t + 1 + (K - 1) - half;   // frame entering at slot K - 1
-#pragma unroll
-        for (int k = 0; k < DW_KMAX; ++k)
-            if (k == K - 1) win[k] = (tn < p.T) ? xb[static_cast<size_t>(tn) * p.C] : 0;
+        win[K - 1] = (tn < p.T) ? xb[static_cast<size_t>(tn) * p.C] : 0;
     }
 }
 

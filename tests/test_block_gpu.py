@@ -77,7 +77,9 @@ def test_glu_projection(ip, orc, B, T, K, C):
 
 
 @pytest.mark.parametrize("B,T,C,K", [(1, 1, 256, 9), (2, 33, 256, 9), (3, 100, 512, 5),
-                                     (32, 375, 1024, 9), (1, 70, 300, 15)])
+                                     (32, 375, 1024, 9), (1, 70, 300, 15), (2, 40, 256, 1),
+                                     (2, 40, 256, 3), (1, 50, 256, 7), (1, 50, 256, 11),
+                                     (1, 50, 256, 13)])
 def test_dwconv_swish(ip, orc, B, T, C, K):
     rng = np.random.default_rng(T * C + K)
     x = rng.integers(-127, 128, size=(B, T, C)).astype(np.int8)
