@@ -451,7 +451,7 @@ def measure_next_rows(dev, peak, pipes, steps: int, cpu: bool):
     rows["layernorm_1024"] = row
     del xs, outs, x0
 
-    # one whole integer Conformer block (Eqs. 1-5): 19 launches
+    # one whole integer Conformer block (Eqs. 1-5): 15 launches
     import synth.block as sblock
     from paper_2609_30846_gb300.block import GPU_LAUNCHES, ConformerBlock
     case = sblock.conformer_block(B, T, seed=7300)
@@ -471,7 +471,7 @@ def measure_next_rows(dev, peak, pipes, steps: int, cpu: bool):
     if ip.status(blk.ws, stream) != 0:
         raise SystemExit("conformer block: a kernel reported an error")
     t_eager = statistics.median(times)
-    # the same nineteen launches captured once into a CUDA graph and replayed
+    # the same fifteen launches captured once into a CUDA graph and replayed
     graph = blk.graph(x)
     times = []
     for _ in range(steps):
@@ -493,8 +493,8 @@ def measure_next_rows(dev, peak, pipes, steps: int, cpu: bool):
            "roofline": {"bound": "tensor+dp4a", "achieved": ops / t / 1e12, "peak": both,
                         "unit": "TOPS", "frac": ops / t / 1e12 / both,
                         "frac_of_mma_peak": ops / t / 1e12 / peak, "traffic": None},
-           "kernel": "19 launches: layernorm x5, linear x8 (2 with Swish, 1 with GLU), "
-                     "relpos_mhsa_fused, dwconv_swish, residual x4",
+           "kernel": "15 launches: layernorm x5, linear x8 (2 with Swish, 1 with GLU, 4 with "
+                     "the residual addition), relpos_mhsa_fused, dwconv_swish",
            "gpu_launches": GPU_LAUNCHES}
     if cpu:
         import oracle

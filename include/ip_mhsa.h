@@ -308,6 +308,20 @@ int ip_linear_glu_i8(const int8_t *x, const int8_t *w, const int32_t *bias, cons
                      const int32_t *s, const ip_swish_params *glu, int B, int T, int K, int N,
                      int8_t *y, void *workspace, size_t workspace_bytes, ip_stream_t stream);
 
+/* A linear layer with the residual addition of its output fused (the
+ * output projection, the second feed-forward projections and the second
+ * pointwise convolution of the block, Eqs. 1-4): y = clamp(round(2^-(31+s_r)
+ * (m_x res + m_y z)), -127, 127) with z the requantised int8 output of
+ * ip_linear_i8 on (x, w, bias, m, s).  Bit-identical to ip_linear_i8 then
+ * ip_residual_i8(res, z, m_x, m_y, s_r).  res: device int8 [B][T][N]
+ * row-major, 16-byte aligned, may not alias y; m_x, m_y in [0, 2^31), s_r in
+ * [0, 31] (else IP_ERR_PARAM).  x: [B][T][K] row-major; y: [B][T][N]
+ * row-major.  Other arguments and errors as ip_linear_i8. */
+int ip_linear_residual_i8(const int8_t *x, const int8_t *w, const int32_t *bias,
+                          const int32_t *m, const int32_t *s, const int8_t *res, int32_t m_x,
+                          int32_t m_y, int32_t s_r, int B, int T, int K, int N, int8_t *y,
+                          void *workspace, size_t workspace_bytes, ip_stream_t stream);
+
 /* GLU constants for the grids S_a, S_b of the two halves and S_y of the
  * output (host, float64): q_c = round(2c / S_b), q_one = round(1 / S_t),
  * S_t = |a| (S_b/2)^2, m 2^-(31+s) = S_a S_t / (2 S_y). */

@@ -34,7 +34,7 @@ EXPORTS = (
     "ip_layernorm_i8", "ip_layernorm_constants", "ip_relpos_mhsa_i8_ex", "ip_residual_i8",
     "ip_residual_params", "ip_linear_glu_i8", "ip_glu_params", "ip_dwconv_swish_i8",
     "ip_swish16_params_from_scales", "ip_relpos_mhsa_i8_host_async", "ip_relpos_mhsa_host_status",
-    "ip_set_workspace", "ip_probe_int8_mix",
+    "ip_set_workspace", "ip_probe_int8_mix", "ip_linear_residual_i8",
 )
 
 ROWS = 0    # IP_LAYOUT_ROWS:  [B][T][C]
@@ -150,6 +150,9 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
         lib.ip_linear_glu_i8.argtypes = [P, P, P, P, P, ctypes.POINTER(SwishParams), I, I, I, I, P,
                                          P, ctypes.c_size_t, P]
         lib.ip_linear_glu_i8.restype = I
+        lib.ip_linear_residual_i8.argtypes = [P, P, P, P, P, P, I, I, I, I, I, I, I, P, P,
+                                              ctypes.c_size_t, P]
+        lib.ip_linear_residual_i8.restype = I
         lib.ip_glu_params.argtypes = [D, D, D, ctypes.POINTER(SwishParams)]
         lib.ip_glu_params.restype = I
         lib.ip_dwconv_swish_i8.argtypes = [P, I, I, I, P, I, P, P, P, ctypes.POINTER(Swish16Params),
@@ -435,6 +438,30 @@ def linear_i8(x, w, bias, m, s, *, x_layout: int = ROWS, y_layout: int = ROWS, g
     return out
 
 
+def linear_residual_i8(x, w, bias, m, s, res, m_x: int, m_y: int, s_r: int, *, out=None,
+                       workspace=None, stream=None):
+    """Integer linear layer with the residual addition of its output fused:
+    out = residual(res, linear(x)) with (m_x, m_y, s_r) from residual_params.
+    x: int8 [B, T, K]; w: int8 [N, K]; bias, m, s as linear_i8; res: int8
+    [B, T, N] (not aliasing out); all CUDA tensors, row-major."""
+    import torch
+    N, K = w.shape
+    B, T, _ = x.shape
+    if out is None:
+        out = torch.empty((B, T, N), dtype=torch.int8, device=w.device)
+    if workspace is None:
+        workspace = torch.zeros(256, dtype=torch.uint8, device=w.device)
+    bp = None if bias is None else _dev_ptr(bias, "bias", torch.int32, (N,))
+    rc = load().ip_linear_residual_i8(
+        _dev_ptr(x, "x", torch.int8, (B, T, K)), _dev_ptr(w, "w", torch.int8, (N, K)), bp,
+        _dev_ptr(m, "m", torch.int32, (N,)), _dev_ptr(s, "s", torch.int32, (N,)),
+        _dev_ptr(res, "res", torch.int8, (B, T, N)), int(m_x), int(m_y), int(s_r), B, T, K, N,
+        _dev_ptr(out, "out", torch.int8, (B, T, N)), ctypes.c_void_p(workspace.data_ptr()),
+        workspace.numel(), _stream_handle(stream))
+    _check("ip_linear_residual_i8", rc)
+    return out
+
+
 def swish_params_from_scales(S_z: float, S_y: float) -> tuple[int, int, int, int]:
     """Integer constants (q_c, q_one, m, s) of the minimax Swish for an int8
     input on grid S_z and an int8 output on grid S_y (Eqs. 12-13)."""
@@ -636,5 +663,5 @@ __all__ = ["build", "load", "relpos_mhsa_i8", "relpos_mhsa_i8_host", "status", "
            "linear_constants", "ROWS", "HEADS", "linear_swish_i8", "swish_params_from_scales",
            "layernorm_i8", "layernorm_constants", "NormConstants", "residual_i8",
            "residual_params", "linear_glu_i8", "glu_params", "dwconv_swish_i8", "swish16_params",
-           "host_status", "set_workspace", "int8_pipe_rates",
+           "host_status", "set_workspace", "int8_pipe_rates", "linear_residual_i8",
            "IpError", "LibraryError", "EXPORTS"]

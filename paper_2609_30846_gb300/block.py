@@ -2,14 +2,15 @@
 library's kernels, every integer constant derived by the library's own
 offline helpers from the declared grids:
 
-  Z1 = X  + 1/2 FFN1(LN1(X))              (Eq. 1)  LayerNorm, linear + Swish, linear, residual
+  Z1 = X  + 1/2 FFN1(LN1(X))              (Eq. 1)  LayerNorm, linear + Swish, linear + residual
   Z2 = Z1 + MHSA(LN2(Z1))                 (Eq. 2)  LayerNorm, Q/K/V head-split, rel-pos MHSA
-                                                   (row-major output), output projection, residual
+                                                   (row-major output), output projection + residual
   Z3 = Z2 + Conv(LN3(Z2))                 (Eqs. 3, 5) LayerNorm, pointwise + GLU, depthwise
-                                                   + BatchNorm (INT16) + Swish, pointwise, residual
+                                                   + BatchNorm (INT16) + Swish, pointwise + residual
   H  = LN5(Z3 + 1/2 FFN2(LN4(Z3)))        (Eq. 4)
 
-Nineteen launches on one stream, all of them CUDA kernels of this library;
+Each residual addition is fused into the projection before it.  Fifteen
+launches on one stream, all of them CUDA kernels of this library;
 `ConformerBlock.graph` captures them into a CUDA graph that replays with no
 host work per launch.
 The parameter object carries int8 weights with per-channel grids, real
@@ -21,11 +22,11 @@ from __future__ import annotations
 import numpy as np
 
 from . import (HEADS, ROWS, dwconv_swish_i8, glu_params, layer_constants, layernorm_constants,
-               layernorm_i8, linear_constants, linear_glu_i8, linear_i8, linear_swish_i8,
-               relpos_mhsa_i8, residual_i8, residual_params, swish16_params,
+               layernorm_i8, linear_constants, linear_glu_i8, linear_i8, linear_residual_i8,
+               linear_swish_i8, relpos_mhsa_i8, residual_params, swish16_params,
                swish_params_from_scales, workspace_bytes)
 
-GPU_LAUNCHES = 19
+GPU_LAUNCHES = 15
 
 
 class ConformerBlock:
@@ -96,38 +97,39 @@ class ConformerBlock:
             w, b, m, s = self.lin[name]
             linear_i8(src, w, b, m, s, out=dst, workspace=ws, stream=st, **kw)
 
-        def ffn(pre, sw, src):
+        def lin_res(name, src, res, rp, dst):
+            # the projection with the residual addition of its output fused
+            w, b, m, s = self.lin[name]
+            linear_residual_i8(src, w, b, m, s, res, *rp, out=dst, workspace=ws, stream=st)
+
+        def ffn(pre, sw, src, res, rp, dst):
             w, b, m, s = self.lin[pre + "a"]
             linear_swish_i8(src, w, b, m, s, sw, out=h, workspace=ws, stream=st)
-            lin(pre + "b", h, f)
+            lin_res(pre + "b", h, res, rp, dst)
 
         # Eq. 1
         ln("ln1", x, a)
-        ffn("ff1", self.sw1, a)
-        residual_i8(x, f, *self.res[0], out=z[0], stream=st)
+        ffn("ff1", self.sw1, a, x, self.res[0], z[0])
         # Eq. 2
         ln("ln2", z[0], a)
         lin("qkv", a, self.qkv, y_layout=HEADS, groups=3)
         relpos_mhsa_i8(self.qkv[0], self.qkv[1], self.qkv[2], self.p, self.u, self.vb, self.attn,
                        out=self.o, workspace=ws, stream=st, out_layout=ROWS)
-        lin("out", self.o.view(self.B, self.T, self.D), f)
-        residual_i8(z[0], f, *self.res[1], out=z[1], stream=st)
+        lin_res("out", self.o.view(self.B, self.T, self.D), z[0], self.res[1], z[1])
         # Eqs. 3, 5
         ln("ln3", z[1], a)
         w, b, m, s = self.lin["pw1"]
         linear_glu_i8(a, w, b, m, s, self.glu, out=self.g, workspace=ws, stream=st)
         dwconv_swish_i8(self.g, *self.dw, self.sw16, out=a, workspace=ws, stream=st)
-        lin("pw2", a, f)
-        residual_i8(z[1], f, *self.res[2], out=z[2], stream=st)
+        lin_res("pw2", a, z[1], self.res[2], z[2])
         # Eq. 4
         ln("ln4", z[2], a)
-        ffn("ff2", self.sw2, a)
-        residual_i8(z[2], f, *self.res[3], out=z[3], stream=st)
+        ffn("ff2", self.sw2, a, z[2], self.res[3], z[3])
         ln("ln5", z[3], self.out)
         return self.out
 
     def graph(self, x, warmup: int = 2):
-        """Captures the block's nineteen launches on `x` (a fixed int8 [B, T,
+        """Captures the block's fifteen launches on `x` (a fixed int8 [B, T,
         D] CUDA tensor) into a CUDA graph and returns it: `g.replay()` runs
         the block again on whatever `x` then holds, with no host work per
         launch.  The eager call runs `warmup` times first, so that the

@@ -26,15 +26,6 @@ struct ResidualParams {
     int m_x, m_y, s;
 };
 
-// round((m_x x + m_y y) / 2^(31+s)) clamped: |m_x x + m_y y| < 2^39, so the
-// quotient by 2^31 is a 32-bit value (funnel shift), then a shift by s.
-__device__ __forceinline__ int residual_one(int x, int y, const ResidualParams &p) {
-    const long long v = static_cast<long long>(p.m_x) * x + static_cast<long long>(p.m_y) * y +
-                        (1ll << (30 + p.s));
-    const int h = static_cast<int>(__funnelshift_r(static_cast<uint32_t>(v),
-                                                   static_cast<uint32_t>(v >> 32), 31));
-    return clamp127(h >> p.s);
-}
 
 __global__ void __launch_bounds__(RES_THREADS) residual_i8_kernel(const ResidualParams p) {
     pdl_launch_dependents();
@@ -45,26 +36,15 @@ __global__ void __launch_bounds__(RES_THREADS) residual_i8_kernel(const Residual
          i += stride) {
         const uint4 a = __ldcs(reinterpret_cast<const uint4 *>(p.x) + i);
         const uint4 b = __ldcs(reinterpret_cast<const uint4 *>(p.y) + i);
-        const uint32_t aw[4] = {a.x, a.y, a.z, a.w}, bw[4] = {b.x, b.y, b.z, b.w};
-        uint32_t o[4];
-#pragma unroll
-        for (int q = 0; q < 4; ++q) {
-            uint32_t w = 0;
-#pragma unroll
-            for (int e = 0; e < 4; ++e) {
-                const int xa = static_cast<int>(static_cast<int8_t>((aw[q] >> (8 * e)) & 0xffu));
-                const int yb = static_cast<int>(static_cast<int8_t>((bw[q] >> (8 * e)) & 0xffu));
-                w |= (static_cast<uint32_t>(residual_one(xa, yb, p)) & 0xffu) << (8 * e);
-            }
-            o[q] = w;
-        }
-        __stcs(reinterpret_cast<uint4 *>(p.z) + i, make_uint4(o[0], o[1], o[2], o[3]));
+        __stcs(reinterpret_cast<uint4 *>(p.z) + i,
+               make_uint4(residual4(a.x, b.x, p.m_x, p.m_y, p.s), residual4(a.y, b.y, p.m_x, p.m_y, p.s),
+                          residual4(a.z, b.z, p.m_x, p.m_y, p.s), residual4(a.w, b.w, p.m_x, p.m_y, p.s)));
     }
     // the tail of n (fewer than 16 bytes)
     const long long tail = nv << 4;
     const long long k = tail + static_cast<long long>(blockIdx.x) * RES_THREADS + threadIdx.x;
     if (k < p.n && k < tail + 16)
-        p.z[k] = static_cast<int8_t>(residual_one(p.x[k], p.y[k], p));
+        p.z[k] = static_cast<int8_t>(residual_one(p.x[k], p.y[k], p.m_x, p.m_y, p.s));
 }
 
 struct DwParams {

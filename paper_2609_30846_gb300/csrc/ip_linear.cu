@@ -78,6 +78,9 @@ int ensure_smem() {
                              ipl::SMEM_LAUNCH) != cudaSuccess ||
         cudaFuncSetAttribute(ipl::linear_i8_kernel<ipl::EPI_GLU>,
                              cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             ipl::SMEM_LAUNCH) != cudaSuccess ||
+        cudaFuncSetAttribute(ipl::linear_i8_kernel<ipl::EPI_RES>,
+                             cudaFuncAttributeMaxDynamicSharedMemorySize,
                              ipl::SMEM_LAUNCH) != cudaSuccess)
         return IP_ERR_CUDA;
     g_smem_set[dev] = 1;
@@ -92,10 +95,16 @@ int check_swish(const ip_swish_params *p) {
     return IP_OK;
 }
 
+// Residual operand of the RES epilogue: the tensor added and its constants.
+struct ResidualArg {
+    const int8_t *x;
+    int32_t m_x, m_y, s;
+};
+
 int linear_launch(const int8_t *x, int x_layout, const int8_t *w, const int32_t *bias,
                   const int32_t *m, const int32_t *s, const ip_swish_params *sw, int epi, int B,
                   int T, int K, int N, int G, int8_t *y, int y_layout, void *workspace,
-                  size_t workspace_bytes, ip_stream_t stream) {
+                  size_t workspace_bytes, ip_stream_t stream, const ResidualArg *res = nullptr) {
     if ((x_layout != IP_LAYOUT_ROWS && x_layout != IP_LAYOUT_HEADS) ||
         (y_layout != IP_LAYOUT_ROWS && y_layout != IP_LAYOUT_HEADS))
         return IP_ERR_PARAM;
@@ -158,6 +167,10 @@ int linear_launch(const int8_t *x, int x_layout, const int8_t *w, const int32_t 
     prm.sw_qone = sw ? sw->q_one : 0;
     prm.sw_m = sw ? sw->m : 0;
     prm.sw_e = sw ? 31 + sw->s : 0;
+    prm.res = res ? res->x : nullptr;
+    prm.res_mx = res ? res->m_x : 0;
+    prm.res_my = res ? res->m_y : 0;
+    prm.res_s = res ? res->s : 0;
     const int nsm = sm_count();
     if (nsm <= 0) return IP_ERR_CUDA;
     const unsigned grid = prm.ntiles < static_cast<unsigned>(nsm) ? prm.ntiles
@@ -169,6 +182,9 @@ int linear_launch(const int8_t *x, int x_layout, const int8_t *w, const int32_t 
                               ipl::SMEM_LAUNCH, st, tm_x, tm_w, prm);
     else if (epi == ipl::EPI_GLU)
         lrc = iph::launch_pdl(ipl::linear_i8_kernel<ipl::EPI_GLU>, dim3(grid), dim3(ipl::THREADS),
+                              ipl::SMEM_LAUNCH, st, tm_x, tm_w, prm);
+    else if (epi == ipl::EPI_RES)
+        lrc = iph::launch_pdl(ipl::linear_i8_kernel<ipl::EPI_RES>, dim3(grid), dim3(ipl::THREADS),
                               ipl::SMEM_LAUNCH, st, tm_x, tm_w, prm);
     else
         lrc = iph::launch_pdl(ipl::linear_i8_kernel<ipl::EPI_PLAIN>, dim3(grid), dim3(ipl::THREADS),
@@ -207,6 +223,18 @@ int ip_linear_glu_i8(const int8_t *x, const int8_t *w, const int32_t *bias, cons
     if (rc != IP_OK) return rc;
     return linear_launch(x, IP_LAYOUT_ROWS, w, bias, m, s, glu, ipl::EPI_GLU, B, T, K, N, 1, y,
                          IP_LAYOUT_ROWS, workspace, workspace_bytes, stream);
+}
+
+int ip_linear_residual_i8(const int8_t *x, const int8_t *w, const int32_t *bias,
+                          const int32_t *m, const int32_t *s, const int8_t *res, int32_t m_x,
+                          int32_t m_y, int32_t s_r, int B, int T, int K, int N, int8_t *y,
+                          void *workspace, size_t workspace_bytes, ip_stream_t stream) {
+    if (m_x < 0 || m_y < 0 || s_r < 0 || s_r > 31) return IP_ERR_PARAM;
+    if (B > 0 && !res) return IP_ERR_NULL;
+    if (res && !aligned(res, 16)) return IP_ERR_ALIGN;
+    const ResidualArg ra{res, m_x, m_y, s_r};
+    return linear_launch(x, IP_LAYOUT_ROWS, w, bias, m, s, nullptr, ipl::EPI_RES, B, T, K, N, 1, y,
+                         IP_LAYOUT_ROWS, workspace, workspace_bytes, stream, &ra);
 }
 
 int ip_swish_params_from_scales(double S_z, double S_y, ip_swish_params *out) {

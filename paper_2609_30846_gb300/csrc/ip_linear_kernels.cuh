@@ -80,6 +80,9 @@ struct LinearParams {
     long long timeout_cycles;
     // minimax Swish of the requantised output (Eqs. 12-13), SWISH kernels only
     int sw_qc, sw_qone, sw_m, sw_e;
+    // residual addition of the output to res (Eqs. 1-4), RES kernels only
+    const int8_t *res;        // [B][T][N], row-major like the output
+    int res_mx, res_my, res_s;
 };
 
 struct Tile {
@@ -132,6 +135,7 @@ __device__ __forceinline__ int glu_i8(int a, int b, const LinearParams &p) {
 constexpr int EPI_PLAIN = 0;   // requantised int8
 constexpr int EPI_SWISH = 1;   // + minimax Swish
 constexpr int EPI_GLU = 2;     // interleaved pairs (a_c, b_c) -> a_c sigma(b_c)
+constexpr int EPI_RES = 3;     // requantised int8, then the residual addition to res
 
 // Offset in Y of tile row r (0 .. BM - 1) at tile column col, or -1 past the
 // last frame.  Row-major Y [B][T][N] (or [B][T][N / 2] for the gated unit,
@@ -343,7 +347,14 @@ __global__ void __launch_bounds__(THREADS, 1)
                     }
                     const int col = prm.y_layout == LAYOUT_ROWS ? n0 + c0 : c0;
                     const long long off = y_offset(prm, L, r0 + i, col, prm.N, hh, grp);
-                    if (off >= 0) *reinterpret_cast<uint2 *>(prm.y + off) = make_uint2(w[0], w[1]);
+                    if (off >= 0) {
+                        if (EPI == EPI_RES) {
+                            const uint2 xr = *reinterpret_cast<const uint2 *>(prm.res + off);
+                            w[0] = residual4(xr.x, w[0], prm.res_mx, prm.res_my, prm.res_s);
+                            w[1] = residual4(xr.y, w[1], prm.res_mx, prm.res_my, prm.res_s);
+                        }
+                        *reinterpret_cast<uint2 *>(prm.y + off) = make_uint2(w[0], w[1]);
+                    }
                 }
             }
         }
@@ -476,10 +487,19 @@ __global__ void __launch_bounds__(THREADS, 1)
 #pragma unroll
         for (int it = 0; it < 2; ++it) {
             const int r = 32 * it + lane;
-            const uint4 v = lds128(ob + r * OUT_ROW);
+            uint4 v = lds128(ob + r * OUT_ROW);
             const int col = prm.y_layout == LAYOUT_ROWS ? n0 + 16 * wn : 16 * wn;
             const long long off = y_offset(prm, L, 64 * wm + r, col, prm.N, hh, grp);
-            if (off >= 0) *reinterpret_cast<uint4 *>(prm.y + off) = v;
+            if (off >= 0) {
+                if (EPI == EPI_RES) {
+                    const uint4 xr = *reinterpret_cast<const uint4 *>(prm.res + off);
+                    v = make_uint4(residual4(xr.x, v.x, prm.res_mx, prm.res_my, prm.res_s),
+                                   residual4(xr.y, v.y, prm.res_mx, prm.res_my, prm.res_s),
+                                   residual4(xr.z, v.z, prm.res_mx, prm.res_my, prm.res_s),
+                                   residual4(xr.w, v.w, prm.res_mx, prm.res_my, prm.res_s));
+                }
+                *reinterpret_cast<uint4 *>(prm.y + off) = v;
+            }
         }
         __syncwarp();
     }

@@ -202,6 +202,29 @@ __device__ __forceinline__ int clamp127(long long x) {
     return x > 127 ? 127 : (x < -127 ? -127 : static_cast<int>(x));
 }
 
+// Residual addition of Eqs. 1-4 for one element: round((m_x x + m_y y) /
+// 2^(31+s)) clamped to [-127, 127]; |m_x x + m_y y| < 2^39, so the quotient
+// by 2^31 is a 32-bit value (funnel shift), then a shift by s.
+__device__ __forceinline__ int residual_one(int x, int y, int m_x, int m_y, int s) {
+    const long long v = static_cast<long long>(m_x) * x + static_cast<long long>(m_y) * y +
+                        (1ll << (30 + s));
+    const int h = static_cast<int>(__funnelshift_r(static_cast<uint32_t>(v),
+                                                   static_cast<uint32_t>(v >> 32), 31));
+    return clamp127(h >> s);
+}
+
+// Residual addition of four packed int8 pairs (byte e of x with byte e of y).
+__device__ __forceinline__ uint32_t residual4(uint32_t x, uint32_t y, int m_x, int m_y, int s) {
+    uint32_t w = 0;
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+        const int xa = static_cast<int>(static_cast<int8_t>((x >> (8 * e)) & 0xffu));
+        const int yb = static_cast<int>(static_cast<int8_t>((y >> (8 * e)) & 0xffu));
+        w |= (static_cast<uint32_t>(residual_one(xa, yb, m_x, m_y, s)) & 0xffu) << (8 * e);
+    }
+    return w;
+}
+
 // (c << 16) | (sat8(a) << 8) | sat8(b): two int32 values saturated to
 // [-128, 127] and packed below the low half of c (cvt.pack.sat).
 __device__ __forceinline__ uint32_t pack_sat2(int a, int b, uint32_t c) {

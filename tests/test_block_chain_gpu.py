@@ -1,4 +1,4 @@
-"""The whole integer Conformer block (Sec. 2.1 Eqs. 1-5) on the GPU, nineteen
+"""The whole integer Conformer block (Sec. 2.1 Eqs. 1-5) on the GPU, fifteen
 kernel launches, against the oracle's composition of the same block:
 bit-exact on every output."""
 import numpy as np
@@ -34,7 +34,7 @@ def test_block_matches_oracle(ip, B, T, seed):
 
 
 def test_block_graph_replay_matches_oracle(ip):
-    # the nineteen launches captured once into a CUDA graph; each replay on a
+    # the fifteen launches captured once into a CUDA graph; each replay on a
     # new input equals the oracle's block on that input
     import synth.block as sb
     from oracle.block import conformer_block as oracle_block

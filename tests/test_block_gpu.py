@@ -1,5 +1,5 @@
 """Parity of the remaining Conformer-block kernels with the oracle (bit-exact):
-residual additions, the GLU projection, the depthwise convolution with
+residual additions (alone and fused into a projection), the GLU projection, the depthwise convolution with
 folded BatchNorm on INT16 followed by the Swish."""
 import numpy as np
 import pytest
@@ -47,6 +47,26 @@ def test_residual(ip, orc, n, alpha):
     m_x, m_y, s = orc.residual_params(0.05, 0.03, 0.06, alpha)
     got = ip.residual_i8(_d(x), _d(y), m_x, m_y, s).cpu().numpy()
     assert_same(got, orc.residual(x, y, m_x, m_y, s))
+
+
+@pytest.mark.parametrize("B,T,K,N,alpha", [(1, 5, 128, 128, 1.0), (2, 130, 256, 384, 0.5),
+                                           (3, 200, 1024, 256, 0.5), (32, 375, 1024, 1024, 1.0)])
+def test_linear_residual(ip, orc, B, T, K, N, alpha):
+    # the projection with the residual addition fused, against the oracle's
+    # linear layer followed by its residual addition; the tile's last frames
+    # (B T not a multiple of 128) and both column halves of every tile
+    lc = synth.linear(B, T, K, N, seed=700 + T + N)
+    m, s = orc.linear_constants(lc.s_x, lc.s_w, lc.s_y_per_channel())
+    rng = np.random.default_rng(T + N)
+    res = rng.integers(-127, 128, size=(B, T, N)).astype(np.int8)
+    s_y = float(lc.s_y[0])
+    rp = orc.residual_params(0.05, s_y, 1.2 * max(0.05, s_y), alpha)   # both ratios below 1
+    want = orc.residual(res, orc.linear(lc.x, lc.w, lc.bias, m, s), *rp)
+    ws = torch.zeros(256, dtype=torch.uint8, device="cuda")
+    got = ip.linear_residual_i8(_d(lc.x), _d(lc.w), _d(lc.bias), _d(m), _d(s), _d(res), *rp,
+                                workspace=ws)
+    assert ip.status(ws) == 0
+    assert_same(got.cpu().numpy(), want)
 
 
 def interleave(w):
