@@ -244,6 +244,31 @@ def test_descriptor_cache_across_buffers(ip, orc):
             assert_same(out.cpu().numpy(), want[i])
 
 
+def test_descriptor_cache_same_pointer_other_shape(ip, orc):
+    # One allocation seen as two problem shapes at the same base address:
+    # the cached TMA descriptors are keyed by pointer and shape, so each
+    # call must still see its own shape.
+    shapes = [(2, 2, 100), (1, 2, 200), (2, 2, 100)]
+    n = max(b * h * t * 128 for b, h, t in shapes)
+    np_ = max(h * (2 * t - 1) * 128 for b, h, t in shapes)
+    bufs = {k: torch.empty(n, dtype=torch.int8, device="cuda") for k in "qkv"}
+    pbuf = torch.empty(np_, dtype=torch.int8, device="cuda")
+    ws = torch.zeros(256, dtype=torch.uint8, device="cuda")
+    for i, (B, H, T) in enumerate(shapes):
+        lay = synth.draw(B, H, T, 128, seed=1400 + i, p_mode="sinusoid")
+        c = ip.layer_constants(lay.scales)
+        views = {}
+        for k, a in (("q", lay.q), ("k", lay.k), ("v", lay.v)):
+            views[k] = bufs[k][:a.size].view(a.shape)
+            views[k].copy_(torch.from_numpy(np.ascontiguousarray(a)))
+        pv = pbuf[:lay.p.size].view(lay.p.shape)
+        pv.copy_(torch.from_numpy(np.ascontiguousarray(lay.p)))
+        out = ip.relpos_mhsa_i8(views["q"], views["k"], views["v"], pv, _dev(lay.u), _dev(lay.vb),
+                                c, workspace=ws)
+        assert ip.status(ws) == 0
+        assert_same(out.cpu().numpy(), oracle_out(orc, lay, c))
+
+
 def test_back_to_back_launches_see_the_previous_output(ip, orc):
     # Each launch may be scheduled while the one before it on the stream
     # finishes (programmatic dependent launch) and must wait for it before
