@@ -6,21 +6,33 @@ import numpy as np
 import pytest
 
 import synth
+import ibert_bounds as ib
 from fp64_ref import attention_f64
 
-# Stated agreement of the integer layer with the float64 rel-pos attention
-# (Eqs. 8-9, real scales, fused score clipped to its grid, exact softmax,
-# output quantised onto S_O), in output LSB: (max, mean) by the fineness of
-# the score grid, q_ln2 = floor(ln2 / S_s).  The integer path rounds the
-# fused score onto its int8 grid, approximates exp, and keeps probabilities
-# on the grid 2^-8; on a coarse score grid the integer exponential dominates
-# the error (see test_oracle_softmax.lsb_bound).
-def layer_bound(q_ln2: int) -> tuple[float, float]:
-    if q_ln2 >= 16:
-        return 6, 0.85
-    if q_ln2 >= 10:
-        return 12, 1.0
-    return 32, 3.0
+def derived_bound(lay, c, lengths=None):
+    """Per-output bound of |O_int - O_ref| in output steps, derived from the
+    roundings of the method (tests/ibert_bounds.py, step 6): the fused
+    score's rounding onto its int8 grid, the integer exponential's floors and
+    its halving every floor(ln2 / S_s) steps, the floor onto the probability
+    grid 2^-8, and the two roundings onto the output grid.  O_ref is the
+    float64 rel-pos attention of fp64_ref (real scales, fused score clipped
+    to its grid, exact softmax, output quantised onto S_O)."""
+    _, want, probs, scores = attention_f64(lay, lengths)
+    r = lay.scales["S_V"] / lay.scales["S_O"]
+    bound = ib.layer_output_bound(probs, scores, lay.v, lay.scales["S_s"], c.shifts[0], r,
+                                  c.multipliers[2], c.shifts[1])
+    return bound, want
+
+
+def _check_layer(oracle_lib, lay):
+    c = oracle_lib.layer_constants(lay.scales, lay.q.shape[-1])
+    got = oracle_lib.relpos_mhsa(lay.q, lay.k, lay.v, lay.p, lay.u, lay.vb, c, lay.lengths)
+    bound, want = derived_bound(lay, c, lay.lengths)
+    err = np.abs(got.astype(np.int64) - want)
+    worst = np.unravel_index(np.argmax(err - bound), err.shape)
+    assert (err <= bound).all(), (c.softmax, int(err[worst]), float(bound[worst]), worst)
+    assert (got != -128).all()
+    return err, bound
 
 
 CASES = [
@@ -40,23 +52,35 @@ def test_layer_vs_float64_attention(oracle_lib, w, B, T, seed):
     W = synth.WORKLOADS[w]
     lay = synth.draw(B, W.H, T, W.dh, seed=1000 * w + seed, p_mode=W.p_mode,
                      dist=W.dist, masked=W.masked)
-    c = oracle_lib.layer_constants(lay.scales, W.dh)
-    got = oracle_lib.relpos_mhsa(lay.q, lay.k, lay.v, lay.p, lay.u, lay.vb, c, lay.lengths)
-    _, want, _, _ = attention_f64(lay, lay.lengths)
-    err = np.abs(got.astype(np.int64) - want)
-    mx, mean = layer_bound(c.softmax[0])
-    assert err.max() <= mx, (c.softmax, err.max())
-    assert err.mean() <= mean, (c.softmax, err.mean())
-    assert (got != -128).all()
+    _check_layer(oracle_lib, lay)
+
+
+def _first_utterance(lay):
+    return synth.Layer(q=lay.q[:1], k=lay.k[:1], v=lay.v[:1], p=lay.p, u=lay.u, vb=lay.vb,
+                       lengths=None if lay.lengths is None else lay.lengths[:1],
+                       scales=lay.scales)
+
+
+# The benchmark's encoder layers on the coarsest score grids: layer 13
+# (q_ln2 = 7), layers 1 and 2 (q_ln2 = 8), layer 7 (q_ln2 = 9); one
+# utterance each, with the layer's own scales.
+@pytest.mark.parametrize("index,q_ln2", [(13, 7), (1, 8), (2, 8), (7, 9)])
+def test_encoder_layer_coarse_grid(oracle_lib, index, q_ln2):
+    lay = _first_utterance(synth.layer(3, index))
+    c = oracle_lib.layer_constants(lay.scales, 128)
+    assert c.softmax[0] == q_ln2
+    err, bound = _check_layer(oracle_lib, lay)
+    # informative, not a pin: the error stays well inside the bound on average
+    assert err.mean() <= bound.mean()
 
 
 def test_layer_detects_dropped_terms(oracle_lib):
-    # The float64 comparison is sharp enough to see a missing bias or a
-    # mirrored relative shift: perturbing the inputs that way moves the
-    # result far outside the stated bound.
+    # The derived bound is sharp enough to see a missing bias or a mirrored
+    # relative shift: perturbing the inputs that way moves some outputs
+    # outside it.
     lay = synth.draw(1, 8, 96, 128, seed=4242, p_mode="sinusoid")
     c = oracle_lib.layer_constants(lay.scales, 128)
-    _, want, _, _ = attention_f64(lay)
+    bound, want = derived_bound(lay, c)
     for bad in ("u", "vb", "pflip"):
         q, k, v, p, u, vb = lay.q, lay.k, lay.v, lay.p, lay.u, lay.vb
         if bad == "u":
@@ -67,8 +91,7 @@ def test_layer_detects_dropped_terms(oracle_lib):
             p = np.ascontiguousarray(p[:, ::-1, :])
         got = oracle_lib.relpos_mhsa(q, k, v, p, u, vb, c)
         err = np.abs(got.astype(np.int64) - want)
-        mx, mean = layer_bound(c.softmax[0])
-        assert err.max() > mx and err.mean() > mean, (bad, err.max(), err.mean())
+        assert (err > bound).sum() > 100, (bad, int((err > bound).sum()))
 
 
 def test_masked_layer_equals_truncated_problem(oracle_lib):

@@ -1,9 +1,9 @@
 """The pins must catch plausible mistakes in the oracle.
 
-Each case plants one mistake in a copy of the oracle's C source (on the
-CPU, in a temporary directory), rebuilds it there and runs the fast pins
-against the copy in a subprocess: every mutant must make at least one pin
-fail.
+Each case plants one mistake in a copy of the oracle's C source or of its
+offline constants (on the CPU, in a temporary directory), rebuilds it there
+and runs the fast pins against the copy in a subprocess: every mutant must
+make at least one pin fail.
 """
 import os
 import shutil
@@ -119,10 +119,26 @@ BLOCK_MUTANTS = {
 
 BLOCK_PINS = ["tests/test_oracle_block.py"]
 
+# mistakes in the offline softmax constants that show only on coarse score
+# grids (q_ln2 = 7..9, where one grid step is a large share of ln2 and b):
+# rounding instead of the floors of I-BERT's constants
+CONST_MUTANTS = {
+    "qb_round": ("q_b = math.floor(IBERT_B / S)", "q_b = math.floor(IBERT_B / S + 0.5)"),
+    "qc_round": ("q_c = math.floor(IBERT_C / (IBERT_A * (S * S)))",
+                 "q_c = math.floor(IBERT_C / (IBERT_A * (S * S)) + 0.5)"),
+    "qln2_round": ("q_ln2 = math.floor(LN2 / S)", "q_ln2 = math.floor(LN2 / S + 0.5)"),
+}
+
+CONST_PINS = [
+    "tests/test_oracle_softmax.py::test_iexp_within_derived_bounds",
+    "tests/test_oracle_softmax.py::test_softmax_two_keys_coarse",
+    "tests/test_oracle_layer.py::test_encoder_layer_coarse_grid",
+]
+
 PINS = [
     "tests/test_oracle_relshift.py",
     "tests/test_oracle_scores.py",
-    "tests/test_oracle_softmax.py::test_iexp_polynomial_accuracy",
+    "tests/test_oracle_softmax.py::test_iexp_within_derived_bounds",
     "tests/test_oracle_softmax.py::test_iexp_halving_identity",
     "tests/test_oracle_softmax.py::test_softmax_uniform_closed_form",
     "tests/test_oracle_softmax.py::test_softmax_single_key_is_255",
@@ -139,7 +155,8 @@ def _copy_tree(dst):
 
 
 GROUPS = [(MUTANTS, PINS, "ipo_mhsa.c"), (LINEAR_MUTANTS, LINEAR_PINS, "ipo_linear.c"),
-          (NORM_MUTANTS, NORM_PINS, "ipo_norm.c"), (BLOCK_MUTANTS, BLOCK_PINS, "ipo_block.c")]
+          (NORM_MUTANTS, NORM_PINS, "ipo_norm.c"), (BLOCK_MUTANTS, BLOCK_PINS, "ipo_block.c"),
+          (CONST_MUTANTS, CONST_PINS, "consts.py")]
 
 
 @pytest.mark.slow

@@ -1,12 +1,15 @@
 """Pins of the oracle's integer softmax (I-BERT's integer exponential and
 normalisation, which I-Parakeet uses for the attention, Sec. 2.2 and the
-text after Eq. 11).  Constants from tests/golden/ibert_exp.txt."""
+text after Eq. 11).  Constants from tests/golden/ibert_exp.txt; the error
+bounds against the real exponential and softmax are derived step by step in
+tests/ibert_bounds.py."""
 import math
 import os
 
 import numpy as np
 import pytest
 
+import ibert_bounds as ib
 import synth
 
 GOLDEN = os.path.join(os.path.dirname(__file__), "golden", "ibert_exp.txt")
@@ -23,16 +26,44 @@ def _golden():
     return vals
 
 
+# Score grids of the benchmark's encoder layers that are coarse (q_ln2 = 7,
+# 8, 9): layer 13 (q_ln2 = 7), layers 1 and 2 (8, with frac(b / S) = 0.56
+# and 0.68), layer 7 (9).  9 of the 24 layers have q_ln2 <= 9.
+COARSE_LAYERS = (13, 1, 2, 7)
+_COARSE = None
+_GRIDS = None
+
+
+def _coarse_grids():
+    global _COARSE
+    if _COARSE is None:
+        out = [synth.layer(3, i).scales["S_s"] for i in COARSE_LAYERS]
+        # q_ln2 = 7, 8, 9 with frac(b / S) on both sides of 1/2, so that a
+        # rounded q_b differs from the floored one on some of them
+        for q in (7, 8, 9):
+            for f in (0.1, 0.5, 0.9):
+                out.append(math.log(2) / (q + f))
+        # b / S just above an integer (q_ln2 = 7, 8, 9): the floor of q_b
+        # then loses almost nothing, and a q_c rounded up (frac(c / (a S^2))
+        # = 0.885, 0.664, 0.926 here) shows above the fit
+        for n, f in ((14, 0.01), (17, 0.01), (18, 0.005)):
+            out.append(1.353 / (n + f))
+        _COARSE = out
+    return list(_COARSE)
+
+
 def _grid_params(oracle_lib):
-    out = []
-    for w in range(5):
-        lay = synth.layer(w, 0) if w != 3 else synth.draw(1, 8, 375, 128, 3000, p_mode="sinusoid")
-        S = lay.scales["S_s"]
-        out.append((S, oracle_lib.isoftmax_params(S)))
-    for q in (5, 8, 16, 32, 100, 400):
-        S = math.log(2) / (q + 0.25)
-        out.append((S, oracle_lib.isoftmax_params(S)))
-    return out
+    global _GRIDS
+    if _GRIDS is None:
+        grids = []
+        for w in range(5):
+            lay = synth.layer(w, 0) if w != 3 else synth.draw(1, 8, 375, 128, 3000, p_mode="sinusoid")
+            grids.append(lay.scales["S_s"])
+        grids += _coarse_grids()
+        for q in (5, 16, 32, 100, 400):
+            grids.append(math.log(2) / (q + 0.25))
+        _GRIDS = grids
+    return [(S, oracle_lib.isoftmax_params(S)) for S in _GRIDS]
 
 
 def test_constants_match_golden(oracle_lib):
@@ -55,6 +86,15 @@ def test_params_closed_form(oracle_lib):
     assert q_c == math.floor(0.344 * 10.5 ** 2 / (0.3585 * math.log(2) ** 2))
 
 
+def test_params_worked_values(oracle_lib):
+    # Worked by hand: S = ln2 / 8.5 gives ln2 / S = 8.5, b / S = 1.353 * 8.5 /
+    # 0.693147 = 16.592 and c / (a S^2) = 0.344 * 72.25 / (0.3585 * 0.480453)
+    # = 144.30: (q_ln2, q_b, q_c) = (8, 16, 144), each constant floored.
+    # S = ln2 / 7.9: 7.9, 15.421, 124.64 -> (7, 15, 124).
+    assert oracle_lib.isoftmax_params(math.log(2) / 8.5) == (8, 16, 144)
+    assert oracle_lib.isoftmax_params(math.log(2) / 7.9) == (7, 15, 124)
+
+
 def test_iexp_monotone_exhaustive(oracle_lib):
     for S, prm in _grid_params(oracle_lib):
         e = [oracle_lib.iexp(d, prm) for d in range(-254, 1)]
@@ -70,56 +110,60 @@ def test_iexp_halving_identity(oracle_lib):
             assert oracle_lib.iexp(d - q_ln2, prm) == oracle_lib.iexp(d, prm) // 2
 
 
-def test_iexp_polynomial_accuracy(oracle_lib):
-    # For -q_ln2 < d <= 0 no shift happens and e(d) a S^2 approximates
-    # exp(d S) up to the fit error (2.5e-3) plus the floors of q_b and q_c
-    # (|dL| <= 2 (b/S) + 2 in units of a S^2).
+def test_iexp_within_derived_bounds(oracle_lib):
+    # Every value of the integer exponential against the real fit with the
+    # error its floors allow (tests/ibert_bounds.py, steps 1-3): above it by
+    # nothing (every floor rounds down), below it by less than
+    # (2 a S (x + b)) 2^-z + a S^2.
     for S, prm in _grid_params(oracle_lib):
-        q_ln2 = prm[0]
-        bound = 2.5e-3 + (2 * 1.353 / S + 2) * 0.3585 * S * S
-        for d in range(-q_ln2 + 1, 1):
-            approx = oracle_lib.iexp(d, prm) * 0.3585 * S * S
-            assert abs(approx - math.exp(d * S)) <= bound, (S, d)
+        d = np.arange(-254, 1)
+        e = np.array([oracle_lib.iexp(int(x), prm) for x in d], dtype=np.float64)
+        lo, hi = ib.iexp_bounds(S, d)
+        got = e * ib.A * S * S
+        assert (got <= hi * (1 + ib.REL)).all(), (S, prm, int(d[np.argmax(got - hi)]))
+        assert (got > lo - ib.REL).all(), (S, prm, int(d[np.argmin(got - lo)]))
 
 
-def _softmax_f64(scores, S, valid):
-    x = scores.astype(np.float64) * S
-    n = scores.shape[-1]
-    mask = np.arange(n)[None, :] < valid[:, None]
-    x = np.where(mask, x, -np.inf)
-    mx = np.max(x, axis=-1, keepdims=True)
-    e = np.where(mask, np.exp(x - np.where(np.isfinite(mx), mx, 0)), 0.0)
-    den = e.sum(-1, keepdims=True)
-    return 256.0 * np.divide(e, den, out=np.zeros_like(e), where=den > 0)
-
-
-# Stated bound of |a_j - 256 softmax_f64(S_s q_s)_j| in output LSB (grid
-# 2^-8), by the fineness of the score grid.  The integer exponential halves
-# every q_ln2 = floor(ln2 / S) steps instead of every ln2 / S, and q_b, q_c
-# are floored; on a coarse int8 score grid that costs up to tens of LSB on
-# a single probability, on a fine grid about one.
-def lsb_bound(q_ln2: int) -> float:
-    if q_ln2 >= 24:
-        return 3.0
-    if q_ln2 >= 16:
-        return 10.0
-    if q_ln2 >= 11:
-        return 24.0
-    return 64.0
+def test_iexp_derived_bounds_worked_value(oracle_lib):
+    # S = ln2 / 8.5 (q_ln2 = 8): at d = 0 there is no shift and x = 0, so
+    # a S^2 e(0) lies in (g(0) - 2 a b S - a S^2, g(0)] = (0.918781, 1.000273];
+    # e(0) = 16^2 + 144 = 400 and 400 a S^2 = 0.953591.
+    S = math.log(2) / 8.5
+    lo, hi = ib.iexp_bounds(S, np.array([0.0]))
+    assert abs(hi[0] - 1.000273) < 1e-6
+    assert abs(lo[0] - 0.918781) < 1e-6
+    assert oracle_lib.iexp(0, oracle_lib.isoftmax_params(S)) == 400
+    assert lo[0] < 400 * 0.3585 * S * S <= hi[0]
 
 
 @pytest.mark.parametrize("n", [1, 2, 7, 64, 375, 1500])
 def test_softmax_vs_float64(oracle_lib, n):
+    # Each probability within the derived bounds of tests/ibert_bounds.py
+    # (steps 4-5) around 256 times the real softmax of the same scores.
     rng = np.random.default_rng(n)
     for S, prm in _grid_params(oracle_lib):
         for sig in (5, 30, 90):
             sc = np.clip(np.rint(rng.normal(0, sig, size=(40, n))), -127, 127).astype(np.int8)
             valid = rng.integers(1, n, size=40, endpoint=True).astype(np.int32)
             a = oracle_lib.isoftmax(sc, prm, valid).astype(np.float64)
-            ref = _softmax_f64(sc, S, valid)
-            err = np.abs(a - ref)
-            assert err.max() <= lsb_bound(prm[0]), (S, prm, sig, err.max())
-            assert err.mean() <= max(1.5, lsb_bound(prm[0]) / 8), (S, prm, sig, err.mean())
+            lower, upper, _ = ib.softmax_bounds(sc, S, valid)
+            assert (a <= upper).all(), (S, prm, sig, float(np.max(a - upper)))
+            assert (a >= lower).all(), (S, prm, sig, float(np.max(lower - a)))
+
+
+def test_softmax_two_keys_coarse(oracle_lib):
+    # Two keys q_ln2 grid steps apart on a coarse grid: the real weights are
+    # 1 and exp(-q_ln2 S) (between 1/2 and 0.55), the integer ones L(0) and
+    # floor(L(0) / 2).  The result lies within the derived bounds, and the
+    # bounds are tight here: less than 5 steps wide.
+    for S in _coarse_grids():
+        prm = oracle_lib.isoftmax_params(S)
+        sc = np.array([[100, 100 - prm[0]]], np.int8)
+        valid = np.array([2], np.int32)
+        a = oracle_lib.isoftmax(sc, prm, valid).astype(np.float64)
+        lower, upper, _ = ib.softmax_bounds(sc, S, valid)
+        assert ((lower <= a) & (a <= upper)).all(), (S, a, lower, upper)
+        assert (upper - lower < 5).all(), (S, lower, upper)
 
 
 def test_softmax_row_sum_bounds(oracle_lib):
