@@ -15,10 +15,14 @@ far above the 129 MB L2, so nothing is reused across steps from L2).
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
 
-Multi-GPU: the path shards with no exchange step; each rank runs its own
-replica of the workload (weak scaling) and `value` sums the ranks' work over
-the slowest rank's time.  `--impl reference` times the CPU oracle on the
-host cores instead (rank 0 only).
+Multi-GPU: the path shards with no exchange step (Sec. 3.1 works per
+utterance and head, so replicas need no collective on the data path); each
+rank runs its own replica of the workload (weak scaling) and `value` sums
+the ranks' work over the slowest rank's time.  `--gpus N` with N > 1 and no
+WORLD_SIZE in the environment re-launches this script as N ranks under
+torch.distributed.run; launched that way already (WORLD_SIZE set), it runs
+as one of them.  `--impl reference` times the CPU oracle on the host cores
+instead (rank 0 only).
 """
 from __future__ import annotations
 
@@ -153,6 +157,78 @@ def useful_ops(B, H, T, dh, layers):
     return 6 * dh * T * T * B * H * layers
 
 
+def spawn_replicas(nproc: int, argv: list[str], env: dict | None = None) -> int:
+    """Runs `python argv...` as `nproc` ranks of one node under
+    torch.distributed.run (rendezvous on 127.0.0.1, a free port) and returns
+    its exit status; the ranks read RANK / LOCAL_RANK / WORLD_SIZE."""
+    import socket
+    with socket.socket() as so:
+        so.bind(("127.0.0.1", 0))
+        port = so.getsockname()[1]
+    cmd = [sys.executable, "-m", "torch.distributed.run", "--nnodes", "1",
+           "--nproc-per-node", str(nproc), "--master-addr", "127.0.0.1",
+           "--master-port", str(port)] + list(argv)
+    run_env = dict(os.environ if env is None else env)
+    for k in ("WORLD_SIZE", "RANK", "LOCAL_RANK"):
+        run_env.pop(k, None)
+    return subprocess.run(cmd, env=run_env).returncode
+
+
+class HostTimer:
+    """Wall-clock timer of a timed region (host work, or GPU work followed
+    by a synchronisation inside the region)."""
+
+    def start(self):
+        self.t0 = time.perf_counter()
+
+    def stop(self) -> float:
+        return (time.perf_counter() - self.t0) * 1e3
+
+
+class EventTimer:
+    """CUDA events on the launching stream; stop() waits for the end event."""
+
+    def __init__(self, stream):
+        import torch
+        self.stream = stream
+        self.e0 = torch.cuda.Event(enable_timing=True)
+        self.e1 = torch.cuda.Event(enable_timing=True)
+
+    def start(self):
+        self.e0.record(self.stream)
+
+    def stop(self) -> float:
+        self.e1.record(self.stream)
+        self.e1.synchronize()
+        return self.e0.elapsed_time(self.e1)
+
+
+def time_replicas(step, steps: int, dist, timer, sync=lambda: None, device=None):
+    """Times `steps` calls of `step` on this rank, bracketed by a barrier and
+    `sync` on both sides, and returns (this rank's ms, the slowest rank's
+    ms).  Every rank runs its own replica; the job ends with its slowest."""
+    if dist is not None:
+        dist.barrier()
+    sync()
+    timer.start()
+    for _ in range(steps):
+        step()
+    ms = timer.stop()
+    sync()
+    if dist is not None:
+        dist.barrier()
+    return ms, slowest(dist, ms, device)
+
+
+def replica_fields(world: int, ops_per_step: float, steps: int, job_ms: float) -> dict:
+    """The bench line's job-level fields for `world` replicas of one step of
+    `ops_per_step` useful ops each: the value counts every rank's work over
+    the slowest rank's time (weak scaling)."""
+    return {"value": job_tops(ops_per_step * steps, world, job_ms * 1e-3), "n_gpus": world,
+            "ms_per_step": job_ms / steps, "scaling": "weak",
+            "parallelism": f"replicas x{world}" if world > 1 else "1 GPU"}
+
+
 def slowest(dist, x: float, device=None) -> float:
     """Max of a per-rank time over all ranks (x itself without a process
     group): the job ends when its slowest replica ends."""
@@ -269,7 +345,7 @@ def run_reference(args):
     ms = dt / args.steps * 1e3
     sample = f"per step {w.layers} layers x 1 of {w.B} utterances (T={w.T}, H={w.H})"
     line = {
-        "impl": "reference", "metric": METRIC, "value": value, "unit": "TOPS", "n_gpus": args.gpus,
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "TOPS", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "int64", "data": "synthetic",
         "config": {"workload": f"{w.name} (sampled: 1 utterance per layer)", "B": 1, "T": w.T,
@@ -615,30 +691,21 @@ def run_ours(args):
     # the stream (a layer's kernel may then be scheduled while the previous
     # one finishes; it waits for it before touching memory), so the timed
     # region has one pair of events and the per-launch time is its average.
-    t0 = torch.cuda.Event(enable_timing=True)
-    t1 = torch.cuda.Event(enable_timing=True)
     clocks = ClockSampler(local)
     clocks.start()
-    if dist:
-        dist.barrier()
-    torch.cuda.synchronize(dev)
-    t0.record(stream)
-    for s in range(args.steps):
-        step()
-    t1.record(stream)
-    torch.cuda.synchronize(dev)
-    if dist:
-        dist.barrier()
+    own_ms, total_ms = time_replicas(step, args.steps, dist, EventTimer(stream),
+                                     sync=lambda: torch.cuda.synchronize(dev), device=dev)
     clk = clocks.stop()
-    total_ms = t0.elapsed_time(t1)
     if ip.status(ws, stream) != 0:
         raise SystemExit("kernel reported a barrier timeout in the timed region")
-
-    total_ms = slowest(dist, total_ms, dev)
+    if world > 1:
+        print(json.dumps({"rank": rank, "ms": own_ms, "steps": args.steps}), file=sys.stderr,
+              flush=True)
 
     ops_step = useful_ops(B, H, T, dh, NL)
-    value = job_tops(ops_step * args.steps, world, total_ms * 1e-3)
-    ms_step = total_ms / args.steps
+    job = replica_fields(world, ops_step, args.steps, total_ms)
+    value = job["value"]
+    ms_step = job["ms_per_step"]
     ops_layer = useful_ops(B, H, T, dh, 1)
     avg_layer_ms = total_ms / (args.steps * NL)   # launch gaps included
     achieved = ops_layer / (avg_layer_ms * 1e-3) / 1e12
@@ -701,13 +768,13 @@ def run_ours(args):
 
     bytes_layer = 4 * B * H * T * dh + H * (2 * T - 1) * dh + 2 * H * dh
     line = {
-        "metric": METRIC, "value": value, "unit": "TOPS", "n_gpus": world, "steps": args.steps,
-        "warmup": max(args.warmup, 3), "ms_per_step": ms_step, "higher_is_better": True,
-        "scaling": "weak", "vs_baseline": None, "dtype": "s8xs8->s32 (int32/int64 epilogue)",
+        "metric": METRIC, "value": value, "unit": "TOPS", "n_gpus": job["n_gpus"],
+        "steps": args.steps, "warmup": max(args.warmup, 3), "ms_per_step": ms_step,
+        "higher_is_better": True, "scaling": job["scaling"], "vs_baseline": None, "dtype": "s8xs8->s32 (int32/int64 epilogue)",
         "data": "synthetic",
         "config": {"workload": w.name + (" (REDUCED, profiling only)" if reduced else ""),
                    "B": B, "H": H, "T": T, "dh": dh, "layers": NL,
-                   "parallelism": f"replicas x{world}" if world > 1 else "1 GPU",
+                   "parallelism": job["parallelism"],
                    "l2": "inputs larger than L2 (%.2f GB per step, L2 129 MB)" % (bytes_layer * NL / 1e9)},
         "rtf": ms_step * 1e-3 / (B * UTT_SECONDS),
         "paper_rtf_npu_full_model": 0.048,
@@ -737,6 +804,17 @@ def run_ours(args):
 
 def main():
     args = parse_args()
+    if args.gpus > 1 and "WORLD_SIZE" not in os.environ:
+        # N replicas were asked for without a launcher: become N ranks
+        if args.impl == "ours":
+            import torch
+            have = torch.cuda.device_count() if torch.cuda.is_available() else 0
+            if have < args.gpus:
+                raise SystemExit(f"--gpus {args.gpus}: only {have} CUDA device(s) visible")
+        return spawn_replicas(args.gpus, [os.path.abspath(__file__)] + sys.argv[1:])
+    world, _, _ = dist_env()
+    if world != args.gpus and args.gpus > 1:
+        raise SystemExit(f"--gpus {args.gpus} but WORLD_SIZE={world}")
     if args.impl == "reference":
         return run_reference(args)
     return run_ours(args)
