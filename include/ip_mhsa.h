@@ -454,6 +454,40 @@ int ip_dyadic_pair(double r_c, double r_p, int32_t *m_c, int32_t *m_p, int32_t *
 /* I-BERT exponential constants on the score grid S_s (see the struct). */
 int ip_isoftmax_params_from_scale(double S_s, ip_isoftmax_params *out);
 
+/* Every integer constant of one attention layer from its real scales
+ * (offline, float64, as the paper precomputes its multipliers, Sec. 2.2
+ * under Eq. 7), ready for ip_relpos_mhsa_i8:
+ *   Eq. 11: the branch ratios r_c = S_Q S_K / (S_s sqrt(dh)) and
+ *     r_p = S_Q S_P / (S_s sqrt(dh)) (u and v live on Q's grid, so the
+ *     content and position branches carry S_Q S_K and S_Q S_P) as one
+ *     dyadic pair on a shared shift (ip_dyadic_pair): multipliers[0..1] =
+ *     {m_c, m_p}, shifts[0] = s_s;
+ *   Eq. 7 after Eq. 9: the probabilities sit on the grid 2^-8, so the
+ *     output ratio is r_o = 2^-8 S_V / S_O: multipliers[2] = m_o,
+ *     shifts[1] = s_o (ip_dyadic_multiplier);
+ *   the I-BERT exponential constants on S_s (ip_isoftmax_params_from_scale).
+ * S_Q, S_K, S_P, S_V: the int8 grids of Q (and u, v), K, P and V; S_s: the
+ * fused score's int8 grid; S_O: the output's; dh: head size (the scale of
+ * Eq. 8 is 1/sqrt(dh)).  multipliers (3), shifts (2), softmax: host memory
+ * owned by the caller.  Returns IP_OK; IP_ERR_NULL for a NULL output;
+ * IP_ERR_PARAM when a scale is not positive and finite, dh < 1, or a ratio
+ * cannot be encoded (the outputs are then left untouched). */
+int ip_relpos_layer_constants(double S_Q, double S_K, double S_P, double S_V, double S_s,
+                              double S_O, int dh, int32_t *multipliers, int32_t *shifts,
+                              ip_isoftmax_params *softmax);
+
+/* Per-output-channel constants of Eq. 7 for ip_linear_i8 and its variants
+ * (offline, float64): weights carry one scale per output channel (Sec. 2.2),
+ * so channel n < N requantises with m[n] 2^-(31+s[n]), the dyadic nearest
+ * to S_x S_w[n] / S_y[n] (ip_dyadic_multiplier).  S_x: the input's grid;
+ * S_w, S_y: host arrays of N weight and output grids (repeat one output grid
+ * for a per-tensor output); m, s: host int32 arrays of N owned by the
+ * caller.  Returns IP_OK; IP_ERR_NULL for a NULL array; IP_ERR_PARAM when
+ * N < 1, a scale is not positive and finite or a ratio cannot be encoded
+ * (m and s are then left untouched). */
+int ip_linear_constants(double S_x, const double *S_w, const double *S_y, int N, int32_t *m,
+                        int32_t *s);
+
 #ifdef __cplusplus
 }
 #endif

@@ -9,7 +9,6 @@ streams only.
 from __future__ import annotations
 
 import ctypes
-import math
 import threading
 from dataclasses import dataclass
 
@@ -35,6 +34,7 @@ EXPORTS = (
     "ip_residual_params", "ip_linear_glu_i8", "ip_glu_params", "ip_dwconv_swish_i8",
     "ip_swish16_params_from_scales", "ip_relpos_mhsa_i8_host_async", "ip_relpos_mhsa_host_status",
     "ip_set_workspace", "ip_probe_int8_mix", "ip_linear_residual_i8",
+    "ip_relpos_layer_constants", "ip_linear_constants",
 )
 
 ROWS = 0    # IP_LAYOUT_ROWS:  [B][T][C]
@@ -121,6 +121,13 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
         lib.ip_dyadic_pair.restype = I
         lib.ip_isoftmax_params_from_scale.argtypes = [ctypes.c_double, ctypes.POINTER(SoftmaxParams)]
         lib.ip_isoftmax_params_from_scale.restype = I
+        D_ = ctypes.c_double
+        lib.ip_relpos_layer_constants.argtypes = [D_] * 6 + [I, P, P, ctypes.POINTER(SoftmaxParams)]
+        lib.ip_relpos_layer_constants.restype = I
+        lib.ip_linear_constants.argtypes = [D_, ctypes.POINTER(D_), ctypes.POINTER(D_), I,
+                                            ctypes.POINTER(ctypes.c_int32),
+                                            ctypes.POINTER(ctypes.c_int32)]
+        lib.ip_linear_constants.restype = I
         lib.ip_relpos_mhsa_i8_ex.argtypes = [P] * 6 + [P, P, ctypes.POINTER(SoftmaxParams), P] + [
             I] * 4 + [P, I, P, ctypes.c_size_t, P]
         lib.ip_relpos_mhsa_i8_ex.restype = I
@@ -205,15 +212,15 @@ def isoftmax_params_from_scale(S_s: float) -> tuple[int, int, int]:
 
 
 def layer_constants(scales: dict, dh: int = IP_DH) -> LayerConstants:
-    """Integer constants of one layer from its real scales (offline, Eq. 7
-    and Eq. 11; probabilities on the grid 2^-8)."""
-    root = math.sqrt(dh)
-    r_c = scales["S_Q"] * scales["S_K"] / (scales["S_s"] * root)
-    r_p = scales["S_Q"] * scales["S_P"] / (scales["S_s"] * root)
-    r_o = scales["S_V"] / (scales["S_O"] * 256.0)
-    m_c, m_p, s_s = dyadic_pair(r_c, r_p)
-    m_o, s_o = dyadic_multiplier(r_o)
-    return LayerConstants((m_c, m_p, m_o), (s_s, s_o), isoftmax_params_from_scale(scales["S_s"]))
+    """Integer constants of one layer from its real scales S_Q, S_K, S_P,
+    S_V, S_s, S_O (offline, Eq. 7 and Eq. 11), by ip_relpos_layer_constants."""
+    mult = (ctypes.c_int32 * 3)()
+    sh = (ctypes.c_int32 * 2)()
+    sm = SoftmaxParams()
+    _check("ip_relpos_layer_constants", load().ip_relpos_layer_constants(
+        float(scales["S_Q"]), float(scales["S_K"]), float(scales["S_P"]), float(scales["S_V"]),
+        float(scales["S_s"]), float(scales["S_O"]), int(dh), mult, sh, ctypes.byref(sm)))
+    return LayerConstants(tuple(mult), tuple(sh), (sm.q_ln2, sm.q_b, sm.q_c))
 
 
 # ---------------------------------------------------------------- device path
@@ -396,15 +403,20 @@ def set_workspace(workspace) -> None:
 
 
 def linear_constants(s_x: float, s_w, s_y):
-    """Per-output-channel constants of Eq. 7 (offline): int32 arrays m, s
-    with m[n] 2^-(31+s[n]) the dyadic nearest to S_x S_w[n] / S_y[n]."""
+    """Per-output-channel constants of Eq. 7 (offline), by
+    ip_linear_constants: int32 arrays m, s of the length of s_w (s_y: one
+    grid per channel, or one for all)."""
     import numpy as np
-    s_w = np.asarray(s_w, dtype=np.float64)
-    s_y = np.broadcast_to(np.asarray(s_y, dtype=np.float64), s_w.shape)
+    s_w = np.ascontiguousarray(s_w, dtype=np.float64).reshape(-1)
+    s_y = np.ascontiguousarray(np.broadcast_to(np.asarray(s_y, dtype=np.float64).reshape(-1)
+                                               if np.ndim(s_y) else np.float64(s_y), s_w.shape))
     m = np.empty(s_w.shape, dtype=np.int32)
     s = np.empty(s_w.shape, dtype=np.int32)
-    for n in range(s_w.size):
-        m[n], s[n] = dyadic_multiplier(float(s_x) * float(s_w[n]) / float(s_y[n]))
+    dp = ctypes.POINTER(ctypes.c_double)
+    ip32 = ctypes.POINTER(ctypes.c_int32)
+    _check("ip_linear_constants", load().ip_linear_constants(
+        float(s_x), s_w.ctypes.data_as(dp), s_y.ctypes.data_as(dp), int(s_w.size),
+        m.ctypes.data_as(ip32), s.ctypes.data_as(ip32)))
     return m, s
 
 

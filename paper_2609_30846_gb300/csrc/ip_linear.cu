@@ -237,6 +237,22 @@ int ip_linear_residual_i8(const int8_t *x, const int8_t *w, const int32_t *bias,
                          IP_LAYOUT_ROWS, workspace, workspace_bytes, stream, &ra);
 }
 
+int ip_linear_constants(double S_x, const double *S_w, const double *S_y, int N, int32_t *m,
+                        int32_t *s) {
+    if (!S_w || !S_y || !m || !s) return IP_ERR_NULL;
+    if (N < 1 || !(S_x > 0.0) || !std::isfinite(S_x)) return IP_ERR_PARAM;
+    for (int n = 0; n < N; ++n)   // every channel valid before any output is written
+        if (!(S_w[n] > 0.0) || !std::isfinite(S_w[n]) || !(S_y[n] > 0.0) || !std::isfinite(S_y[n]))
+            return IP_ERR_PARAM;
+    for (int n = 0; n < N; ++n) {
+        int32_t mm = 0, ss = 0;
+        if (ip_dyadic_multiplier(S_x * S_w[n] / S_y[n], &mm, &ss) != IP_OK) return IP_ERR_PARAM;
+    }
+    for (int n = 0; n < N; ++n)
+        ip_dyadic_multiplier(S_x * S_w[n] / S_y[n], &m[n], &s[n]);
+    return IP_OK;
+}
+
 int ip_swish_params_from_scales(double S_z, double S_y, ip_swish_params *out) {
     if (!out) return IP_ERR_NULL;
     if (!(S_z > 0.0) || !(S_y > 0.0) || !std::isfinite(S_z) || !std::isfinite(S_y))

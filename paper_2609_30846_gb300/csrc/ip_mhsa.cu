@@ -564,6 +564,33 @@ int ip_isoftmax_params_from_scale(double S_s, ip_isoftmax_params *out) {
     return IP_OK;
 }
 
+int ip_relpos_layer_constants(double S_Q, double S_K, double S_P, double S_V, double S_s,
+                              double S_O, int dh, int32_t *multipliers, int32_t *shifts,
+                              ip_isoftmax_params *softmax) {
+    if (!multipliers || !shifts || !softmax) return IP_ERR_NULL;
+    const double sc[6] = {S_Q, S_K, S_P, S_V, S_s, S_O};
+    for (double x : sc)
+        if (!(x > 0.0) || !isfinite(x)) return IP_ERR_PARAM;
+    if (dh < 1) return IP_ERR_PARAM;
+    const double root = sqrt(static_cast<double>(dh));
+    const double r_c = S_Q * S_K / (S_s * root);   // Eq. 11, content branch
+    const double r_p = S_Q * S_P / (S_s * root);   // Eq. 11, position branch
+    const double r_o = S_V / (S_O * 256.0);        // Eq. 7, probabilities on 2^-8
+    int32_t m_c = 0, m_p = 0, s_s = 0, m_o = 0, s_o = 0;
+    ip_isoftmax_params sm{};
+    int rc = ip_dyadic_pair(r_c, r_p, &m_c, &m_p, &s_s);
+    if (rc == IP_OK) rc = ip_dyadic_multiplier(r_o, &m_o, &s_o);
+    if (rc == IP_OK) rc = ip_isoftmax_params_from_scale(S_s, &sm);
+    if (rc != IP_OK) return rc;
+    multipliers[0] = m_c;
+    multipliers[1] = m_p;
+    multipliers[2] = m_o;
+    shifts[0] = s_s;
+    shifts[1] = s_o;
+    *softmax = sm;
+    return IP_OK;
+}
+
 long long ip_probe_int8_mma(int blocks, int iters, int *sink, ip_stream_t stream) {
     if (blocks < 1 || iters < 1 || !sink) return -1;
     ipk::int8_mma_probe_kernel<<<blocks, ipk::PROBE_THREADS, 0,

@@ -136,6 +136,74 @@ def test_constants_match_oracle(lib):
         assert (c1.multipliers, c1.shifts, c1.softmax) == (c2.multipliers, c2.shifts, c2.softmax)
 
 
+def test_layer_constants_entry_point_matches_oracle(lib):
+    # ip_relpos_layer_constants composes Eq. 11's and Eq. 7's ratios itself;
+    # on random scales it agrees with the oracle's float64 composition, and
+    # both refuse the same unencodable ones.
+    import oracle
+    rng = np.random.default_rng(11)
+    agree = 0
+    for _ in range(400):
+        sc = dict(zip(("S_Q", "S_K", "S_P", "S_V", "S_s", "S_O"), 10.0 ** rng.uniform(-3, 0.3, 6)))
+        dh = int(rng.choice([16, 64, 128]))
+        try:
+            want = oracle.layer_constants(sc, dh)
+        except ValueError:
+            want = None
+        if want is None:
+            with pytest.raises(ip.IpError):
+                ip.layer_constants(sc, dh)
+            continue
+        got = ip.layer_constants(sc, dh)
+        assert (got.multipliers, got.shifts, got.softmax) == \
+            (want.multipliers, want.shifts, want.softmax), sc
+        agree += 1
+    assert agree > 100
+
+
+def test_layer_constants_entry_point_errors(lib):
+    m = (ctypes.c_int32 * 3)(7, 7, 7)
+    sh = (ctypes.c_int32 * 2)(7, 7)
+    sm = ip.SoftmaxParams(7, 7, 7)
+    f = lib.ip_relpos_layer_constants
+    assert f(0.01, 0.01, 0.01, 0.01, 0.1, 0.02, 128, None, sh, ctypes.byref(sm)) == -1
+    for bad in ((0.0, 0.01, 0.01, 0.01, 0.1, 0.02, 128), (0.01, 0.01, 0.01, 0.01, -0.1, 0.02, 128),
+                (0.01, 0.01, 0.01, float("inf"), 0.1, 0.02, 128), (0.01, 0.01, 0.01, 0.01, 0.1, 0.02, 0),
+                (4.0, 4.0, 4.0, 0.01, 0.1, 0.02, 128)):   # the last: r_c >= 1/2, unencodable
+        assert f(*bad, m, sh, ctypes.byref(sm)) == -7, bad
+    assert tuple(m) == (7, 7, 7) and tuple(sh) == (7, 7) and sm.q_ln2 == 7   # untouched
+
+
+def test_linear_constants_entry_point_matches_oracle(lib):
+    import oracle
+    rng = np.random.default_rng(12)
+    for n in (1, 5, 64, 1000):
+        s_x = float(10.0 ** rng.uniform(-3, -1))
+        s_w = 10.0 ** rng.uniform(-4, -1, n)
+        for s_y in (10.0 ** rng.uniform(-3, -1, n), float(10.0 ** rng.uniform(-2, -1))):
+            got = ip.linear_constants(s_x, s_w, s_y)
+            want = oracle.linear_constants(s_x, s_w, s_y)
+            np.testing.assert_array_equal(got[0], want[0])
+            np.testing.assert_array_equal(got[1], want[1])
+    with pytest.raises(ip.IpError):
+        ip.linear_constants(0.01, np.array([1e-3, -1e-3]), 0.01)
+    with pytest.raises(ip.IpError):
+        ip.linear_constants(0.01, np.array([], dtype=np.float64), 0.01)
+    with pytest.raises(ip.IpError):
+        ip.linear_constants(1.0, np.array([1.0]), 0.5)          # ratio 2, unencodable
+
+
+def test_binding_holds_no_scale_arithmetic():
+    # the binding marshals the scales to the C helpers; the ratios of Eq. 7
+    # and Eq. 11 are composed behind the C ABI
+    src = open(os.path.join(ROOT, "paper_2609_30846_gb300", "__init__.py")).read()
+    for fn in ("def layer_constants", "def linear_constants"):
+        start = src.index(fn)
+        body = src[start:src.index("\ndef ", start + 1)]
+        for pat in (r"sqrt", r"\* 256", r"/ \(", r"dyadic_multiplier\(", r"\bfor\s+\w+\s+in\b"):
+            assert not re.search(pat, body), (fn, pat)
+
+
 def test_constants_reject_bad_ratios(lib):
     with pytest.raises(ip.IpError):
         ip.dyadic_multiplier(1.0)
