@@ -18,7 +18,11 @@ def ip():
     return mod
 
 
-@pytest.mark.parametrize("B,T,seed", [(2, 64, 1), (3, 150, 2)])
+# (32, 375): the benchmark's block shape (30 s utterances, 12000 frames);
+# (3, 301): 903 frames, not a multiple of the 128-frame tiles of the
+# projections, and T not a multiple of the attention's 64-row tiles.
+@pytest.mark.parametrize("B,T,seed", [(2, 64, 1), (3, 150, 2), (3, 301, 4), (4, 375, 3),
+                                      (32, 375, 5)])
 def test_block_matches_oracle(ip, B, T, seed):
     import synth.block as sb
     from oracle.block import conformer_block as oracle_block
@@ -30,7 +34,9 @@ def test_block_matches_oracle(ip, B, T, seed):
     assert ip.status(blk.ws) == 0
     got = got.cpu().numpy()
     bad = got != want
-    assert not bad.any(), f"{int(bad.sum())} of {got.size} outputs differ"
+    if bad.any():
+        idx = np.argwhere(bad)[0].tolist()
+        raise AssertionError(f"{int(bad.sum())} of {got.size} outputs differ; first at {idx}")
 
 
 def test_block_graph_replay_matches_oracle(ip):

@@ -4,6 +4,8 @@ folded BatchNorm on INT16 followed by the Swish."""
 import numpy as np
 import pytest
 
+from guard import Guarded
+
 import synth
 
 pytestmark = pytest.mark.gpu
@@ -45,7 +47,9 @@ def test_residual(ip, orc, n, alpha):
     x = rng.integers(-127, 128, size=n).astype(np.int8)
     y = rng.integers(-127, 128, size=n).astype(np.int8)
     m_x, m_y, s = orc.residual_params(0.05, 0.03, 0.06, alpha)
-    got = ip.residual_i8(_d(x), _d(y), m_x, m_y, s).cpu().numpy()
+    g = Guarded(x.shape, torch.int8)
+    got = ip.residual_i8(_d(x), _d(y), m_x, m_y, s, out=g.view).cpu().numpy()
+    g.check()
     assert_same(got, orc.residual(x, y, m_x, m_y, s))
 
 
@@ -63,9 +67,11 @@ def test_linear_residual(ip, orc, B, T, K, N, alpha):
     rp = orc.residual_params(0.05, s_y, 1.2 * max(0.05, s_y), alpha)   # both ratios below 1
     want = orc.residual(res, orc.linear(lc.x, lc.w, lc.bias, m, s), *rp)
     ws = torch.zeros(256, dtype=torch.uint8, device="cuda")
+    g = Guarded(want.shape, torch.int8)
     got = ip.linear_residual_i8(_d(lc.x), _d(lc.w), _d(lc.bias), _d(m), _d(s), _d(res), *rp,
-                                workspace=ws)
+                                out=g.view, workspace=ws)
     assert ip.status(ws) == 0
+    g.check()
     assert_same(got.cpu().numpy(), want)
 
 
@@ -90,9 +96,11 @@ def test_glu_projection(ip, orc, B, T, K, C):
     perm[0::2] = np.arange(C)
     perm[1::2] = np.arange(C) + C
     ws = torch.zeros(256, dtype=torch.uint8, device="cuda")
+    gd = Guarded(want.shape, torch.int8)
     got = ip.linear_glu_i8(_d(lc.x), _d(interleave(lc.w)), _d(lc.bias[perm]), _d(m[perm]),
-                           _d(s[perm]), (g.q_c, g.q_one, g.m, g.s), workspace=ws)
+                           _d(s[perm]), (g.q_c, g.q_one, g.m, g.s), out=gd.view, workspace=ws)
     assert ip.status(ws) == 0
+    gd.check()
     assert_same(got.cpu().numpy(), want)
 
 
@@ -111,9 +119,11 @@ def test_dwconv_swish(ip, orc, B, T, C, K):
     p16 = orc.swish16_params(s_bn, 5.0 / 127)
     want = orc.swish16(orc.dwconv(x, w, bias, m, s), p16)
     ws = torch.zeros(256, dtype=torch.uint8, device="cuda")
+    g = Guarded(want.shape, torch.int8)
     got = ip.dwconv_swish_i8(_d(x), _d(w), _d(bias), _d(m), _d(s),
-                             (p16.q_c, p16.q_one, p16.m, p16.s), workspace=ws)
+                             (p16.q_c, p16.q_one, p16.m, p16.s), out=g.view, workspace=ws)
     assert ip.status(ws) == 0
+    g.check()
     assert_same(got.cpu().numpy(), want)
 
 

@@ -3,6 +3,8 @@ CPU oracle: bit-exact on every output."""
 import numpy as np
 import pytest
 
+from guard import Guarded
+
 import synth
 
 pytestmark = pytest.mark.gpu
@@ -32,10 +34,13 @@ def _d(a):
 
 def run_both(ip, orc, x, w, bias, m, s, x_layout=0, y_layout=0, groups=1):
     ws = torch.zeros(256, dtype=torch.uint8, device="cuda")
-    got = ip.linear_i8(_d(x), _d(w), None if bias is None else _d(bias), _d(m), _d(s),
-                       x_layout=x_layout, y_layout=y_layout, groups=groups, workspace=ws)
-    st = ip.status(ws)
     want = orc.linear(x, w, bias, m, s, x_layout=x_layout, y_layout=y_layout, groups=groups)
+    g = Guarded(want.shape, torch.int8)
+    got = ip.linear_i8(_d(x), _d(w), None if bias is None else _d(bias), _d(m), _d(s),
+                       x_layout=x_layout, y_layout=y_layout, groups=groups, out=g.view,
+                       workspace=ws)
+    st = ip.status(ws)
+    g.check()
     return got.cpu().numpy(), want, st
 
 
@@ -163,10 +168,12 @@ def swish_case(orc, B, T, K, N, seed):
 
 def run_swish(ip, orc, c, m, s, sw):
     ws = torch.zeros(256, dtype=torch.uint8, device="cuda")
-    got = ip.linear_swish_i8(_d(c.x), _d(c.w), None if c.bias is None else _d(c.bias), _d(m),
-                             _d(s), (sw.q_c, sw.q_one, sw.m, sw.s), workspace=ws)
-    st = ip.status(ws)
     z = orc.linear(c.x, c.w, c.bias, m, s)
+    g = Guarded(z.shape, torch.int8)
+    got = ip.linear_swish_i8(_d(c.x), _d(c.w), None if c.bias is None else _d(c.bias), _d(m),
+                             _d(s), (sw.q_c, sw.q_one, sw.m, sw.s), out=g.view, workspace=ws)
+    st = ip.status(ws)
+    g.check()
     return got.cpu().numpy(), orc.swish(z, sw), st
 
 

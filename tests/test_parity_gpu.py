@@ -8,6 +8,7 @@ import numpy as np
 import pytest
 
 import synth
+from guard import Guarded
 
 pytestmark = pytest.mark.gpu
 
@@ -38,9 +39,11 @@ def run_gpu(ip, lay, consts, lengths=None):
     B, H, T, dh = lay.q.shape
     ws = torch.zeros(ip.workspace_bytes(B, H, T, dh), dtype=torch.uint8, device="cuda")
     lens = None if lengths is None else _dev(lengths.astype(np.int32))
+    g = Guarded((B, H, T, dh), torch.int8)
     out = ip.relpos_mhsa_i8(_dev(lay.q), _dev(lay.k), _dev(lay.v), _dev(lay.p), _dev(lay.u),
-                            _dev(lay.vb), consts, lengths=lens, workspace=ws)
+                            _dev(lay.vb), consts, lengths=lens, out=g.view, workspace=ws)
     assert ip.status(ws) == 0
+    g.check()
     return out.cpu().numpy()
 
 

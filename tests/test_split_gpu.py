@@ -12,6 +12,7 @@ import numpy as np
 import pytest
 
 import synth
+from guard import Guarded
 from test_parity_gpu import assert_same, oracle_out, run_gpu
 
 pytestmark = pytest.mark.gpu
@@ -95,9 +96,11 @@ def test_row_major_output_is_the_transpose(ip, orc, mode, T, masked):
     d = lambda a: torch.from_numpy(np.ascontiguousarray(a)).cuda()
     ws = torch.zeros(ip.workspace_bytes(3, 8, T, 128), dtype=torch.uint8, device="cuda")
     lens = None if lay.lengths is None else d(lay.lengths.astype(np.int32))
+    g = Guarded((3, T, 8, 128), torch.int8)
     got = ip.relpos_mhsa_i8(d(lay.q), d(lay.k), d(lay.v), d(lay.p), d(lay.u), d(lay.vb), c,
-                            lengths=lens, workspace=ws, out_layout=ip.ROWS)
+                            lengths=lens, out=g.view, workspace=ws, out_layout=ip.ROWS)
     assert ip.status(ws) == 0
+    g.check()
     assert_same(got.cpu().numpy(), np.ascontiguousarray(want.transpose(0, 2, 1, 3)))
 
 
@@ -116,7 +119,8 @@ def test_every_tile_split_is_repeatable(ip):
                      device="cuda")
     ip.set_split_mode(0)
     want = ip.relpos_mhsa_i8(q, k, v, p, u, vb, c, workspace=ws).clone()
-    out = torch.empty_like(want)
+    g = Guarded(want.shape, torch.int8)
+    out = g.view
     bad = 0
     for m in (1, 2):
         ip.set_split_mode(m)
@@ -125,4 +129,5 @@ def test_every_tile_split_is_repeatable(ip):
             bad += int(not torch.equal(out, want))
     ip.set_split_mode(-1)
     assert ip.status(ws) == 0
+    g.check()
     assert bad == 0, f"{bad} of 40 runs differ"
