@@ -71,6 +71,11 @@ def parse_args():
                     help="skip the projection and feed-forward measurements")
     ap.add_argument("--rows-only", action="store_true",
                     help="profiling: only the projection and feed-forward measurements")
+    ap.add_argument("--no-configs", action="store_true",
+                    help="skip the measurements of the other attention workloads")
+    ap.add_argument("--configs-only", type=int, default=None, metavar="W",
+                    help="profiling: only the attention workload W (0, 1, 2 or 4), "
+                         "--steps launch groups")
     return ap.parse_args()
 
 
@@ -376,6 +381,106 @@ NEXT_ROWS = [
 ]
 
 
+# The other attention workloads, each one layer: shapes, distributions and
+# (workload 2) key-padding lengths as drawn by synth; launches per timed
+# group so that a group lasts well above the event timer's ~2 us tick.
+CONFIG_WORKLOADS = (0, 1, 2, 4)
+CONFIG_GROUP = {0: 200, 1: 200, 2: 20, 4: 8}
+
+
+def valid_ops(w, lengths) -> float:
+    """Useful ops of one layer of workload w: 6 dh len^2 per (b, h), len the
+    utterance's valid length (T without a key-padding mask)."""
+    if lengths is None:
+        return float(useful_ops(w.B, w.H, w.T, w.dh, 1))
+    lens = np.clip(np.asarray(lengths, dtype=np.int64), 0, w.T)
+    return float(6 * w.dh * w.H * int(np.sum(lens * lens)))
+
+
+def measure_configs(dev, peak, pipes, steps: int, cpu: bool, only=None):
+    """Per-launch device time of one layer of each other workload: groups of
+    CONFIG_GROUP[w] back-to-back launches between one pair of CUDA events on
+    the launching stream, L2 flushed before every group (the small workloads
+    then read their inputs from HBM in the first launch of a group and from
+    L2 after it), median over `steps` groups; useful ops on the valid
+    frames; with `cpu`, the oracle timed on the same layer on the host
+    cores."""
+    import torch
+    import paper_2609_30846_gb300 as ip
+    stream = torch.cuda.current_stream(dev)
+    hstream = ctypes.c_void_p(stream.cuda_stream)
+    lib = ip.load()
+    flush_w = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    rows = {}
+    for wk in (CONFIG_WORKLOADS if only is None else (only,)):
+        w = synth.WORKLOADS[wk]
+        lay = synth.layer(w, 0)
+        c = ip.layer_constants(lay.scales)
+        to = lambda a: torch.from_numpy(np.ascontiguousarray(a)).to(dev)
+        d = dict(q=to(lay.q), k=to(lay.k), v=to(lay.v), p=to(lay.p), u=to(lay.u), vb=to(lay.vb))
+        lens = None if lay.lengths is None else to(lay.lengths.astype(np.int32))
+        out = torch.empty((w.B, w.H, w.T, w.dh), dtype=torch.int8, device=dev)
+        ws = torch.zeros(ip.workspace_bytes(w.B, w.H, w.T, w.dh), dtype=torch.uint8, device=dev)
+        sm = ip.SoftmaxParams(*c.softmax)
+        mult = (ctypes.c_int32 * 3)(*c.multipliers)
+        sh = (ctypes.c_int32 * 2)(*c.shifts)
+        P = lambda t: None if t is None else ctypes.c_void_p(t.data_ptr())
+        args = (P(d["q"]), P(d["k"]), P(d["v"]), P(d["p"]), P(d["u"]), P(d["vb"]), mult, sh,
+                ctypes.byref(sm), P(lens), w.B, w.H, w.T, w.dh, P(out), P(ws), ws.numel(), hstream)
+        n = CONFIG_GROUP[wk]
+
+        def group():
+            for _ in range(n):
+                rc = lib.ip_relpos_mhsa_i8(*args)
+                if rc != 0:
+                    raise ip.IpError("ip_relpos_mhsa_i8", rc, ip.strerror(rc))
+        group()
+        times = []
+        for _ in range(max(steps, 1)):
+            flush_w.zero_()
+            torch.cuda._sleep(200_000)   # the events and launches queue behind it
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            group()
+            e1.record(stream)
+            e1.synchronize()
+            times.append(e0.elapsed_time(e1) * 1e-3 / n)
+        if ip.status(ws, stream) != 0:
+            raise SystemExit(f"workload {w.name}: kernel reported an error")
+        t = statistics.median(times)
+        ops = valid_ops(w, lay.lengths)
+        tops = ops / t / 1e12
+        bytes_layer = 4 * w.B * w.H * w.T * w.dh + w.H * (2 * w.T - 1) * w.dh
+        row = {"workload": w.name, "B": w.B, "H": w.H, "T": w.T, "dh": w.dh,
+               "masked": w.masked, "dist": w.dist, "us_per_launch": t * 1e6,
+               "value": tops, "unit": "TOPS", "useful_ops": ops,
+               "ops_basis": "6 dh len^2 per (b, h), len the valid length" if w.masked
+                            else "6 dh T^2 per (b, h)",
+               "items": w.B * w.H * ((w.T + 63) // 64),
+               "roofline": {"bound": "tensor", "achieved": tops, "peak": peak,
+                            "frac": tops / peak,
+                            "frac_of_both_integer_pipes": tops / pipes["imma_plus_dp4a"],
+                            "hbm_floor_frac": (bytes_layer / (HBM_GBS * 1e9)) / t},
+               "timing": f"{n} launches per event pair, L2 flushed before each group, "
+                         f"median of {max(steps, 1)} groups",
+               "gpu_launches": n * (max(steps, 1) + 1)}
+        if cpu:
+            import oracle
+            oracle.build()
+            threads = os.cpu_count() or 1
+            oracle.set_threads(threads)
+            oc = oracle.layer_constants(lay.scales, w.dh)
+            t0 = time.perf_counter()
+            oracle.relpos_mhsa(lay.q, lay.k, lay.v, lay.p, lay.u, lay.vb, oc, lay.lengths)
+            dt = time.perf_counter() - t0
+            row["cpu_baseline"] = {"value": ops / dt / 1e12, "unit": "TOPS", "cores": threads,
+                                   "kind": "oracle", "seconds": dt,
+                                   "sample": f"the whole layer (B={w.B}, T={w.T})"}
+        rows[w.name] = row
+        del d, out, ws
+    return rows
+
+
 def measure_next_rows(dev, peak, pipes, steps: int, cpu: bool):
     """Each projection timed alone (CUDA events per launch, L2 flushed before
     every timed launch: a 256 MB write, then a 256 MB read so that no dirty
@@ -643,6 +748,15 @@ def run_ours(args):
             dist.destroy_process_group()
         return 0
 
+    if args.configs_only is not None:
+        if rank == 0:
+            rows = measure_configs(dev, ip.int8_mma_peak_tops(), ip.int8_pipe_rates(),
+                                   max(args.steps, 1), cpu=False, only=args.configs_only)
+            print(json.dumps({"configs": rows}), flush=True)
+        if dist:
+            dist.destroy_process_group()
+        return 0
+
     w = synth.WORKLOADS[WORKLOAD]
     B, H, T, dh, NL = w.B, w.H, w.T, w.dh, w.layers
     if args.layers:
@@ -761,6 +875,10 @@ def run_ours(args):
     cpu = None
     if world == 1 and not args.no_cpu_baseline:
         cpu = cpu_sample(layers, os.cpu_count() or 1, args.cpu_seconds)
+    configs = None
+    if not args.no_configs and not reduced:
+        configs = measure_configs(dev, peak, pipes, max(args.steps, 5),
+                                  cpu=world == 1 and not args.no_cpu_baseline)
     next_rows = None
     if not args.no_next_rows and not reduced:
         next_rows = measure_next_rows(dev, peak, pipes, max(args.steps, 5),
@@ -794,6 +912,7 @@ def run_ours(args):
         "e2e": e2e,
         "gpu_launches": NL * args.steps,
         "clocks": clk,
+        "configs": configs,
         "next_rows": next_rows,
     }
     print(json.dumps(line), flush=True)
