@@ -264,6 +264,25 @@ def _counters():
         return {}
 
 
+ROWS_TRAFFIC_FILE = os.path.join(ROOT, "profiles", "next_rows_traffic.json")
+
+
+def rows_traffic() -> dict:
+    """DRAM bytes per launch of the widened rows' kernels from the committed
+    ncu record, if every kernel source it names is unchanged (else {})."""
+    if not os.path.exists(ROWS_TRAFFIC_FILE):
+        return {}
+    try:
+        rec = json.load(open(ROWS_TRAFFIC_FILE))
+        csrc = os.path.join(ROOT, "paper_2609_30846_gb300", "csrc")
+        for f, h in rec.get("kernel_sha256", {}).items():
+            if hashlib.sha256(open(os.path.join(csrc, f), "rb").read()).hexdigest() != h:
+                return {}
+        return {k: v["dram_bytes_per_launch"] for k, v in rec.get("rows", {}).items()}
+    except (OSError, ValueError, KeyError):
+        return {}
+
+
 def traffic_per_launch():
     """DRAM bytes per fused-kernel launch from the committed ncu summary,
     if it was taken on the current kernel source (else None)."""
@@ -508,6 +527,7 @@ def measure_next_rows(dev, peak, pipes, steps: int, cpu: bool):
         torch.cuda._sleep(200_000)
 
     rows = {}
+    traffic = rows_traffic()
     for name, K, N, G, xl, yl, sw in NEXT_ROWS:
         case = synth.linear(B, T, K, N, seed=7000 + K + N + G, groups=G)
         m, s = ip.linear_constants(case.s_x, case.s_w, case.s_y_per_channel())
@@ -549,7 +569,8 @@ def measure_next_rows(dev, peak, pipes, steps: int, cpu: bool):
                          "swish": sw},
                "roofline": {"bound": "tensor+dp4a", "achieved": ops / t / 1e12, "peak": both,
                             "unit": "TOPS", "frac": ops / t / 1e12 / both,
-                            "frac_of_mma_peak": ops / t / 1e12 / peak, "traffic": None,
+                            "frac_of_mma_peak": ops / t / 1e12 / peak,
+                            "traffic": traffic.get(name),
                             "peak_source": "measured in this run: integer MMA and dp4a pipes "
                                            "together (ip_probe_int8_mix)"},
                "kernel": "linear_i8_kernel" + ("<swish>" if sw else ""), "gpu_launches": 1}
@@ -611,7 +632,8 @@ def measure_next_rows(dev, peak, pipes, steps: int, cpu: bool):
            "shape": {"rows": B * T, "d": d},
            "roofline": {"bound": "alu", "achieved": ops / t / 1e12, "peak": alu_peak,
                         "unit": "Tops/s (int32 lane ops)", "frac": ops / t / 1e12 / alu_peak,
-                        "traffic": None, "hbm_frac": elems * 2 / t / 1e9 / HBM_GBS},
+                        "traffic": traffic.get("layernorm_1024"),
+                        "hbm_frac": elems * 2 / t / 1e9 / HBM_GBS},
            "kernel": "layernorm_i8_kernel<2>", "gpu_launches": NORM_BUFS,
            "timing": f"{NORM_BUFS} launches on {NORM_BUFS} input/output pairs per event pair"}
     if cpu:
@@ -673,7 +695,11 @@ def measure_next_rows(dev, peak, pipes, steps: int, cpu: bool):
            "frames_per_s": B * T / t, "shape": {"B": B, "T": T, "d": 1024, "ff": 4096, "heads": 8},
            "roofline": {"bound": "tensor+dp4a", "achieved": ops / t / 1e12, "peak": both,
                         "unit": "TOPS", "frac": ops / t / 1e12 / both,
-                        "frac_of_mma_peak": ops / t / 1e12 / peak, "traffic": None},
+                        "frac_of_mma_peak": ops / t / 1e12 / peak, "traffic": None,
+                        "traffic_parts": {k: v for k, v in traffic.items() if k.startswith("block_")},
+                        "traffic_note": "per kernel in profiles/next_rows_traffic.json; two of "
+                                        "the block's fifteen launches (the 1024 -> 1024 "
+                                        "projections with the residual) were not captured"},
            "kernel": "15 launches: layernorm x5, linear x8 (2 with Swish, 1 with GLU, 4 with "
                      "the residual addition), relpos_mhsa_fused, dwconv_swish",
            "gpu_launches": GPU_LAUNCHES}

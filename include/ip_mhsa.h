@@ -159,8 +159,10 @@ int ip_relpos_mhsa_i8_host(const int8_t *q, const int8_t *k, const int8_t *v,
  * no allocation: no cudaMalloc, cudaFree or allocating library routine.
  *
  * The first call on a device looks up the device address of the array
- * (cudaGetSymbolAddress, with that device current) and caches it; make that
- * first call before any stream capture.  Every call shares the array and
+ * (cudaGetSymbolAddress, with that device current) and caches it for the
+ * life of the process; make that first call before any stream capture.  A
+ * device reset (cudaDeviceReset) after that first call is not supported:
+ * the cached address would belong to the destroyed context.  Every call shares the array and
  * clears its status word in stream order before launching; calls that
  * overlap on the GPU (concurrent streams) race on it.  Kernel-side barrier
  * timeouts are recorded there and are not reported by this entry point; a
@@ -314,8 +316,10 @@ int ip_linear_glu_i8(const int8_t *x, const int8_t *w, const int32_t *bias, cons
  * (m_x res + m_y z)), -127, 127) with z the requantised int8 output of
  * ip_linear_i8 on (x, w, bias, m, s).  Bit-identical to ip_linear_i8 then
  * ip_residual_i8(res, z, m_x, m_y, s_r).  res: device int8 [B][T][N]
- * row-major, 16-byte aligned, may not alias y; m_x, m_y in [0, 2^31), s_r in
- * [0, 31] (else IP_ERR_PARAM).  x: [B][T][K] row-major; y: [B][T][N]
+ * row-major, 16-byte aligned; it may be y itself (in place: each element
+ * is read by the thread that then writes it), but a partial overlap with y
+ * is rejected with IP_ERR_PARAM; m_x, m_y in [0, 2^31), s_r in [0, 31]
+ * (else IP_ERR_PARAM).  x: [B][T][K] row-major; y: [B][T][N]
  * row-major.  Other arguments and errors as ip_linear_i8. */
 int ip_linear_residual_i8(const int8_t *x, const int8_t *w, const int32_t *bias,
                           const int32_t *m, const int32_t *s, const int8_t *res, int32_t m_x,

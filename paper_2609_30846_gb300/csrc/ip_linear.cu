@@ -232,6 +232,14 @@ int ip_linear_residual_i8(const int8_t *x, const int8_t *w, const int32_t *bias,
     if (m_x < 0 || m_y < 0 || s_r < 0 || s_r > 31) return IP_ERR_PARAM;
     if (B > 0 && !res) return IP_ERR_NULL;
     if (res && !aligned(res, 16)) return IP_ERR_ALIGN;
+    if (res && y && res != y && B > 0 && T > 0 && N > 0) {
+        // in place (res == y) is fine: every element is read by the thread
+        // that then writes it; a partial overlap would race across CTAs
+        const uintptr_t a = reinterpret_cast<uintptr_t>(res), b = reinterpret_cast<uintptr_t>(y);
+        const uintptr_t n = static_cast<uintptr_t>(B) * static_cast<uintptr_t>(T) *
+                            static_cast<uintptr_t>(N);
+        if (a < b + n && b < a + n) return IP_ERR_PARAM;
+    }
     const ResidualArg ra{res, m_x, m_y, s_r};
     return linear_launch(x, IP_LAYOUT_ROWS, w, bias, m, s, nullptr, ipl::EPI_RES, B, T, K, N, 1, y,
                          IP_LAYOUT_ROWS, workspace, workspace_bytes, stream, &ra);

@@ -193,6 +193,22 @@ def test_linear_constants_entry_point_matches_oracle(lib):
         ip.linear_constants(1.0, np.array([1.0]), 0.5)          # ratio 2, unencodable
 
 
+def test_linear_residual_rejects_partial_overlap(lib):
+    # res overlapping y other than exactly (in place) is refused before any
+    # device work (the fake addresses are never dereferenced)
+    P = ctypes.c_void_p
+    fake = P(1 << 20)
+    y = P(1 << 24)
+    ws = P(1 << 21)
+
+    def call(res):
+        return lib.ip_linear_residual_i8(fake, fake, None, fake, fake, res, 1 << 30, 1 << 30, 0,
+                                         1, 4, 256, 256, y, ws, 256, None)
+    assert call(P((1 << 24) + 16)) == -7
+    assert call(P((1 << 24) - 512)) == -7           # ends inside y
+    assert call(P((1 << 24) + 512)) == -7           # starts inside y
+
+
 def test_binding_holds_no_scale_arithmetic():
     # the binding marshals the scales to the C helpers; the ratios of Eq. 7
     # and Eq. 11 are composed behind the C ABI

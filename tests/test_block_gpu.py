@@ -75,6 +75,62 @@ def test_linear_residual(ip, orc, B, T, K, N, alpha):
     assert_same(got.cpu().numpy(), want)
 
 
+# Hand-picked constants at the edges of the residual's domain: the largest
+# multipliers, the shortest and longest shifts, and (2^30, 2^30, 0), where
+# (x + y) / 2 lands on a half step for every odd sum (the round-half-up tie).
+EDGE_RESIDUAL = [(2 ** 31 - 1, 2 ** 31 - 1, 31), (2 ** 31 - 1, 1, 0), (1, 2 ** 31 - 1, 0),
+                 (2 ** 30, 2 ** 30, 0), (2 ** 30, 2 ** 29, 1), (0, 2 ** 31 - 1, 31),
+                 (12345, 2 ** 31 - 1, 7), (2 ** 31 - 1, 0, 30)]
+
+
+@pytest.mark.parametrize("m_x,m_y,s_r", EDGE_RESIDUAL)
+def test_residual_edge_constants(ip, orc, m_x, m_y, s_r):
+    # every (x, y) pair of int8 values, bit for bit against the oracle
+    v = np.arange(-128, 128, dtype=np.int16)
+    x = np.repeat(v, 256).astype(np.int8)
+    y = np.tile(v, 256).astype(np.int8)
+    g = Guarded(x.shape, torch.int8)
+    got = ip.residual_i8(_d(x), _d(y), m_x, m_y, s_r, out=g.view).cpu().numpy()
+    g.check()
+    assert_same(got, orc.residual(x, y, m_x, m_y, s_r))
+
+
+@pytest.mark.parametrize("m_x,m_y,s_r", EDGE_RESIDUAL)
+def test_linear_residual_edge_constants(ip, orc, m_x, m_y, s_r):
+    B, T, K, N = 2, 70, 256, 256
+    lc = synth.linear(B, T, K, N, seed=731)
+    m, s = orc.linear_constants(lc.s_x, lc.s_w, lc.s_y_per_channel())
+    rng = np.random.default_rng(s_r + 7)
+    res = rng.integers(-128, 128, size=(B, T, N)).astype(np.int8)
+    want = orc.residual(res, orc.linear(lc.x, lc.w, lc.bias, m, s), m_x, m_y, s_r)
+    ws = torch.zeros(256, dtype=torch.uint8, device="cuda")
+    g = Guarded(want.shape, torch.int8)
+    got = ip.linear_residual_i8(_d(lc.x), _d(lc.w), _d(lc.bias), _d(m), _d(s), _d(res), m_x, m_y,
+                                s_r, out=g.view, workspace=ws)
+    assert ip.status(ws) == 0
+    g.check()
+    assert_same(got.cpu().numpy(), want)
+
+
+def test_linear_residual_in_place(ip, orc):
+    # res and y the same buffer: the residual stream updated in place
+    B, T, K, N = 3, 130, 256, 384
+    lc = synth.linear(B, T, K, N, seed=732)
+    m, s = orc.linear_constants(lc.s_x, lc.s_w, lc.s_y_per_channel())
+    res = np.random.default_rng(5).integers(-127, 128, size=(B, T, N)).astype(np.int8)
+    rp = orc.residual_params(0.05, float(lc.s_y[0]), 1.2 * max(0.05, float(lc.s_y[0])), 0.5)
+    want = orc.residual(res, orc.linear(lc.x, lc.w, lc.bias, m, s), *rp)
+    ws = torch.zeros(256, dtype=torch.uint8, device="cuda")
+    g = Guarded(res.shape, torch.int8)
+    g.view.copy_(_d(res))
+    got = ip.linear_residual_i8(_d(lc.x), _d(lc.w), _d(lc.bias), _d(m), _d(s), g.view, *rp,
+                                out=g.view, workspace=ws)
+    assert ip.status(ws) == 0
+    g.check()
+    assert got.data_ptr() == g.view.data_ptr()
+    assert_same(got.cpu().numpy(), want)
+
+
 def interleave(w):
     N2 = w.shape[0]
     C = N2 // 2
