@@ -68,7 +68,7 @@ typedef struct {
 #define IP_ERR_WORKSPACE (-8)   /* workspace smaller than ip_relpos_mhsa_workspace_bytes */
 
 #define IP_DH 128
-#define IP_MAX_T 2048   /* frames; the int8 scores of a 64-row tile stay in shared memory */
+#define IP_MAX_T 2048   /* frames; the int8 scores of a 64-row tile stay on chip or in L2 */
 #define IP_MAX_B 65535
 #define IP_MAX_H 65535
 /* B H ceil(T / 64) (the 64-row query tiles of a call) must stay below this:
@@ -80,8 +80,13 @@ typedef struct {
  * its first use; ip_relpos_mhsa_status reads and clears it.  The workspace
  * also holds the work-item counters of the attention kernel (its CTAs claim
  * query tiles from them), which every call returns to zero when it ends;
- * calls that share a workspace must not overlap on the GPU.  0 if the shape
- * is invalid. */
+ * calls that share a workspace must not overlap on the GPU.
+ * For T > 384 the size also counts a region for the int8 scores of every
+ * resident CTA of the current device (4 warps x 16 rows x T, rounded up to
+ * 64 keys, per CTA): a call given that much keeps the scores between the
+ * softmax passes there (in L2) and fits two CTAs per SM; a call given only
+ * the first 256 bytes keeps them in shared memory, one CTA per SM, with the
+ * same result.  The region needs no zero fill.  0 if the shape is invalid. */
 size_t ip_relpos_mhsa_workspace_bytes(int B, int H, int T, int dh);
 
 /* The whole layer on the GPU.

@@ -120,40 +120,70 @@ bool cached_map(CUtensorMap *m, const void *base, unsigned long long d1, unsigne
     return true;
 }
 
-std::mutex g_attr_mu;
-int g_attr_smem[64] = {0};
+// The fused kernel in its two forms: int8 scores kept in shared memory, or
+// (gs, long sequences) in the caller's workspace.
+using FusedKernel = void (*)(const CUtensorMap, const CUtensorMap, const CUtensorMap,
+                             const CUtensorMap, const ipk::FusedParams);
+FusedKernel fused_kernel(bool gs) {
+    return gs ? ipk::relpos_mhsa_fused_kernel<true> : ipk::relpos_mhsa_fused_kernel<false>;
+}
 
-int ensure_smem(int bytes) {
+std::mutex g_attr_mu;
+int g_attr_smem[2][64] = {{0}};
+
+int ensure_smem(bool gs, int bytes) {
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return IP_ERR_CUDA;
     std::lock_guard<std::mutex> lock(g_attr_mu);
-    if (g_attr_smem[dev] >= bytes) return IP_OK;
-    if (cudaFuncSetAttribute(ipk::relpos_mhsa_fused_kernel,
-                             cudaFuncAttributeMaxDynamicSharedMemorySize, bytes) != cudaSuccess)
+    if (g_attr_smem[gs][dev] >= bytes) return IP_OK;
+    if (cudaFuncSetAttribute(fused_kernel(gs), cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             bytes) != cudaSuccess)
         return IP_ERR_CUDA;
-    g_attr_smem[dev] = bytes;
+    g_attr_smem[gs][dev] = bytes;
     return IP_OK;
 }
 
 // CTAs of the fused kernel resident on the whole GPU at once (its SMs x the
-// CTAs an SM holds at this shared-memory size), cached for the last query.
+// CTAs an SM holds at this shared-memory size), cached for the last query
+// of each form.
 std::mutex g_occ_mu;
-int g_occ_dev = -1, g_occ_smem = -1, g_occ_slots = 0;
+int g_occ_dev[2] = {-1, -1}, g_occ_smem[2] = {-1, -1}, g_occ_slots[2] = {0, 0};
 
-int resident_ctas(int smem) {
+int resident_ctas(bool gs, int smem) {
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return 0;
     std::lock_guard<std::mutex> lock(g_occ_mu);
-    if (dev == g_occ_dev && smem == g_occ_smem) return g_occ_slots;
+    if (dev == g_occ_dev[gs] && smem == g_occ_smem[gs]) return g_occ_slots[gs];
     int nsm = 0, per_sm = 0;
-    if (cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
-        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, ipk::relpos_mhsa_fused_kernel,
-                                                      ipk::NTHREADS, smem) != cudaSuccess)
+    if (ensure_smem(gs, smem) != IP_OK ||
+        cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
+        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fused_kernel(gs), ipk::NTHREADS,
+                                                      smem) != cudaSuccess)
         return 0;
-    g_occ_dev = dev;
-    g_occ_smem = smem;
-    g_occ_slots = nsm * per_sm;
-    return g_occ_slots;
+    g_occ_dev[gs] = dev;
+    g_occ_smem[gs] = smem;
+    g_occ_slots[gs] = nsm * per_sm;
+    return g_occ_slots[gs];
+}
+
+// Sequences longer than this keep their scores in the workspace when it
+// has room: the shared-memory slices of T <= 384 (6 chunks) let two CTAs
+// share an SM, longer ones only one.
+constexpr int GS_MIN_T = 6 * ipk::NK + 1;
+
+int fused_smem(int T, bool gs) {
+    return ipk::smem_layout((T + ipk::NK - 1) / ipk::NK, gs).total + 1024;
+}
+
+// Bytes of the workspace's score region for T (0 when the scores stay in
+// shared memory or the device cannot be queried): one slice of nchunk KB
+// per consumer warp of every resident CTA.
+size_t gs_scores_bytes(int T) {
+    if (T < GS_MIN_T) return 0;
+    const int slots = resident_ctas(true, fused_smem(T, true));
+    if (slots < 1) return 0;
+    return static_cast<size_t>(slots) * ipk::NCWARPS *
+           static_cast<size_t>((T + ipk::NK - 1) / ipk::NK) * ipk::CHUNK_SCORE_BYTES;
 }
 
 // Work items of the persistent kernel.  The N whole tiles run on G resident
@@ -196,7 +226,7 @@ extern "C" {
 
 size_t ip_relpos_mhsa_workspace_bytes(int B, int H, int T, int dh) {
     if (check_shape(B, H, T, dh) != IP_OK) return 0;
-    return ws_bytes();
+    return ws_bytes() + gs_scores_bytes(T);
 }
 
 int ip_relpos_mhsa_i8(const int8_t *q, const int8_t *k, const int8_t *v, const int8_t *p,
@@ -254,8 +284,11 @@ int ip_relpos_mhsa_i8_ex(const int8_t *q, const int8_t *k, const int8_t *v, cons
     const long long N = static_cast<long long>(B) * H * ntiles;   // whole tiles
     if (N >= IP_MAX_TILES) return IP_ERR_SHAPE;   // item indices stay below 2^31
     const int nchunk_max = (T + ipk::NK - 1) / ipk::NK;
-    const int smem = ipk::smem_layout(nchunk_max).total + 1024;
-    rc = ensure_smem(smem);
+    // long sequences: scores in the workspace when it holds their region
+    const size_t gsb = gs_scores_bytes(T);
+    const bool gs = gsb > 0 && workspace_bytes >= ws_bytes() + gsb;
+    const int smem = fused_smem(T, gs);
+    rc = ensure_smem(gs, smem);
     if (rc != IP_OK) return rc;
 
     ipk::FusedParams prm;
@@ -288,7 +321,7 @@ int ip_relpos_mhsa_i8_ex(const int8_t *q, const int8_t *k, const int8_t *v, cons
     prm.f24 = !g_wide_sums && e0 > 256ull ? 1 : 0;
     prm.timeout_cycles = g_timeout_cycles;
     prm.stall_injection = g_stall_injection;
-    const int slots = resident_ctas(smem);
+    const int slots = resident_ctas(gs, smem);
     if (slots < 1) return IP_ERR_CUDA;
     const ItemPlan ip = plan_items(N, slots);
     prm.ntiles = ntiles;
@@ -298,10 +331,11 @@ int ip_relpos_mhsa_i8_ex(const int8_t *q, const int8_t *k, const int8_t *v, cons
     prm.split_log2 = ip.split_log2;
     prm.nitems = ip.nitems;
     prm.out_rows = out_layout == IP_LAYOUT_ROWS ? 1 : 0;
+    prm.gscores = gs ? static_cast<uint8_t *>(workspace) + ws_bytes() : nullptr;
     // Programmatic dependent launch: this grid may be scheduled while the
     // kernel before it on the stream finishes (the kernel waits for that
     // grid before its first global access, so the order of the two is kept).
-    if (iph::launch_pdl(ipk::relpos_mhsa_fused_kernel, dim3(ip.grid), dim3(ipk::NTHREADS),
+    if (iph::launch_pdl(fused_kernel(gs), dim3(ip.grid), dim3(ipk::NTHREADS),
                         static_cast<size_t>(smem), st, tm_q, tm_k, tm_v, tm_p, prm) != cudaSuccess)
         return IP_ERR_CUDA;
     if (cudaGetLastError() != cudaSuccess) return IP_ERR_CUDA;
@@ -342,7 +376,7 @@ size_t ip_relpos_mhsa_host_arena_bytes(int B, int H, int T, int dh) {
     const size_t pb = align_up(static_cast<size_t>(H) * (2ull * T - 1) * dh, 256);
     const size_t bias = align_up(static_cast<size_t>(H) * dh, 256);
     const size_t lens = align_up(4ull * (B > 0 ? B : 1), 256);
-    return 4 * act + pb + 2 * bias + lens + ws_bytes();
+    return 4 * act + pb + 2 * bias + lens + ws_bytes() + gs_scores_bytes(T);
 }
 
 namespace {
@@ -375,7 +409,7 @@ HostArena host_arena(void *arena, int B, int H, int T, int dh) {
     h.u = reinterpret_cast<int8_t *>(take(nb));
     h.vb = reinterpret_cast<int8_t *>(take(nb));
     h.len = reinterpret_cast<int32_t *>(take(4ull * (B > 0 ? B : 1)));
-    h.ws = take(ws_bytes());
+    h.ws = take(ws_bytes() + gs_scores_bytes(T));
     return h;
 }
 
@@ -409,7 +443,8 @@ int host_enqueue(const int8_t *q, const int8_t *k, const int8_t *v, const int8_t
         if (c.n && cudaMemcpyAsync(c.dst, c.src, c.n, cudaMemcpyHostToDevice, st) != cudaSuccess)
             return IP_ERR_CUDA;
     rc = ip_relpos_mhsa_i8(h.q, h.k, h.v, h.p, h.u, h.vb, multipliers, shifts, sm,
-                           lengths ? h.len : nullptr, B, H, T, dh, h.out, h.ws, ws_bytes(),
+                           lengths ? h.len : nullptr, B, H, T, dh, h.out, h.ws,
+                           ws_bytes() + gs_scores_bytes(T),
                            stream);
     if (rc != IP_OK) return rc;
     if (nact && cudaMemcpyAsync(out, h.out, nact, cudaMemcpyDeviceToHost, st) != cudaSuccess)

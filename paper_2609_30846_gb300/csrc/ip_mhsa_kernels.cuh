@@ -69,13 +69,14 @@ struct SmemLayout {
     int stages, qtile, scores, remap, lut, bars, total;
 };
 
-// Offsets from a 1024-byte aligned base.
-__host__ __device__ inline SmemLayout smem_layout(int nchunk_max) {
+// Offsets from a 1024-byte aligned base.  With global_scores the consumer
+// warps keep their int8 scores in the caller's workspace instead (ScoreBuf).
+__host__ __device__ inline SmemLayout smem_layout(int nchunk_max, bool global_scores = false) {
     SmemLayout L;
     L.stages = 0;
     L.qtile = NSTAGE * STAGE_BYTES;   // 1024-byte aligned (128-byte swizzle); Ring::qtile
     L.scores = L.qtile + Q_TILE_BYTES;
-    L.remap = L.scores + NCWARPS * nchunk_max * CHUNK_SCORE_BYTES;
+    L.remap = L.scores + (global_scores ? 0 : NCWARPS * nchunk_max * CHUNK_SCORE_BYTES);
     L.lut = L.remap + NCWARPS * REMAP_BYTES;
     L.bars = L.lut + LUT_ENTRIES * LUT_COPIES * 4;
     L.total = L.bars + 128;
@@ -108,7 +109,44 @@ struct FusedParams {
     uint32_t nwhole, nitems;           // nitems < 2^31
     int split_log2;                    // 1: halves, 2: quarters
     int out_rows;             // output [B][T][H][DH] instead of [B][H][T][DH]
+    uint8_t *gscores;         // global mode: score slices, NCWARPS per CTA, nchunk_max KB each
 };
+
+// Where a consumer warp keeps the int8 scores of its 16 rows between the
+// three passes (CHUNK_SCORE_BYTES per key chunk, each thread's bytes at the
+// same offsets in both places): its slice of shared memory, or, for long
+// sequences whose slices would leave room for one CTA per SM only, a slice
+// of the caller's workspace in global memory (written and read back by the
+// same thread, cached in L2).
+struct ScoreBuf {
+    uint32_t s;    // shared-memory address of the slice
+    uint8_t *g;    // global address of the slice
+};
+
+template <bool GS>
+__device__ __forceinline__ void sc_st128(const ScoreBuf &b, uint32_t off, uint32_t x, uint32_t y,
+                                         uint32_t z, uint32_t w) {
+    if constexpr (GS) stg128_cg(b.g + off, x, y, z, w);
+    else sts128(b.s + off, x, y, z, w);
+}
+
+template <bool GS>
+__device__ __forceinline__ uint4 sc_ld128(const ScoreBuf &b, uint32_t off) {
+    if constexpr (GS) return ldg128_cg(b.g + off);
+    else return lds128(b.s + off);
+}
+
+template <bool GS>
+__device__ __forceinline__ void sc_st64(const ScoreBuf &b, uint32_t off, int x, int y) {
+    if constexpr (GS) stg64_cg(b.g + off, x, y);
+    else sts64(b.s + off, x, y);
+}
+
+template <bool GS>
+__device__ __forceinline__ int2 sc_ld64(const ScoreBuf &b, uint32_t off) {
+    if constexpr (GS) return ldg64_cg(b.g + off);
+    else return lds64(b.s + off);
+}
 
 // Offset of output row `row` of (b, h).
 __device__ __forceinline__ size_t out_offset(const FusedParams &p, int b, int h, int row) {
@@ -312,18 +350,18 @@ __device__ __forceinline__ uint32_t score_tile(const int (&c)[4], int nt, uint32
 }
 
 // Eq. 11 for a whole chunk (8 tiles) and the store of the packed scores.
-template <bool MASK>
+template <bool MASK, bool GS>
 __device__ __forceinline__ void score_epilogue(const int (&cacc)[8][4], uint32_t remap,
-                                               uint32_t sdst, int lane, long long m_c,
-                                               long long m_p, long long half_s, int s_s,
-                                               int kvalid, int &mx0, int &mx1) {
+                                               const ScoreBuf &sb, uint32_t soff, int lane,
+                                               long long m_c, long long m_p, long long half_s,
+                                               int s_s, int kvalid, int &mx0, int &mx1) {
     uint32_t packed[8];
 #pragma unroll
     for (int nt = 0; nt < 8; ++nt)
         packed[nt] = score_tile<MASK>(cacc[nt], nt, remap, lane, m_c, m_p, half_s, s_s, kvalid,
                                       mx0, mx1);
-    sts128(sdst + lane * 16, packed[0], packed[1], packed[2], packed[3]);
-    sts128(sdst + 512 + lane * 16, packed[4], packed[5], packed[6], packed[7]);
+    sc_st128<GS>(sb, soff + lane * 16, packed[0], packed[1], packed[2], packed[3]);
+    sc_st128<GS>(sb, soff + 512 + lane * 16, packed[4], packed[5], packed[6], packed[7]);
 }
 
 // Sum of the integer exponentials of one stored half chunk (16 scores per
@@ -623,8 +661,9 @@ struct Ring {
 // Passes 1-3 and the output of one whole 64-row tile by one consumer warp
 // (its 16-row strip), with ring uses u0 .. u0 + 2 nchunks - 1; the item's
 // Q tile has landed.  Returns false after a barrier wait ran out.
+template <bool GS>
 __device__ __forceinline__ bool consume_whole(const FusedParams &prm, const Item &it, int u0,
-                                              const Ring &R, uint32_t remap, uint32_t scores,
+                                              const Ring &R, uint32_t remap, const ScoreBuf &scores,
                                               uint32_t lut, int warp, int lane) {
     const int T = prm.T, len = it.len, nchunks = it.nchunks;
     const int g = lane >> 2, t4 = lane & 3;
@@ -658,9 +697,10 @@ __device__ __forceinline__ bool consume_whole(const FusedParams &prm, const Item
         int cacc[8][4];
         content_mma(cacc, qa, R.stage(u), R.stage(u) + KU_OFF, lane);
         if (c > 0) {
-            const uint32_t sprev = scores + (c - 1) * CHUNK_SCORE_BYTES;
-            sts128(sprev + lane * 16, packed[0], packed[1], packed[2], packed[3]);
-            sts128(sprev + 512 + lane * 16, packed[4], packed[5], packed[6], packed[7]);
+            const uint32_t oprev = (c - 1) * CHUNK_SCORE_BYTES;
+            sc_st128<GS>(scores, oprev + lane * 16, packed[0], packed[1], packed[2], packed[3]);
+            sc_st128<GS>(scores, oprev + 512 + lane * 16, packed[4], packed[5], packed[6],
+                         packed[7]);
         }
         __syncwarp();
 #pragma unroll
@@ -669,7 +709,7 @@ __device__ __forceinline__ bool consume_whole(const FusedParams &prm, const Item
             sts64(remap + ((g + 8) * REMAP_STRIDE + nt * 8 + 2 * t4) * 4, bacc[nt][2], bacc[nt][3]);
         }
         release_stage(R.empty(u), lane);
-        const uint32_t sdst = scores + c * CHUNK_SCORE_BYTES;
+        const uint32_t sdst = c * CHUNK_SCORE_BYTES;
         if (c + 1 < nchunks) {
             if (!warp_wait(R.ready(u + 1), Ring::parity(u + 1), prm.timeout_cycles)) {
                 if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_READY);
@@ -715,11 +755,11 @@ __device__ __forceinline__ bool consume_whole(const FusedParams &prm, const Item
             __syncwarp();
             const int kvalid = len - c * NK;
             if (kvalid < NK)
-                score_epilogue<true>(cacc, remap, sdst, lane, m_c, m_p, half_s, s_s, kvalid,
-                                     mx0, mx1);
+                score_epilogue<true, GS>(cacc, remap, scores, sdst, lane, m_c, m_p, half_s, s_s,
+                                         kvalid, mx0, mx1);
             else
-                score_epilogue<false>(cacc, remap, sdst, lane, m_c, m_p, half_s, s_s, kvalid,
-                                      mx0, mx1);
+                score_epilogue<false, GS>(cacc, remap, scores, sdst, lane, m_c, m_p, half_s, s_s,
+                                          kvalid, mx0, mx1);
         }
     }
 
@@ -735,13 +775,31 @@ __device__ __forceinline__ bool consume_whole(const FusedParams &prm, const Item
     const uint32_t lut_g = lut + 4 * (g & (LUT_COPIES - 1));
     const uint32_t mx4h = max4h(mx0, mx1);
     unsigned long long sum0 = 0, sum1 = 0;
-    if (prm.sum32) {
+    if constexpr (GS) {
+        // scores from L2: each chunk's two words are requested one chunk ahead
+        uint4 nx0 = sc_ld128<GS>(scores, lane * 16), nx1 = sc_ld128<GS>(scores, 512 + lane * 16);
+        for (int c = 0; c < nchunks; ++c) {
+            const int kvalid = len - c * NK;
+            const uint4 sv0 = nx0, sv1 = nx1;
+            if (c + 1 < nchunks) {
+                nx0 = sc_ld128<GS>(scores, (c + 1) * CHUNK_SCORE_BYTES + lane * 16);
+                nx1 = sc_ld128<GS>(scores, (c + 1) * CHUNK_SCORE_BYTES + 512 + lane * 16);
+            }
+            if (kvalid < NK) {
+                exp_sums<true>(sv0, lut_g, mx4h, t4, 0, kvalid, sum0, sum1);
+                exp_sums<true>(sv1, lut_g, mx4h, t4, 32, kvalid, sum0, sum1);
+            } else {
+                exp_sums<false>(sv0, lut_g, mx4h, t4, 0, kvalid, sum0, sum1);
+                exp_sums<false>(sv1, lut_g, mx4h, t4, 32, kvalid, sum0, sum1);
+            }
+        }
+    } else if (prm.sum32) {
         uint32_t a[4] = {0u, 0u, 0u, 0u};
         for (int c = 0; c < nchunks; ++c) {
             const int kvalid = len - c * NK;
 #pragma unroll
             for (int hf = 0; hf < 2; ++hf) {
-                const uint4 sv = lds128(scores + c * CHUNK_SCORE_BYTES + hf * 512 + lane * 16);
+                const uint4 sv = sc_ld128<GS>(scores, c * CHUNK_SCORE_BYTES + hf * 512 + lane * 16);
                 if (kvalid < NK)
                     exp_sums32<true>(sv, lut_g, mx4h, t4, 32 * hf, kvalid, a);
                 else
@@ -755,7 +813,7 @@ __device__ __forceinline__ bool consume_whole(const FusedParams &prm, const Item
             const int kvalid = len - c * NK;
 #pragma unroll
             for (int hf = 0; hf < 2; ++hf) {
-                const uint4 sv = lds128(scores + c * CHUNK_SCORE_BYTES + hf * 512 + lane * 16);
+                const uint4 sv = sc_ld128<GS>(scores, c * CHUNK_SCORE_BYTES + hf * 512 + lane * 16);
                 if (kvalid < NK)
                     exp_sums<true>(sv, lut_g, mx4h, t4, 32 * hf, kvalid, sum0, sum1);
                 else
@@ -781,7 +839,7 @@ __device__ __forceinline__ bool consume_whole(const FusedParams &prm, const Item
         uint32_t af[4];
         const int kvalid_last = len - (nchunks - 1) * NK;   // valid keys of the last chunk
         {
-            const uint4 sv = lds128(scores + lane * 16);
+            const uint4 sv = sc_ld128<GS>(scores, lane * 16);
             uint32_t pw[4] = {prob_word<F24>(sv.x, lut_g, mx4h, fa, fb),
                               prob_word<F24>(sv.y, lut_g, mx4h, fa, fb),
                               prob_word<F24>(sv.z, lut_g, mx4h, fa, fb),
@@ -802,8 +860,8 @@ __device__ __forceinline__ bool consume_whole(const FusedParams &prm, const Item
 #pragma unroll
             for (int ks = 0; ks < 2; ++ks) {
                 const int nxt = min(2 * c + ks + 1, nsteps - 1);
-                const uint4 svn =
-                    lds128(scores + (nxt >> 1) * CHUNK_SCORE_BYTES + (nxt & 1) * 512 + lane * 16);
+                const uint4 svn = sc_ld128<GS>(
+                    scores, (nxt >> 1) * CHUNK_SCORE_BYTES + (nxt & 1) * 512 + lane * 16);
                 const uint32_t wn[4] = {svn.x, svn.y, svn.z, svn.w};
                 uint32_t pw[4];
 #pragma unroll
@@ -866,9 +924,10 @@ __device__ __forceinline__ bool consume_whole(const FusedParams &prm, const Item
 // exponential sums and attn.V partial sums through their exchange areas
 // behind the strip pair's barrier (four phases per half: maxima, sums,
 // partials, and the partner done reading before the areas are reused).
+template <bool GS>
 __device__ __forceinline__ bool consume_half(const FusedParams &prm, const Item &it, int u0,
                                              const Ring &R, uint32_t remap,
-                                             uint32_t scores, uint32_t lut, uint32_t pair,
+                                             const ScoreBuf &scores, uint32_t lut, uint32_t pair,
                                              int warp, int lane) {
     const int len = it.len, nchunks = it.nchunks;
     const int g = lane >> 2, t4 = lane & 3;
@@ -920,7 +979,8 @@ __device__ __forceinline__ bool consume_half(const FusedParams &prm, const Item 
                 pk[i] = score_tile<false>(hc[i], nt0 + i, remap, lane, m_c, m_p, half_s, s_s,
                                           kvalid, mx0, mx1);
         }
-        sts128(scores + c * CHUNK_SCORE_BYTES + hk * 512 + lane * 16, pk[0], pk[1], pk[2], pk[3]);
+        sc_st128<GS>(scores, c * CHUNK_SCORE_BYTES + hk * 512 + lane * 16, pk[0], pk[1], pk[2],
+                     pk[3]);
     }
     release_stage(R.qempty(), lane);   // done with the Q tile
     mx0 = max(mx0, __shfl_xor_sync(0xffffffffu, mx0, 1));
@@ -946,7 +1006,7 @@ __device__ __forceinline__ bool consume_half(const FusedParams &prm, const Item 
     unsigned long long sum0 = 0, sum1 = 0;
     for (int c = 0; c < nchunks; ++c) {
         const int kvalid = len - c * NK;
-        const uint4 sv = lds128(scores + c * CHUNK_SCORE_BYTES + hk * 512 + lane * 16);
+        const uint4 sv = sc_ld128<GS>(scores, c * CHUNK_SCORE_BYTES + hk * 512 + lane * 16);
         if (kvalid < NK)
             exp_sums<true>(sv, lut_g, mx4h, t4, 32 * hk, kvalid, sum0, sum1);
         else
@@ -981,7 +1041,7 @@ __device__ __forceinline__ bool consume_half(const FusedParams &prm, const Item 
     for (int nt = 0; nt < 16; ++nt) oacc[nt][0] = oacc[nt][1] = oacc[nt][2] = oacc[nt][3] = 0;
     const int kvalid_last = len - (nchunks - 1) * NK;
     for (int c = 0; c < nchunks; ++c) {
-        const uint4 sv = lds128(scores + c * CHUNK_SCORE_BYTES + hk * 512 + lane * 16);
+        const uint4 sv = sc_ld128<GS>(scores, c * CHUNK_SCORE_BYTES + hk * 512 + lane * 16);
         uint32_t pw[4] = {prob_word<false>(sv.x, lut_g, mx4h, f0, f1),
                           prob_word<false>(sv.y, lut_g, mx4h, f0, f1),
                           prob_word<false>(sv.z, lut_g, mx4h, f0, f1),
@@ -1093,9 +1153,10 @@ __device__ __forceinline__ void quarter_chunk_mma(int (&bacc)[4][4], int (&cacc)
 // steps).  Row maxima, exponential sums and the attn.V partial sums (warp w
 // finishes d = 32 w .. 32 w + 31) are combined through the warps' exchange
 // areas behind the quad barrier, eight phases per quarter.
+template <bool GS>
 __device__ __forceinline__ bool consume_quarter(const FusedParams &prm, const Item &it, int u0,
                                                 const Ring &R, uint32_t remap, uint32_t remap0,
-                                                uint32_t scores, uint32_t lut, uint32_t quad,
+                                                const ScoreBuf &scores, uint32_t lut, uint32_t quad,
                                                 int warp, int lane) {
     const int len = it.len, nchunks = it.nchunks;
     const int g = lane >> 2, t4 = lane & 3;
@@ -1154,7 +1215,7 @@ __device__ __forceinline__ bool consume_quarter(const FusedParams &prm, const It
                 pk[i] = score_tile<false>(qc[i], i, remap, lane, m_c, m_p, half_s, s_s, kvalid,
                                           mx0, mx1);
         }
-        sts64(scores + c * CHUNK_SCORE_BYTES + lane * 8, static_cast<int>(pk[0]),
+        sc_st64<GS>(scores, c * CHUNK_SCORE_BYTES + lane * 8, static_cast<int>(pk[0]),
               static_cast<int>(pk[1]));
     }
     release_stage(R.qempty(), lane);   // done with the Q tile
@@ -1177,7 +1238,7 @@ __device__ __forceinline__ bool consume_quarter(const FusedParams &prm, const It
     unsigned long long sum0 = 0, sum1 = 0;
     for (int c = 0; c < nchunks; ++c) {
         const int kvalid = len - c * NK - 16 * warp;
-        const int2 wv = lds64(scores + c * CHUNK_SCORE_BYTES + lane * 8);
+        const int2 wv = sc_ld64<GS>(scores, c * CHUNK_SCORE_BYTES + lane * 8);
         const uint32_t w2[2] = {static_cast<uint32_t>(wv.x), static_cast<uint32_t>(wv.y)};
 #pragma unroll
         for (int q = 0; q < 2; ++q) {
@@ -1219,7 +1280,7 @@ __device__ __forceinline__ bool consume_quarter(const FusedParams &prm, const It
     const int vkey = 16 * warp + 8 * ((lane >> 3) & 1) + (lane & 7);
     for (int c = 0; c < nchunks; ++c) {
         const int kvalid = len - c * NK - 16 * warp;
-        const int2 wv = lds64(scores + c * CHUNK_SCORE_BYTES + lane * 8);
+        const int2 wv = sc_ld64<GS>(scores, c * CHUNK_SCORE_BYTES + lane * 8);
         uint32_t pw0 = prob_word<false>(static_cast<uint32_t>(wv.x), lut_g, mx4h, f0, f1);
         uint32_t pw1 = prob_word<false>(static_cast<uint32_t>(wv.y), lut_g, mx4h, f0, f1);
         if (kvalid < 16) {
@@ -1322,6 +1383,7 @@ __device__ __forceinline__ void zero_rows(const FusedParams &p, const Item &it, 
             make_int4(0, 0, 0, 0);
 }
 
+template <bool GS>
 __global__ void __launch_bounds__(NTHREADS, 2)
     relpos_mhsa_fused_kernel(const __grid_constant__ CUtensorMap tm_q,
                              const __grid_constant__ CUtensorMap tm_k,
@@ -1330,7 +1392,7 @@ __global__ void __launch_bounds__(NTHREADS, 2)
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-    const SmemLayout L = smem_layout(prm.nchunk_max);
+    const SmemLayout L = smem_layout(prm.nchunk_max, GS);
     const int T = prm.T;
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
@@ -1539,7 +1601,11 @@ __global__ void __launch_bounds__(NTHREADS, 2)
 
     // ------------------------------------------------------------ consumers
     const uint32_t remap = smem_u32(smem + L.remap) + warp * REMAP_BYTES;
-    const uint32_t scores = smem_u32(smem + L.scores) + warp * (prm.nchunk_max * CHUNK_SCORE_BYTES);
+    ScoreBuf scores;
+    scores.s = smem_u32(smem + L.scores) + warp * (prm.nchunk_max * CHUNK_SCORE_BYTES);
+    scores.g = GS ? prm.gscores + (static_cast<size_t>(blockIdx.x) * NCWARPS + warp) *
+                                      static_cast<size_t>(prm.nchunk_max) * CHUNK_SCORE_BYTES
+                  : nullptr;
     if (prm.stall_injection && !warp_wait(never_bar, 0, prm.timeout_cycles)) {
         if (lane == 0) atomicOr(prm.err, ERR_TIMEOUT_INJECTED);
         return;
@@ -1554,10 +1620,10 @@ __global__ void __launch_bounds__(NTHREADS, 2)
         if (item == NO_ITEM) return;
         const Item it = decode_item(prm, item);
         const bool ok =
-            it.nparts == 1   ? consume_whole(prm, it, u0, R, remap, scores, lut, warp, lane)
-            : it.nparts == 2 ? consume_half(prm, it, u0, R, remap, scores, lut, pair_bar(warp >> 1),
+            it.nparts == 1   ? consume_whole<GS>(prm, it, u0, R, remap, scores, lut, warp, lane)
+            : it.nparts == 2 ? consume_half<GS>(prm, it, u0, R, remap, scores, lut, pair_bar(warp >> 1),
                                             warp, lane)
-                             : consume_quarter(prm, it, u0, R, remap, smem_u32(smem + L.remap),
+                             : consume_quarter<GS>(prm, it, u0, R, remap, smem_u32(smem + L.remap),
                                                scores, lut, R.quad(), warp, lane);
         if (!ok) return;
         u0 += 2 * it.nchunks;

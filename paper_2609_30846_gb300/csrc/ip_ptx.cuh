@@ -157,6 +157,34 @@ __device__ __forceinline__ void sts128(uint32_t addr, uint32_t x, uint32_t y, ui
                  : "memory");
 }
 
+// Global memory cached in L2 only (.cg): the long-sequence score slices,
+// written and read back by the same thread.
+__device__ __forceinline__ void stg128_cg(void *addr, uint32_t x, uint32_t y, uint32_t z,
+                                          uint32_t w) {
+    asm volatile("st.global.cg.v4.u32 [%0], {%1,%2,%3,%4};" ::"l"(addr), "r"(x), "r"(y), "r"(z),
+                 "r"(w)
+                 : "memory");
+}
+
+__device__ __forceinline__ uint4 ldg128_cg(const void *addr) {
+    uint4 v;
+    asm volatile("ld.global.cg.v4.u32 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                 : "l"(addr)
+                 : "memory");
+    return v;
+}
+
+__device__ __forceinline__ void stg64_cg(void *addr, int x, int y) {
+    asm volatile("st.global.cg.v2.s32 [%0], {%1,%2};" ::"l"(addr), "r"(x), "r"(y) : "memory");
+}
+
+__device__ __forceinline__ int2 ldg64_cg(const void *addr) {
+    int2 v;
+    asm volatile("ld.global.cg.v2.s32 {%0,%1}, [%2];" : "=r"(v.x), "=r"(v.y) : "l"(addr) : "memory");
+    return v;
+}
+
 // D += A B with A 16x32 s8 (row), B 32x8 s8 (col), D 16x8 s32.
 __device__ __forceinline__ void mma_s8s8(int (&d)[4], const uint32_t (&a)[4], uint32_t b0,
                                          uint32_t b1) {

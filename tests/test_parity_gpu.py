@@ -128,6 +128,29 @@ def test_longest_sequence(ip, orc):
     assert_same(run_gpu(ip, lay, c), oracle_out(orc, lay, c))
 
 
+@pytest.mark.parametrize("T,masked", [(450, False), (520, True), (1100, False)])
+def test_long_sequences_in_both_score_modes(ip, orc, T, masked):
+    # Beyond 384 frames the int8 scores move to the workspace when it holds
+    # their region (ip_relpos_mhsa_workspace_bytes counts it): two CTAs per
+    # SM instead of one.  With only the 256-byte status workspace the kernel
+    # keeps them in shared memory.  Both equal the oracle.
+    B, H = 2, 3
+    lens = np.array([T, T // 2 + 7], np.int32) if masked else None
+    lay = synth.draw(B, H, T, 128, seed=1300 + T, p_mode="sinusoid", lengths=lens)
+    c = ip.layer_constants(lay.scales)
+    want = oracle_out(orc, lay, c, lens)
+    assert ip.workspace_bytes(B, H, T) > 256
+    for ws_bytes in (ip.workspace_bytes(B, H, T), 256):
+        ws = torch.zeros(ws_bytes, dtype=torch.uint8, device="cuda")
+        dl = None if lens is None else _dev(lens)
+        g = Guarded((B, H, T, 128), torch.int8)
+        out = ip.relpos_mhsa_i8(_dev(lay.q), _dev(lay.k), _dev(lay.v), _dev(lay.p), _dev(lay.u),
+                                _dev(lay.vb), c, lengths=dl, out=g.view, workspace=ws)
+        assert ip.status(ws) == 0
+        g.check()
+        assert_same(out.cpu().numpy(), want)
+
+
 def test_empty_batch(ip):
     lay = synth.draw(0, 8, 10, 128, seed=1)
     c = ip.layer_constants(synth.draw(1, 8, 10, 128, seed=1).scales)

@@ -44,7 +44,7 @@ def mode(request, ip):
     ip.set_split_mode(-1)
 
 
-@pytest.mark.parametrize("T", [1, 2, 31, 32, 33, 63, 64, 65, 96, 97, 129, 200])
+@pytest.mark.parametrize("T", [1, 2, 31, 32, 33, 63, 64, 65, 96, 97, 129, 200, 450])
 def test_ragged_T(ip, orc, mode, T):
     lay = synth.draw(2, 3, T, 128, seed=900 + T, p_mode="sinusoid")
     c = ip.layer_constants(lay.scales)
