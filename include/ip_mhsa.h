@@ -170,8 +170,7 @@ int ip_relpos_mhsa_i8_host(const int8_t *q, const int8_t *k, const int8_t *v,
  * the cached address would belong to the destroyed context.  Every call shares the array and
  * clears its status word in stream order before launching; calls that
  * overlap on the GPU (concurrent streams) race on it.  Kernel-side barrier
- * timeouts are recorded there and are not reported by this entry point; a
- * caller that needs them uses ip_relpos_mhsa_i8 with a workspace.
+ * timeouts are recorded there; ip_relpos_mhsa_noalloc_status reads them.
  * Returns IP_OK or an IP_ERR_* code as ip_relpos_mhsa_i8. */
 #define IP_NOALLOC_SCRATCH_BYTES 256
 int ip_relpos_mhsa_i8_noalloc(const int8_t *q, const int8_t *k, const int8_t *v,
@@ -179,6 +178,16 @@ int ip_relpos_mhsa_i8_noalloc(const int8_t *q, const int8_t *k, const int8_t *v,
                               const int32_t *multipliers, const int32_t *shifts,
                               const ip_isoftmax_params *sm, const int32_t *lengths,
                               int B, int H, int T, int dh, int8_t *out, ip_stream_t stream);
+
+/* Device-side status of the ip_relpos_mhsa_i8_noalloc calls made on the
+ * current device since the last call of this function or of the entry
+ * point itself (each call clears the word before its kernel): synchronises
+ * `stream`, returns IP_OK, IP_ERR_TIMEOUT (a bounded barrier wait ran out)
+ * or IP_ERR_PARAM (a device-side constant out of its domain), and clears
+ * the word.  Read it after the call whose result is in question, on the
+ * call's stream, before the next call.  Allocates nothing; IP_OK if the
+ * entry point was never called on this device. */
+int ip_relpos_mhsa_noalloc_status(ip_stream_t stream);
 
 /* ---- integer linear layer (Sec. 2.2, Eqs. 6-7) ------------------------
  *

@@ -34,7 +34,7 @@ EXPORTS = (
     "ip_residual_params", "ip_linear_glu_i8", "ip_glu_params", "ip_dwconv_swish_i8",
     "ip_swish16_params_from_scales", "ip_relpos_mhsa_i8_host_async", "ip_relpos_mhsa_host_status",
     "ip_set_workspace", "ip_probe_int8_mix", "ip_linear_residual_i8",
-    "ip_relpos_layer_constants", "ip_linear_constants",
+    "ip_relpos_layer_constants", "ip_linear_constants", "ip_relpos_mhsa_noalloc_status",
 )
 
 ROWS = 0    # IP_LAYOUT_ROWS:  [B][T][C]
@@ -101,6 +101,8 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
         lib.ip_relpos_mhsa_i8_host.restype = I
         lib.ip_relpos_mhsa_i8_noalloc.argtypes = sig[:15] + [P]
         lib.ip_relpos_mhsa_i8_noalloc.restype = I
+        lib.ip_relpos_mhsa_noalloc_status.argtypes = [P]
+        lib.ip_relpos_mhsa_noalloc_status.restype = I
         lib.ip_relpos_mhsa_status.argtypes = [P, P]
         lib.ip_relpos_mhsa_status.restype = I
         lib.ip_set_workspace.argtypes = [P, ctypes.c_size_t]
@@ -378,6 +380,13 @@ def status(workspace=None, stream=None) -> int:
     workspace registered by set_workspace."""
     ptr = None if workspace is None else ctypes.c_void_p(workspace.data_ptr())
     return load().ip_relpos_mhsa_status(ptr, _stream_handle(stream))
+
+
+def noalloc_status(stream=None) -> int:
+    """Synchronises the stream and returns the device-side status code of
+    the ip_relpos_mhsa_i8_noalloc calls on the current device since the
+    last read (0 = ok), clearing it."""
+    return load().ip_relpos_mhsa_noalloc_status(_stream_handle(stream))
 
 
 _default_workspace = None

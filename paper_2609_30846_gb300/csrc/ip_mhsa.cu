@@ -547,6 +547,19 @@ int ip_relpos_mhsa_i8_noalloc(const int8_t *q, const int8_t *k, const int8_t *v,
                              out, scratch, IP_NOALLOC_SCRATCH_BYTES, stream);
 }
 
+int ip_relpos_mhsa_noalloc_status(ip_stream_t stream) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return IP_ERR_CUDA;
+    {
+        std::lock_guard<std::mutex> lock(g_noalloc_mu);
+        if (g_noalloc_addr[dev] == nullptr) return IP_OK;   // no call on this device yet
+    }
+    void *scratch = nullptr;
+    const int rc = noalloc_scratch(&scratch);
+    if (rc != IP_OK) return rc;
+    return ip_relpos_mhsa_status(scratch, stream);
+}
+
 int ip_dyadic_multiplier(double ratio, int32_t *m, int32_t *s) {
     if (!m || !s) return IP_ERR_NULL;
     if (!(ratio > 0.0) || !isfinite(ratio)) return IP_ERR_PARAM;

@@ -8,8 +8,10 @@ test calls it through the C ABI twice in a row and checks that both calls
 give exactly the output of ip_relpos_mhsa_i8, the entry point that takes a
 caller-owned workspace (integer path: the tolerance is bit-exactness), and
 issues two calls back to back on one stream with no synchronisation between
-them, which is where the shared scratch is reused.  It lives in a file of
-its own that pytest collects last.
+them, which is where the shared scratch is reused.  A barrier wait that runs
+out inside such a call (the stall-injection hook with a short bound) is read
+back by ip_relpos_mhsa_noalloc_status.  It lives in a file of its own that
+pytest collects last.
 """
 import ctypes
 
@@ -56,7 +58,7 @@ def test_noalloc_matches_workspace_entry_point(masked):
             None if dlen is None else _ptr(dlen), B, H, T, dh, _ptr(got),
             ctypes.c_void_p(stream.cuda_stream))
         assert rc == 0, ip.strerror(rc)
-        torch.cuda.synchronize()
+        assert ip.noalloc_status() == 0
         np.testing.assert_array_equal(got.cpu().numpy(), want.cpu().numpy())
 
 
@@ -100,9 +102,43 @@ def test_noalloc_calls_back_to_back_in_stream_order():
     torch.cuda.synchronize()
     for dev, c, dlen, shape, got, _ in todo:      # back to back, no sync between
         _noalloc_call(lib, ip, dev, c, dlen, shape, got, stream)
-    torch.cuda.synchronize()
+    assert ip.noalloc_status() == 0
     for _, _, _, _, got, want in todo:
         np.testing.assert_array_equal(got.cpu().numpy(), want.cpu().numpy())
+
+
+def test_noalloc_reports_barrier_timeout():
+    # every consumer warp first waits on a barrier nobody arrives on, with a
+    # bound of about a millisecond: the wait runs out, the kernel records
+    # IP_ERR_TIMEOUT in the library's scratch word and returns; the status
+    # reader reports it once and clears it, and the next call is exact
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import oracle
+    import paper_2609_30846_gb300 as ip
+    lib = ip.load()
+    B, H, T, dh = 2, 8, 200, 128
+    lay = synth.draw(B, H, T, dh, seed=8301, p_mode="sinusoid")
+    c = ip.layer_constants(lay.scales)
+    dev = {n: torch.from_numpy(np.ascontiguousarray(getattr(lay, n))).cuda()
+           for n in ("q", "k", "v", "p", "u", "vb")}
+    out = torch.zeros((B, H, T, dh), dtype=torch.int8, device="cuda")
+    stream = torch.cuda.current_stream()
+    assert ip.noalloc_status() == 0
+    try:
+        ip.set_timeout_cycles(2_000_000)
+        ip.set_stall_injection(True)
+        _noalloc_call(lib, ip, dev, c, None, (B, H, T, dh), out, stream)
+        assert ip.noalloc_status() == -6     # IP_ERR_TIMEOUT, read and cleared
+        assert ip.noalloc_status() == 0
+    finally:
+        ip.set_stall_injection(False)
+        ip.set_timeout_cycles(-1)
+    _noalloc_call(lib, ip, dev, c, None, (B, H, T, dh), out, stream)
+    assert ip.noalloc_status() == 0
+    want = oracle.relpos_mhsa(lay.q, lay.k, lay.v, lay.p, lay.u, lay.vb,
+                              oracle.layer_constants(lay.scales, 128))
+    np.testing.assert_array_equal(out.cpu().numpy(), want)
 
 
 def test_noalloc_rejects_bad_shapes():
