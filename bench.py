@@ -275,10 +275,13 @@ def rows_traffic() -> dict:
     try:
         rec = json.load(open(ROWS_TRAFFIC_FILE))
         csrc = os.path.join(ROOT, "paper_2609_30846_gb300", "csrc")
-        for f, h in rec.get("kernel_sha256", {}).items():
-            if hashlib.sha256(open(os.path.join(csrc, f), "rb").read()).hexdigest() != h:
-                return {}
-        return {k: v["dram_bytes_per_launch"] for k, v in rec.get("rows", {}).items()}
+        out = {}
+        for k, v in rec.get("rows", {}).items():
+            # each row names the sources of its kernel and their hashes at capture
+            if all(hashlib.sha256(open(os.path.join(csrc, f), "rb").read()).hexdigest() == h
+                   for f, h in v["kernel_sha256"].items()):
+                out[k] = v["dram_bytes_per_launch"]
+        return out
     except (OSError, ValueError, KeyError):
         return {}
 
@@ -654,6 +657,64 @@ def measure_next_rows(dev, peak, pipes, steps: int, cpu: bool):
     rows["layernorm_1024"] = row
     del xs, outs, x0
 
+    # the ConvBlock's depthwise convolution (K = 9) with the folded
+    # BatchNorm onto INT16 and the Swish, on the block's B x T x 1024
+    # frames; timed like the LayerNorm (a group of NORM_BUFS launches on as
+    # many input/output pairs after the flush)
+    C, Kd = 1024, 9
+    rng = np.random.default_rng(7200)
+    xd0 = torch.from_numpy(rng.integers(-127, 128, size=(B, T, C)).astype(np.int8)).to(dev)
+    wd = torch.from_numpy(rng.integers(-127, 128, size=(C, Kd)).astype(np.int8)).to(dev)
+    bd = torch.from_numpy(rng.integers(-20000, 20000, size=C).astype(np.int32)).to(dev)
+    s_bn = 40.0 / 32767
+    md, sd = ip.linear_constants(0.04, rng.uniform(0.001, 0.01, C), np.full(C, s_bn))
+    md, sd = torch.from_numpy(md).to(dev), torch.from_numpy(sd).to(dev)
+    p16 = ip.swish16_params(s_bn, 5.0 / 127)
+    xs = [xd0] + [xd0.clone() for _ in range(NORM_BUFS - 1)]
+    outs = [torch.empty_like(xd0) for _ in range(NORM_BUFS)]
+    ws = torch.zeros(256, dtype=torch.uint8, device=dev)
+    call = lambda i: ip.dwconv_swish_i8(xs[i], wd, bd, md, sd, p16, out=outs[i], workspace=ws,
+                                        stream=stream)
+    for i in range(NORM_BUFS):
+        call(i)
+    times = []
+    for _ in range(steps):
+        flush()
+        torch.cuda._sleep(1_500_000)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for i in range(NORM_BUFS):
+            call(i)
+        e1.record(stream)
+        e1.synchronize()
+        times.append(e0.elapsed_time(e1) * 1e-3 / NORM_BUFS)
+    if ip.status(ws, stream) != 0:
+        raise SystemExit("dwconv: kernel reported an error")
+    t = statistics.median(times)
+    elems = B * T * C
+    ops = (2 * Kd + DW_OPS_PER_ELEMENT) * elems
+    row = {"value": elems * 2 / t / 1e9, "unit": "GB/s", "us_per_launch": t * 1e6,
+           "shape": {"B": B, "T": T, "C": C, "K": Kd},
+           "roofline": {"bound": "alu", "achieved": ops / t / 1e12, "peak": alu_peak,
+                        "unit": "Tops/s (int32 lane ops)", "frac": ops / t / 1e12 / alu_peak,
+                        "traffic": traffic.get("block_dwconv_swish_k9"),
+                        "hbm_frac": elems * 2 / t / 1e9 / HBM_GBS},
+           "kernel": f"dwconv_swish_x4_kernel<{Kd}>", "gpu_launches": NORM_BUFS,
+           "timing": f"{NORM_BUFS} launches on {NORM_BUFS} input/output pairs per event pair"}
+    if cpu:
+        import oracle
+        oracle.build()
+        mh, sh = md.cpu().numpy(), sd.cpu().numpy()
+        xh, wh, bh = xd0[:1].cpu().numpy(), wd.cpu().numpy(), bd.cpu().numpy()
+        t0 = time.perf_counter()
+        oracle.swish16(oracle.dwconv(xh, wh, bh, mh, sh), oracle.Swish16Params(*p16))
+        dt = time.perf_counter() - t0
+        row["cpu_baseline"] = {"value": T * C * 2 / dt / 1e9, "unit": "GB/s",
+                               "cores": 1, "kind": "oracle",
+                               "sample": f"1 of {B} utterances (T={T}), {dt:.2f} s"}
+    rows["dwconv_swish_k9_1024"] = row
+    del xs, outs, xd0
+
     # one whole integer Conformer block (Eqs. 1-5): 15 launches
     import synth.block as sblock
     from paper_2609_30846_gb300.block import GPU_LAUNCHES, ConformerBlock
@@ -723,6 +784,12 @@ def measure_next_rows(dev, peak, pipes, steps: int, cpu: bool):
 # sum and sum of squares (2), centring d q - sum (2), c f with rounding and
 # shift (3), M n + B with rounding and shift (3), clamp (2).
 NORM_OPS_PER_ELEMENT = 12
+# Of the depthwise convolution + INT16 requantisation + Swish, besides the
+# K multiply-adds (2 K): bias (1), m acc with rounding and shift (3), clamp
+# to INT16 (2), |z| and min(|z|, q_c) - q_c (3), its square and q_one - D^2
+# (2), the sign term q_one + sgn(z) L (2), z t (1), m_sw z t with rounding
+# and shift (3), clamp (2).
+DW_OPS_PER_ELEMENT = 19
 def _hbm_gbs() -> float:
     """Measured copy bandwidth of this GPU type (MEASURED_PEAKS.json, written
     by the pool's driver), else the 6.8 TB/s fallback."""

@@ -30,6 +30,48 @@ int sm_count() {
     return g_sms[dev];
 }
 
+// Resident CTAs of dwconv_swish_x4_kernel<K> on the current device (SMs x
+// CTAs per SM), looked up once per device and K.
+int g_dw4_slots[64][ipb::DW_KMAX + 1] = {{0}};
+
+template <int K>
+cudaError_t launch_dw4(ipb::DwParams p, cudaStream_t st) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+    int slots = 0;
+    {
+        std::lock_guard<std::mutex> lock(g_mu);
+        slots = g_dw4_slots[dev][K];
+    }
+    if (slots == 0) {
+        int per_sm = 0;
+        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, ipb::dwconv_swish_x4_kernel<K>,
+                                                          ipb::DW4_THREADS, 0);
+        if (e != cudaSuccess) return e;
+        slots = (per_sm > 0 ? per_sm : 1) * sm_count();
+        if (slots <= 0) return cudaErrorInvalidValue;
+        std::lock_guard<std::mutex> lock(g_mu);
+        g_dw4_slots[dev][K] = slots;
+    }
+    // channel blocks of 256 channels; the frames of each split evenly over
+    // the slots left for it
+    const int ncb = (p.C / 4 + ipb::DW4_THREADS - 1) / ipb::DW4_THREADS;
+    const long long frames = static_cast<long long>(p.B) * p.T;
+    long long per_block = slots / ncb > 0 ? slots / ncb : 1;
+    // a multiple of the frames of one step, so that only utterance ends
+    // leave a partly used step
+    constexpr int step = 4 * ipb::DW4_BLOCKS;
+    const long long per = ((frames + per_block - 1) / per_block + step - 1) / step * step;
+    per_block = (frames + per - 1) / per;
+    p.frames_per_cta = static_cast<uint32_t>(per);
+    p.t_magic = iph::div_magic(static_cast<unsigned long long>(p.T));
+    return iph::launch_pdl(ipb::dwconv_swish_x4_kernel<K>,
+                           dim3(static_cast<unsigned>(per_block), static_cast<unsigned>(ncb)),
+                           dim3(ipb::DW4_THREADS), 0, st, p);
+}
+
 int check_swish16(const ip_swish16_params *p) {
     if (p->q_c < 1 || p->q_c >= (1 << 16) || p->q_one < 1 || p->q_one >= (1ll << 31) ||
         p->q_one < static_cast<long long>(p->q_c) * p->q_c || p->m < 0 || p->s < 0 || p->s > 31)
@@ -100,10 +142,26 @@ int ip_dwconv_swish_i8(const int8_t *x, int B, int T, int C, const int8_t *w, in
     p.sw_m = sw->m;
     p.sw_s = sw->s;
     p.err = static_cast<int *>(workspace);
-    const dim3 grid((C + ipb::DW_THREADS - 1) / ipb::DW_THREADS,
-                    (T + ipb::DW_FRAMES - 1) / ipb::DW_FRAMES, B);
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
     cudaError_t lrc;
+    if (C % 4 == 0 && aligned(x, 4) && aligned(y, 4) && aligned(w, 4) &&
+        static_cast<long long>(B) * T < (1ll << 31)) {
+        // four channels per thread, one CTA per resident slot
+        switch (K) {   // odd, 1 .. DW_KMAX (checked above)
+            case 1: lrc = launch_dw4<1>(p, st); break;
+            case 3: lrc = launch_dw4<3>(p, st); break;
+            case 5: lrc = launch_dw4<5>(p, st); break;
+            case 7: lrc = launch_dw4<7>(p, st); break;
+            case 9: lrc = launch_dw4<9>(p, st); break;
+            case 11: lrc = launch_dw4<11>(p, st); break;
+            case 13: lrc = launch_dw4<13>(p, st); break;
+            default: lrc = launch_dw4<15>(p, st); break;
+        }
+        if (lrc != cudaSuccess) return IP_ERR_CUDA;
+        return cudaGetLastError() == cudaSuccess ? IP_OK : IP_ERR_CUDA;
+    }
+    const dim3 grid((C + ipb::DW_THREADS - 1) / ipb::DW_THREADS,
+                    (T + ipb::DW_FRAMES - 1) / ipb::DW_FRAMES, B);
     switch (K) {   // odd, 1 .. DW_KMAX (checked above)
         case 1: lrc = iph::launch_pdl(ipb::dwconv_swish_kernel<1>, grid, dim3(ipb::DW_THREADS), 0, st, p); break;
         case 3: lrc = iph::launch_pdl(ipb::dwconv_swish_kernel<3>, grid, dim3(ipb::DW_THREADS), 0, st, p); break;

@@ -160,10 +160,13 @@ def test_glu_projection(ip, orc, B, T, K, C):
     assert_same(got.cpu().numpy(), want)
 
 
+# C a multiple of 4 takes the four-channels-per-thread kernel (C = 300 and
+# 260: a partly filled CTA), C = 258 and 66 the one-channel kernel.
 @pytest.mark.parametrize("B,T,C,K", [(1, 1, 256, 9), (2, 33, 256, 9), (3, 100, 512, 5),
                                      (32, 375, 1024, 9), (1, 70, 300, 15), (2, 40, 256, 1),
                                      (2, 40, 256, 3), (1, 50, 256, 7), (1, 50, 256, 11),
-                                     (1, 50, 256, 13)])
+                                     (1, 50, 256, 13), (2, 37, 260, 15), (1, 33, 4, 3),
+                                     (1, 40, 258, 9), (2, 45, 66, 5)])
 def test_dwconv_swish(ip, orc, B, T, C, K):
     rng = np.random.default_rng(T * C + K)
     x = rng.integers(-127, 128, size=(B, T, C)).astype(np.int8)
@@ -181,6 +184,63 @@ def test_dwconv_swish(ip, orc, B, T, C, K):
     assert ip.status(ws) == 0
     g.check()
     assert_same(got.cpu().numpy(), want)
+
+
+def _dw_case(rng, B, T, C, K):
+    x = rng.integers(-127, 128, size=(B, T, C)).astype(np.int8)
+    w = rng.integers(-127, 128, size=(C, K)).astype(np.int8)
+    bias = rng.integers(-20000, 20000, size=C).astype(np.int32)
+    m, s = (rng.integers(1, 2 ** 31, size=C).astype(np.int32),
+            rng.integers(10, 20, size=C).astype(np.int32))
+    return x, w, bias, m, s
+
+
+def test_dwconv_unaligned_buffers_take_the_one_channel_kernel(ip, orc):
+    # x and y one byte off a 4-byte boundary (C a multiple of 4): the
+    # one-channel kernel runs and gives the same bytes as the oracle
+    rng = np.random.default_rng(77)
+    B, T, C, K = 2, 50, 256, 9
+    x, w, bias, m, s = _dw_case(rng, B, T, C, K)
+    p16 = orc.swish16_params(40.0 / 32767, 5.0 / 127)
+    want = orc.swish16(orc.dwconv(x, w, bias, m, s), p16)
+    xs = torch.zeros(B * T * C + 1, dtype=torch.int8, device="cuda")
+    xs[1:] = _d(x).flatten()
+    ys = torch.zeros(B * T * C + 1, dtype=torch.int8, device="cuda")
+    got = ip.dwconv_swish_i8(xs[1:].view(B, T, C), _d(w), _d(bias), _d(m), _d(s),
+                             (p16.q_c, p16.q_one, p16.m, p16.s), out=ys[1:].view(B, T, C))
+    assert_same(got.cpu().numpy(), want)
+    assert int(ys[0]) == 0
+
+
+@pytest.mark.parametrize("C", [256, 258])
+def test_dwconv_extreme_constants(ip, orc, C):
+    # multipliers 0, 1 and 2^31 - 1, shifts 0, 1, 30 and 31, biases at the
+    # domain's edges, and Swish constants at the edges of theirs (q_one =
+    # 2^31 - 1 with the largest q_c it allows; m_sw = 2^31 - 1 at s = 0 and
+    # 31): every rounding and both clamps, in both kernels
+    rng = np.random.default_rng(C)
+    B, T, K = 1, 64, 9
+    x = rng.integers(-127, 128, size=(B, T, C)).astype(np.int8)
+    x[0, ::7] = 127
+    x[0, 3::7] = -127
+    w = rng.integers(-127, 128, size=(C, K)).astype(np.int8)
+    w[::5] = 127
+    mv = np.array([0, 1, 2 ** 31 - 1, 2 ** 30, 123456789], np.int64)
+    sv = np.array([0, 1, 30, 31, 17], np.int64)
+    bv = np.array([2 ** 30 - 1, -(2 ** 30 - 1), 0, 12345, -54321], np.int64)
+    m = mv[rng.integers(0, 5, C)].astype(np.int32)
+    s = sv[rng.integers(0, 5, C)].astype(np.int32)
+    bias = bv[rng.integers(0, 5, C)].astype(np.int32)
+    for p16 in (orc.Swish16Params(46340, 2 ** 31 - 1, 2 ** 31 - 1, 31),
+                orc.Swish16Params(46340, 2 ** 31 - 1, 2 ** 31 - 1, 0),
+                orc.Swish16Params(1, 1, 2 ** 31 - 1, 31),
+                orc.Swish16Params(300, 90000, 1, 0)):
+        want = orc.swish16(orc.dwconv(x, w, bias, m, s), p16)
+        ws = torch.zeros(256, dtype=torch.uint8, device="cuda")
+        got = ip.dwconv_swish_i8(_d(x), _d(w), _d(bias), _d(m), _d(s),
+                                 (p16.q_c, p16.q_one, p16.m, p16.s), workspace=ws)
+        assert ip.status(ws) == 0
+        assert_same(got.cpu().numpy(), want)
 
 
 def test_dwconv_saturating_int16(ip, orc):
