@@ -997,6 +997,8 @@ def run_ours(args):
                      "alu_floor": issue_floor(dev, avg_layer_ms * 1e3,
                                               (clk or {}).get("sm_mhz") or 2070.0),
                      "integer_pipes_tops": pipes,
+                     "frac_of_both_pipes": (achieved / pipes["imma_plus_dp4a"]
+                                            if (pipes or {}).get("imma_plus_dp4a") else None),
                      "integer_pipes_note": "measured in this run: the integer MMA pipe and the "
                                            "dp4a pipe alone and together (ip_probe_int8_mix); "
                                            "the fused kernel's contractions use the MMA pipe",
