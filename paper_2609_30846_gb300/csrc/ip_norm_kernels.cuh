@@ -1,7 +1,8 @@
 // Device code of the integer LayerNorm (I-Parakeet, Sec. 2.1, Eqs. 1-4, with
 // the integer kernel of Sec. 2.2) for sm_103a.  Integer arithmetic only: no
 // floating-point type, no division by a run-time value (d is a compile-time
-// multiple of 512; the square root and the reciprocal are digit-by-digit).
+// multiple of 512; the square root and the reciprocal are Newton iterations
+// with multiplications only, each settled exactly by a final comparison).
 //
 // One warp per batch of four rows of d channels, batches dealt warp-major
 // over a grid of one CTA per SM, so that every warp takes two or more
@@ -42,35 +43,61 @@ struct NormParams {
     int *err;
 };
 
-// floor(sqrt(n)) for 0 <= n < 2^42, digit by digit (no division).
+// floor(sqrt(n)) for 0 <= n < 2^42 by Newton's iteration on 1 / sqrt, with
+// multiplications only.  An even shift normalises n to m = n 4^k in [2^40,
+// 2^42), M = m / 2^42 in [1/4, 1).  y approximates 2^30 / sqrt(M): it starts
+// from the chord of that function over [1/4, 1/2) or [1/2, 1) (y0 = a - b q
+// with q = M 2^10; relative error under 3 %), and each step y <- y (3 - M
+// y^2) / 2, in fixed point (t = M y^2 2^60 by a 64 x 64 high product, y' =
+// y (3 2^60 - t) / 2^61), squares the error: after three steps it is below
+// 2^-28 with the truncations.  sqrt(m) is then m y / 2^51, and its integer
+// part shifted right by k lies within one of floor(sqrt(n)); two
+// comparisons each way settle it.
 __device__ __forceinline__ unsigned long long isqrt_u42(unsigned long long n) {
-    unsigned long long r = 0;
-    // the root has at most (bit length of n + 1) / 2 bits: start there
-    const int k0 = n == 0 ? -1 : (63 - __clzll(static_cast<long long>(n))) >> 1;
-#pragma unroll 1
-    for (int k = k0; k >= 0; --k) {
-        const unsigned long long bit = 1ull << (2 * k);
-        const bool take = n >= r + bit;
-        n -= take ? r + bit : 0ull;
-        r = (r >> 1) + (take ? bit : 0ull);
+    if (n == 0) return 0;
+    const int k = (__clzll(static_cast<long long>(n)) - 22) >> 1;
+    const unsigned long long m = n << (2 * k);
+    const unsigned long long q = m >> 32;   // M 2^10, in [256, 1024)
+    // chord of 2^30 / sqrt(q / 2^10) through q = 256, 512 and q = 512, 1024
+    unsigned long long y = q < 512 ? 2776467046ull - 2456966ull * q : 1963258675ull - 868669ull * q;
+#pragma unroll
+    for (int it = 0; it < 3; ++it) {
+        const unsigned long long t = __umul64hi(m << 22, y * y);
+        y = __umul64hi(y << 32, 3ull * (1ull << 60) - t) >> 29;
     }
-    return r;
+    unsigned long long s = (__umul64hi(m << 22, y << 10) >> 19) >> k;
+    s -= s * s > n ? 1ull : 0ull;
+    s -= s * s > n ? 1ull : 0ull;
+    s += (s + 1) * (s + 1) <= n ? 1ull : 0ull;
+    s += (s + 1) * (s + 1) <= n ? 1ull : 0ull;
+    return s;
 }
 
-// floor(2^31 / s) for 1 <= s < 2^32 by restoring binary long division.
-__device__ __forceinline__ uint32_t recip_2pow31(unsigned long long s) {
-    unsigned long long rem = 1ull << 31;
-    uint32_t quo = 0;
-    // s >= 2^(L-1) for bit length L, so the quotient is below 2^(32 - L)
-    const int top = __clzll(static_cast<long long>(s)) - 32;   // 32 - L
-#pragma unroll 1
-    for (int bit = top < 31 ? top : 31; bit >= 0; --bit) {
-        const unsigned long long t = s << bit;          // s < 2^32: no overflow
-        const bool take = t <= rem;
-        rem -= take ? t : 0ull;
-        quo |= take ? (1u << bit) : 0u;
+// floor(2^31 / s) for 1 <= s < 2^22 by Newton's iteration on the
+// reciprocal of the normalised divisor, with multiplications only.  With L
+// the bit length of s, x = s 2^(22-L) lies in [2^21, 2^22), X = x / 2^22 in
+// [1/2, 1), and floor(2^31 / s) = floor(floor(2^52 / x) / 2^(L-1)).  r
+// approximates 2^52 / x: the start 2^30 (48 - 32 X) / 17 has relative error
+// at most 1/17, and each step r += r (2^52 - x r) / 2^52 squares it (three
+// steps: below 2^-29 with the truncations).  q = r / 2^(L-1) is then within
+// one of the quotient, and the remainder 2^31 - q s settles it.
+__device__ __forceinline__ uint32_t recip_2pow31(unsigned long long s64) {
+    const long long s = static_cast<long long>(s64);
+    const int L = 64 - __clzll(s);
+    const long long x = s << (22 - L);
+    long long r = (51539607552ll - 8192ll * x) / 17;   // 2^30 (48 - 32 X) / 17
+#pragma unroll
+    for (int it = 0; it < 3; ++it) {
+        const long long e = (1ll << 52) - x * r;       // |e| < 2^48
+        r += (r * (e >> 21)) >> 31;
     }
-    return quo;
+    long long q = r >> (L - 1);
+    long long rem = (1ll << 31) - q * s;
+    if (rem < 0) { --q; rem += s; }
+    if (rem < 0) { --q; rem += s; }
+    if (rem >= s) { ++q; rem -= s; }
+    if (rem >= s) { ++q; }
+    return static_cast<uint32_t>(q);
 }
 
 // C = d / 512 segments of 16 channels per lane.  A warp takes NB rows at a

@@ -71,6 +71,36 @@ def test_special_rows(ip, orc):
         assert_same(*run_both(ip, orc, x, gamma, beta, s_x, s_y, eps))
 
 
+def test_sigma_and_reciprocal_over_their_range(ip, orc):
+    # sigma = isqrt(floor(sum c^2 / d) + eps_c) and f = floor(2^31 / sigma)
+    # are Newton iterations in the kernel: rows with one to three nonzero
+    # values (and constant rows) give floor(sum c^2 / d) = d sum q^2 -
+    # (sum q)^2 over a wide spread, and eps_c from 0 to 2^40 (powers of two
+    # and their neighbours, where the normalisation changes) moves sigma
+    # from 1 to 2^20; every output against the oracle
+    d, rows = 512, 2048
+    rng = np.random.default_rng(12)
+    x = np.zeros((rows, d), np.int8)
+    for r in range(rows):
+        k = int(rng.integers(0, 4))
+        x[r, rng.choice(d, size=k, replace=False)] = rng.integers(-127, 128, size=k)
+    x[::97] = rng.integers(-127, 128)
+    _, gamma, beta, s_x, s_y, _ = case(1, d, seed=13)
+    c = orc.layernorm_constants(s_x, gamma, beta, s_y, 1e-5)
+    eps_values = [0, 1, 2, 3, 5, 2 ** 40]
+    for k in range(2, 40, 3):
+        eps_values += [2 ** k - 1, 2 ** k, 2 ** k + 1]
+    eps_values += [int(v) for v in rng.integers(0, 2 ** 40, size=6)]
+    ws = torch.zeros(256, dtype=torch.uint8, device="cuda")
+    xd = _d(x)
+    Md, Bd, Ed = _d(c.M), _d(c.B), _d(c.E)
+    for eps_c in eps_values:
+        got = ip.layernorm_i8(xd, Md, Bd, Ed, eps_c, workspace=ws)
+        assert ip.status(ws) == 0
+        want = orc.layernorm(x, orc.NormConstants(M=c.M, B=c.B, E=c.E, eps_c=eps_c))
+        assert_same(got.cpu().numpy(), want)
+
+
 def test_small_variance_rows(ip, orc):
     assert_same(*run_both(ip, orc, *case(64, 1024, seed=6, eps=2e-4, spread=0.6)))
 
